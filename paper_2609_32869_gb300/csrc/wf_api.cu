@@ -1,0 +1,823 @@
+// Host orchestration of the Whisper-Flash decode step and the C ABI (wf.h).
+//
+// Per call the host enqueues kernels on the caller's stream; it never waits
+// for the device except where an entry point says so (wf_compact,
+// wf_get_state, wf_get_error).  All device memory is carved from the caller's
+// workspace; the library allocates nothing on the device.
+#include <algorithm>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "wf_device.cuh"
+#include "wf_internal.h"
+
+using namespace wf;
+
+struct wf_handle {
+  wf_config cfg;
+  int Bmax = 0, ctx = 0, Mmax = 0, d = 0, H = 0, F = 0, V = 0, K = 0, nl = 0, nd = 0;
+  std::vector<wf_layer_weights> tl, dl;
+  wf_target_weights tw;
+  wf_drafter_weights dw;
+  // per-slot state
+  int32_t *L, *anchor, *remaining, *done, *step, *snap_L, *snap_anchor, *snap_rem;
+  int32_t *active, *n_active_dev, *cand;
+  uint32_t *err;
+  // caches
+  bf16 *self_k, *self_v, *cross_k, *cross_v, *hist_k, *hist_v;
+  // activations
+  float *x, *xd, *hproj;
+  bf16 *xn, *q, *att, *h1, *taps, *hn;
+  // scratch
+  float *partial;
+  int32_t *gemm_counters;
+  size_t partial_floats;
+  int gemm_counter_cap;
+  float *apart;
+  int32_t *attn_counters;
+  size_t apart_floats;
+  int attn_counter_cap;
+  HeadRec *recs_t, *recs_d;
+  HeadOut *hout_t, *hout_d;
+  float *logits_t, *logits_d;
+  float2 *rope;
+  int n_vtiles = 0;
+  int n_active = 0;
+  int launches = 0;
+  bool in_step = false;
+  bool keep_logits = false;
+};
+
+namespace {
+
+constexpr int kAlign = 256;
+
+struct Carver {
+  char *base;
+  size_t off = 0;
+  template <typename T>
+  T *take(size_t count) {
+    off = (off + kAlign - 1) / kAlign * kAlign;
+    T *p = base ? reinterpret_cast<T *>(base + off) : nullptr;
+    off += count * sizeof(T);
+    return p;
+  }
+};
+
+bool cfg_ok(const wf_config *c) {
+  if (!c) return false;
+  if (c->d_model <= 0 || c->n_heads <= 0 || c->d_model != c->n_heads * 64) return false;
+  if (c->d_model % 64 || c->d_ff % 64 || c->d_ff <= 0) return false;
+  if (c->d_model > 1536) return false;
+  if (c->n_layers <= 0 || c->n_layers > WF_MAX_LAYERS) return false;
+  if (c->n_draft_layers <= 0 || c->n_draft_layers > 8) return false;
+  if (c->vocab <= 0 || c->max_pos <= 0 || c->max_pos > 4096 || c->enc_frames <= 0) return false;
+  if (c->block_k < 1 || c->block_k > 8) return false;
+  if (c->n_taps < 1 || c->n_taps > WF_MAX_TAPS) return false;
+  for (int i = 0; i < c->n_taps; ++i)
+    if (c->taps[i] < 0 || c->taps[i] >= c->n_layers) return false;
+  if (c->eos_id < 0 || c->eos_id >= c->vocab) return false;
+  return true;
+}
+
+int rows_max(const wf_config *c, int Bmax, int ctx) {
+  return std::max(Bmax * (c->block_k + 1), ctx);
+}
+
+// Largest split-K scratch (floats per token row) over the per-step projections.
+size_t partial_per_row(const wf_config *c) {
+  const int d = c->d_model, F = c->d_ff;
+  const int shapes[][2] = {{3 * d, d}, {d, d}, {F, d}, {d, F}, {d, c->n_taps * d}, {2 * d, d}};
+  size_t best = 0;
+  for (auto &sh : shapes) {
+    const int s = gemm_splits(sh[0], sh[1]);
+    if (s > 1) best = std::max(best, static_cast<size_t>(s) * sh[0]);
+  }
+  return best;
+}
+
+// Lay the workspace out (base == nullptr: only measure).
+size_t layout(wf_handle *h, const wf_config *c, int Bmax, int ctx, char *base) {
+  Carver cv{base};
+  const int d = c->d_model, H = c->n_heads, F = c->d_ff, V = c->vocab, K = c->block_k;
+  const int nl = c->n_layers, nd = c->n_draft_layers, T = c->enc_frames;
+  const int Mmax = rows_max(c, Bmax, ctx);
+  const size_t sl = static_cast<size_t>(Bmax);
+  wf_handle tmp;
+  wf_handle *o = h ? h : &tmp;
+  o->L = cv.take<int32_t>(sl);
+  o->anchor = cv.take<int32_t>(sl);
+  o->remaining = cv.take<int32_t>(sl);
+  o->done = cv.take<int32_t>(sl);
+  o->step = cv.take<int32_t>(sl);
+  o->snap_L = cv.take<int32_t>(sl);
+  o->snap_anchor = cv.take<int32_t>(sl);
+  o->snap_rem = cv.take<int32_t>(sl);
+  o->active = cv.take<int32_t>(sl);
+  o->n_active_dev = cv.take<int32_t>(1);
+  o->cand = cv.take<int32_t>(sl * K);
+  o->err = cv.take<uint32_t>(1);
+  const size_t self_sz = static_cast<size_t>(nl) * sl * H * ctx * 64;
+  o->self_k = cv.take<bf16>(self_sz);
+  o->self_v = cv.take<bf16>(self_sz);
+  const size_t cross_sz = static_cast<size_t>(nl + nd) * sl * H * T * 64;
+  o->cross_k = cv.take<bf16>(cross_sz);
+  o->cross_v = cv.take<bf16>(cross_sz);
+  const size_t hist_sz = static_cast<size_t>(nd) * sl * H * ctx * 64;
+  o->hist_k = cv.take<bf16>(hist_sz);
+  o->hist_v = cv.take<bf16>(hist_sz);
+  const size_t M = static_cast<size_t>(Mmax);
+  o->x = cv.take<float>(M * d);
+  o->xd = cv.take<float>(M * d);
+  o->hproj = cv.take<float>(M * d);
+  o->xn = cv.take<bf16>(M * d);
+  o->q = cv.take<bf16>(M * d);
+  o->att = cv.take<bf16>(M * d);
+  o->hn = cv.take<bf16>(M * d);
+  o->h1 = cv.take<bf16>(M * F);
+  o->taps = cv.take<bf16>(M * c->n_taps * d);
+  o->partial_floats = M * partial_per_row(c);
+  o->partial = cv.take<float>(std::max<size_t>(o->partial_floats, 1));
+  o->gemm_counter_cap = 1 << 16;
+  o->gemm_counters = cv.take<int32_t>(o->gemm_counter_cap);
+  const int groups = Bmax + Mmax / kAttnQGroup + 1;
+  const int chunks = (std::max(ctx, T) + kAttnChunk - 1) / kAttnChunk;
+  o->apart_floats = static_cast<size_t>(groups) * H * chunks * kAttnQGroup * 66;
+  o->apart = cv.take<float>(o->apart_floats);
+  o->attn_counter_cap = groups * H;
+  o->attn_counters = cv.take<int32_t>(o->attn_counter_cap);
+  const int vt = (V + 127) / 128;
+  o->recs_t = cv.take<HeadRec>(M * vt);
+  o->recs_d = cv.take<HeadRec>(M * vt);
+  o->hout_t = cv.take<HeadOut>(M);
+  o->hout_d = cv.take<HeadOut>(M);
+  o->logits_t = cv.take<float>(M * V);
+  o->logits_d = cv.take<float>(M * V);
+  o->rope = cv.take<float2>(static_cast<size_t>(c->max_pos) * 32);
+  return cv.off + kAlign;
+}
+
+inline cudaStream_t S(void *s) { return static_cast<cudaStream_t>(s); }
+
+#define WF_TRY(expr)                               \
+  do {                                             \
+    cudaError_t _e = (expr);                       \
+    if (_e != cudaSuccess) return WF_ERR_CUDA;     \
+  } while (0)
+
+constexpr bool kPDL = true;
+
+// ---------------------------------------------------------------- GEMMs --
+GemmParams gemm_base(wf_handle *h, int M, int N, int K, int epi) {
+  GemmParams p = {};
+  p.M = M;
+  p.N = N;
+  p.K = K;
+  p.epi = epi;
+  p.splits = gemm_splits(N, K);
+  p.partial = h->partial;
+  p.counters = h->gemm_counters;
+  p.err = h->err;
+  p.d_model = h->d;
+  p.n_heads = h->H;
+  return p;
+}
+
+cudaError_t gemm(wf_handle *h, const void *X, const void *W, GemmParams p, cudaStream_t s) {
+  if (p.splits > 1) {
+    if (gemm_partial_floats(p.M, p.N, p.splits) > h->partial_floats) return cudaErrorInvalidValue;
+    if (gemm_counter_slots(p.M, p.N) > h->gemm_counter_cap) return cudaErrorInvalidValue;
+  }
+  h->launches++;
+  return launch_gemm(X, W, p, s, kPDL);
+}
+
+cudaError_t layernorm(wf_handle *h, const float *x, int stride, int off, const void *g,
+                      const void *b, bf16 *y, int rows, cudaStream_t s) {
+  h->launches++;
+  return launch_layernorm(x, stride, off, static_cast<const bf16 *>(g),
+                          static_cast<const bf16 *>(b), y, rows, h->d, h->cfg.ln_eps, s, kPDL);
+}
+
+cudaError_t attention(wf_handle *h, const bf16 *q, const bf16 *kc, const bf16 *vc,
+                      const int32_t *slots, int n_seq, int rps, int ctx, int mode, bool rope,
+                      cudaStream_t s) {
+  AttnParams p = {};
+  p.q = q;
+  p.kc = kc;
+  p.vc = vc;
+  p.out = h->att;
+  p.seq_slot = slots;
+  p.pos_base = h->L;
+  p.rope_tab = rope ? h->rope : nullptr;
+  p.part = h->apart;
+  p.counters = h->attn_counters;
+  p.err = h->err;
+  p.n_seq = n_seq;
+  p.rps = rps;
+  p.n_heads = h->H;
+  p.ctx = ctx;
+  p.mode = mode;
+  if (attn_partial_floats(n_seq, rps, h->H, ctx) > h->apart_floats) return cudaErrorInvalidValue;
+  if (attn_counter_slots(n_seq, rps, h->H) > h->attn_counter_cap) return cudaErrorInvalidValue;
+  h->launches++;
+  return launch_attention(p, s, kPDL);
+}
+
+size_t layer_cache_off(wf_handle *h, int layer, int positions) {
+  return static_cast<size_t>(layer) * h->Bmax * h->H * positions * 64;
+}
+
+struct Pass {
+  int n_seq, rps;
+  const int32_t *slots;
+  bool drafter;
+  float *x;
+  bool taps;
+};
+
+// One pre-LayerNorm Whisper block over the pass's rows.
+cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, int layer,
+                      cudaStream_t s) {
+  const int M = ps.n_seq * ps.rps, d = h->d;
+  cudaError_t e;
+  bf16 *kc, *vc, *xkc, *xvc;
+  if (ps.drafter) {
+    kc = h->hist_k + layer_cache_off(h, layer, h->ctx);
+    vc = h->hist_v + layer_cache_off(h, layer, h->ctx);
+    xkc = h->cross_k + layer_cache_off(h, h->nl + layer, h->cfg.enc_frames);
+    xvc = h->cross_v + layer_cache_off(h, h->nl + layer, h->cfg.enc_frames);
+  } else {
+    kc = h->self_k + layer_cache_off(h, layer, h->ctx);
+    vc = h->self_v + layer_cache_off(h, layer, h->ctx);
+    xkc = h->cross_k + layer_cache_off(h, layer, h->cfg.enc_frames);
+    xvc = h->cross_v + layer_cache_off(h, layer, h->cfg.enc_frames);
+  }
+  // self-attention
+  if ((e = layernorm(h, ps.x, 1, 0, lw.ln1_g, lw.ln1_b, h->xn, M, s)) != cudaSuccess) return e;
+  {
+    GemmParams p = gemm_base(h, M, 3 * d, d, EPI_KV);
+    p.bias = static_cast<const bf16 *>(lw.qkv_b);
+    p.out_bf16 = h->q;
+    p.ld_out = d;
+    p.q_cols = d;
+    p.kc = kc;
+    p.vc = vc;
+    p.ctx = h->ctx;
+    p.rows_per_seq = ps.rps;
+    p.seq_slot = ps.slots;
+    p.pos_base = h->L;
+    if ((e = gemm(h, h->xn, lw.qkv_w, p, s)) != cudaSuccess) return e;
+  }
+  if ((e = attention(h, h->q, kc, vc, ps.slots, ps.n_seq, ps.rps, h->ctx, ps.drafter ? 1 : 0,
+                     ps.drafter, s)) != cudaSuccess)
+    return e;
+  {
+    GemmParams p = gemm_base(h, M, d, d, EPI_RESID);
+    p.bias = static_cast<const bf16 *>(lw.out_b);
+    p.resid = ps.x;
+    p.ld_resid = d;
+    if ((e = gemm(h, h->att, lw.out_w, p, s)) != cudaSuccess) return e;
+  }
+  // cross-attention
+  if ((e = layernorm(h, ps.x, 1, 0, lw.ln2_g, lw.ln2_b, h->xn, M, s)) != cudaSuccess) return e;
+  {
+    GemmParams p = gemm_base(h, M, d, d, EPI_BF16);
+    p.bias = static_cast<const bf16 *>(lw.xq_b);
+    p.out_bf16 = h->q;
+    p.ld_out = d;
+    if ((e = gemm(h, h->xn, lw.xq_w, p, s)) != cudaSuccess) return e;
+  }
+  if ((e = attention(h, h->q, xkc, xvc, ps.slots, ps.n_seq, ps.rps, h->cfg.enc_frames, 2, false,
+                     s)) != cudaSuccess)
+    return e;
+  {
+    GemmParams p = gemm_base(h, M, d, d, EPI_RESID);
+    p.bias = static_cast<const bf16 *>(lw.xout_b);
+    p.resid = ps.x;
+    p.ld_resid = d;
+    if ((e = gemm(h, h->att, lw.xout_w, p, s)) != cudaSuccess) return e;
+  }
+  // feed-forward
+  if ((e = layernorm(h, ps.x, 1, 0, lw.ln3_g, lw.ln3_b, h->xn, M, s)) != cudaSuccess) return e;
+  {
+    GemmParams p = gemm_base(h, M, h->F, d, EPI_GELU);
+    p.bias = static_cast<const bf16 *>(lw.fc1_b);
+    p.out_bf16 = h->h1;
+    p.ld_out = h->F;
+    if ((e = gemm(h, h->xn, lw.fc1_w, p, s)) != cudaSuccess) return e;
+  }
+  {
+    GemmParams p = gemm_base(h, M, d, h->F, EPI_RESID);
+    p.bias = static_cast<const bf16 *>(lw.fc2_b);
+    p.resid = ps.x;
+    p.ld_resid = d;
+    if (ps.taps) {
+      // the block's output residual stream, before the final LayerNorm (App. A.2)
+      int found = 0;
+      for (int t = 0; t < h->cfg.n_taps; ++t) {
+        if (h->cfg.taps[t] != layer) continue;
+        bf16 *dst = h->taps + static_cast<size_t>(t) * d;
+        if (found == 0) p.tap0 = dst;
+        else if (found == 1) p.tap1 = dst;
+        ++found;
+      }
+      p.ld_tap = h->cfg.n_taps * d;
+    }
+    if ((e = gemm(h, h->h1, lw.fc2_w, p, s)) != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+// Final LayerNorm (the target's, shared with the drafter) and the tied head.
+cudaError_t head(wf_handle *h, const float *x, int stride, int off, int rows, const int32_t *slots,
+                 int rps, HeadRec *recs, HeadOut *out, float *logits, const wf_sample_params *sp,
+                 uint32_t tag, int32_t *cand, cudaStream_t s) {
+  cudaError_t e;
+  if ((e = layernorm(h, x, stride, off, h->tw.lnf_g, h->tw.lnf_b, h->xn, rows, s)) != cudaSuccess)
+    return e;
+  const bool sampling = sp && sp->temperature > 0.f;
+  GemmParams p = gemm_base(h, rows, h->V, h->d, EPI_HEAD);
+  p.recs = recs;
+  p.logits = (sampling || h->keep_logits) ? logits : nullptr;
+  p.keep_logits = h->keep_logits ? 1 : 0;
+  p.temperature = sampling ? sp->temperature : 0.f;
+  p.seed = sp ? sp->seed : 0;
+  p.suppress = sp ? sp->d_suppress : nullptr;
+  p.step = h->step;
+  p.tag = tag;
+  p.rows_per_seq = rps;
+  p.seq_slot = slots;
+  if ((e = gemm(h, h->xn, h->tw.tok_emb, p, s)) != cudaSuccess) return e;
+  HeadReduceParams r = {};
+  r.recs = recs;
+  r.out = out;
+  r.rows = rows;
+  r.n_tiles = h->n_vtiles;
+  r.cand = cand;
+  r.seq_slot = slots;
+  r.rps = rps;
+  r.K = h->K;
+  r.sampling = sampling ? 1 : 0;
+  h->launches++;
+  return launch_head_reduce(r, s, kPDL);
+}
+
+// History memory (Sec. 3.2, App. A.2): project the tapped residual streams of
+// the pass's rows, normalise, and write each drafter block's keys/values at
+// the rows' text positions (L + j).
+cudaError_t ingest(wf_handle *h, int n_seq, int rps, const int32_t *slots, cudaStream_t s) {
+  const int M = n_seq * rps, d = h->d;
+  cudaError_t e;
+  {
+    GemmParams p = gemm_base(h, M, d, h->cfg.n_taps * d, EPI_F32);
+    p.bias = static_cast<const bf16 *>(h->dw.proj_b);
+    p.out_f32 = h->hproj;
+    p.ld_out = d;
+    if ((e = gemm(h, h->taps, h->dw.proj_w, p, s)) != cudaSuccess) return e;
+  }
+  if ((e = layernorm(h, h->hproj, 1, 0, h->dw.hln_g, h->dw.hln_b, h->hn, M, s)) != cudaSuccess)
+    return e;
+  for (int l = 0; l < h->nd; ++l) {
+    const wf_layer_weights &lw = h->dl[l];
+    GemmParams p = gemm_base(h, M, 2 * d, d, EPI_KV);
+    p.bias = static_cast<const bf16 *>(lw.qkv_b) + d;
+    p.q_cols = 0;
+    p.kc = h->hist_k + layer_cache_off(h, l, h->ctx);
+    p.vc = h->hist_v + layer_cache_off(h, l, h->ctx);
+    p.ctx = h->ctx;
+    p.rows_per_seq = rps;
+    p.seq_slot = slots;
+    p.pos_base = h->L;
+    const bf16 *wkv = static_cast<const bf16 *>(lw.qkv_w) + static_cast<size_t>(d) * d;
+    if ((e = gemm(h, h->hn, wkv, p, s)) != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t target_pass(wf_handle *h, int n_seq, int rps, const int32_t *slots, int src,
+                        const int32_t *prompt, int P, const int32_t *forced, bool taps,
+                        cudaStream_t s) {
+  EmbedParams ep = {};
+  ep.tok_emb = static_cast<const bf16 *>(h->tw.tok_emb);
+  ep.pos_emb = static_cast<const bf16 *>(h->tw.pos_emb);
+  ep.seq_slot = slots;
+  ep.L = h->L;
+  ep.anchor = h->anchor;
+  ep.cand_in = h->cand;
+  ep.cand_out = h->cand;
+  ep.forced = forced;
+  ep.prompt = prompt;
+  ep.x = h->x;
+  ep.n_seq = n_seq;
+  ep.rps = rps;
+  ep.d = h->d;
+  ep.K = h->K;
+  ep.P = P;
+  ep.vocab = h->V;
+  ep.src = src;
+  ep.drafter = 0;
+  ep.err = h->err;
+  h->launches++;
+  cudaError_t e = launch_embed(ep, s, kPDL);
+  if (e != cudaSuccess) return e;
+  Pass ps{n_seq, rps, slots, false, h->x, taps};
+  for (int l = 0; l < h->nl; ++l)
+    if ((e = run_block(h, ps, h->tl[l], l, s)) != cudaSuccess) return e;
+  return cudaSuccess;
+}
+
+wf_status check_weights(const wf_layer_weights &w) {
+  const void *ptrs[] = {w.ln1_g, w.ln1_b, w.qkv_w, w.qkv_b, w.out_w, w.out_b, w.ln2_g,
+                        w.ln2_b, w.xq_w,  w.xq_b,  w.xkv_w, w.xkv_b, w.xout_w, w.xout_b,
+                        w.ln3_g, w.ln3_b, w.fc1_w, w.fc1_b, w.fc2_w, w.fc2_b};
+  for (const void *p : ptrs) {
+    if (!p) return WF_ERR_INVALID;
+    if (reinterpret_cast<uintptr_t>(p) & 15) return WF_ERR_INVALID;
+  }
+  return WF_OK;
+}
+
+}  // namespace
+
+// ====================================================================== ABI
+extern "C" {
+
+const char *wf_status_str(wf_status s) {
+  switch (s) {
+    case WF_OK: return "ok";
+    case WF_ERR_INVALID: return "invalid argument";
+    case WF_ERR_CAPACITY: return "capacity exceeded";
+    case WF_ERR_CUDA: return "CUDA error";
+    case WF_ERR_UNSUPPORTED: return "unsupported shape";
+    case WF_ERR_DEVICE: return "device error word set";
+  }
+  return "unknown status";
+}
+
+wf_status wf_workspace_bytes(const wf_config *cfg, int32_t max_batch, int32_t max_ctx,
+                             size_t *out_bytes) {
+  if (!out_bytes || !cfg) return WF_ERR_INVALID;
+  if (!cfg_ok(cfg)) return WF_ERR_UNSUPPORTED;
+  if (max_batch <= 0 || max_ctx <= cfg->block_k + 1 || max_ctx > cfg->max_pos) return WF_ERR_INVALID;
+  *out_bytes = layout(nullptr, cfg, max_batch, max_ctx, nullptr);
+  return WF_OK;
+}
+
+wf_status wf_create(const wf_config *cfg, const wf_target_weights *tw, const wf_drafter_weights *dw,
+                    int32_t max_batch, int32_t max_ctx, void *d_workspace, size_t workspace_bytes,
+                    void *stream, wf_handle **out) {
+  if (!cfg || !tw || !dw || !out || !d_workspace) return WF_ERR_INVALID;
+  *out = nullptr;
+  size_t need = 0;
+  wf_status st = wf_workspace_bytes(cfg, max_batch, max_ctx, &need);
+  if (st != WF_OK) return st;
+  if (workspace_bytes < need) return WF_ERR_CAPACITY;
+  if (reinterpret_cast<uintptr_t>(d_workspace) % kAlign) return WF_ERR_INVALID;
+  if (!tw->tok_emb || !tw->pos_emb || !tw->lnf_g || !tw->lnf_b || !tw->layers) return WF_ERR_INVALID;
+  if (!dw->layers || !dw->proj_w || !dw->proj_b || !dw->hln_g || !dw->hln_b || !dw->mask_emb)
+    return WF_ERR_INVALID;
+  int dev = 0, major = 0, minor = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return WF_ERR_CUDA;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+    return WF_ERR_CUDA;
+  if (major != 10 || minor != 3) return WF_ERR_UNSUPPORTED;
+  wf_handle *h = new (std::nothrow) wf_handle;
+  if (!h) return WF_ERR_CAPACITY;
+  h->cfg = *cfg;
+  h->Bmax = max_batch;
+  h->ctx = max_ctx;
+  h->Mmax = rows_max(cfg, max_batch, max_ctx);
+  h->d = cfg->d_model;
+  h->H = cfg->n_heads;
+  h->F = cfg->d_ff;
+  h->V = cfg->vocab;
+  h->K = cfg->block_k;
+  h->nl = cfg->n_layers;
+  h->nd = cfg->n_draft_layers;
+  h->n_vtiles = (cfg->vocab + 127) / 128;
+  h->tl.assign(tw->layers, tw->layers + cfg->n_layers);
+  h->dl.assign(dw->layers, dw->layers + cfg->n_draft_layers);
+  for (auto &w : h->tl)
+    if (check_weights(w) != WF_OK) { delete h; return WF_ERR_INVALID; }
+  for (auto &w : h->dl)
+    if (check_weights(w) != WF_OK) { delete h; return WF_ERR_INVALID; }
+  h->tw = *tw;
+  h->tw.layers = h->tl.data();
+  h->dw = *dw;
+  h->dw.layers = h->dl.data();
+  layout(h, cfg, max_batch, max_ctx, static_cast<char *>(d_workspace));
+  cudaStream_t s = S(stream);
+  const size_t sl = static_cast<size_t>(max_batch) * sizeof(int32_t);
+  bool ok = cudaMemsetAsync(h->L, 0, sl, s) == cudaSuccess &&
+            cudaMemsetAsync(h->anchor, 0, sl, s) == cudaSuccess &&
+            cudaMemsetAsync(h->remaining, 0, sl, s) == cudaSuccess &&
+            cudaMemsetAsync(h->done, 0x01, sl, s) == cudaSuccess &&  // no slot is active yet
+            cudaMemsetAsync(h->step, 0, sl, s) == cudaSuccess &&
+            cudaMemsetAsync(h->cand, 0, sl * h->K, s) == cudaSuccess &&
+            cudaMemsetAsync(h->n_active_dev, 0, sizeof(int32_t), s) == cudaSuccess &&
+            cudaMemsetAsync(h->err, 0, sizeof(uint32_t), s) == cudaSuccess &&
+            cudaMemsetAsync(h->gemm_counters, 0, h->gemm_counter_cap * sizeof(int32_t), s) == cudaSuccess &&
+            cudaMemsetAsync(h->attn_counters, 0, h->attn_counter_cap * sizeof(int32_t), s) == cudaSuccess &&
+            launch_rope_table(h->rope, cfg->max_pos, cfg->rope_base, s) == cudaSuccess;
+  if (!ok) {
+    delete h;
+    return WF_ERR_CUDA;
+  }
+  *out = h;
+  return WF_OK;
+}
+
+wf_status wf_destroy(wf_handle *h) {
+  if (!h) return WF_ERR_INVALID;
+  delete h;
+  return WF_OK;
+}
+
+int32_t wf_last_launch_count(const wf_handle *h) { return h ? h->launches : -1; }
+
+wf_status wf_set_option(wf_handle *h, int32_t option, int32_t value) {
+  if (!h) return WF_ERR_INVALID;
+  if (option == WF_OPT_KEEP_LOGITS) {
+    h->keep_logits = value != 0;
+    return WF_OK;
+  }
+  return WF_ERR_INVALID;
+}
+
+wf_status wf_debug_view(wf_handle *h, int32_t which, void **d_ptr, size_t *bytes) {
+  if (!h || !d_ptr || !bytes) return WF_ERR_INVALID;
+  const size_t M = static_cast<size_t>(h->Mmax);
+  switch (which) {
+    case WF_VIEW_TARGET_LOGITS:
+      *d_ptr = h->logits_t;
+      *bytes = M * h->V * sizeof(float);
+      return WF_OK;
+    case WF_VIEW_DRAFT_LOGITS:
+      *d_ptr = h->logits_d;
+      *bytes = M * h->V * sizeof(float);
+      return WF_OK;
+    case WF_VIEW_TAPS:
+      *d_ptr = h->taps;
+      *bytes = M * h->cfg.n_taps * h->d * sizeof(bf16);
+      return WF_OK;
+    case WF_VIEW_CANDIDATES:
+      *d_ptr = h->cand;
+      *bytes = static_cast<size_t>(h->Bmax) * h->K * sizeof(int32_t);
+      return WF_OK;
+  }
+  return WF_ERR_INVALID;
+}
+
+wf_status wf_prefill_cross_kv(wf_handle *h, int32_t n, const int32_t *d_slots, const void *d_enc,
+                              const int32_t *d_prompt, int32_t P, const int32_t *d_budget,
+                              int32_t *d_first, const wf_sample_params *sp, void *stream) {
+  if (!h || !d_slots || !d_enc || !d_prompt || !d_budget || n <= 0 || P <= 0) return WF_ERR_INVALID;
+  if (h->n_active + n > h->Bmax) return WF_ERR_CAPACITY;
+  if (P + h->K + 1 > h->ctx || P > h->Mmax) return WF_ERR_CAPACITY;
+  if (reinterpret_cast<uintptr_t>(d_enc) & 15) return WF_ERR_INVALID;
+  cudaStream_t s = S(stream);
+  h->launches = 0;
+  const int d = h->d, T = h->cfg.enc_frames;
+  // acoustic keys/values of every target and drafter block (App. A.5)
+  for (int l = 0; l < h->nl + h->nd; ++l) {
+    const wf_layer_weights &lw = l < h->nl ? h->tl[l] : h->dl[l - h->nl];
+    GemmParams p = gemm_base(h, n * T, 2 * d, d, EPI_KV);
+    p.splits = 1;
+    p.bias = static_cast<const bf16 *>(lw.xkv_b);
+    p.q_cols = 0;
+    p.kc = h->cross_k + layer_cache_off(h, l, T);
+    p.vc = h->cross_v + layer_cache_off(h, l, T);
+    p.ctx = T;
+    p.rows_per_seq = T;
+    p.seq_slot = d_slots;
+    p.pos_base = nullptr;
+    WF_TRY(gemm(h, d_enc, lw.xkv_w, p, s));
+  }
+  StateParams sp0 = {};
+  sp0.op = 0;
+  sp0.n = n;
+  sp0.slots = d_slots;
+  sp0.max_batch = h->Bmax;
+  sp0.L = h->L;
+  sp0.anchor = h->anchor;
+  sp0.remaining = h->remaining;
+  sp0.done = h->done;
+  sp0.step = h->step;
+  h->launches++;
+  WF_TRY(launch_state(sp0, s, kPDL));
+  const int g = std::max(1, std::min(n, h->Mmax / P));
+  const bool sampling = sp && sp->temperature > 0.f;
+  for (int i0 = 0; i0 < n; i0 += g) {
+    const int gn = std::min(g, n - i0);
+    const int32_t *slots = d_slots + i0;
+    WF_TRY(target_pass(h, gn, P, slots, TOK_PROMPT, d_prompt + static_cast<size_t>(i0) * P, P,
+                       nullptr, true, s));
+    WF_TRY(ingest(h, gn, P, slots, s));
+    WF_TRY(head(h, h->x, P, P - 1, gn, slots, 1, h->recs_t, h->hout_t, h->logits_t, sp, kTagBonus,
+                nullptr, s));
+    StateParams sp1 = sp0;
+    sp1.op = 1;
+    sp1.n = gn;
+    sp1.slots = slots;
+    sp1.budget = d_budget + i0;
+    sp1.hout = h->hout_t;
+    sp1.first = d_first ? d_first + i0 : nullptr;
+    sp1.P = P;
+    sp1.eos = h->cfg.eos_id;
+    sp1.sampling = sampling ? 1 : 0;
+    sp1.snap_L = h->snap_L;
+    sp1.snap_anchor = h->snap_anchor;
+    sp1.snap_remaining = h->snap_rem;
+    sp1.active = h->active;
+    sp1.n_active_dev = h->n_active_dev;
+    sp1.active_offset = h->n_active + i0;
+    h->launches++;
+    WF_TRY(launch_state(sp1, s, kPDL));
+  }
+  h->n_active += n;
+  return WF_OK;
+}
+
+wf_status wf_draft(wf_handle *h, const wf_sample_params *sp, void *stream) {
+  if (!h) return WF_ERR_INVALID;
+  h->launches = 0;
+  if (h->n_active == 0) return WF_OK;
+  cudaStream_t s = S(stream);
+  const int n = h->n_active, rps = h->K + 1;
+  EmbedParams ep = {};
+  ep.tok_emb = static_cast<const bf16 *>(h->tw.tok_emb);
+  ep.mask_emb = static_cast<const bf16 *>(h->dw.mask_emb);
+  ep.seq_slot = h->active;
+  ep.anchor = h->anchor;
+  ep.x = h->xd;
+  ep.n_seq = n;
+  ep.rps = rps;
+  ep.d = h->d;
+  ep.K = h->K;
+  ep.vocab = h->V;
+  ep.src = TOK_ANCHOR;
+  ep.drafter = 1;
+  ep.err = h->err;
+  h->launches++;
+  WF_TRY(launch_embed(ep, s, kPDL));
+  Pass ps{n, rps, h->active, true, h->xd, false};
+  for (int l = 0; l < h->nd; ++l) WF_TRY(run_block(h, ps, h->dl[l], l, s));
+  WF_TRY(head(h, h->xd, 1, 0, n * rps, h->active, rps, h->recs_d, h->hout_d, h->logits_d, sp,
+              kTagDraft, h->cand, s));
+  return WF_OK;
+}
+
+wf_status wf_verify_accept(wf_handle *h, const wf_sample_params *sp, const int32_t *d_forced,
+                           int32_t *d_out_tokens, int32_t *d_out_count, void *stream) {
+  if (!h || !d_out_tokens || !d_out_count) return WF_ERR_INVALID;
+  cudaStream_t s = S(stream);
+  if (!h->in_step) h->launches = 0;
+  const int n = h->n_active, rps = h->K + 1;
+  if (n > 0) {
+    WF_TRY(target_pass(h, n, rps, h->active, TOK_VERIFY, nullptr, 0, d_forced, true, s));
+    WF_TRY(head(h, h->x, 1, 0, n * rps, h->active, rps, h->recs_t, h->hout_t, h->logits_t, sp,
+                kTagBonus, nullptr, s));
+    WF_TRY(ingest(h, n, rps, h->active, s));
+  }
+  AcceptParams ap = {};
+  ap.seq_slot = h->active;
+  ap.n_seq = n;
+  ap.rps = rps;
+  ap.K = h->K;
+  ap.max_batch = h->Bmax;
+  ap.vocab = h->V;
+  ap.eos = h->cfg.eos_id;
+  ap.max_ctx = h->ctx;
+  ap.greedy_step = 0;
+  ap.tout = h->hout_t;
+  ap.dout = h->hout_d;
+  ap.cand = h->cand;
+  ap.tlogits = h->logits_t;
+  ap.dlogits = h->logits_d;
+  ap.suppress = sp ? sp->d_suppress : nullptr;
+  ap.temperature = (sp && sp->temperature > 0.f) ? sp->temperature : 0.f;
+  ap.seed = sp ? sp->seed : 0;
+  ap.L = h->L;
+  ap.anchor = h->anchor;
+  ap.remaining = h->remaining;
+  ap.done = h->done;
+  ap.step = h->step;
+  ap.out_tokens = d_out_tokens;
+  ap.out_count = d_out_count;
+  ap.err = h->err;
+  h->launches++;
+  WF_TRY(launch_accept(ap, s, kPDL));
+  return WF_OK;
+}
+
+wf_status wf_step(wf_handle *h, const wf_sample_params *sp, const int32_t *d_forced,
+                  int32_t *d_out_tokens, int32_t *d_out_count, void *stream) {
+  if (!h) return WF_ERR_INVALID;
+  wf_status st = wf_draft(h, sp, stream);
+  if (st != WF_OK) return st;
+  h->in_step = true;
+  st = wf_verify_accept(h, sp, d_forced, d_out_tokens, d_out_count, stream);
+  h->in_step = false;
+  return st;
+}
+
+wf_status wf_greedy_step(wf_handle *h, const wf_sample_params *sp, int32_t *d_out_tokens,
+                         int32_t *d_out_count, void *stream) {
+  if (!h || !d_out_tokens || !d_out_count) return WF_ERR_INVALID;
+  cudaStream_t s = S(stream);
+  h->launches = 0;
+  const int n = h->n_active;
+  if (n > 0) {
+    WF_TRY(target_pass(h, n, 1, h->active, TOK_ANCHOR, nullptr, 0, nullptr, false, s));
+    WF_TRY(head(h, h->x, 1, 0, n, h->active, 1, h->recs_t, h->hout_t, h->logits_t, sp, kTagBonus,
+                nullptr, s));
+  }
+  AcceptParams ap = {};
+  ap.seq_slot = h->active;
+  ap.n_seq = n;
+  ap.rps = 1;
+  ap.K = h->K;
+  ap.max_batch = h->Bmax;
+  ap.vocab = h->V;
+  ap.eos = h->cfg.eos_id;
+  ap.max_ctx = h->ctx;
+  ap.greedy_step = 1;
+  ap.tout = h->hout_t;
+  ap.cand = h->cand;
+  ap.temperature = (sp && sp->temperature > 0.f) ? sp->temperature : 0.f;
+  ap.seed = sp ? sp->seed : 0;
+  ap.L = h->L;
+  ap.anchor = h->anchor;
+  ap.remaining = h->remaining;
+  ap.done = h->done;
+  ap.step = h->step;
+  ap.out_tokens = d_out_tokens;
+  ap.out_count = d_out_count;
+  ap.err = h->err;
+  h->launches++;
+  WF_TRY(launch_accept(ap, s, kPDL));
+  return WF_OK;
+}
+
+wf_status wf_compact(wf_handle *h, void *stream, int32_t *h_n_active) {
+  if (!h) return WF_ERR_INVALID;
+  cudaStream_t s = S(stream);
+  h->launches = 1;
+  WF_TRY(launch_compact(h->done, h->Bmax, h->active, h->n_active_dev, s));
+  int32_t n = 0;
+  WF_TRY(cudaMemcpyAsync(&n, h->n_active_dev, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
+  WF_TRY(cudaStreamSynchronize(s));
+  h->n_active = n;
+  if (h_n_active) *h_n_active = n;
+  return WF_OK;
+}
+
+wf_status wf_reset_slots(wf_handle *h, int32_t n, const int32_t *d_slots, void *stream) {
+  if (!h || !d_slots || n <= 0) return WF_ERR_INVALID;
+  StateParams p = {};
+  p.op = 2;
+  p.n = n;
+  p.slots = d_slots;
+  p.max_batch = h->Bmax;
+  p.L = h->L;
+  p.anchor = h->anchor;
+  p.remaining = h->remaining;
+  p.done = h->done;
+  p.step = h->step;
+  p.snap_L = h->snap_L;
+  p.snap_anchor = h->snap_anchor;
+  p.snap_remaining = h->snap_rem;
+  h->launches = 1;
+  WF_TRY(launch_state(p, S(stream), kPDL));
+  return WF_OK;
+}
+
+wf_status wf_get_state(wf_handle *h, int32_t *h_len, int32_t *h_anchor, int32_t *h_remaining,
+                       int32_t *h_done, void *stream) {
+  if (!h) return WF_ERR_INVALID;
+  cudaStream_t s = S(stream);
+  const size_t sz = static_cast<size_t>(h->Bmax) * sizeof(int32_t);
+  if (h_len) WF_TRY(cudaMemcpyAsync(h_len, h->L, sz, cudaMemcpyDeviceToHost, s));
+  if (h_anchor) WF_TRY(cudaMemcpyAsync(h_anchor, h->anchor, sz, cudaMemcpyDeviceToHost, s));
+  if (h_remaining) WF_TRY(cudaMemcpyAsync(h_remaining, h->remaining, sz, cudaMemcpyDeviceToHost, s));
+  if (h_done) WF_TRY(cudaMemcpyAsync(h_done, h->done, sz, cudaMemcpyDeviceToHost, s));
+  WF_TRY(cudaStreamSynchronize(s));
+  return WF_OK;
+}
+
+wf_status wf_get_error(wf_handle *h, uint32_t *h_err, int32_t clear, void *stream) {
+  if (!h || !h_err) return WF_ERR_INVALID;
+  cudaStream_t s = S(stream);
+  WF_TRY(cudaMemcpyAsync(h_err, h->err, sizeof(uint32_t), cudaMemcpyDeviceToHost, s));
+  WF_TRY(cudaStreamSynchronize(s));
+  if (clear) {
+    WF_TRY(cudaMemsetAsync(h->err, 0, sizeof(uint32_t), s));
+    WF_TRY(cudaStreamSynchronize(s));
+  }
+  return WF_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,459 @@
+// Skinny-M bf16 GEMM on the sm_103a tensor cores (tcgen05 + TMEM + TMA).
+//
+// Every projection of the decode step is Y = X W^T with few token rows
+// (M = 9 per sequence: the anchor and K = 8 proposals, Sec. 3.1) against a
+// large weight matrix, so the weights stream from HBM once and set the time.
+// The kernel computes a 128 x BT tile of D = W_tile X_tile^T ("swap-AB"): the
+// 128 weight rows fill the MMA's M side, the token tile (a multiple of 16,
+// <= 256) its N side.  Weight and token tiles stream into shared memory by
+// TMA (128-byte swizzle) through an mbarrier ring; one thread issues
+// tcgen05.mma into a TMEM accumulator; four warps read it back with
+// tcgen05.ld for a fused epilogue (bias, GELU, residual add, taps, key/value
+// cache scatter, or the output-head reduction).
+//
+// K is split into a fixed number of chunks per (N, K) shape so that ~150 CTAs
+// stream weights even for a single sequence; partial tiles go to a scratch
+// buffer and the last CTA of a tile (atomic ticket, no waiting) sums them in
+// split order, so results are deterministic and independent of M.
+//
+// With programmatic dependent launch the weight tiles of the first pipeline
+// stages are requested before griddepcontrol.wait: they do not depend on the
+// previous kernel, so their HBM latency overlaps its tail.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <mutex>
+#include <map>
+#include <tuple>
+
+#include "wf_device.cuh"
+#include "wf_internal.h"
+
+namespace wf {
+
+constexpr int kBlockN = 128;   // weight rows per tile (MMA M)
+constexpr int kBlockK = 64;    // K per pipeline stage (one 128-byte swizzle atom)
+constexpr int kStageA = kBlockN * kBlockK * 2;  // 16 KB
+constexpr int kSmemBudget = 200 * 1024;
+
+struct __align__(16) RedEntry {
+  float m, s, gm;
+  int arg, garg;
+};
+
+__device__ __forceinline__ void head_combine(float &m, float &s, int &arg, float &gm, int &garg,
+                                             float m2, float s2, int arg2, float gm2, int garg2) {
+  const float M = fmaxf(m, m2);
+  float ns = 0.f;
+  if (M != -INFINITY) {
+    ns = (m == -INFINITY ? 0.f : s * __expf(m - M)) + (m2 == -INFINITY ? 0.f : s2 * __expf(m2 - M));
+  }
+  if (m2 > m || (m2 == m && arg2 < arg)) arg = arg2;
+  m = M;
+  s = ns;
+  if (gm2 > gm || (gm2 == gm && garg2 < garg)) {
+    gm = gm2;
+    garg = garg2;
+  }
+}
+
+template <int EPI>
+__device__ __forceinline__ void epilogue_store(const GemmParams &p, int t, int n, float acc) {
+  if (t >= p.M || n >= p.N) return;
+  float v = acc + (p.bias ? bf2f(p.bias[n]) : 0.f);
+  if constexpr (EPI == EPI_F32) {
+    p.out_f32[static_cast<size_t>(t) * p.ld_out + n] = v;
+  } else if constexpr (EPI == EPI_BF16) {
+    p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(v);
+  } else if constexpr (EPI == EPI_GELU) {
+    p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(gelu_erf(v));
+  } else if constexpr (EPI == EPI_RESID) {
+    float *r = p.resid + static_cast<size_t>(t) * p.ld_resid + n;
+    const float nr = *r + v;
+    *r = nr;
+    if (p.tap0) p.tap0[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
+    if (p.tap1) p.tap1[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
+  } else if constexpr (EPI == EPI_KV) {
+    if (n < p.q_cols) {
+      p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(v);
+      return;
+    }
+    const int c = n - p.q_cols;
+    const int which = c / p.d_model;
+    const int hd = c - which * p.d_model;
+    const int h = hd >> 6, dd = hd & 63;
+    const int i = t / p.rows_per_seq, j = t - i * p.rows_per_seq;
+    const int slot = p.seq_slot[i];
+    const int pos = (p.pos_base ? p.pos_base[slot] : 0) + j;
+    if (pos >= p.ctx) {
+      set_error(p.err, WF_DEV_ERR_CAPACITY);
+      return;
+    }
+    bf16 *dst = which == 0 ? p.kc : p.vc;
+    dst[((static_cast<size_t>(slot) * p.n_heads + h) * p.ctx + pos) * 64 + dd] =
+        __float2bfloat16(v);
+  }
+}
+
+template <int EPI>
+__global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW,
+                                                      const __grid_constant__ CUtensorMap tmX,
+                                                      const GemmParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  uint8_t *smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+  const int BT = p.BT, stages = p.stages, kps = p.kps;
+  const uint32_t stageB = static_cast<uint32_t>(BT) * kBlockK * 2;
+  uint8_t *sA = smem;
+  uint8_t *sB = smem + static_cast<size_t>(stages) * kStageA;
+  uint64_t *full = reinterpret_cast<uint64_t *>(sB + static_cast<size_t>(stages) * stageB);
+  uint64_t *empty = full + stages;
+  uint64_t *done = empty + stages;
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
+  int *flag = reinterpret_cast<int *>(tmem_slot + 1);
+  RedEntry *red = reinterpret_cast<RedEntry *>(smem + static_cast<size_t>(stages) * (kStageA + stageB) +
+                                               (2 * stages + 1) * 8 + 16 + 16);
+  red = reinterpret_cast<RedEntry *>((reinterpret_cast<uintptr_t>(red) + 15) & ~uintptr_t(15));
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int tt = blockIdx.x, ntile = blockIdx.y, split = blockIdx.z;
+  const int n0 = ntile * kBlockN, t0 = tt * BT, kit0 = split * kps;
+
+  if (threadIdx.x == 0) {
+    tma_prefetch_desc(&tmW);
+    tma_prefetch_desc(&tmX);
+    for (int s = 0; s < stages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(done, 1);
+    fence_barrier_init();
+    fence_proxy_async();
+  }
+  if (warp == 2) tmem_alloc(tmem_slot, p.tmem_cols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_launch_dependents();
+
+  if (warp == 0 && lane == 0) {
+    // ---------------- TMA producer
+    const int npre = kps < stages ? kps : stages;
+    const uint32_t tx = kStageA + stageB;
+    for (int i = 0; i < npre; ++i) {
+      mbar_arrive_expect_tx(&full[i], tx);
+      tma_load_2d(sA + static_cast<size_t>(i) * kStageA, &tmW, (kit0 + i) * kBlockK, n0, &full[i]);
+    }
+    pdl_wait();  // token rows come from the previous kernel
+    for (int i = 0; i < npre; ++i)
+      tma_load_2d(sB + static_cast<size_t>(i) * stageB, &tmX, (kit0 + i) * kBlockK, t0, &full[i]);
+    for (int it = npre; it < kps; ++it) {
+      const int s = it % stages;
+      const uint32_t ph = static_cast<uint32_t>((it / stages) - 1) & 1u;
+      if (!mbar_wait(&empty[s], ph, p.err)) break;
+      mbar_arrive_expect_tx(&full[s], tx);
+      tma_load_2d(sA + static_cast<size_t>(s) * kStageA, &tmW, (kit0 + it) * kBlockK, n0, &full[s]);
+      tma_load_2d(sB + static_cast<size_t>(s) * stageB, &tmX, (kit0 + it) * kBlockK, t0, &full[s]);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ---------------- MMA issuer
+    const uint32_t idesc = umma_idesc_bf16(kBlockN, BT);
+    for (int it = 0; it < kps; ++it) {
+      const int s = it % stages;
+      const uint32_t ph = static_cast<uint32_t>(it / stages) & 1u;
+      if (!mbar_wait(&full[s], ph, p.err)) break;
+      tc_fence_after();
+      const uint32_t a0 = smem_u32(sA + static_cast<size_t>(s) * kStageA);
+      const uint32_t b0 = smem_u32(sB + static_cast<size_t>(s) * stageB);
+#pragma unroll
+      for (int kk = 0; kk < kBlockK / 16; ++kk) {
+        umma_bf16(tmem, umma_desc_sw128(a0 + kk * 32), umma_desc_sw128(b0 + kk * 32), idesc,
+                  (it | kk) != 0 ? 1u : 0u);
+      }
+      umma_commit(&empty[s]);
+    }
+    umma_commit(done);
+  }
+  __syncwarp();
+
+  // ---------------- epilogue: warp w owns TMEM lanes [32w, 32w+32) = weight rows
+  pdl_wait();
+  const bool ok = mbar_wait(done, 0, p.err);
+  tc_fence_after();
+  __syncwarp();
+  const int n = n0 + warp * 32 + lane;
+  const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+
+  if constexpr (EPI == EPI_HEAD) {
+    const bool sampling = p.temperature > 0.f;
+    const int n_tiles = gridDim.y;
+    const bool masked = n >= p.N || (p.suppress && p.suppress[n]);
+    for (int c = 0; c < BT / 16; ++c) {
+      float v[16];
+      tmem_ld16(trow + c * 16, v);
+#pragma unroll
+      for (int jj = 0; jj < 16; ++jj) {
+        const int t = t0 + c * 16 + jj;
+        float z = v[jj];
+        if (ok && p.logits && t < p.M && n < p.N)
+          p.logits[static_cast<size_t>(t) * p.N + n] = z;
+        float x = masked ? -INFINITY : (sampling ? __fdiv_rn(z, p.temperature) : z);
+        float m = x, s = masked ? 0.f : 1.f, gm = -INFINITY;
+        int arg = n, garg = n;
+        if (sampling && !masked && t < p.M) {
+          const int i = t / p.rows_per_seq, j = t - i * p.rows_per_seq;
+          const int slot = p.seq_slot[i];
+          gm = x + gumbel(p.seed, static_cast<uint32_t>(slot), static_cast<uint32_t>(p.step[slot]),
+                          static_cast<uint32_t>(j), p.tag, static_cast<uint32_t>(n));
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+          const float m2 = __shfl_down_sync(0xffffffffu, m, off);
+          const float s2 = __shfl_down_sync(0xffffffffu, s, off);
+          const float gm2 = __shfl_down_sync(0xffffffffu, gm, off);
+          const int a2 = __shfl_down_sync(0xffffffffu, arg, off);
+          const int ga2 = __shfl_down_sync(0xffffffffu, garg, off);
+          head_combine(m, s, arg, gm, garg, m2, s2, a2, gm2, ga2);
+        }
+        if (lane == 0) {
+          RedEntry e;
+          e.m = m;
+          e.s = s;
+          e.gm = gm;
+          e.arg = arg;
+          e.garg = garg;
+          red[warp * BT + c * 16 + jj] = e;
+        }
+      }
+    }
+    __syncthreads();
+    for (int col = threadIdx.x; col < BT; col += blockDim.x) {
+      const int t = t0 + col;
+      if (t >= p.M) continue;
+      RedEntry e = red[col];
+      for (int w = 1; w < 4; ++w) {
+        const RedEntry f = red[w * BT + col];
+        head_combine(e.m, e.s, e.arg, e.gm, e.garg, f.m, f.s, f.arg, f.gm, f.garg);
+      }
+      HeadRec r;
+      r.m = e.m;
+      r.s = e.s;
+      r.gm = e.gm;
+      r.arg = e.arg;
+      r.garg = e.garg;
+      r._pad[0] = r._pad[1] = r._pad[2] = 0;
+      p.recs[static_cast<size_t>(t) * n_tiles + ntile] = r;
+    }
+  } else {
+    if (p.splits == 1) {
+      for (int c = 0; c < BT / 16; ++c) {
+        float v[16];
+        tmem_ld16(trow + c * 16, v);
+        if (ok) {
+#pragma unroll
+          for (int jj = 0; jj < 16; ++jj) epilogue_store<EPI>(p, t0 + c * 16 + jj, n, v[jj]);
+        }
+      }
+    } else {
+      // write this split's partial tile, then the last CTA of the tile reduces
+      for (int c = 0; c < BT / 16; ++c) {
+        float v[16];
+        tmem_ld16(trow + c * 16, v);
+#pragma unroll
+        for (int jj = 0; jj < 16; ++jj) {
+          const int t = t0 + c * 16 + jj;
+          if (t < p.M && n < p.N)
+            p.partial[(static_cast<size_t>(split) * p.M + t) * p.N + n] = v[jj];
+        }
+      }
+      __threadfence();
+      __syncthreads();
+      const int tile_id = ntile * p.n_tt + tt;
+      if (threadIdx.x == 0) {
+        const int prev = atomicAdd(&p.counters[tile_id], 1);
+        *flag = (prev == p.splits - 1);
+      }
+      __syncthreads();
+      if (*flag) {
+        __threadfence();
+        const int tend = min(BT, p.M - t0);
+        if (n < p.N) {
+          for (int jj = 0; jj < tend; ++jj) {
+            const int t = t0 + jj;
+            float acc = 0.f;
+            for (int sp = 0; sp < p.splits; ++sp)
+              acc += __ldcg(&p.partial[(static_cast<size_t>(sp) * p.M + t) * p.N + n]);
+            if (ok) epilogue_store<EPI>(p, t, n, acc);
+          }
+        }
+        if (threadIdx.x == 0) p.counters[tile_id] = 0;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 2) tmem_dealloc(tmem, p.tmem_cols);
+}
+
+// --------------------------------------------------------------- host ----
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
+
+const CUtensorMap *tmap_bf16_2d(const void *ptr, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+  static std::mutex mu;
+  static std::map<std::tuple<uintptr_t, uint64_t, uint64_t, uint32_t>, CUtensorMap *> cache;
+  std::lock_guard<std::mutex> lock(mu);
+  auto key = std::make_tuple(reinterpret_cast<uintptr_t>(ptr), rows, cols, box_rows);
+  auto it = cache.find(key);
+  if (it != cache.end()) return it->second;
+  auto fn = encode_fn();
+  if (!fn) return nullptr;
+  if ((reinterpret_cast<uintptr_t>(ptr) & 15) || (cols * 2) % 16 || box_rows == 0 || box_rows > 256)
+    return nullptr;
+  CUtensorMap *m = new CUtensorMap;
+  cuuint64_t gdim[2] = {cols, rows};
+  cuuint64_t gstride[1] = {cols * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(kBlockK), box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), gdim, gstride,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    delete m;
+    return nullptr;
+  }
+  cache.emplace(key, m);
+  return m;
+}
+
+void gemm_token_tiling(int M, int *BT, int *n_tt) {
+  const int nt = (M + 255) / 256;
+  const int per = (M + nt - 1) / nt;
+  *n_tt = nt;
+  *BT = ((per + 15) / 16) * 16;
+}
+
+int gemm_splits(int N, int K) {
+  const int n_tiles = (N + kBlockN - 1) / kBlockN;
+  const int k_iters = K / kBlockK;
+  int best = 1;
+  for (int s = 1; s <= k_iters; ++s) {
+    if (k_iters % s) continue;
+    if (n_tiles * s > 160) break;
+    if (k_iters / s < 2) break;
+    best = s;
+  }
+  return best;
+}
+
+size_t gemm_partial_floats(int M, int N, int splits) {
+  return splits > 1 ? static_cast<size_t>(splits) * M * N : 0;
+}
+
+int gemm_counter_slots(int M, int N) {
+  int BT, n_tt;
+  gemm_token_tiling(M, &BT, &n_tt);
+  return n_tt * ((N + kBlockN - 1) / kBlockN);
+}
+
+template <int EPI>
+static cudaError_t launch_typed(const CUtensorMap *tw, const CUtensorMap *tx, const GemmParams &p,
+                                size_t smem, cudaStream_t s, bool pdl) {
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<EPI>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.n_tt, (p.N + kBlockN - 1) / kBlockN, p.splits);
+  cfg.blockDim = dim3(128, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<EPI>, *tw, *tx, p);
+}
+
+cudaError_t launch_gemm(const void *X, const void *W, GemmParams p, cudaStream_t s, bool pdl) {
+  if (p.M <= 0 || p.N <= 0 || p.K <= 0 || p.K % kBlockK) return cudaErrorInvalidValue;
+  gemm_token_tiling(p.M, &p.BT, &p.n_tt);
+  if (p.epi == EPI_HEAD) p.splits = 1;
+  if (p.splits < 1) p.splits = 1;
+  const int k_iters = p.K / kBlockK;
+  if (k_iters % p.splits) return cudaErrorInvalidValue;
+  p.kps = k_iters / p.splits;
+  const size_t stage = kStageA + static_cast<size_t>(p.BT) * kBlockK * 2;
+  const size_t red = (p.epi == EPI_HEAD) ? 4 * static_cast<size_t>(p.BT) * sizeof(RedEntry) : 0;
+  int stages = static_cast<int>((kSmemBudget - red) / stage);
+  if (stages > p.kps) stages = p.kps;
+  if (stages > 16) stages = 16;
+  if (stages < 1) return cudaErrorInvalidValue;
+  p.stages = stages;
+  uint32_t cols = 32;
+  while (cols < static_cast<uint32_t>(p.BT)) cols <<= 1;
+  p.tmem_cols = cols;
+  const size_t smem = 1024 + stages * stage + (2 * stages + 1) * 8 + 32 + 16 + red;
+  const CUtensorMap *tw = tmap_bf16_2d(W, p.N, p.K, kBlockN);
+  const CUtensorMap *tx = tmap_bf16_2d(X, p.M, p.K, p.BT);
+  if (!tw || !tx) return cudaErrorInvalidValue;
+  switch (p.epi) {
+    case EPI_F32: return launch_typed<EPI_F32>(tw, tx, p, smem, s, pdl);
+    case EPI_BF16: return launch_typed<EPI_BF16>(tw, tx, p, smem, s, pdl);
+    case EPI_GELU: return launch_typed<EPI_GELU>(tw, tx, p, smem, s, pdl);
+    case EPI_RESID: return launch_typed<EPI_RESID>(tw, tx, p, smem, s, pdl);
+    case EPI_KV: return launch_typed<EPI_KV>(tw, tx, p, smem, s, pdl);
+    case EPI_HEAD: return launch_typed<EPI_HEAD>(tw, tx, p, smem, s, pdl);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace wf
+
+// ------------------------------------------------------- C entry points --
+extern "C" size_t wf_gemm_scratch_bytes(int32_t M, int32_t N, int32_t K) {
+  if (M <= 0 || N <= 0 || K <= 0 || K % 64) return 0;
+  const int s = wf::gemm_splits(N, K);
+  return wf::gemm_partial_floats(M, N, s) * sizeof(float) +
+         static_cast<size_t>(wf::gemm_counter_slots(M, N)) * sizeof(int32_t) + 256;
+}
+
+extern "C" wf_status wf_gemm_bf16(const void *d_x, const void *d_w, const void *d_b, float *d_y,
+                                  int32_t M, int32_t N, int32_t K, void *d_scratch,
+                                  size_t scratch_bytes, void *stream) {
+  if (!d_x || !d_w || !d_y || M <= 0 || N <= 0 || K <= 0) return WF_ERR_INVALID;
+  if (K % 64) return WF_ERR_UNSUPPORTED;
+  if (scratch_bytes < wf_gemm_scratch_bytes(M, N, K) || (!d_scratch && scratch_bytes)) return WF_ERR_CAPACITY;
+  wf::GemmParams p = {};
+  p.M = M;
+  p.N = N;
+  p.K = K;
+  p.epi = wf::EPI_F32;
+  p.bias = static_cast<const wf::bf16 *>(d_b);
+  p.out_f32 = d_y;
+  p.ld_out = N;
+  p.splits = wf::gemm_splits(N, K);
+  const size_t pf = wf::gemm_partial_floats(M, N, p.splits);
+  p.partial = static_cast<float *>(d_scratch);
+  p.counters = reinterpret_cast<int32_t *>(static_cast<char *>(d_scratch) + pf * sizeof(float));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(p.counters, 0, wf::gemm_counter_slots(M, N) * sizeof(int32_t), s) != cudaSuccess)
+    return WF_ERR_CUDA;
+  return wf::launch_gemm(d_x, d_w, p, s, false) == cudaSuccess ? WF_OK : WF_ERR_CUDA;
+}

@@ -1,0 +1,173 @@
+// Host-side declarations shared by the translation units of libwf: kernel
+// parameter blocks and launchers.  Not part of the public ABI.
+#pragma once
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/wf.h"
+
+namespace wf {
+
+using bf16 = __nv_bfloat16;
+
+// ------------------------------------------------------------------ GEMM --
+// Y[t, n] = sum_k X[t, k] W[n, k] for token rows t < M and features n < N,
+// computed as a 128 x BT tile of D = W_tile * X_tile^T on tcgen05 ("swap-AB":
+// the weights fill the 128-row MMA side, the few tokens the N side).
+enum EpiMode : int {
+  EPI_F32 = 0,    // out_f32[t*ld_out + n] = y + b
+  EPI_BF16 = 1,   // out_bf16[t*ld_out + n] = bf16(y + b)
+  EPI_GELU = 2,   // out_bf16[t*ld_out + n] = bf16(gelu(y + b))
+  EPI_RESID = 3,  // resid[t*ld_resid + n] += y + b; optional bf16 copies (taps)
+  EPI_KV = 4,     // n < q_cols: out_bf16 (query); else keys/values into a cache
+  EPI_HEAD = 5    // output-head records: per (token, 128-id tile) max/argmax,
+                  // sum of exponentials and Gumbel-max (sampling)
+};
+
+struct HeadRec {  // one (token row, 128-id vocabulary tile) of the output head
+  float m;        // max of x = z/T (z when greedy) over the tile
+  float s;        // sum of exp(x - m) over the tile
+  float gm;       // max of x + Gumbel noise (sampling only)
+  int32_t arg;    // lowest id attaining m
+  int32_t garg;   // lowest id attaining gm
+  int32_t _pad[3];
+};
+
+struct GemmParams {
+  int M, N, K;
+  int BT, n_tt, splits, kps, stages;
+  uint32_t tmem_cols;
+  int epi;
+  const bf16 *bias;
+  float *out_f32;
+  bf16 *out_bf16;
+  int ld_out;
+  float *resid;
+  int ld_resid;
+  bf16 *tap0, *tap1;
+  int ld_tap;
+  // EPI_KV: row t -> sequence i = t / rows_per_seq, j = t % rows_per_seq;
+  // slot = seq_slot[i]; position = (pos_base ? pos_base[slot] : 0) + j;
+  // cache layout [slot][head][ctx][64].
+  int q_cols, d_model, n_heads, ctx, rows_per_seq;
+  bf16 *kc, *vc;
+  const int32_t *seq_slot, *pos_base;
+  // EPI_HEAD
+  HeadRec *recs;  // [M][n_tiles]
+  float *logits;  // nullable [M][N] raw logits (sampling, or kept for inspection)
+  int keep_logits;
+  float temperature;  // 0: greedy
+  uint64_t seed;
+  const uint8_t *suppress;
+  const int32_t *step;  // per slot
+  uint32_t tag;
+  // split-K
+  float *partial;
+  int32_t *counters;
+  uint32_t *err;
+};
+
+// Cache of TMA descriptors keyed by (address, rows, cols, box rows).
+const CUtensorMap *tmap_bf16_2d(const void *ptr, uint64_t rows, uint64_t cols, uint32_t box_rows);
+
+// Token tile for M rows: a multiple of 16, at most 256.
+void gemm_token_tiling(int M, int *BT, int *n_tt);
+// Split-K count for a projection of N outputs over K inputs (a function of
+// the shape only, so a row's result never depends on how many rows run).
+int gemm_splits(int N, int K);
+size_t gemm_partial_floats(int M, int N, int splits);
+int gemm_counter_slots(int M, int N);
+
+// Launch one GEMM.  W is [N, K] bf16, X is [M, K] bf16 (row stride K).
+cudaError_t launch_gemm(const void *X, const void *W, GemmParams p, cudaStream_t s, bool pdl);
+
+// ------------------------------------------------------------- attention --
+struct AttnParams {
+  const bf16 *q;
+  const bf16 *kc, *vc;
+  bf16 *out;
+  const int32_t *seq_slot, *pos_base;
+  const float2 *rope_tab;  // [max_pos][32] (cos, sin); nullable
+  float *part;
+  int32_t *counters;
+  uint32_t *err;
+  int n_seq, rps, n_heads, ctx, mode, n_chunks, qgroups;
+};
+constexpr int kAttnChunk = 64;   // keys per CTA, aligned to absolute positions
+constexpr int kAttnQGroup = 16;  // query rows per CTA
+size_t attn_partial_floats(int n_seq, int rps, int n_heads, int ctx);
+int attn_counter_slots(int n_seq, int rps, int n_heads);
+cudaError_t launch_attention(const AttnParams &p, cudaStream_t s, bool pdl);
+cudaError_t launch_rope_table(float2 *tab, int max_pos, float base, cudaStream_t s);
+
+// -------------------------------------------------------- small kernels --
+enum TokSrc : int { TOK_VERIFY = 0, TOK_PROMPT = 1, TOK_ANCHOR = 2 };
+struct EmbedParams {
+  const bf16 *tok_emb, *pos_emb, *mask_emb;
+  const int32_t *seq_slot, *L, *anchor, *cand_in, *forced, *prompt;
+  int32_t *cand_out;   // effective proposals (after forcing) [slot][K]
+  float *x;
+  int n_seq, rps, d, K, P, vocab, src, drafter;
+  uint32_t *err;
+};
+cudaError_t launch_embed(const EmbedParams &p, cudaStream_t s, bool pdl);
+
+// y[r] = LN(x[r*in_stride + in_off]) as bf16 (fp32 statistics).
+cudaError_t launch_layernorm(const float *x, int in_stride, int in_off, const bf16 *g,
+                             const bf16 *b, bf16 *y, int rows, int d, float eps, cudaStream_t s,
+                             bool pdl);
+
+// Reduce head records over the vocabulary tiles of each row.
+struct HeadOut {
+  int32_t arg;   // greedy argmax
+  int32_t garg;  // Gumbel-max sample
+  float lse;     // log sum exp(x) (x = z/T)
+  float m;
+};
+struct HeadReduceParams {
+  const HeadRec *recs;
+  HeadOut *out;
+  int rows, n_tiles;
+  // drafter: write proposals cand[slot*K + j-1] for rows j >= 1
+  int32_t *cand;
+  const int32_t *seq_slot;
+  int rps, K, sampling;
+};
+cudaError_t launch_head_reduce(const HeadReduceParams &p, cudaStream_t s, bool pdl);
+
+struct AcceptParams {
+  const int32_t *seq_slot;
+  int n_seq, rps, K, max_batch, vocab, eos, max_ctx;
+  int greedy_step;  // 1: plain autoregressive step (k = 0)
+  const HeadOut *tout, *dout;
+  const int32_t *cand;  // effective proposals [slot][K]
+  const float *tlogits, *dlogits;  // sampling: raw logits [rows][V]
+  const uint8_t *suppress;
+  float temperature;
+  uint64_t seed;
+  int32_t *L, *anchor, *remaining, *done, *step;
+  int32_t *out_tokens, *out_count;
+  uint32_t *err;
+};
+cudaError_t launch_accept(const AcceptParams &p, cudaStream_t s, bool pdl);
+
+struct StateParams {
+  int op;  // 0: begin prefill, 1: finish prefill, 2: reset to snapshot, 3: append active
+  int n;
+  const int32_t *slots;
+  const int32_t *budget;
+  const HeadOut *hout;
+  int32_t *first;
+  int P, eos, sampling, max_batch;
+  int32_t *L, *anchor, *remaining, *done, *step;
+  int32_t *snap_L, *snap_anchor, *snap_remaining;
+  int32_t *active, *n_active_dev;
+  int active_offset;
+};
+cudaError_t launch_state(const StateParams &p, cudaStream_t s, bool pdl);
+cudaError_t launch_compact(const int32_t *done, int max_batch, int32_t *active,
+                           int32_t *n_active_dev, cudaStream_t s);
+
+}  // namespace wf

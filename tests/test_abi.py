@@ -1,0 +1,55 @@
+"""The C-ABI library builds, loads without a GPU, and exports every entry point
+include/wf.h declares; the binding's signature table covers the same set."""
+import ctypes
+import os
+import re
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "wf.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(wf_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for must in ("wf_create", "wf_prefill_cross_kv", "wf_draft", "wf_verify_accept", "wf_step",
+                 "wf_greedy_step", "wf_workspace_bytes", "wf_destroy", "wf_get_state"):
+        assert must in names
+
+
+def test_library_exports_every_declared_symbol():
+    from paper_2609_32869_gb300 import build
+    path = build.build()
+    lib = ctypes.CDLL(path)
+    missing = [n for n in _declared() if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def test_binding_covers_the_header():
+    from paper_2609_32869_gb300 import binding
+    assert sorted(binding.EXPORTED) == _declared()
+
+
+def test_host_validation_without_gpu():
+    """Argument checks run on the host and need no device."""
+    from paper_2609_32869_gb300 import binding as B
+    from paper_2609_32869_gb300 import synthetic as syn
+    cfg = B.make_config(syn.LARGE)
+    n = B.wf_workspace_bytes(cfg, 1, 448)
+    assert n > 2 * 32 * 448 * 1280 * 2          # at least the target's key/value cache
+    bad = B.make_config(syn.LARGE)
+    bad.n_heads = 7                              # head_dim would not be 64
+    try:
+        B.wf_workspace_bytes(bad, 1, 448)
+        raise AssertionError("expected failure")
+    except B.WfError as e:
+        assert e.status == B.WF_ERR_UNSUPPORTED
+    try:
+        B.wf_workspace_bytes(cfg, 1, 449)           # beyond the learned positions
+        raise AssertionError("expected failure")
+    except B.WfError as e:
+        assert e.status == B.WF_ERR_INVALID
+    assert B.wf_gemm_scratch_bytes(9, 1280, 1000) == 0   # K not a multiple of 64
