@@ -55,8 +55,8 @@ typedef enum wf_status {
 #define WF_MAX_TAPS 8
 #define WF_MAX_LAYERS 64
 
-/* Model shape.  Supported: head_dim = d_model / n_heads = 64; d_model, d_ff and
- * n_taps*d_model multiples of 64; block_k <= 8; max_pos <= 4096. */
+/* Model shape.  Supported: head_dim = d_model / n_heads = 64; d_model a multiple
+ * of 128 and at most 1536; d_ff a multiple of 64; block_k <= 8; max_pos <= 4096. */
 typedef struct wf_config {
   int32_t d_model;        /* 1280 (Whisper large), 384 (tiny) */
   int32_t n_heads;        /* 20, 6 */
@@ -208,11 +208,32 @@ int32_t wf_last_launch_count(const wf_handle *h);
  *   WF_VIEW_TAPS           bf16 [rows][n_taps*d] tapped residual streams (App. A.2)
  *   WF_VIEW_CANDIDATES     int32 [max_batch][K] proposals verified by the last step */
 #define WF_OPT_KEEP_LOGITS 1
+#define WF_OPT_PROFILE 2     /* 1: bracket every launch with CUDA events (serialises launches) */
+#define WF_OPT_PDL 4         /* 1 (default): kernels use programmatic dependent launch */
+#define WF_OPT_GRAPHS 3      /* 1 (default): wf_step / wf_greedy_step replay a CUDA graph
+                                captured on first use per (active count, forcing, sampling
+                                parameters); 0: launch kernel by kernel */
 #define WF_VIEW_TARGET_LOGITS 1
 #define WF_VIEW_DRAFT_LOGITS 2
 #define WF_VIEW_TAPS 3
 #define WF_VIEW_CANDIDATES 4
 wf_status wf_set_option(wf_handle *h, int32_t option, int32_t value);
+
+/* Kernel families reported by wf_profile_read. */
+#define WF_FAM_GEMM 0       /* tcgen05 projections (all but the output head) */
+#define WF_FAM_HEAD 1       /* tcgen05 output head with its fused reduction records */
+#define WF_FAM_ATTN_SELF 2  /* causal verify / prompt attention and the drafter's block attention */
+#define WF_FAM_ATTN_CROSS 3 /* cross-attention over the encoder frames */
+#define WF_FAM_LAYERNORM 4
+#define WF_FAM_OTHER 5      /* embeddings, head reduction, accept, slot state */
+#define WF_PROF_FAMILIES 6
+/* With WF_OPT_PROFILE on: synchronise `stream`, then return per family the
+ * summed kernel time (ms, CUDA events on the launching stream), the number of
+ * launches and, for the GEMM and head families, the algorithmic bytes those
+ * launches move (weights + token rows in + results out; split-K scratch is
+ * not counted).  Each array has WF_PROF_FAMILIES entries; accumulators reset. */
+wf_status wf_profile_read(wf_handle *h, void *stream, double *h_ms, int32_t *h_launches,
+                          double *h_bytes);
 wf_status wf_debug_view(wf_handle *h, int32_t which, void **d_ptr, size_t *bytes);
 
 const char *wf_status_str(wf_status s);
@@ -224,7 +245,9 @@ const char *wf_status_str(wf_status s);
 
 /* Y = X W^T (+ b): the skinny-M tcgen05 GEMM of every projection in the step.
  *   d_x bf16 [M, K], d_w bf16 [N, K], d_b bf16 [N] (nullable), d_y fp32 [M, N].
- *   K % 64 == 0, 1 <= M, 1 <= N.  d_scratch: at least wf_gemm_scratch_bytes. */
+ *   K % 64 == 0, 1 <= M, 1 <= N.  Split-K partial sums are reduced on chip
+ *   (thread-block cluster shared memory), so wf_gemm_scratch_bytes returns 0 and
+ *   d_scratch may be null. */
 wf_status wf_gemm_bf16(const void *d_x, const void *d_w, const void *d_b, float *d_y,
                        int32_t M, int32_t N, int32_t K, void *d_scratch,
                        size_t scratch_bytes, void *stream);

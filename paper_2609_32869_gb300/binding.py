@@ -19,6 +19,10 @@ WF_OK, WF_ERR_INVALID, WF_ERR_CAPACITY, WF_ERR_CUDA, WF_ERR_UNSUPPORTED, WF_ERR_
 WF_DEV_ERR_TIMEOUT, WF_DEV_ERR_CAPACITY, WF_DEV_ERR_TOKEN = 1, 2, 4
 WF_MAX_TAPS = 8
 WF_OPT_KEEP_LOGITS = 1
+WF_OPT_PROFILE = 2
+WF_OPT_GRAPHS = 3
+WF_OPT_PDL = 4
+WF_FAMILIES = ("gemm", "head", "attn_self", "attn_cross", "layernorm", "other")
 WF_VIEW_TARGET_LOGITS, WF_VIEW_DRAFT_LOGITS, WF_VIEW_TAPS, WF_VIEW_CANDIDATES = 1, 2, 3, 4
 
 
@@ -81,6 +85,7 @@ _SIGS = {
     "wf_last_launch_count": (_I, [_P]),
     "wf_set_option": (_I, [_P, _I, _I]),
     "wf_debug_view": (_I, [_P, _I, C.POINTER(_P), C.POINTER(_SZ)]),
+    "wf_profile_read": (_I, [_P, _P, _P, _P, _P]),
     "wf_status_str": (C.c_char_p, [_I]),
     "wf_gemm_bf16": (_I, [_P, _P, _P, _P, _I, _I, _I, _P, _SZ, _P]),
     "wf_gemm_scratch_bytes": (_SZ, [_I, _I, _I]),
@@ -260,6 +265,15 @@ def wf_debug_view(h, which):
     p, n = C.c_void_p(), C.c_size_t()
     _check("wf_debug_view", lib().wf_debug_view(h, which, C.byref(p), C.byref(n)))
     return p.value, n.value
+
+
+def wf_profile_read(h, stream=None) -> dict:
+    n = len(WF_FAMILIES)
+    ms, cnt, by = np.zeros(n), np.zeros(n, np.int32), np.zeros(n)
+    _check("wf_profile_read", lib().wf_profile_read(h, _stream(stream), ms.ctypes.data,
+                                                    cnt.ctypes.data, by.ctypes.data))
+    return {f: {"ms": float(ms[i]), "launches": int(cnt[i]), "bytes": float(by[i])}
+            for i, f in enumerate(WF_FAMILIES)}
 
 
 def wf_gemm_scratch_bytes(M, N, K) -> int:

@@ -6,7 +6,9 @@
 // workspace; the library allocates nothing on the device.
 #include <algorithm>
 #include <cstring>
+#include <map>
 #include <new>
+#include <tuple>
 #include <vector>
 
 #include "wf_device.cuh"
@@ -30,10 +32,6 @@ struct wf_handle {
   float *x, *xd, *hproj;
   bf16 *xn, *q, *att, *h1, *taps, *hn;
   // scratch
-  float *partial;
-  int32_t *gemm_counters;
-  size_t partial_floats;
-  int gemm_counter_cap;
   float *apart;
   int32_t *attn_counters;
   size_t apart_floats;
@@ -45,8 +43,37 @@ struct wf_handle {
   int n_vtiles = 0;
   int n_active = 0;
   int launches = 0;
-  bool in_step = false;
   bool keep_logits = false;
+  // profiling (WF_OPT_PROFILE)
+  bool profile = false;
+  std::vector<cudaEvent_t> ev_pool;
+  size_t ev_next = 0;
+  struct Rec {
+    int fam;
+    cudaEvent_t a, b;
+    double bytes;
+  };
+  std::vector<Rec> prof;
+  cudaEvent_t pending = nullptr;
+  // CUDA graphs of the hot entry points, keyed by what changes their launches
+  struct GraphKey {
+    int kind, n_active, forced;
+    float temperature;
+    uint64_t seed;
+    const void *suppress;
+    bool operator<(const GraphKey &o) const {
+      return std::tie(kind, n_active, forced, temperature, seed, suppress) <
+             std::tie(o.kind, o.n_active, o.forced, o.temperature, o.seed, o.suppress);
+    }
+  };
+  struct GraphEntry {
+    cudaGraphExec_t exec;
+    int launches;
+  };
+  std::map<GraphKey, GraphEntry> graphs;
+  bool use_graphs = true;
+  cudaStream_t cap_stream = nullptr;
+  int32_t *forced_buf = nullptr, *tok_buf = nullptr, *cnt_buf = nullptr;
 };
 
 namespace {
@@ -68,7 +95,7 @@ struct Carver {
 bool cfg_ok(const wf_config *c) {
   if (!c) return false;
   if (c->d_model <= 0 || c->n_heads <= 0 || c->d_model != c->n_heads * 64) return false;
-  if (c->d_model % 64 || c->d_ff % 64 || c->d_ff <= 0) return false;
+  if (c->d_model % 128 || c->d_ff % 64 || c->d_ff <= 0) return false;
   if (c->d_model > 1536) return false;
   if (c->n_layers <= 0 || c->n_layers > WF_MAX_LAYERS) return false;
   if (c->n_draft_layers <= 0 || c->n_draft_layers > 8) return false;
@@ -83,18 +110,6 @@ bool cfg_ok(const wf_config *c) {
 
 int rows_max(const wf_config *c, int Bmax, int ctx) {
   return std::max(Bmax * (c->block_k + 1), ctx);
-}
-
-// Largest split-K scratch (floats per token row) over the per-step projections.
-size_t partial_per_row(const wf_config *c) {
-  const int d = c->d_model, F = c->d_ff;
-  const int shapes[][2] = {{3 * d, d}, {d, d}, {F, d}, {d, F}, {d, c->n_taps * d}, {2 * d, d}};
-  size_t best = 0;
-  for (auto &sh : shapes) {
-    const int s = gemm_splits(sh[0], sh[1]);
-    if (s > 1) best = std::max(best, static_cast<size_t>(s) * sh[0]);
-  }
-  return best;
 }
 
 // Lay the workspace out (base == nullptr: only measure).
@@ -118,6 +133,9 @@ size_t layout(wf_handle *h, const wf_config *c, int Bmax, int ctx, char *base) {
   o->n_active_dev = cv.take<int32_t>(1);
   o->cand = cv.take<int32_t>(sl * K);
   o->err = cv.take<uint32_t>(1);
+  o->forced_buf = cv.take<int32_t>(sl * K);
+  o->tok_buf = cv.take<int32_t>(sl * (K + 1));
+  o->cnt_buf = cv.take<int32_t>(sl);
   const size_t self_sz = static_cast<size_t>(nl) * sl * H * ctx * 64;
   o->self_k = cv.take<bf16>(self_sz);
   o->self_v = cv.take<bf16>(self_sz);
@@ -137,12 +155,8 @@ size_t layout(wf_handle *h, const wf_config *c, int Bmax, int ctx, char *base) {
   o->hn = cv.take<bf16>(M * d);
   o->h1 = cv.take<bf16>(M * F);
   o->taps = cv.take<bf16>(M * c->n_taps * d);
-  o->partial_floats = M * partial_per_row(c);
-  o->partial = cv.take<float>(std::max<size_t>(o->partial_floats, 1));
-  o->gemm_counter_cap = 1 << 16;
-  o->gemm_counters = cv.take<int32_t>(o->gemm_counter_cap);
   const int groups = Bmax + Mmax / kAttnQGroup + 1;
-  const int chunks = (std::max(ctx, T) + kAttnChunk - 1) / kAttnChunk;
+  const int chunks = (std::max(ctx, T) + kAttnKeysPerCTA - 1) / kAttnKeysPerCTA;
   o->apart_floats = static_cast<size_t>(groups) * H * chunks * kAttnQGroup * 66;
   o->apart = cv.take<float>(o->apart_floats);
   o->attn_counter_cap = groups * H;
@@ -166,7 +180,46 @@ inline cudaStream_t S(void *s) { return static_cast<cudaStream_t>(s); }
     if (_e != cudaSuccess) return WF_ERR_CUDA;     \
   } while (0)
 
-constexpr bool kPDL = true;
+// Programmatic dependent launch for every kernel of a call (WF_OPT_PDL).
+static bool g_pdl = true;
+#define kPDL g_pdl
+
+cudaEvent_t prof_event(wf_handle *h) {
+  if (h->ev_next == h->ev_pool.size()) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    h->ev_pool.push_back(e);
+  }
+  return h->ev_pool[h->ev_next++];
+}
+void prof_begin(wf_handle *h, cudaStream_t s) {
+  if (!h->profile) return;
+  h->pending = prof_event(h);
+  if (h->pending) cudaEventRecord(h->pending, s);
+}
+void prof_end(wf_handle *h, cudaStream_t s, int fam, double bytes) {
+  if (!h->profile || !h->pending) return;
+  cudaEvent_t b = prof_event(h);
+  if (!b) return;
+  cudaEventRecord(b, s);
+  h->prof.push_back({fam, h->pending, b, bytes});
+  h->pending = nullptr;
+}
+// Algorithmic bytes of one projection: weights, token rows in, results out.
+double gemm_bytes(const GemmParams &p) {
+  double b = 2.0 * p.N * p.K + 2.0 * p.M * p.K + (p.bias ? 2.0 * p.N : 0.0);
+  switch (p.epi) {
+    case EPI_F32: b += 4.0 * p.M * p.N; break;
+    case EPI_RESID:
+      b += 8.0 * p.M * p.N + (p.tap0 ? 2.0 * p.M * p.N : 0.0) + (p.tap1 ? 2.0 * p.M * p.N : 0.0);
+      break;
+    case EPI_HEAD:
+      b += 32.0 * p.M * ((p.N + 127) / 128) + (p.logits ? 4.0 * p.M * p.N : 0.0);
+      break;
+    default: b += 2.0 * p.M * p.N; break;
+  }
+  return b;
+}
 
 // ---------------------------------------------------------------- GEMMs --
 GemmParams gemm_base(wf_handle *h, int M, int N, int K, int epi) {
@@ -176,8 +229,6 @@ GemmParams gemm_base(wf_handle *h, int M, int N, int K, int epi) {
   p.K = K;
   p.epi = epi;
   p.splits = gemm_splits(N, K);
-  p.partial = h->partial;
-  p.counters = h->gemm_counters;
   p.err = h->err;
   p.d_model = h->d;
   p.n_heads = h->H;
@@ -185,19 +236,22 @@ GemmParams gemm_base(wf_handle *h, int M, int N, int K, int epi) {
 }
 
 cudaError_t gemm(wf_handle *h, const void *X, const void *W, GemmParams p, cudaStream_t s) {
-  if (p.splits > 1) {
-    if (gemm_partial_floats(p.M, p.N, p.splits) > h->partial_floats) return cudaErrorInvalidValue;
-    if (gemm_counter_slots(p.M, p.N) > h->gemm_counter_cap) return cudaErrorInvalidValue;
-  }
   h->launches++;
-  return launch_gemm(X, W, p, s, kPDL);
+  prof_begin(h, s);
+  cudaError_t e = launch_gemm(X, W, p, s, kPDL);
+  prof_end(h, s, p.epi == EPI_HEAD ? WF_FAM_HEAD : WF_FAM_GEMM, gemm_bytes(p));
+  return e;
 }
 
 cudaError_t layernorm(wf_handle *h, const float *x, int stride, int off, const void *g,
                       const void *b, bf16 *y, int rows, cudaStream_t s) {
   h->launches++;
-  return launch_layernorm(x, stride, off, static_cast<const bf16 *>(g),
-                          static_cast<const bf16 *>(b), y, rows, h->d, h->cfg.ln_eps, s, kPDL);
+  prof_begin(h, s);
+  cudaError_t e = launch_layernorm(x, stride, off, static_cast<const bf16 *>(g),
+                                   static_cast<const bf16 *>(b), y, rows, h->d, h->cfg.ln_eps, s,
+                                   kPDL);
+  prof_end(h, s, WF_FAM_LAYERNORM, 6.0 * rows * h->d);
+  return e;
 }
 
 cudaError_t attention(wf_handle *h, const bf16 *q, const bf16 *kc, const bf16 *vc,
@@ -222,7 +276,10 @@ cudaError_t attention(wf_handle *h, const bf16 *q, const bf16 *kc, const bf16 *v
   if (attn_partial_floats(n_seq, rps, h->H, ctx) > h->apart_floats) return cudaErrorInvalidValue;
   if (attn_counter_slots(n_seq, rps, h->H) > h->attn_counter_cap) return cudaErrorInvalidValue;
   h->launches++;
-  return launch_attention(p, s, kPDL);
+  prof_begin(h, s);
+  cudaError_t e = launch_attention(p, s, kPDL);
+  prof_end(h, s, mode == 2 ? WF_FAM_ATTN_CROSS : WF_FAM_ATTN_SELF, 0.0);
+  return e;
 }
 
 size_t layer_cache_off(wf_handle *h, int layer, int positions) {
@@ -361,7 +418,10 @@ cudaError_t head(wf_handle *h, const float *x, int stride, int off, int rows, co
   r.K = h->K;
   r.sampling = sampling ? 1 : 0;
   h->launches++;
-  return launch_head_reduce(r, s, kPDL);
+  prof_begin(h, s);
+  e = launch_head_reduce(r, s, kPDL);
+  prof_end(h, s, WF_FAM_OTHER, 0.0);
+  return e;
 }
 
 // History memory (Sec. 3.2, App. A.2): project the tapped residual streams of
@@ -420,7 +480,9 @@ cudaError_t target_pass(wf_handle *h, int n_seq, int rps, const int32_t *slots, 
   ep.drafter = 0;
   ep.err = h->err;
   h->launches++;
+  prof_begin(h, s);
   cudaError_t e = launch_embed(ep, s, kPDL);
+  prof_end(h, s, WF_FAM_OTHER, 0.0);
   if (e != cudaSuccess) return e;
   Pass ps{n_seq, rps, slots, false, h->x, taps};
   for (int l = 0; l < h->nl; ++l)
@@ -519,10 +581,12 @@ wf_status wf_create(const wf_config *cfg, const wf_target_weights *tw, const wf_
             cudaMemsetAsync(h->cand, 0, sl * h->K, s) == cudaSuccess &&
             cudaMemsetAsync(h->n_active_dev, 0, sizeof(int32_t), s) == cudaSuccess &&
             cudaMemsetAsync(h->err, 0, sizeof(uint32_t), s) == cudaSuccess &&
-            cudaMemsetAsync(h->gemm_counters, 0, h->gemm_counter_cap * sizeof(int32_t), s) == cudaSuccess &&
             cudaMemsetAsync(h->attn_counters, 0, h->attn_counter_cap * sizeof(int32_t), s) == cudaSuccess &&
             launch_rope_table(h->rope, cfg->max_pos, cfg->rope_base, s) == cudaSuccess;
+  ok = ok && gemm_init() == cudaSuccess && attention_init() == cudaSuccess &&
+       cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) == cudaSuccess;
   if (!ok) {
+    if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
     delete h;
     return WF_ERR_CUDA;
   }
@@ -532,6 +596,9 @@ wf_status wf_create(const wf_config *cfg, const wf_target_weights *tw, const wf_
 
 wf_status wf_destroy(wf_handle *h) {
   if (!h) return WF_ERR_INVALID;
+  for (cudaEvent_t e : h->ev_pool) cudaEventDestroy(e);
+  for (auto &kv : h->graphs) cudaGraphExecDestroy(kv.second.exec);
+  if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
   delete h;
   return WF_OK;
 }
@@ -544,7 +611,44 @@ wf_status wf_set_option(wf_handle *h, int32_t option, int32_t value) {
     h->keep_logits = value != 0;
     return WF_OK;
   }
+  if (option == WF_OPT_PDL) {
+    g_pdl = value != 0;
+    for (auto &kv : h->graphs) cudaGraphExecDestroy(kv.second.exec);
+    h->graphs.clear();
+    return WF_OK;
+  }
+  if (option == WF_OPT_GRAPHS) {
+    h->use_graphs = value != 0;
+    return WF_OK;
+  }
+  if (option == WF_OPT_PROFILE) {
+    h->profile = value != 0;
+    h->prof.clear();
+    h->ev_next = 0;
+    return WF_OK;
+  }
   return WF_ERR_INVALID;
+}
+
+wf_status wf_profile_read(wf_handle *h, void *stream, double *h_ms, int32_t *h_launches,
+                          double *h_bytes) {
+  if (!h || !h_ms || !h_launches || !h_bytes) return WF_ERR_INVALID;
+  WF_TRY(cudaStreamSynchronize(S(stream)));
+  for (int f = 0; f < WF_PROF_FAMILIES; ++f) {
+    h_ms[f] = 0.0;
+    h_launches[f] = 0;
+    h_bytes[f] = 0.0;
+  }
+  for (auto &r : h->prof) {
+    float ms = 0.f;
+    WF_TRY(cudaEventElapsedTime(&ms, r.a, r.b));
+    h_ms[r.fam] += ms;
+    h_launches[r.fam] += 1;
+    h_bytes[r.fam] += r.bytes;
+  }
+  h->prof.clear();
+  h->ev_next = 0;
+  return WF_OK;
 }
 
 wf_status wf_debug_view(wf_handle *h, int32_t which, void **d_ptr, size_t *bytes) {
@@ -641,11 +745,8 @@ wf_status wf_prefill_cross_kv(wf_handle *h, int32_t n, const int32_t *d_slots, c
   return WF_OK;
 }
 
-wf_status wf_draft(wf_handle *h, const wf_sample_params *sp, void *stream) {
-  if (!h) return WF_ERR_INVALID;
-  h->launches = 0;
+static wf_status draft_body(wf_handle *h, const wf_sample_params *sp, cudaStream_t s) {
   if (h->n_active == 0) return WF_OK;
-  cudaStream_t s = S(stream);
   const int n = h->n_active, rps = h->K + 1;
   EmbedParams ep = {};
   ep.tok_emb = static_cast<const bf16 *>(h->tw.tok_emb);
@@ -662,7 +763,9 @@ wf_status wf_draft(wf_handle *h, const wf_sample_params *sp, void *stream) {
   ep.drafter = 1;
   ep.err = h->err;
   h->launches++;
+  prof_begin(h, s);
   WF_TRY(launch_embed(ep, s, kPDL));
+  prof_end(h, s, WF_FAM_OTHER, 0.0);
   Pass ps{n, rps, h->active, true, h->xd, false};
   for (int l = 0; l < h->nd; ++l) WF_TRY(run_block(h, ps, h->dl[l], l, s));
   WF_TRY(head(h, h->xd, 1, 0, n * rps, h->active, rps, h->recs_d, h->hout_d, h->logits_d, sp,
@@ -670,11 +773,8 @@ wf_status wf_draft(wf_handle *h, const wf_sample_params *sp, void *stream) {
   return WF_OK;
 }
 
-wf_status wf_verify_accept(wf_handle *h, const wf_sample_params *sp, const int32_t *d_forced,
-                           int32_t *d_out_tokens, int32_t *d_out_count, void *stream) {
-  if (!h || !d_out_tokens || !d_out_count) return WF_ERR_INVALID;
-  cudaStream_t s = S(stream);
-  if (!h->in_step) h->launches = 0;
+static wf_status verify_body(wf_handle *h, const wf_sample_params *sp, const int32_t *d_forced,
+                             int32_t *d_out_tokens, int32_t *d_out_count, cudaStream_t s) {
   const int n = h->n_active, rps = h->K + 1;
   if (n > 0) {
     WF_TRY(target_pass(h, n, rps, h->active, TOK_VERIFY, nullptr, 0, d_forced, true, s));
@@ -709,26 +809,14 @@ wf_status wf_verify_accept(wf_handle *h, const wf_sample_params *sp, const int32
   ap.out_count = d_out_count;
   ap.err = h->err;
   h->launches++;
+  prof_begin(h, s);
   WF_TRY(launch_accept(ap, s, kPDL));
+  prof_end(h, s, WF_FAM_OTHER, 0.0);
   return WF_OK;
 }
 
-wf_status wf_step(wf_handle *h, const wf_sample_params *sp, const int32_t *d_forced,
-                  int32_t *d_out_tokens, int32_t *d_out_count, void *stream) {
-  if (!h) return WF_ERR_INVALID;
-  wf_status st = wf_draft(h, sp, stream);
-  if (st != WF_OK) return st;
-  h->in_step = true;
-  st = wf_verify_accept(h, sp, d_forced, d_out_tokens, d_out_count, stream);
-  h->in_step = false;
-  return st;
-}
-
-wf_status wf_greedy_step(wf_handle *h, const wf_sample_params *sp, int32_t *d_out_tokens,
-                         int32_t *d_out_count, void *stream) {
-  if (!h || !d_out_tokens || !d_out_count) return WF_ERR_INVALID;
-  cudaStream_t s = S(stream);
-  h->launches = 0;
+static wf_status greedy_body(wf_handle *h, const wf_sample_params *sp, int32_t *d_out_tokens,
+                             int32_t *d_out_count, cudaStream_t s) {
   const int n = h->n_active;
   if (n > 0) {
     WF_TRY(target_pass(h, n, 1, h->active, TOK_ANCHOR, nullptr, 0, nullptr, false, s));
@@ -758,7 +846,108 @@ wf_status wf_greedy_step(wf_handle *h, const wf_sample_params *sp, int32_t *d_ou
   ap.out_count = d_out_count;
   ap.err = h->err;
   h->launches++;
+  prof_begin(h, s);
   WF_TRY(launch_accept(ap, s, kPDL));
+  prof_end(h, s, WF_FAM_OTHER, 0.0);
+  return WF_OK;
+}
+
+}  // extern "C"
+
+// Run `body` through a CUDA graph captured once per key on the handle's capture
+// stream and replayed on the caller's stream; eager when graphs are off, when
+// profiling, or when the caller's stream is itself being captured.
+template <typename Body>
+static wf_status run_graphed(wf_handle *h, wf_handle::GraphKey key, cudaStream_t s, Body body) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (s && cudaStreamIsCapturing(s, &cs) != cudaSuccess) return WF_ERR_CUDA;
+  if (!h->use_graphs || h->profile || cs != cudaStreamCaptureStatusNone) {
+    h->launches = 0;
+    return body(s);
+  }
+  auto it = h->graphs.find(key);
+  if (it == h->graphs.end()) {
+    if (cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess)
+      return WF_ERR_CUDA;
+    h->launches = 0;
+    wf_status st = body(h->cap_stream);
+    cudaGraph_t g = nullptr;
+    cudaError_t e = cudaStreamEndCapture(h->cap_stream, &g);
+    if (st != WF_OK || e != cudaSuccess) {
+      if (g) cudaGraphDestroy(g);
+      return st != WF_OK ? st : WF_ERR_CUDA;
+    }
+    cudaGraphExec_t ex = nullptr;
+    e = cudaGraphInstantiate(&ex, g, 0);
+    cudaGraphDestroy(g);
+    if (e != cudaSuccess) return WF_ERR_CUDA;
+    it = h->graphs.emplace(key, wf_handle::GraphEntry{ex, h->launches}).first;
+  }
+  h->launches = it->second.launches;
+  WF_TRY(cudaGraphLaunch(it->second.exec, s));
+  return WF_OK;
+}
+
+static wf_handle::GraphKey graph_key(wf_handle *h, int kind, const wf_sample_params *sp,
+                                     bool forced) {
+  wf_handle::GraphKey k;
+  k.kind = kind;
+  k.n_active = h->n_active;
+  k.forced = forced ? 1 : 0;
+  const bool sampling = sp && sp->temperature > 0.f;
+  k.temperature = sampling ? sp->temperature : 0.f;
+  k.seed = sampling ? sp->seed : 0;
+  k.suppress = sp ? sp->d_suppress : nullptr;
+  return k;
+}
+
+extern "C" {
+
+wf_status wf_draft(wf_handle *h, const wf_sample_params *sp, void *stream) {
+  if (!h) return WF_ERR_INVALID;
+  h->launches = 0;
+  return draft_body(h, sp, S(stream));
+}
+
+wf_status wf_verify_accept(wf_handle *h, const wf_sample_params *sp, const int32_t *d_forced,
+                           int32_t *d_out_tokens, int32_t *d_out_count, void *stream) {
+  if (!h || !d_out_tokens || !d_out_count) return WF_ERR_INVALID;
+  h->launches = 0;
+  return verify_body(h, sp, d_forced, d_out_tokens, d_out_count, S(stream));
+}
+
+wf_status wf_step(wf_handle *h, const wf_sample_params *sp, const int32_t *d_forced,
+                  int32_t *d_out_tokens, int32_t *d_out_count, void *stream) {
+  if (!h || !d_out_tokens || !d_out_count) return WF_ERR_INVALID;
+  cudaStream_t s = S(stream);
+  const size_t kb = static_cast<size_t>(h->Bmax) * h->K * sizeof(int32_t);
+  if (d_forced) WF_TRY(cudaMemcpyAsync(h->forced_buf, d_forced, kb, cudaMemcpyDeviceToDevice, s));
+  const int32_t *forced = d_forced ? h->forced_buf : nullptr;
+  wf_status st = run_graphed(h, graph_key(h, 1, sp, d_forced != nullptr), s,
+                             [&](cudaStream_t cs) -> wf_status {
+                               wf_status r = draft_body(h, sp, cs);
+                               if (r != WF_OK) return r;
+                               return verify_body(h, sp, forced, h->tok_buf, h->cnt_buf, cs);
+                             });
+  if (st != WF_OK) return st;
+  WF_TRY(cudaMemcpyAsync(d_out_tokens, h->tok_buf, kb / h->K * (h->K + 1), cudaMemcpyDeviceToDevice, s));
+  WF_TRY(cudaMemcpyAsync(d_out_count, h->cnt_buf, static_cast<size_t>(h->Bmax) * sizeof(int32_t),
+                         cudaMemcpyDeviceToDevice, s));
+  return WF_OK;
+}
+
+wf_status wf_greedy_step(wf_handle *h, const wf_sample_params *sp, int32_t *d_out_tokens,
+                         int32_t *d_out_count, void *stream) {
+  if (!h || !d_out_tokens || !d_out_count) return WF_ERR_INVALID;
+  cudaStream_t s = S(stream);
+  wf_status st = run_graphed(h, graph_key(h, 2, sp, false), s, [&](cudaStream_t cs) -> wf_status {
+    return greedy_body(h, sp, h->tok_buf, h->cnt_buf, cs);
+  });
+  if (st != WF_OK) return st;
+  const size_t kb = static_cast<size_t>(h->Bmax) * (h->K + 1) * sizeof(int32_t);
+  WF_TRY(cudaMemcpyAsync(d_out_tokens, h->tok_buf, kb, cudaMemcpyDeviceToDevice, s));
+  WF_TRY(cudaMemcpyAsync(d_out_count, h->cnt_buf, static_cast<size_t>(h->Bmax) * sizeof(int32_t),
+                         cudaMemcpyDeviceToDevice, s));
   return WF_OK;
 }
 

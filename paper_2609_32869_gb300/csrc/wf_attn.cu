@@ -9,31 +9,83 @@
 //    positions [0, L) and the 9 block positions [L, L+9), bidirectional inside
 //    the block, with RoPE on queries and keys (Sec. 3.2, App. A.2);
 //  - mode 2, cross: all encoder frames (cross-attention, Sec. 3.2).
-// A CTA takes one (sequence, head, group of <= 16 queries, chunk of 64 keys);
-// chunks are aligned to absolute positions and combined by the last CTA of a
-// (sequence, head, group) in chunk order with the log-sum-exp rule, so a
-// query's result does not depend on how many other rows run with it.
+//
+// A CTA takes one (sequence, head, group of <= 16 query rows, block of 256
+// keys).  Keys and values stream into XOR-swizzled shared memory with
+// cp.async (rows past the cache length are zero-filled); each of the four
+// warps multiplies the 16 query rows against its 64 keys on the tensor cores
+// (mma.sync m16n8k16, bf16 in, fp32 accumulate), keeps the row maxima and
+// sums in fp32 and forms P V the same way.  Warps combine in order, and the
+// blocks of a (sequence, head, group) are combined by the last CTA in block
+// order.  Blocks and warps are aligned to absolute key positions and a key a
+// query cannot see contributes an exact zero, so a query's result does not
+// depend on how many other rows run with it.
+#include <mutex>
+
 #include "wf_device.cuh"
 #include "wf_internal.h"
 
 namespace wf {
 
-constexpr int kCK = kAttnChunk;
-constexpr int kQG = kAttnQGroup;
-constexpr int kPartStride = 2 + 64;  // m, l, o[64]
+constexpr int kKB = kAttnKeysPerCTA;  // 256 keys per CTA, 64 per warp
+constexpr int kQG = kAttnQGroup;      // 16 query rows per CTA
+constexpr int kPartStride = 2 + 64;   // m, l, o[64]
+constexpr int kSmemK = kKB * 128;     // bytes
+constexpr int kSmemQ = kQG * 128;
+constexpr int kSmemAttn = 2 * kSmemK + kSmemQ + 4 * kQG * (2 + 64) * 4 + 16;
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, bool valid) {
+  const int n = valid ? 16 : 0;  // zero-fill when the source row is past the cache
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(n)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
+                                        uint32_t &r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
+                                          uint32_t &r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                         uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t *>(&v);
+}
+// byte offset of 16-byte chunk `ch` of row `row` in a [rows][64] bf16 tile
+__device__ __forceinline__ uint32_t swz(int row, int ch) {
+  return static_cast<uint32_t>(row * 128 + ((ch ^ (row & 7)) << 4));
+}
 
 __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
-  __shared__ float sq[kQG][64];
-  __shared__ float sk[kCK][65];
-  __shared__ float sv[kCK][64];
-  __shared__ float sp[kQG][kCK];
+  extern __shared__ __align__(128) uint8_t smem[];
+  uint8_t *sK = smem;
+  uint8_t *sV = smem + kSmemK;
+  uint8_t *sQ = smem + 2 * kSmemK;
+  float *sm = reinterpret_cast<float *>(smem + 2 * kSmemK + kSmemQ);  // [4][16]
+  float *sl = sm + 4 * kQG;                                          // [4][16]
+  float *so = sl + 4 * kQG;                                          // [4][16][64]
   __shared__ int s_last;
 
-  const int c = blockIdx.x;
+  const int blk = blockIdx.x;
   const int h = blockIdx.y % p.n_heads;
   const int qg = blockIdx.y / p.n_heads;
   const int i = blockIdx.z;
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
   pdl_wait();
   pdl_launch_dependents();
@@ -51,143 +103,263 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
     n_keys = base + q0 + nq;  // keys visible to the last query of the group
   if (n_keys > p.ctx || (p.mode != 2 && base + p.rps > p.ctx)) {
     // the block would pass the cache: record it and leave the output untouched
-    if (c == 0 && tid == 0) set_error(p.err, WF_DEV_ERR_CAPACITY);
+    if (blk == 0 && tid == 0) set_error(p.err, WF_DEV_ERR_CAPACITY);
     return;
   }
-  const int n_chunks = (n_keys + kCK - 1) / kCK;
-  if (c >= n_chunks) return;
+  const int n_blocks = (n_keys + kKB - 1) / kKB;
+  if (blk >= n_blocks) return;
 
   const int d_model = p.n_heads * 64;
   const size_t cache_off = (static_cast<size_t>(slot) * p.n_heads + h) * p.ctx;
+  const int key0 = blk * kKB;
 
-  // ---- queries (pre-scaled by 1/8 = 1/sqrt(64): exact in binary)
-  for (int e = tid; e < kQG * 64; e += blockDim.x) {
-    const int qi = e >> 6, dd = e & 63;
-    float v = 0.f;
-    if (qi < nq) {
-      const bf16 *qrow = p.q + static_cast<size_t>(i * p.rps + q0 + qi) * d_model + h * 64;
-      v = bf2f(qrow[dd]);
-      if (p.rope_tab) {
-        const int pos = base + q0 + qi;
-        const int pr = dd & 31;
-        const float2 cs = p.rope_tab[pos * 32 + pr];
-        const float other = bf2f(qrow[dd ^ 32]);
+  // ---- keys and values: cp.async, zero-filled past the cache length
+  {
+    const uint32_t k_u32 = smem_u32(sK), v_u32 = smem_u32(sV);
+#pragma unroll 4
+    for (int idx = tid; idx < kKB * 8; idx += 128) {
+      const int kr = idx >> 3, ch = idx & 7;
+      const int pos = key0 + kr;
+      const bool valid = pos < n_keys;
+      const size_t off = (cache_off + (valid ? pos : 0)) * 64 + ch * 8;
+      cp_async16(k_u32 + swz(kr, ch), p.kc + off, valid);
+      cp_async16(v_u32 + swz(kr, ch), p.vc + off, valid);
+    }
+  }
+  // ---- queries, pre-scaled by 1/8 = 1/sqrt(64) (exact in binary), RoPE in fp32
+  {
+    const int r = tid >> 3, ch = tid & 7;
+    uint4 raw = make_uint4(0, 0, 0, 0), par = make_uint4(0, 0, 0, 0);
+    if (r < nq) {
+      const bf16 *qrow = p.q + static_cast<size_t>(i * p.rps + q0 + r) * d_model + h * 64;
+      raw = *reinterpret_cast<const uint4 *>(qrow + ch * 8);
+      if (p.rope_tab) par = *reinterpret_cast<const uint4 *>(qrow + ((ch * 8) ^ 32));
+    }
+    const bf16 *qv = reinterpret_cast<const bf16 *>(&raw);
+    const bf16 *qp = reinterpret_cast<const bf16 *>(&par);
+    float f[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      float v = bf2f(qv[e]);
+      if (p.rope_tab && r < nq) {
+        const int dd = ch * 8 + e;
+        const float2 cs = __ldg(p.rope_tab + (base + q0 + r) * 32 + (dd & 31));
+        const float other = bf2f(qp[e]);
         v = dd < 32 ? v * cs.x - other * cs.y : v * cs.x + other * cs.y;
       }
+      f[e] = v * 0.125f;
     }
-    sq[qi][dd] = v * 0.125f;
+    uint4 o;
+    o.x = pack_bf16(f[0], f[1]);
+    o.y = pack_bf16(f[2], f[3]);
+    o.z = pack_bf16(f[4], f[5]);
+    o.w = pack_bf16(f[6], f[7]);
+    *reinterpret_cast<uint4 *>(sQ + swz(r, ch)) = o;
   }
-  // ---- keys and values of this chunk
-  for (int e = tid; e < kCK * 64; e += blockDim.x) {
-    const int kk = e >> 6, dd = e & 63;
-    const int pos = c * kCK + kk;
-    float kv = 0.f, vv = 0.f;
-    if (pos < n_keys) {
-      const bf16 *krow = p.kc + (cache_off + pos) * 64;
-      kv = bf2f(krow[dd]);
-      vv = bf2f(p.vc[(cache_off + pos) * 64 + dd]);
-      if (p.rope_tab) {
-        const int pr = dd & 31;
-        const float2 cs = p.rope_tab[pos * 32 + pr];
-        const float other = bf2f(krow[dd ^ 32]);
-        kv = dd < 32 ? kv * cs.x - other * cs.y : kv * cs.x + other * cs.y;
+  cp_async_wait_all();
+  __syncthreads();
+
+  // ---- RoPE on the keys (drafter): dims i and i+32 rotate by pos * base^(-2i/64)
+  if (p.rope_tab) {
+    for (int idx = tid; idx < kKB * 4; idx += 128) {
+      const int kr = idx >> 2, c = idx & 3;  // chunk c (dims 8c..8c+7) pairs with chunk c+4
+      const int pos = key0 + kr;
+      if (pos >= n_keys) continue;
+      uint4 *lo = reinterpret_cast<uint4 *>(sK + swz(kr, c));
+      uint4 *hi = reinterpret_cast<uint4 *>(sK + swz(kr, c + 4));
+      uint4 a = *lo, b = *hi;
+      bf16 *av = reinterpret_cast<bf16 *>(&a);
+      bf16 *bv = reinterpret_cast<bf16 *>(&b);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        const float2 cs = __ldg(p.rope_tab + pos * 32 + c * 8 + e);
+        const float x1 = bf2f(av[e]), x2 = bf2f(bv[e]);
+        av[e] = __float2bfloat16(x1 * cs.x - x2 * cs.y);
+        bv[e] = __float2bfloat16(x2 * cs.x + x1 * cs.y);
       }
+      *lo = a;
+      *hi = b;
     }
-    sk[kk][dd] = kv;
-    sv[kk][dd] = vv;
+    __syncthreads();
+  }
+
+  // ---- per warp: 16 query rows x 64 keys on the tensor cores
+  const int g = lane >> 2, c4 = lane & 3;
+  const int kw = warp * 64;  // first key of this warp within the block
+  const uint32_t q_u32 = smem_u32(sQ), k_u32 = smem_u32(sK), v_u32 = smem_u32(sV);
+  float s[8][4];
+#pragma unroll
+  for (int nt = 0; nt < 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+#pragma unroll
+  for (int ks = 0; ks < 4; ++ks) {
+    uint32_t a0, a1, a2, a3;
+    {
+      const int mi = lane >> 3;
+      ldsm_x4(q_u32 + swz((mi & 1) * 8 + (lane & 7), 2 * ks + (mi >> 1)), a0, a1, a2, a3);
+    }
+#pragma unroll
+    for (int np = 0; np < 4; ++np) {
+      uint32_t b0, b1, b2, b3;
+      const int mi = lane >> 3;
+      ldsm_x4(k_u32 + swz(kw + np * 16 + (mi >> 1) * 8 + (lane & 7), 2 * ks + (mi & 1)), b0, b1, b2,
+              b3);
+      mma_bf16(s[2 * np], a0, a1, a2, a3, b0, b1);
+      mma_bf16(s[2 * np + 1], a0, a1, a2, a3, b2, b3);
+    }
+  }
+  // masks, row maxima and exponentials (rows g and g+8 of the group)
+  float mrow[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+  for (int nt = 0; nt < 8; ++nt) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int row = g + (e >> 1) * 8;
+      const int pos = key0 + kw + nt * 8 + c4 * 2 + (e & 1);
+      bool vis = row < nq && pos < n_keys;
+      if (p.mode == 0) vis = vis && pos <= base + q0 + row;
+      s[nt][e] = vis ? s[nt][e] : -INFINITY;
+      mrow[e >> 1] = fmaxf(mrow[e >> 1], s[nt][e]);
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    mrow[r] = fmaxf(mrow[r], __shfl_xor_sync(0xffffffffu, mrow[r], 1));
+    mrow[r] = fmaxf(mrow[r], __shfl_xor_sync(0xffffffffu, mrow[r], 2));
+  }
+  float lrow[2] = {0.f, 0.f};
+#pragma unroll
+  for (int nt = 0; nt < 8; ++nt) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float v = s[nt][e] == -INFINITY ? 0.f : expf(s[nt][e] - mrow[e >> 1]);
+      s[nt][e] = v;
+      lrow[e >> 1] += v;
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 1);
+    lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 2);
+  }
+  // O = P V (P rounded to bf16 as the A operand)
+  float o[8][4];
+#pragma unroll
+  for (int nd = 0; nd < 8; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
+#pragma unroll
+  for (int kk = 0; kk < 4; ++kk) {
+    const uint32_t a0 = pack_bf16(s[2 * kk][0], s[2 * kk][1]);
+    const uint32_t a1 = pack_bf16(s[2 * kk][2], s[2 * kk][3]);
+    const uint32_t a2 = pack_bf16(s[2 * kk + 1][0], s[2 * kk + 1][1]);
+    const uint32_t a3 = pack_bf16(s[2 * kk + 1][2], s[2 * kk + 1][3]);
+#pragma unroll
+    for (int dp = 0; dp < 4; ++dp) {
+      uint32_t b0, b1, b2, b3;
+      const int mi = lane >> 3;
+      ldsm_x4_t(v_u32 + swz(kw + kk * 16 + (mi & 1) * 8 + (lane & 7), 2 * dp + (mi >> 1)), b0, b1,
+                b2, b3);
+      mma_bf16(o[2 * dp], a0, a1, a2, a3, b0, b1);
+      mma_bf16(o[2 * dp + 1], a0, a1, a2, a3, b2, b3);
+    }
+  }
+  // stage this warp's (m, l, O) for the in-order combine
+  if (c4 == 0) {
+    sm[warp * kQG + g] = mrow[0];
+    sm[warp * kQG + g + 8] = mrow[1];
+    sl[warp * kQG + g] = lrow[0];
+    sl[warp * kQG + g + 8] = lrow[1];
+  }
+#pragma unroll
+  for (int nd = 0; nd < 8; ++nd) {
+    float *o0 = so + (warp * kQG + g) * 64 + nd * 8 + c4 * 2;
+    float *o1 = so + (warp * kQG + g + 8) * 64 + nd * 8 + c4 * 2;
+    o0[0] = o[nd][0];
+    o0[1] = o[nd][1];
+    o1[0] = o[nd][2];
+    o1[1] = o[nd][3];
   }
   __syncthreads();
 
-  // ---- scores: thread -> (query qi = tid/8, keys kg + 8m)
-  const int qi = tid >> 3, kg = tid & 7;
-  float s[8];
-  float mloc = -INFINITY;
+  // ---- combine the four warps in order: thread -> (row qi, dims d0..d0+7)
+  const int qi = tid >> 3, d0 = (tid & 7) * 8;
+  float M = -INFINITY;
 #pragma unroll
-  for (int m = 0; m < 8; ++m) {
-    const int kk = kg + 8 * m;
-    const int pos = c * kCK + kk;
-    bool vis = qi < nq && pos < n_keys;
-    if (p.mode == 0) vis = vis && pos <= base + q0 + qi;
-    float acc = -INFINITY;
-    if (vis) {
-      acc = 0.f;
-#pragma unroll 16
-      for (int dd = 0; dd < 64; ++dd) acc = fmaf(sq[qi][dd], sk[kk][dd], acc);
-    }
-    s[m] = acc;
-    mloc = fmaxf(mloc, acc);
-  }
-  mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, 4));
-  mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, 2));
-  mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, 1));
-  float l = 0.f;
+  for (int w = 0; w < 4; ++w) M = fmaxf(M, sm[w * kQG + qi]);
+  float L = 0.f, acc[8];
 #pragma unroll
-  for (int m = 0; m < 8; ++m) {
-    const float pv = (s[m] == -INFINITY) ? 0.f : expf(s[m] - mloc);
-    sp[qi][kg + 8 * m] = pv;
-    l += pv;
-  }
-  l += __shfl_xor_sync(0xffffffffu, l, 4);
-  l += __shfl_xor_sync(0xffffffffu, l, 2);
-  l += __shfl_xor_sync(0xffffffffu, l, 1);
-  __syncthreads();
-
-  // ---- partial output: thread -> (query qi, dims d0..d0+7)
-  const int d0 = kg * 8;
-  float o[8];
+  for (int e = 0; e < 8; ++e) acc[e] = 0.f;
 #pragma unroll
-  for (int e = 0; e < 8; ++e) o[e] = 0.f;
-  if (qi < nq) {
-    for (int kk = 0; kk < kCK; ++kk) {
-      const float pv = sp[qi][kk];
+  for (int w = 0; w < 4; ++w) {
+    const float mw = sm[w * kQG + qi];
+    const float wt = (mw == -INFINITY) ? 0.f : expf(mw - M);
+    L += sl[w * kQG + qi] * wt;
 #pragma unroll
-      for (int e = 0; e < 8; ++e) o[e] = fmaf(pv, sv[kk][d0 + e], o[e]);
-    }
+    for (int e = 0; e < 8; ++e) acc[e] += so[(w * kQG + qi) * 64 + d0 + e] * wt;
   }
 
+  if (n_blocks == 1) {
+    if (qi < nq) {
+      const float inv = 1.0f / L;
+      bf16 *orow = p.out + static_cast<size_t>(i * p.rps + q0 + qi) * d_model + h * 64 + d0;
+      uint4 ov;
+      ov.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+      ov.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+      ov.z = pack_bf16(acc[4] * inv, acc[5] * inv);
+      ov.w = pack_bf16(acc[6] * inv, acc[7] * inv);
+      *reinterpret_cast<uint4 *>(orow) = ov;
+    }
+    return;
+  }
+
+  // ---- several key blocks: partials to global, the last CTA combines in order
   const int group_id = (i * p.n_heads + h) * p.qgroups + qg;
-  float *part = p.part + (static_cast<size_t>(group_id) * p.n_chunks + c) * kQG * kPartStride;
+  float *part = p.part + (static_cast<size_t>(group_id) * p.n_chunks + blk) * kQG * kPartStride;
   if (qi < nq) {
     float *pe = part + qi * kPartStride;
-    if (kg == 0) {
-      pe[0] = mloc;
-      pe[1] = l;
+    if (d0 == 0) {
+      pe[0] = M;
+      pe[1] = L;
     }
 #pragma unroll
-    for (int e = 0; e < 8; ++e) pe[2 + d0 + e] = o[e];
+    for (int e = 0; e < 8; ++e) pe[2 + d0 + e] = acc[e];
   }
   __threadfence();
   __syncthreads();
   if (tid == 0) {
     const int prev = atomicAdd(&p.counters[group_id], 1);
-    s_last = (prev == n_chunks - 1);
+    s_last = (prev == n_blocks - 1);
   }
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-
-  // ---- the last CTA combines the chunks in order
+  // A block the query cannot see carries m = -inf, l = 0, o = 0 and gets
+  // weight 0, so it adds exact zeros; the loads of all blocks are independent.
   if (qi < nq) {
     const float *pg = p.part + static_cast<size_t>(group_id) * p.n_chunks * kQG * kPartStride;
-    float M = -INFINITY;
-    for (int cc = 0; cc < n_chunks; ++cc) M = fmaxf(M, __ldcg(pg + (cc * kQG + qi) * kPartStride));
-    float L = 0.f;
-    float acc[8];
+    float MM = -INFINITY;
+    for (int u = 0; u < n_blocks; ++u) MM = fmaxf(MM, __ldcg(pg + (u * kQG + qi) * kPartStride));
+    float LL = 0.f, oo[8];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) acc[e] = 0.f;
-    for (int cc = 0; cc < n_chunks; ++cc) {
-      const float *pe = pg + (cc * kQG + qi) * kPartStride;
+    for (int e = 0; e < 8; ++e) oo[e] = 0.f;
+    for (int u = 0; u < n_blocks; ++u) {
+      const float *pe = pg + (u * kQG + qi) * kPartStride;
       const float mc = __ldcg(pe);
-      if (mc == -INFINITY) continue;
-      const float w = expf(mc - M);
-      L += __ldcg(pe + 1) * w;
+      const float lc = __ldcg(pe + 1);
+      float ov[8];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) acc[e] += __ldcg(pe + 2 + d0 + e) * w;
+      for (int e = 0; e < 8; ++e) ov[e] = __ldcg(pe + 2 + d0 + e);
+      const float wt = (mc == -INFINITY) ? 0.f : expf(mc - MM);
+      LL += lc * wt;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) oo[e] += ov[e] * wt;
     }
-    const float inv = 1.0f / L;
+    const float inv = 1.0f / LL;
     bf16 *orow = p.out + static_cast<size_t>(i * p.rps + q0 + qi) * d_model + h * 64 + d0;
-#pragma unroll
-    for (int e = 0; e < 8; ++e) orow[e] = __float2bfloat16(acc[e] * inv);
+    uint4 ov;
+    ov.x = pack_bf16(oo[0] * inv, oo[1] * inv);
+    ov.y = pack_bf16(oo[2] * inv, oo[3] * inv);
+    ov.z = pack_bf16(oo[4] * inv, oo[5] * inv);
+    ov.w = pack_bf16(oo[6] * inv, oo[7] * inv);
+    *reinterpret_cast<uint4 *>(orow) = ov;
   }
   if (tid == 0) p.counters[group_id] = 0;
 }
@@ -205,21 +377,32 @@ __global__ void rope_table_kernel(float2 *tab, int max_pos, float base) {
 
 size_t attn_partial_floats(int n_seq, int rps, int n_heads, int ctx) {
   const int qgroups = (rps + kQG - 1) / kQG;
-  const int n_chunks = (ctx + kCK - 1) / kCK;
-  return static_cast<size_t>(n_seq) * n_heads * qgroups * n_chunks * kQG * kPartStride;
+  const int n_blocks = (ctx + kKB - 1) / kKB;
+  return static_cast<size_t>(n_seq) * n_heads * qgroups * n_blocks * kQG * kPartStride;
 }
 
 int attn_counter_slots(int n_seq, int rps, int n_heads) {
   return n_seq * n_heads * ((rps + kQG - 1) / kQG);
 }
 
+cudaError_t attention_init() {
+  static cudaError_t status = cudaErrorNotReady;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    status = cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  kSmemAttn);
+  });
+  return status;
+}
+
 cudaError_t launch_attention(const AttnParams &p0, cudaStream_t s, bool pdl) {
   AttnParams p = p0;
   p.qgroups = (p.rps + kQG - 1) / kQG;
-  p.n_chunks = (p.ctx + kCK - 1) / kCK;
+  p.n_chunks = (p.ctx + kKB - 1) / kKB;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.n_chunks, p.n_heads * p.qgroups, p.n_seq);
   cfg.blockDim = dim3(128, 1, 1);
+  cfg.dynamicSmemBytes = kSmemAttn;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -256,6 +439,7 @@ extern "C" wf_status wf_attention(const void *d_q, const void *d_kc, const void 
   if (mode != 2 && !d_base) return WF_ERR_INVALID;
   if (scratch_bytes < wf_attention_scratch_bytes(n_seq, RPS, n_heads, ctx) || !d_scratch)
     return WF_ERR_CAPACITY;
+  if (wf::attention_init() != cudaSuccess) return WF_ERR_CUDA;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   wf::AttnParams p = {};
   p.q = static_cast<const wf::bf16 *>(d_q);

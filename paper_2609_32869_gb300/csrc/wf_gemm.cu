@@ -12,9 +12,12 @@
 // cache scatter, or the output-head reduction).
 //
 // K is split into a fixed number of chunks per (N, K) shape so that ~150 CTAs
-// stream weights even for a single sequence; partial tiles go to a scratch
-// buffer and the last CTA of a tile (atomic ticket, no waiting) sums them in
-// split order, so results are deterministic and independent of M.
+// stream weights even for a single sequence.  The S split CTAs of a tile form
+// a thread-block cluster; after the MMAs each stages its fp32 partial tile in
+// its own shared memory and, past a cluster barrier, reduces a slice of the
+// tile by reading the S partials over distributed shared memory in split
+// order, so results are deterministic and independent of M, and no partial
+// ever travels through global memory.
 //
 // With programmatic dependent launch the weight tiles of the first pipeline
 // stages are requested before griddepcontrol.wait: they do not depend on the
@@ -24,6 +27,7 @@
 #include <mutex>
 #include <map>
 #include <tuple>
+#include <algorithm>
 
 #include "wf_device.cuh"
 #include "wf_internal.h"
@@ -56,10 +60,73 @@ __device__ __forceinline__ void head_combine(float &m, float &s, int &arg, float
   }
 }
 
+// Epilogue of 16 consecutive token columns t0..t0+15 for output feature n.
+// acc[] holds the 16 accumulated values; every global load of the chunk (the
+// residual) is issued before its stores so the latencies overlap.
 template <int EPI>
-__device__ __forceinline__ void epilogue_store(const GemmParams &p, int t, int n, float acc) {
-  if (t >= p.M || n >= p.N) return;
-  float v = acc + (p.bias ? bf2f(p.bias[n]) : 0.f);
+__device__ __forceinline__ void epi_chunk(const GemmParams &p, int t0, int n, float bn,
+                                          const float (&acc)[16], const int2 *tok) {
+  if (n >= p.N) return;
+  if constexpr (EPI == EPI_F32) {
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj)
+      if (t0 + jj < p.M) p.out_f32[static_cast<size_t>(t0 + jj) * p.ld_out + n] = acc[jj] + bn;
+  } else if constexpr (EPI == EPI_BF16) {
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj)
+      if (t0 + jj < p.M)
+        p.out_bf16[static_cast<size_t>(t0 + jj) * p.ld_out + n] = __float2bfloat16(acc[jj] + bn);
+  } else if constexpr (EPI == EPI_GELU) {
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj)
+      if (t0 + jj < p.M)
+        p.out_bf16[static_cast<size_t>(t0 + jj) * p.ld_out + n] =
+            __float2bfloat16(gelu_erf(acc[jj] + bn));
+  } else if constexpr (EPI == EPI_RESID) {
+    float r[16];
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj)
+      r[jj] = (t0 + jj < p.M) ? p.resid[static_cast<size_t>(t0 + jj) * p.ld_resid + n] : 0.f;
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj) {
+      if (t0 + jj >= p.M) continue;
+      const float nr = r[jj] + (acc[jj] + bn);
+      p.resid[static_cast<size_t>(t0 + jj) * p.ld_resid + n] = nr;
+      if (p.tap0) p.tap0[static_cast<size_t>(t0 + jj) * p.ld_tap + n] = __float2bfloat16(nr);
+      if (p.tap1) p.tap1[static_cast<size_t>(t0 + jj) * p.ld_tap + n] = __float2bfloat16(nr);
+    }
+  } else if constexpr (EPI == EPI_KV) {
+    if (n < p.q_cols) {
+#pragma unroll
+      for (int jj = 0; jj < 16; ++jj)
+        if (t0 + jj < p.M)
+          p.out_bf16[static_cast<size_t>(t0 + jj) * p.ld_out + n] = __float2bfloat16(acc[jj] + bn);
+      return;
+    }
+    const int c = n - p.q_cols;
+    const int which = c / p.d_model;
+    const int hd = c - which * p.d_model;
+    const int h = hd >> 6, dd = hd & 63;
+    bf16 *dst = which == 0 ? p.kc : p.vc;
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj) {
+      if (t0 + jj >= p.M) continue;
+      const int2 sp = tok[jj];  // (slot, position) of this token row
+      if (sp.y >= p.ctx) {
+        set_error(p.err, WF_DEV_ERR_CAPACITY);
+        continue;
+      }
+      dst[((static_cast<size_t>(sp.x) * p.n_heads + h) * p.ctx + sp.y) * 64 + dd] =
+          __float2bfloat16(acc[jj] + bn);
+    }
+  }
+}
+
+// Epilogue of one (token t, feature n) element.
+template <int EPI>
+__device__ __forceinline__ void epi_one(const GemmParams &p, int t, int n, float y,
+                                        const int2 *tok_local) {
+  const float v = y + (p.bias ? bf2f(p.bias[n]) : 0.f);
   if constexpr (EPI == EPI_F32) {
     p.out_f32[static_cast<size_t>(t) * p.ld_out + n] = v;
   } else if constexpr (EPI == EPI_BF16) {
@@ -80,16 +147,13 @@ __device__ __forceinline__ void epilogue_store(const GemmParams &p, int t, int n
     const int c = n - p.q_cols;
     const int which = c / p.d_model;
     const int hd = c - which * p.d_model;
-    const int h = hd >> 6, dd = hd & 63;
-    const int i = t / p.rows_per_seq, j = t - i * p.rows_per_seq;
-    const int slot = p.seq_slot[i];
-    const int pos = (p.pos_base ? p.pos_base[slot] : 0) + j;
-    if (pos >= p.ctx) {
+    const int2 sp = *tok_local;
+    if (sp.y >= p.ctx) {
       set_error(p.err, WF_DEV_ERR_CAPACITY);
       return;
     }
     bf16 *dst = which == 0 ? p.kc : p.vc;
-    dst[((static_cast<size_t>(slot) * p.n_heads + h) * p.ctx + pos) * 64 + dd] =
+    dst[((static_cast<size_t>(sp.x) * p.n_heads + (hd >> 6)) * p.ctx + sp.y) * 64 + (hd & 63)] =
         __float2bfloat16(v);
   }
 }
@@ -105,14 +169,14 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
   const uint32_t stageB = static_cast<uint32_t>(BT) * kBlockK * 2;
   uint8_t *sA = smem;
   uint8_t *sB = smem + static_cast<size_t>(stages) * kStageA;
-  uint64_t *full = reinterpret_cast<uint64_t *>(sB + static_cast<size_t>(stages) * stageB);
+  uint64_t *full = reinterpret_cast<uint64_t *>(smem + p.pipe_bytes);
   uint64_t *empty = full + stages;
   uint64_t *done = empty + stages;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
-  int *flag = reinterpret_cast<int *>(tmem_slot + 1);
-  RedEntry *red = reinterpret_cast<RedEntry *>(smem + static_cast<size_t>(stages) * (kStageA + stageB) +
-                                               (2 * stages + 1) * 8 + 16 + 16);
+  RedEntry *red = reinterpret_cast<RedEntry *>(smem + p.pipe_bytes + (2 * stages + 1) * 8 + 16 + 16);
   red = reinterpret_cast<RedEntry *>((reinterpret_cast<uintptr_t>(red) + 15) & ~uintptr_t(15));
+  // per-token (slot, position) for EPI_KV, (slot, step) for sampling heads
+  int2 *tok = reinterpret_cast<int2 *>(red + (EPI == EPI_HEAD ? 4 * BT : 0));
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int tt = blockIdx.x, ntile = blockIdx.y, split = blockIdx.z;
@@ -178,6 +242,33 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
 
   // ---------------- epilogue: warp w owns TMEM lanes [32w, 32w+32) = weight rows
   pdl_wait();
+  if constexpr (EPI == EPI_HEAD) {
+    if (p.temperature > 0.f) {
+      for (int j = threadIdx.x; j < BT; j += blockDim.x) {
+        const int t = t0 + j;
+        int2 ss = make_int2(0, 0);
+        if (t < p.M) {
+          const int i = t / p.rows_per_seq;
+          ss.x = p.seq_slot[i];
+          ss.y = p.step[ss.x];
+        }
+        tok[j] = ss;
+      }
+    }
+  }
+  if constexpr (EPI == EPI_KV) {
+    for (int j = threadIdx.x; j < BT; j += blockDim.x) {
+      const int t = t0 + j;
+      int2 sp = make_int2(0, 0x7fffffff);
+      if (t < p.M) {
+        const int i = t / p.rows_per_seq, jr = t - i * p.rows_per_seq;
+        sp.x = p.seq_slot[i];
+        sp.y = (p.pos_base ? p.pos_base[sp.x] : 0) + jr;
+      }
+      tok[j] = sp;
+    }
+  }
+  __syncthreads();
   const bool ok = mbar_wait(done, 0, p.err);
   tc_fence_after();
   __syncwarp();
@@ -201,9 +292,9 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
         float m = x, s = masked ? 0.f : 1.f, gm = -INFINITY;
         int arg = n, garg = n;
         if (sampling && !masked && t < p.M) {
-          const int i = t / p.rows_per_seq, j = t - i * p.rows_per_seq;
-          const int slot = p.seq_slot[i];
-          gm = x + gumbel(p.seed, static_cast<uint32_t>(slot), static_cast<uint32_t>(p.step[slot]),
+          const int j = t % p.rows_per_seq;
+          const int2 ss = tok[c * 16 + jj];
+          gm = x + gumbel(p.seed, static_cast<uint32_t>(ss.x), static_cast<uint32_t>(ss.y),
                           static_cast<uint32_t>(j), p.tag, static_cast<uint32_t>(n));
         }
 #pragma unroll
@@ -245,49 +336,54 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
       p.recs[static_cast<size_t>(t) * n_tiles + ntile] = r;
     }
   } else {
+    const float bn = (p.bias && n < p.N) ? bf2f(p.bias[n]) : 0.f;
     if (p.splits == 1) {
       for (int c = 0; c < BT / 16; ++c) {
         float v[16];
         tmem_ld16(trow + c * 16, v);
-        if (ok) {
-#pragma unroll
-          for (int jj = 0; jj < 16; ++jj) epilogue_store<EPI>(p, t0 + c * 16 + jj, n, v[jj]);
-        }
+        if (ok) epi_chunk<EPI>(p, t0 + c * 16, n, bn, v, tok + c * 16);
       }
     } else {
-      // write this split's partial tile, then the last CTA of the tile reduces
+      // Split-K across the thread-block cluster of this tile: every CTA stages
+      // its fp32 partial tile [BT][128] in its own shared memory (the pipeline
+      // buffers are free once the MMAs completed), then each CTA reduces a
+      // slice of the tile by reading the S partials over DSMEM in split order.
+      float *tile = reinterpret_cast<float *>(smem);
+      const int r = warp * 32 + lane;
       for (int c = 0; c < BT / 16; ++c) {
         float v[16];
         tmem_ld16(trow + c * 16, v);
 #pragma unroll
-        for (int jj = 0; jj < 16; ++jj) {
-          const int t = t0 + c * 16 + jj;
-          if (t < p.M && n < p.N)
-            p.partial[(static_cast<size_t>(split) * p.M + t) * p.N + n] = v[jj];
-        }
+        for (int jj = 0; jj < 16; ++jj) tile[(c * 16 + jj) * kBlockN + r] = v[jj];
       }
-      __threadfence();
-      __syncthreads();
-      const int tile_id = ntile * p.n_tt + tt;
-      if (threadIdx.x == 0) {
-        const int prev = atomicAdd(&p.counters[tile_id], 1);
-        *flag = (prev == p.splits - 1);
-      }
-      __syncthreads();
-      if (*flag) {
-        __threadfence();
-        const int tend = min(BT, p.M - t0);
-        if (n < p.N) {
-          for (int jj = 0; jj < tend; ++jj) {
-            const int t = t0 + jj;
-            float acc = 0.f;
-            for (int sp = 0; sp < p.splits; ++sp)
-              acc += __ldcg(&p.partial[(static_cast<size_t>(sp) * p.M + t) * p.N + n]);
-            if (ok) epilogue_store<EPI>(p, t, n, acc);
+      cluster_sync();
+      const int S = p.splits;
+      const int rank = static_cast<int>(cluster_ctarank());
+      const int cols = min(BT, p.M - t0);
+      const int E = cols * kBlockN;
+      const int lo = static_cast<int>((static_cast<long long>(E) * rank) / S);
+      const int hi = static_cast<int>((static_cast<long long>(E) * (rank + 1)) / S);
+      const uint32_t tile_u32 = smem_u32(tile);
+      for (int e0 = lo; e0 < hi; e0 += 2 * 128) {
+        float acc[2] = {0.f, 0.f};
+#pragma unroll
+        for (int sp = 0; sp < 16; ++sp) {
+          if (sp < S) {
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+              const int e = e0 + u * 128 + threadIdx.x;
+              if (e < hi) acc[u] += dsmem_ld_f32(dsmem_map(tile_u32 + 4u * e, sp));
+            }
           }
         }
-        if (threadIdx.x == 0) p.counters[tile_id] = 0;
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const int e = e0 + u * 128 + threadIdx.x;
+          const int tl = e >> 7, nn = n0 + (e & 127);
+          if (e < hi && ok && nn < p.N) epi_one<EPI>(p, t0 + tl, nn, acc[u], tok + tl);
+        }
       }
+      cluster_sync();
     }
   }
 
@@ -349,7 +445,7 @@ int gemm_splits(int N, int K) {
   const int n_tiles = (N + kBlockN - 1) / kBlockN;
   const int k_iters = K / kBlockK;
   int best = 1;
-  for (int s = 1; s <= k_iters; ++s) {
+  for (int s = 1; s <= k_iters && s <= 16; ++s) {
     if (k_iters % s) continue;
     if (n_tiles * s > 160) break;
     if (k_iters / s < 2) break;
@@ -358,37 +454,92 @@ int gemm_splits(int N, int K) {
   return best;
 }
 
-size_t gemm_partial_floats(int M, int N, int splits) {
-  return splits > 1 ? static_cast<size_t>(splits) * M * N : 0;
-}
-
-int gemm_counter_slots(int M, int N) {
-  int BT, n_tt;
-  gemm_token_tiling(M, &BT, &n_tt);
-  return n_tt * ((N + kBlockN - 1) / kBlockN);
+template <int EPI>
+static cudaError_t cluster_fits(int splits, size_t smem, dim3 grid) {
+  static std::mutex mu;
+  static std::map<std::pair<int, size_t>, int> seen;
+  std::lock_guard<std::mutex> lock(mu);
+  auto key = std::make_pair(splits, smem);
+  auto it = seen.find(key);
+  if (it == seen.end()) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(128, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = 1;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = splits;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    cudaError_t e = cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<EPI>, &cfg);
+    if (e != cudaSuccess) return e;
+    it = seen.emplace(key, n).first;
+  }
+  return it->second > 0 ? cudaSuccess : cudaErrorInvalidConfiguration;
 }
 
 template <int EPI>
 static cudaError_t launch_typed(const CUtensorMap *tw, const CUtensorMap *tx, const GemmParams &p,
                                 size_t smem, cudaStream_t s, bool pdl) {
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<EPI>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+  const dim3 grid(p.n_tt, (p.N + kBlockN - 1) / kBlockN, p.splits);
+  if (p.splits > 1) {
+    cudaError_t e = cluster_fits<EPI>(p.splits, smem, grid);
     if (e != cudaSuccess) return e;
-    configured = true;
   }
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(p.n_tt, (p.N + kBlockN - 1) / kBlockN, p.splits);
+  cfg.gridDim = grid;
   cfg.blockDim = dim3(128, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[2];
+  int na = 0;
+  if (p.splits > 1) {
+    attr[na].id = cudaLaunchAttributeClusterDimension;
+    attr[na].val.clusterDim.x = 1;
+    attr[na].val.clusterDim.y = 1;
+    attr[na].val.clusterDim.z = p.splits;
+    ++na;
+  }
+  if (pdl) {
+    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
+  cfg.numAttrs = na;
   return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<EPI>, *tw, *tx, p);
+}
+
+cudaError_t gemm_init() {
+  static cudaError_t status = cudaErrorNotReady;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    const int lim = 227 * 1024;
+    status = cudaFuncSetAttribute(gemm_tc_kernel<EPI_F32>, cudaFuncAttributeMaxDynamicSharedMemorySize, lim);
+    if (status == cudaSuccess)
+      status = cudaFuncSetAttribute(gemm_tc_kernel<EPI_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize, lim);
+    if (status == cudaSuccess)
+      status = cudaFuncSetAttribute(gemm_tc_kernel<EPI_GELU>, cudaFuncAttributeMaxDynamicSharedMemorySize, lim);
+    if (status == cudaSuccess)
+      status = cudaFuncSetAttribute(gemm_tc_kernel<EPI_RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, lim);
+    if (status == cudaSuccess)
+      status = cudaFuncSetAttribute(gemm_tc_kernel<EPI_KV>, cudaFuncAttributeMaxDynamicSharedMemorySize, lim);
+    if (status == cudaSuccess)
+      status = cudaFuncSetAttribute(gemm_tc_kernel<EPI_HEAD>, cudaFuncAttributeMaxDynamicSharedMemorySize, lim);
+    // split-K clusters of up to 16 CTAs
+    const void *fns[] = {reinterpret_cast<const void *>(gemm_tc_kernel<EPI_F32>),
+                         reinterpret_cast<const void *>(gemm_tc_kernel<EPI_BF16>),
+                         reinterpret_cast<const void *>(gemm_tc_kernel<EPI_GELU>),
+                         reinterpret_cast<const void *>(gemm_tc_kernel<EPI_RESID>),
+                         reinterpret_cast<const void *>(gemm_tc_kernel<EPI_KV>)};
+    for (const void *f : fns)
+      if (status == cudaSuccess)
+        status = cudaFuncSetAttribute(f, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  });
+  return status;
 }
 
 cudaError_t launch_gemm(const void *X, const void *W, GemmParams p, cudaStream_t s, bool pdl) {
@@ -400,7 +551,8 @@ cudaError_t launch_gemm(const void *X, const void *W, GemmParams p, cudaStream_t
   if (k_iters % p.splits) return cudaErrorInvalidValue;
   p.kps = k_iters / p.splits;
   const size_t stage = kStageA + static_cast<size_t>(p.BT) * kBlockK * 2;
-  const size_t red = (p.epi == EPI_HEAD) ? 4 * static_cast<size_t>(p.BT) * sizeof(RedEntry) : 0;
+  const size_t red = (p.epi == EPI_HEAD ? 4 * static_cast<size_t>(p.BT) * sizeof(RedEntry) : 0) +
+                     static_cast<size_t>(p.BT) * sizeof(int2);
   int stages = static_cast<int>((kSmemBudget - red) / stage);
   if (stages > p.kps) stages = p.kps;
   if (stages > 16) stages = 16;
@@ -409,7 +561,11 @@ cudaError_t launch_gemm(const void *X, const void *W, GemmParams p, cudaStream_t
   uint32_t cols = 32;
   while (cols < static_cast<uint32_t>(p.BT)) cols <<= 1;
   p.tmem_cols = cols;
-  const size_t smem = 1024 + stages * stage + (2 * stages + 1) * 8 + 32 + 16 + red;
+  // the split-K cluster reduction reuses the pipeline buffers for a [BT][128] fp32 tile
+  const size_t pipe = std::max<size_t>(stages * stage, p.splits > 1 ? 512 * static_cast<size_t>(p.BT) : 0);
+  const size_t smem = 1024 + pipe + (2 * stages + 1) * 8 + 32 + 16 + red;
+  if (smem > 227 * 1024) return cudaErrorInvalidValue;
+  p.pipe_bytes = static_cast<int>(pipe);
   const CUtensorMap *tw = tmap_bf16_2d(W, p.N, p.K, kBlockN);
   const CUtensorMap *tx = tmap_bf16_2d(X, p.M, p.K, p.BT);
   if (!tw || !tx) return cudaErrorInvalidValue;
@@ -428,18 +584,20 @@ cudaError_t launch_gemm(const void *X, const void *W, GemmParams p, cudaStream_t
 
 // ------------------------------------------------------- C entry points --
 extern "C" size_t wf_gemm_scratch_bytes(int32_t M, int32_t N, int32_t K) {
-  if (M <= 0 || N <= 0 || K <= 0 || K % 64) return 0;
-  const int s = wf::gemm_splits(N, K);
-  return wf::gemm_partial_floats(M, N, s) * sizeof(float) +
-         static_cast<size_t>(wf::gemm_counter_slots(M, N)) * sizeof(int32_t) + 256;
+  // split-K partials are reduced on chip (cluster shared memory): no scratch
+  (void)M;
+  (void)N;
+  (void)K;
+  return 0;
 }
 
 extern "C" wf_status wf_gemm_bf16(const void *d_x, const void *d_w, const void *d_b, float *d_y,
                                   int32_t M, int32_t N, int32_t K, void *d_scratch,
                                   size_t scratch_bytes, void *stream) {
+  (void)d_scratch;
+  (void)scratch_bytes;
   if (!d_x || !d_w || !d_y || M <= 0 || N <= 0 || K <= 0) return WF_ERR_INVALID;
   if (K % 64) return WF_ERR_UNSUPPORTED;
-  if (scratch_bytes < wf_gemm_scratch_bytes(M, N, K) || (!d_scratch && scratch_bytes)) return WF_ERR_CAPACITY;
   wf::GemmParams p = {};
   p.M = M;
   p.N = N;
@@ -449,11 +607,7 @@ extern "C" wf_status wf_gemm_bf16(const void *d_x, const void *d_w, const void *
   p.out_f32 = d_y;
   p.ld_out = N;
   p.splits = wf::gemm_splits(N, K);
-  const size_t pf = wf::gemm_partial_floats(M, N, p.splits);
-  p.partial = static_cast<float *>(d_scratch);
-  p.counters = reinterpret_cast<int32_t *>(static_cast<char *>(d_scratch) + pf * sizeof(float));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (cudaMemsetAsync(p.counters, 0, wf::gemm_counter_slots(M, N) * sizeof(int32_t), s) != cudaSuccess)
-    return WF_ERR_CUDA;
+  if (wf::gemm_init() != cudaSuccess) return WF_ERR_CUDA;
   return wf::launch_gemm(d_x, d_w, p, s, false) == cudaSuccess ? WF_OK : WF_ERR_CUDA;
 }

@@ -37,7 +37,7 @@ struct HeadRec {  // one (token row, 128-id vocabulary tile) of the output head
 
 struct GemmParams {
   int M, N, K;
-  int BT, n_tt, splits, kps, stages;
+  int BT, n_tt, splits, kps, stages, pipe_bytes;
   uint32_t tmem_cols;
   int epi;
   const bf16 *bias;
@@ -63,9 +63,6 @@ struct GemmParams {
   const uint8_t *suppress;
   const int32_t *step;  // per slot
   uint32_t tag;
-  // split-K
-  float *partial;
-  int32_t *counters;
   uint32_t *err;
 };
 
@@ -77,9 +74,9 @@ void gemm_token_tiling(int M, int *BT, int *n_tt);
 // Split-K count for a projection of N outputs over K inputs (a function of
 // the shape only, so a row's result never depends on how many rows run).
 int gemm_splits(int N, int K);
-size_t gemm_partial_floats(int M, int N, int splits);
-int gemm_counter_slots(int M, int N);
 
+// Opt every GEMM instantiation into large dynamic shared memory (once).
+cudaError_t gemm_init();
 // Launch one GEMM.  W is [N, K] bf16, X is [M, K] bf16 (row stride K).
 cudaError_t launch_gemm(const void *X, const void *W, GemmParams p, cudaStream_t s, bool pdl);
 
@@ -95,8 +92,9 @@ struct AttnParams {
   uint32_t *err;
   int n_seq, rps, n_heads, ctx, mode, n_chunks, qgroups;
 };
-constexpr int kAttnChunk = 64;   // keys per CTA, aligned to absolute positions
-constexpr int kAttnQGroup = 16;  // query rows per CTA
+constexpr int kAttnKeysPerCTA = 256;  // keys per CTA (64 per warp), aligned to absolute positions
+constexpr int kAttnQGroup = 16;       // query rows per CTA
+cudaError_t attention_init();
 size_t attn_partial_floats(int n_seq, int rps, int n_heads, int ctx);
 int attn_counter_slots(int n_seq, int rps, int n_heads);
 cudaError_t launch_attention(const AttnParams &p, cudaStream_t s, bool pdl);

@@ -68,47 +68,72 @@ cudaError_t launch_embed(const EmbedParams &p0, cudaStream_t s, bool pdl) {
 }
 
 // ------------------------------------------------------------ LayerNorm --
-// One warp per row; mean then the mean squared deviation (two passes over
-// registers), y = (x - mean) / sqrt(var + eps) * g + b, written as bf16.
-constexpr int kLnMaxPerLane = 48;  // d <= 1536
-__global__ void layernorm_kernel(const float *x, int in_stride, int in_off, const bf16 *g,
-                                 const bf16 *b, bf16 *y, int rows, int d, float eps) {
+// One warp per row; lane l owns the float4 chunks l, l+32, ... of the row.
+// Every load (the row, the gain, the bias) is issued before any arithmetic so
+// their latencies overlap; mean, then the mean squared deviation, then
+// y = (x - mean) / sqrt(var + eps) * g + b written as bf16.
+constexpr int kLnMaxChunks = 12;  // d <= 1536 (d % 128 == 0)
+__global__ void __launch_bounds__(128) layernorm_kernel(const float *__restrict__ x, int in_stride,
+                                                        int in_off, const bf16 *__restrict__ g,
+                                                        const bf16 *__restrict__ b,
+                                                        bf16 *__restrict__ y, int rows, int d,
+                                                        float eps) {
   pdl_wait();
   pdl_launch_dependents();
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (warp >= rows) return;
-  const float *xr = x + static_cast<size_t>(warp * in_stride + in_off) * d;
-  float v[kLnMaxPerLane];
-  const int per = d / 32;
-  float sum = 0.f;
+  const float4 *xr =
+      reinterpret_cast<const float4 *>(x + static_cast<size_t>(warp * in_stride + in_off) * d);
+  const uint2 *gr = reinterpret_cast<const uint2 *>(g);
+  const uint2 *br = reinterpret_cast<const uint2 *>(b);
+  const int chunks = d >> 7;
+  float4 v[kLnMaxChunks];
+  uint2 gv[kLnMaxChunks], bv[kLnMaxChunks];
 #pragma unroll
-  for (int k = 0; k < kLnMaxPerLane; ++k) {
-    if (k < per) {
+  for (int k = 0; k < kLnMaxChunks; ++k) {
+    if (k < chunks) {
       v[k] = xr[k * 32 + lane];
-      sum += v[k];
+      gv[k] = gr[k * 32 + lane];
+      bv[k] = br[k * 32 + lane];
     }
   }
+  float sum = 0.f;
+#pragma unroll
+  for (int k = 0; k < kLnMaxChunks; ++k)
+    if (k < chunks) sum += (v[k].x + v[k].y) + (v[k].z + v[k].w);
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
   const float mean = sum / static_cast<float>(d);
   float sq = 0.f;
 #pragma unroll
-  for (int k = 0; k < kLnMaxPerLane; ++k) {
-    if (k < per) {
-      const float c = v[k] - mean;
-      sq += c * c;
+  for (int k = 0; k < kLnMaxChunks; ++k) {
+    if (k < chunks) {
+      const float a = v[k].x - mean, bb = v[k].y - mean, c = v[k].z - mean, e = v[k].w - mean;
+      sq += (a * a + bb * bb) + (c * c + e * e);
     }
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
   const float rstd = rsqrtf(sq / static_cast<float>(d) + eps);
-  bf16 *yr = y + static_cast<size_t>(warp) * d;
+  uint2 *yr = reinterpret_cast<uint2 *>(y + static_cast<size_t>(warp) * d);
 #pragma unroll
-  for (int k = 0; k < kLnMaxPerLane; ++k) {
-    if (k < per) {
-      const int e = k * 32 + lane;
-      yr[e] = __float2bfloat16((v[k] - mean) * rstd * bf2f(g[e]) + bf2f(b[e]));
+  for (int k = 0; k < kLnMaxChunks; ++k) {
+    if (k < chunks) {
+      const __nv_bfloat162 g01 = *reinterpret_cast<const __nv_bfloat162 *>(&gv[k].x);
+      const __nv_bfloat162 g23 = *reinterpret_cast<const __nv_bfloat162 *>(&gv[k].y);
+      const __nv_bfloat162 b01 = *reinterpret_cast<const __nv_bfloat162 *>(&bv[k].x);
+      const __nv_bfloat162 b23 = *reinterpret_cast<const __nv_bfloat162 *>(&bv[k].y);
+      const __nv_bfloat162 o01 = __floats2bfloat162_rn(
+          (v[k].x - mean) * rstd * __low2float(g01) + __low2float(b01),
+          (v[k].y - mean) * rstd * __high2float(g01) + __high2float(b01));
+      const __nv_bfloat162 o23 = __floats2bfloat162_rn(
+          (v[k].z - mean) * rstd * __low2float(g23) + __low2float(b23),
+          (v[k].w - mean) * rstd * __high2float(g23) + __high2float(b23));
+      uint2 o;
+      o.x = *reinterpret_cast<const uint32_t *>(&o01);
+      o.y = *reinterpret_cast<const uint32_t *>(&o23);
+      yr[k * 32 + lane] = o;
     }
   }
 }
@@ -116,9 +141,9 @@ __global__ void layernorm_kernel(const float *x, int in_stride, int in_off, cons
 cudaError_t launch_layernorm(const float *x, int in_stride, int in_off, const bf16 *g,
                              const bf16 *b, bf16 *y, int rows, int d, float eps, cudaStream_t s,
                              bool pdl) {
-  if (d % 32 || d / 32 > kLnMaxPerLane) return cudaErrorInvalidValue;
+  if (d % 128 || d / 128 > kLnMaxChunks) return cudaErrorInvalidValue;
   void *args[] = {&x, &in_stride, &in_off, &g, &b, &y, &rows, &d, &eps};
-  const int threads = 256;
+  const int threads = 128;
   const int blocks = (rows * 32 + threads - 1) / threads;
   return launch_ex(reinterpret_cast<const void *>(layernorm_kernel), dim3(blocks), dim3(threads),
                    args, s, pdl);
@@ -373,12 +398,10 @@ cudaError_t launch_state(const StateParams &p0, cudaStream_t s, bool pdl) {
 // Active list = slots whose done flag is clear, ascending.
 __global__ void compact_kernel(const int32_t *done, int max_batch, int32_t *active,
                                int32_t *n_active) {
-  __shared__ int count;
   if (threadIdx.x == 0) {
     int c = 0;
     for (int s = 0; s < max_batch; ++s)
       if (!done[s]) active[c++] = s;
-    count = c;
     *n_active = c;
   }
 }
