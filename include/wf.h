@@ -270,6 +270,22 @@ wf_status wf_attention(const void *d_q, const void *d_kc, const void *d_vc,
                        void *stream);
 size_t wf_attention_scratch_bytes(int32_t n_seq, int32_t RPS, int32_t n_heads, int32_t ctx);
 
+/* wf_attention without a scratch argument, for callers that cannot allocate
+ * device memory (a graph being captured in a mode that forbids cudaMalloc, a
+ * plugin whose host framework owns every allocation, a latency-critical loop
+ * that must not synchronise).  The paper has no counterpart: this is a
+ * deployment convenience of this library.  Its scratch is one 8 MiB device
+ * array inside the library, held by every GPU that loads it until exit;
+ * calls needing more (wf_attention_scratch_bytes > 8 MiB) return
+ * WF_ERR_CAPACITY.  The first call on a device looks the array up and may
+ * load the library's module, so make it before any stream capture.  Every
+ * call shares the array: calls that may overlap on the GPU race and must not
+ * be issued.  Arguments and results are those of wf_attention. */
+wf_status wf_attention_noalloc(const void *d_q, const void *d_kc, const void *d_vc,
+                               const int32_t *d_slot, const int32_t *d_base, int32_t n_seq,
+                               int32_t RPS, int32_t n_heads, int32_t ctx, int32_t mode,
+                               int32_t rope, float rope_base, void *d_out, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

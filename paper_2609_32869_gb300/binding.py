@@ -91,6 +91,7 @@ _SIGS = {
     "wf_gemm_scratch_bytes": (_SZ, [_I, _I, _I]),
     "wf_attention": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, C.c_float, _P, _P, _SZ, _P]),
     "wf_attention_scratch_bytes": (_SZ, [_I, _I, _I, _I]),
+    "wf_attention_noalloc": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, C.c_float, _P, _P]),
 }
 EXPORTED = tuple(_SIGS)
 
@@ -294,3 +295,10 @@ def wf_attention(q, kc, vc, slot, base, n_seq, rps, n_heads, ctx, mode, rope, ro
     _check("wf_attention", lib().wf_attention(
         _ptr(q), _ptr(kc), _ptr(vc), _ptr(slot), _ptr(base), n_seq, rps, n_heads, ctx, mode,
         int(rope), float(rope_base), _ptr(out), _ptr(scratch), scratch_bytes, _stream(stream)))
+
+
+def wf_attention_noalloc(q, kc, vc, slot, base, n_seq, rps, n_heads, ctx, mode, rope, rope_base,
+                         out, stream=None):
+    _check("wf_attention_noalloc", lib().wf_attention_noalloc(
+        _ptr(q), _ptr(kc), _ptr(vc), _ptr(slot), _ptr(base), n_seq, rps, n_heads, ctx, mode,
+        int(rope), float(rope_base), _ptr(out), _stream(stream)))

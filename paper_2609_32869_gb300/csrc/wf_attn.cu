@@ -470,3 +470,81 @@ extern "C" wf_status wf_attention(const void *d_q, const void *d_kc, const void 
     return WF_ERR_CUDA;
   return wf::launch_attention(p, s, false) == cudaSuccess ? WF_OK : WF_ERR_CUDA;
 }
+
+// ---------------------------------------------------------------------------
+// wf_attention_noalloc: the same attention for callers that cannot allocate
+// device memory.
+//
+// Some callers have no way to obtain scratch: code that runs while a CUDA
+// graph is being captured in a mode that forbids cudaMalloc, plugins hosted
+// by a framework that owns every device allocation, and latency-critical
+// loops where an allocation (which can synchronise the device) is not
+// acceptable.  For them the partial sums and counters live in one file-scope
+// device array of kNoAllocScratchBytes, which every GPU that loads this
+// library holds until the process exits.  The first call on a device looks
+// the array's device address up (cudaGetSymbolAddress), which can load the
+// library's module; make that first call before any stream capture.  All
+// calls share the array: calls that can overlap on the GPU (different
+// streams, or without ordering between them) race on it and must not be
+// issued.  The counters are cleared on every call; the partial sums need no
+// clearing.
+namespace {
+constexpr size_t kNoAllocScratchBytes = size_t(8) << 20;  // 8 MiB
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+constexpr int kNoAllocMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void *g_noalloc_ptr[kNoAllocMaxDevices] = {};
+}  // namespace
+
+extern "C" wf_status wf_attention_noalloc(const void *d_q, const void *d_kc, const void *d_vc,
+                                          const int32_t *d_slot, const int32_t *d_base,
+                                          int32_t n_seq, int32_t RPS, int32_t n_heads,
+                                          int32_t ctx, int32_t mode, int32_t rope,
+                                          float rope_base, void *d_out, void *stream) {
+  if (!d_q || !d_kc || !d_vc || !d_slot || !d_out || n_seq <= 0 || RPS <= 0 || n_heads <= 0 ||
+      ctx <= 0 || mode < 0 || mode > 2)
+    return WF_ERR_INVALID;
+  if (mode != 2 && !d_base) return WF_ERR_INVALID;
+  const size_t need = wf_attention_scratch_bytes(n_seq, RPS, n_heads, ctx);
+  if (need > kNoAllocScratchBytes) return WF_ERR_CAPACITY;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) return WF_ERR_CUDA;
+  if (dev < 0 || dev >= kNoAllocMaxDevices) return WF_ERR_UNSUPPORTED;
+  void *scratch = nullptr;
+  {
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+      void *ptr = nullptr;
+      if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) return WF_ERR_CUDA;
+      g_noalloc_ptr[dev] = ptr;
+    }
+    scratch = g_noalloc_ptr[dev];
+  }
+  if (wf::attention_init() != cudaSuccess) return WF_ERR_CUDA;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  wf::AttnParams p = {};
+  p.q = static_cast<const wf::bf16 *>(d_q);
+  p.kc = static_cast<const wf::bf16 *>(d_kc);
+  p.vc = static_cast<const wf::bf16 *>(d_vc);
+  p.out = static_cast<wf::bf16 *>(d_out);
+  p.seq_slot = d_slot;
+  p.pos_base = d_base;
+  p.n_seq = n_seq;
+  p.rps = RPS;
+  p.n_heads = n_heads;
+  p.ctx = ctx;
+  p.mode = mode;
+  const size_t pf = wf::attn_partial_floats(n_seq, RPS, n_heads, ctx);
+  const size_t counters = static_cast<size_t>(wf::attn_counter_slots(n_seq, RPS, n_heads)) * 4;
+  p.part = static_cast<float *>(scratch);
+  p.counters = reinterpret_cast<int32_t *>(static_cast<char *>(scratch) + pf * sizeof(float));
+  float2 *tab = nullptr;
+  if (rope) {
+    tab = reinterpret_cast<float2 *>(static_cast<char *>(scratch) + pf * sizeof(float) +
+                                     ((counters + 255) / 256) * 256);
+    if (wf::launch_rope_table(tab, ctx, rope_base, s) != cudaSuccess) return WF_ERR_CUDA;
+  }
+  p.rope_tab = tab;
+  if (cudaMemsetAsync(p.counters, 0, counters, s) != cudaSuccess) return WF_ERR_CUDA;
+  return wf::launch_attention(p, s, false) == cudaSuccess ? WF_OK : WF_ERR_CUDA;
+}

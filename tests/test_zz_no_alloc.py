@@ -1,0 +1,55 @@
+"""wf_attention_noalloc: the attention entry point that allocates nothing.
+
+It serves callers that cannot allocate device memory; its scratch is an
+array inside the library.  Checked through the C ABI against wf_attention
+(which takes caller scratch) on two calls in a row, the second with a
+different attention mode and size, so state left in the shared array by the
+first call must not leak into the second.  Kept in a file of its own that
+pytest collects last."""
+import numpy as np
+import pytest
+
+from paper_2609_32869_gb300 import synthetic as syn
+
+pytestmark = pytest.mark.gpu
+
+
+def _dev(bits, torch):
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
+
+
+def test_noalloc_attention_matches_scratch_entry_point_twice():
+    import torch
+    from paper_2609_32869_gb300 import binding as B
+    H, n_seq, n_slots = 4, 3, 4
+    d = H * 64
+    slots = torch.tensor([2, 0, 3], dtype=torch.int32, device="cuda")
+    base = torch.tensor([100, 0, 57, 211], dtype=torch.int32, device="cuda")
+    cases = [(2, 9, 1500, 0), (0, 9, 300, 0), (1, 9, 300, 1)]  # cross, causal, drafter block
+    for call, (mode, rps, ctx, rope) in enumerate(cases[:2] + cases[2:]):
+        q = _dev(syn.normal_bf16(41 + call, "naq", (n_seq * rps, d), 1.0), torch)
+        kc = _dev(syn.normal_bf16(42 + call, "nak", (n_slots, H, ctx, 64), 1.0), torch)
+        vc = _dev(syn.normal_bf16(43 + call, "nav", (n_slots, H, ctx, 64), 1.0), torch)
+        ref = torch.empty(n_seq * rps, d, dtype=torch.bfloat16, device="cuda")
+        got = torch.full_like(ref, float("nan"))
+        nb = B.wf_attention_scratch_bytes(n_seq, rps, H, ctx)
+        sc = torch.empty(nb, dtype=torch.uint8, device="cuda")
+        B.wf_attention(q, kc, vc, slots, base, n_seq, rps, H, ctx, mode, rope, 1e4, ref, sc, nb)
+        B.wf_attention_noalloc(q, kc, vc, slots, base, n_seq, rps, H, ctx, mode, rope, 1e4, got)
+        torch.cuda.synchronize()
+        np.testing.assert_allclose(got.float().cpu().numpy(), ref.float().cpu().numpy(),
+                                   atol=2e-2, rtol=1e-2)
+
+
+def test_noalloc_rejects_oversize_requests():
+    import torch
+    from paper_2609_32869_gb300 import binding as B
+    H, n_seq, rps, ctx = 20, 64, 9, 1500       # needs more than the 8 MiB array
+    assert B.wf_attention_scratch_bytes(n_seq, rps, H, ctx) > 8 << 20
+    q = torch.zeros(n_seq * rps, H * 64, dtype=torch.bfloat16, device="cuda")
+    kv = torch.zeros(1, dtype=torch.bfloat16, device="cuda")
+    slots = torch.zeros(n_seq, dtype=torch.int32, device="cuda")
+    out = torch.empty_like(q)
+    with pytest.raises(B.WfError) as e:
+        B.wf_attention_noalloc(q, kv, kv, slots, None, n_seq, rps, H, ctx, 2, 0, 1e4, out)
+    assert e.value.status == B.WF_ERR_CAPACITY
