@@ -5,6 +5,8 @@
 // wf_get_state, wf_get_error).  All device memory is carved from the caller's
 // workspace; the library allocates nothing on the device.
 #include <algorithm>
+#include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <map>
 #include <new>
@@ -174,10 +176,19 @@ size_t layout(wf_handle *h, const wf_config *c, int Bmax, int ctx, char *base) {
 
 inline cudaStream_t S(void *s) { return static_cast<cudaStream_t>(s); }
 
-#define WF_TRY(expr)                               \
-  do {                                             \
-    cudaError_t _e = (expr);                       \
-    if (_e != cudaSuccess) return WF_ERR_CUDA;     \
+// With WF_DEBUG set in the environment, failing CUDA calls are reported on
+// stderr (the status code alone says only WF_ERR_CUDA).
+void report_cuda(const char *what, cudaError_t e, int line) {
+  static const bool on = getenv("WF_DEBUG") != nullptr;
+  if (on) fprintf(stderr, "libwf: %s failed (wf_api.cu:%d): %s\n", what, line, cudaGetErrorString(e));
+}
+#define WF_TRY(expr)                                \
+  do {                                              \
+    cudaError_t _e = (expr);                        \
+    if (_e != cudaSuccess) {                        \
+      report_cuda(#expr, _e, __LINE__);             \
+      return WF_ERR_CUDA;                           \
+    }                                               \
   } while (0)
 
 // Programmatic dependent launch for every kernel of a call (WF_OPT_PDL).
@@ -874,13 +885,17 @@ static wf_status run_graphed(wf_handle *h, wf_handle::GraphKey key, cudaStream_t
     cudaGraph_t g = nullptr;
     cudaError_t e = cudaStreamEndCapture(h->cap_stream, &g);
     if (st != WF_OK || e != cudaSuccess) {
+      if (e != cudaSuccess) report_cuda("cudaStreamEndCapture", e, __LINE__);
       if (g) cudaGraphDestroy(g);
       return st != WF_OK ? st : WF_ERR_CUDA;
     }
     cudaGraphExec_t ex = nullptr;
     e = cudaGraphInstantiate(&ex, g, 0);
     cudaGraphDestroy(g);
-    if (e != cudaSuccess) return WF_ERR_CUDA;
+    if (e != cudaSuccess) {
+      report_cuda("cudaGraphInstantiate", e, __LINE__);
+      return WF_ERR_CUDA;
+    }
     it = h->graphs.emplace(key, wf_handle::GraphEntry{ex, h->launches}).first;
   }
   h->launches = it->second.launches;

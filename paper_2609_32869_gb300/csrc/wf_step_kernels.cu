@@ -260,7 +260,7 @@ __device__ int residual_draw(const AcceptParams &p, int slot, int step, int i, c
   return barg;
 }
 
-__global__ void accept_kernel(const AcceptParams p) {
+__global__ void __launch_bounds__(512) accept_kernel(const AcceptParams p) {
   pdl_wait();
   pdl_launch_dependents();
   const int Kp1 = p.K + 1;
@@ -349,7 +349,7 @@ __global__ void accept_kernel(const AcceptParams p) {
 cudaError_t launch_accept(const AcceptParams &p0, cudaStream_t s, bool pdl) {
   AcceptParams p = p0;
   void *args[] = {&p};
-  return launch_ex(reinterpret_cast<const void *>(accept_kernel), dim3(1), dim3(1024), args, s, pdl);
+  return launch_ex(reinterpret_cast<const void *>(accept_kernel), dim3(1), dim3(512), args, s, pdl);
 }
 
 // ---------------------------------------------------------------- state --

@@ -1,0 +1,99 @@
+"""Parity at the full Whisper-large shapes (d=1280, 20 heads, FFN 5120, 32
+layers, vocabulary 51866, 1500 encoder frames) in the launch configuration
+the benchmark uses (graph-replayed steps), on sampled sequences of a batch
+whose caches grow raggedly.  The oracle computes sequences 0 and 3 of the 4
+one by one; the others only make the batch ragged."""
+import numpy as np
+import pytest
+
+from oracle.decoder import WhisperFlashOracle
+from paper_2609_32869_gb300 import synthetic as syn
+
+pytestmark = [pytest.mark.gpu, pytest.mark.slow]
+
+LOGIT_ATOL = 3e-2
+HIDDEN_REL = 1e-2
+MARGIN = 0.05
+
+
+def _margin(row):
+    top = np.partition(np.asarray(row, np.float64), -2)[-2:]
+    return float(top[1] - top[0])
+
+
+def _forced(g, t, a, K, V):
+    cand = [g[t + j] if t + j < len(g) else 0 for j in range(K)]
+    if a < K and t + a < len(g):
+        cand[a] = (g[t + a] + 1) % V
+    return cand
+
+
+def test_large_shapes_two_steps_match_oracle():
+    import torch
+    from paper_2609_32869_gb300 import binding as B
+    from paper_2609_32869_gb300.session import Session
+    cfg = syn.LARGE
+    K, V, d = cfg.block_k, cfg.vocab, cfg.d_model
+    ws = syn.make_weights(cfg, seed=0)
+    n = 4
+    enc = syn.encoder_output(cfg, n, seed=1)
+    prompt = syn.prompts(cfg, n, length=4, seed=1)
+    budgets = np.array([60, 30, 45, 50], np.int32)
+    checked = (0, 3)
+    accept = {0: (8, 3), 3: (2, 6)}
+    s = Session(cfg, ws, max_batch=n, keep_logits=True)
+    first = s.prefill(np.arange(n, dtype=np.int32), enc, prompt, budgets).cpu().numpy()
+    torch.cuda.synchronize()
+    pre_logits = s.view(B.WF_VIEW_TARGET_LOGITS, torch.float32, (n, V)).cpu().numpy()
+
+    o = WhisperFlashOracle(syn.weights_as_float(ws, np.float64), cfg)
+    seqs, greedy = {}, {}
+    for b in checked:
+        encf = syn.bf16_bits_to_f32(enc[b]).astype(np.float64)
+        sq = o.prefill(encf, prompt[b], int(budgets[b]), seq_id=b)
+        assert np.abs(pre_logits[b] - sq._prefill_logits[-1]).max() <= LOGIT_ATOL
+        gseq = o.prefill(encf, prompt[b], int(budgets[b]), seq_id=b)
+        while len(gseq.emitted) < 1 + sum(a + 1 for a in accept[b]) + K and not gseq.done:
+            o.greedy_step(gseq)
+        seqs[b], greedy[b] = sq, gseq.emitted
+    live = [b for b in checked if first[b] == seqs[b].emitted[0] or
+            _margin(seqs[b]._prefill_logits[-1]) <= MARGIN]
+    live = [b for b in live if first[b] == seqs[b].emitted[0]]
+    decisions = steps_equal = 0
+    for step in range(2):
+        forced = syn.random_tokens(cfg, (n, K), seed=50 + step)
+        for b in checked:
+            forced[b] = _forced(greedy[b], len(seqs[b].emitted), accept[b][step], K, V)
+        toks, cnt = s.step(forced=forced.astype(np.int32))
+        torch.cuda.synchronize()
+        dl = s.view(B.WF_VIEW_DRAFT_LOGITS, torch.float32, (n * (K + 1), V)).cpu().numpy()
+        vl = s.view(B.WF_VIEW_TARGET_LOGITS, torch.float32, (n * (K + 1), V)).cpu().numpy()
+        taps = s.view(B.WF_VIEW_TAPS, torch.bfloat16, (n * (K + 1), cfg.n_taps * d)).float().cpu().numpy()
+        toks, cnt = toks.cpu().numpy(), cnt.cpu().numpy()
+        st = s.state()
+        for b in list(live):
+            rec = o.spec_step(seqs[b], forced=forced[b])
+            r0 = b * (K + 1)             # no sequence finished: active order = slot order
+            assert np.abs(dl[r0 + 1:r0 + 1 + K] - rec.draft_logits).max() <= LOGIT_ATOL
+            assert np.abs(vl[r0:r0 + rec.k + 1] - rec.verify_logits).max() <= LOGIT_ATOL
+            rel = (np.linalg.norm(taps[r0:r0 + rec.k + 1] - rec.verify_taps, axis=1)
+                   / np.linalg.norm(rec.verify_taps, axis=1))
+            assert rel.max() <= HIDDEN_REL
+            # every decision with a clear margin is identical (draft and verify rows)
+            for gpu_rows, ora_rows in ((dl[r0 + 1:r0 + 1 + K], rec.draft_logits),
+                                       (vl[r0:r0 + rec.k + 1], rec.verify_logits)):
+                for gr, orow in zip(gpu_rows, ora_rows):
+                    if _margin(orow) > MARGIN:
+                        assert int(np.argmax(gr)) == int(np.argmax(orow))
+                        decisions += 1
+            deciding = [_margin(rec.verify_logits[j]) for j in range(min(rec.accepted + 1, rec.k + 1))]
+            got = [int(x) for x in toks[b, :cnt[b]]]
+            if got == rec.emitted:
+                assert st["len"][b] == seqs[b].L
+                steps_equal += 1
+            else:
+                assert min(deciding) <= MARGIN   # only a near tie may split the trajectories
+                live.remove(b)
+    assert decisions >= 20 and steps_equal >= 1
+    assert s.error() == 0
+    s.close()
