@@ -87,11 +87,16 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
   const int i = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
-  pdl_wait();
-  pdl_launch_dependents();
+  // Before griddepcontrol.wait only data the previous kernel cannot be
+  // writing is touched: the active list and cache lengths change only between
+  // steps (the kernels that precede an attention launch in a call all wait
+  // for their predecessors before allowing it to start), the acoustic memory
+  // only at prefill, and self-attention cache rows below L only in earlier
+  // steps.  Those rows stream in while the producer of this layer's queries
+  // (and of rows L..L+rps-1) finishes.
 
-  const int slot = p.seq_slot[i];
-  const int base = (p.mode == 2 || !p.pos_base) ? 0 : p.pos_base[slot];
+  const int slot = __ldcg(p.seq_slot + i);
+  const int base = (p.mode == 2 || !p.pos_base) ? 0 : __ldcg(p.pos_base + slot);
   const int q0 = qg * kQG;
   const int nq = min(kQG, p.rps - q0);
   int n_keys;
@@ -113,17 +118,34 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
   const size_t cache_off = (static_cast<size_t>(slot) * p.n_heads + h) * p.ctx;
   const int key0 = blk * kKB;
 
-  // ---- keys and values: cp.async, zero-filled past the cache length
+  // ---- keys and values: cp.async, zero-filled past the cache length.  Rows
+  // below `fresh` are settled before this kernel starts; rows from `fresh`
+  // on are written by this step's projection and load after the wait.
+  const int fresh = p.mode == 2 ? n_keys : base;
   {
     const uint32_t k_u32 = smem_u32(sK), v_u32 = smem_u32(sV);
 #pragma unroll 4
     for (int idx = tid; idx < kKB * 8; idx += 128) {
       const int kr = idx >> 3, ch = idx & 7;
       const int pos = key0 + kr;
+      if (pos >= fresh && pos < n_keys) continue;
       const bool valid = pos < n_keys;
       const size_t off = (cache_off + (valid ? pos : 0)) * 64 + ch * 8;
       cp_async16(k_u32 + swz(kr, ch), p.kc + off, valid);
       cp_async16(v_u32 + swz(kr, ch), p.vc + off, valid);
+    }
+  }
+  pdl_wait();
+  pdl_launch_dependents();
+  if (fresh < n_keys && key0 + kKB > fresh) {
+    const uint32_t k_u32 = smem_u32(sK), v_u32 = smem_u32(sV);
+    for (int idx = tid; idx < kKB * 8; idx += 128) {
+      const int kr = idx >> 3, ch = idx & 7;
+      const int pos = key0 + kr;
+      if (pos < fresh || pos >= n_keys) continue;
+      const size_t off = (cache_off + pos) * 64 + ch * 8;
+      cp_async16(k_u32 + swz(kr, ch), p.kc + off, true);
+      cp_async16(v_u32 + swz(kr, ch), p.vc + off, true);
     }
   }
   // ---- queries, pre-scaled by 1/8 = 1/sqrt(64) (exact in binary), RoPE in fp32
