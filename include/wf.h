@@ -19,7 +19,8 @@
  *    allocated by the library on the device: the caller passes one workspace
  *    of at least wf_workspace_bytes() bytes, 256-byte aligned.
  *  - Parameters are bfloat16, row-major; matrices are [out_features, in_features]
- *    (y = x W^T + b).  Token ids are int32.
+ *    (y = x W^T + b); every weight pointer is 16-byte aligned.  Token ids are
+ *    int32.
  *  - Calls are asynchronous and ordered on the given stream unless stated.  The
  *    return value reports host-side validation and launch errors; conditions
  *    found on the device (capacity overflow, a bounded wait that gave up) are
@@ -126,7 +127,8 @@ wf_status wf_workspace_bytes(const wf_config *cfg, int32_t max_batch, int32_t ma
 
 /* Build a handle over caller-owned weights and workspace.  Encodes the TMA
  * descriptors of every weight matrix and clears the per-sequence state on
- * `stream` (asynchronously).  d_workspace must be 256-byte aligned. */
+ * `stream` (asynchronously).  d_workspace must be 256-byte aligned and every
+ * weight pointer 16-byte aligned (else WF_ERR_INVALID). */
 wf_status wf_create(const wf_config *cfg, const wf_target_weights *tw,
                     const wf_drafter_weights *dw, int32_t max_batch, int32_t max_ctx,
                     void *d_workspace, size_t workspace_bytes, void *stream,

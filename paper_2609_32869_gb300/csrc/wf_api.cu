@@ -32,6 +32,8 @@ struct wf_handle {
   bf16 *self_k, *self_v, *cross_k, *cross_v, *hist_k, *hist_v;
   // activations
   float *x, *xd, *hproj;
+  // per row and 128-feature tile (mean, M2) of x, xd, hproj for their LayerNorms
+  float2 *st_x, *st_xd, *st_hp;
   bf16 *xn, *q, *att, *h1, *taps, *hn;
   // scratch
   float *apart;
@@ -151,6 +153,9 @@ size_t layout(wf_handle *h, const wf_config *c, int Bmax, int ctx, char *base) {
   o->x = cv.take<float>(M * d);
   o->xd = cv.take<float>(M * d);
   o->hproj = cv.take<float>(M * d);
+  o->st_x = cv.take<float2>(M * (d / 128));
+  o->st_xd = cv.take<float2>(M * (d / 128));
+  o->st_hp = cv.take<float2>(M * (d / 128));
   o->xn = cv.take<bf16>(M * d);
   o->q = cv.take<bf16>(M * d);
   o->att = cv.take<bf16>(M * d);
@@ -254,15 +259,36 @@ cudaError_t gemm(wf_handle *h, const void *X, const void *W, GemmParams p, cudaS
   return e;
 }
 
-cudaError_t layernorm(wf_handle *h, const float *x, int stride, int off, const void *g,
-                      const void *b, bf16 *y, int rows, cudaStream_t s) {
+cudaError_t layernorm(wf_handle *h, const float *x, const float2 *st, int stride, int off,
+                      const void *g, const void *b, bf16 *y, int rows, cudaStream_t s) {
   h->launches++;
   prof_begin(h, s);
-  cudaError_t e = launch_layernorm(x, stride, off, static_cast<const bf16 *>(g),
+  cudaError_t e = launch_layernorm(x, st, stride, off, static_cast<const bf16 *>(g),
                                    static_cast<const bf16 *>(b), y, rows, h->d, h->cfg.ln_eps, s,
                                    kPDL);
   prof_end(h, s, WF_FAM_LAYERNORM, 6.0 * rows * h->d);
   return e;
+}
+
+// A projection of LN(x): the GEMM normalises its own token operand from the
+// fp32 rows and their tile statistics when its tiles fit in shared memory,
+// otherwise a LayerNorm kernel writes the bf16 rows first.  Both forms give
+// the same bits.
+cudaError_t ln_gemm(wf_handle *h, const float *x, const float2 *st, const void *g, const void *b,
+                    const void *W, GemmParams p, cudaStream_t s) {
+  if (gemm_ln_fits(p.M, p.N, p.K, p.epi)) {
+    p.ln_x = x;
+    p.ln_ld = h->d;
+    p.ln_tiles = h->d / 128;
+    p.ln_stats = st;
+    p.ln_g = static_cast<const bf16 *>(g);
+    p.ln_b = static_cast<const bf16 *>(b);
+    p.ln_eps = h->cfg.ln_eps;
+    return gemm(h, nullptr, W, p, s);
+  }
+  cudaError_t e = layernorm(h, x, st, 1, 0, g, b, h->xn, p.M, s);
+  if (e != cudaSuccess) return e;
+  return gemm(h, h->xn, W, p, s);
 }
 
 cudaError_t attention(wf_handle *h, const bf16 *q, const bf16 *kc, const bf16 *vc,
@@ -302,6 +328,7 @@ struct Pass {
   const int32_t *slots;
   bool drafter;
   float *x;
+  float2 *st;  // LayerNorm statistics of x
   bool taps;
 };
 
@@ -323,7 +350,6 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     xvc = h->cross_v + layer_cache_off(h, layer, h->cfg.enc_frames);
   }
   // self-attention
-  if ((e = layernorm(h, ps.x, 1, 0, lw.ln1_g, lw.ln1_b, h->xn, M, s)) != cudaSuccess) return e;
   {
     GemmParams p = gemm_base(h, M, 3 * d, d, EPI_KV);
     p.bias = static_cast<const bf16 *>(lw.qkv_b);
@@ -336,7 +362,7 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.rows_per_seq = ps.rps;
     p.seq_slot = ps.slots;
     p.pos_base = h->L;
-    if ((e = gemm(h, h->xn, lw.qkv_w, p, s)) != cudaSuccess) return e;
+    if ((e = ln_gemm(h, ps.x, ps.st, lw.ln1_g, lw.ln1_b, lw.qkv_w, p, s)) != cudaSuccess) return e;
   }
   if ((e = attention(h, h->q, kc, vc, ps.slots, ps.n_seq, ps.rps, h->ctx, ps.drafter ? 1 : 0,
                      ps.drafter, s)) != cudaSuccess)
@@ -346,16 +372,16 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.bias = static_cast<const bf16 *>(lw.out_b);
     p.resid = ps.x;
     p.ld_resid = d;
+    p.stats_out = ps.st;
     if ((e = gemm(h, h->att, lw.out_w, p, s)) != cudaSuccess) return e;
   }
   // cross-attention
-  if ((e = layernorm(h, ps.x, 1, 0, lw.ln2_g, lw.ln2_b, h->xn, M, s)) != cudaSuccess) return e;
   {
     GemmParams p = gemm_base(h, M, d, d, EPI_BF16);
     p.bias = static_cast<const bf16 *>(lw.xq_b);
     p.out_bf16 = h->q;
     p.ld_out = d;
-    if ((e = gemm(h, h->xn, lw.xq_w, p, s)) != cudaSuccess) return e;
+    if ((e = ln_gemm(h, ps.x, ps.st, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s)) != cudaSuccess) return e;
   }
   if ((e = attention(h, h->q, xkc, xvc, ps.slots, ps.n_seq, ps.rps, h->cfg.enc_frames, 2, false,
                      s)) != cudaSuccess)
@@ -365,22 +391,23 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.bias = static_cast<const bf16 *>(lw.xout_b);
     p.resid = ps.x;
     p.ld_resid = d;
+    p.stats_out = ps.st;
     if ((e = gemm(h, h->att, lw.xout_w, p, s)) != cudaSuccess) return e;
   }
   // feed-forward
-  if ((e = layernorm(h, ps.x, 1, 0, lw.ln3_g, lw.ln3_b, h->xn, M, s)) != cudaSuccess) return e;
   {
     GemmParams p = gemm_base(h, M, h->F, d, EPI_GELU);
     p.bias = static_cast<const bf16 *>(lw.fc1_b);
     p.out_bf16 = h->h1;
     p.ld_out = h->F;
-    if ((e = gemm(h, h->xn, lw.fc1_w, p, s)) != cudaSuccess) return e;
+    if ((e = ln_gemm(h, ps.x, ps.st, lw.ln3_g, lw.ln3_b, lw.fc1_w, p, s)) != cudaSuccess) return e;
   }
   {
     GemmParams p = gemm_base(h, M, d, h->F, EPI_RESID);
     p.bias = static_cast<const bf16 *>(lw.fc2_b);
     p.resid = ps.x;
     p.ld_resid = d;
+    p.stats_out = ps.st;
     if (ps.taps) {
       // the block's output residual stream, before the final LayerNorm (App. A.2)
       int found = 0;
@@ -399,11 +426,12 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
 }
 
 // Final LayerNorm (the target's, shared with the drafter) and the tied head.
-cudaError_t head(wf_handle *h, const float *x, int stride, int off, int rows, const int32_t *slots,
+cudaError_t head(wf_handle *h, const float *x, const float2 *st, int stride, int off, int rows,
+                 const int32_t *slots,
                  int rps, HeadRec *recs, HeadOut *out, float *logits, const wf_sample_params *sp,
                  uint32_t tag, int32_t *cand, cudaStream_t s) {
   cudaError_t e;
-  if ((e = layernorm(h, x, stride, off, h->tw.lnf_g, h->tw.lnf_b, h->xn, rows, s)) != cudaSuccess)
+  if ((e = layernorm(h, x, st, stride, off, h->tw.lnf_g, h->tw.lnf_b, h->xn, rows, s)) != cudaSuccess)
     return e;
   const bool sampling = sp && sp->temperature > 0.f;
   GemmParams p = gemm_base(h, rows, h->V, h->d, EPI_HEAD);
@@ -446,9 +474,14 @@ cudaError_t ingest(wf_handle *h, int n_seq, int rps, const int32_t *slots, cudaS
     p.bias = static_cast<const bf16 *>(h->dw.proj_b);
     p.out_f32 = h->hproj;
     p.ld_out = d;
+    p.stats_out = h->st_hp;
     if ((e = gemm(h, h->taps, h->dw.proj_w, p, s)) != cudaSuccess) return e;
   }
-  if ((e = layernorm(h, h->hproj, 1, 0, h->dw.hln_g, h->dw.hln_b, h->hn, M, s)) != cudaSuccess)
+  // LN_h is applied inside each drafter block's key/value projection (or by
+  // one LayerNorm kernel ahead of them when their tiles do not fit)
+  const bool fused = gemm_ln_fits(M, 2 * d, d, EPI_KV);
+  if (!fused &&
+      (e = layernorm(h, h->hproj, h->st_hp, 1, 0, h->dw.hln_g, h->dw.hln_b, h->hn, M, s)) != cudaSuccess)
     return e;
   for (int l = 0; l < h->nd; ++l) {
     const wf_layer_weights &lw = h->dl[l];
@@ -462,7 +495,18 @@ cudaError_t ingest(wf_handle *h, int n_seq, int rps, const int32_t *slots, cudaS
     p.seq_slot = slots;
     p.pos_base = h->L;
     const bf16 *wkv = static_cast<const bf16 *>(lw.qkv_w) + static_cast<size_t>(d) * d;
-    if ((e = gemm(h, h->hn, wkv, p, s)) != cudaSuccess) return e;
+    if (fused) {
+      p.ln_x = h->hproj;
+      p.ln_ld = d;
+      p.ln_tiles = d / 128;
+      p.ln_stats = h->st_hp;
+      p.ln_g = static_cast<const bf16 *>(h->dw.hln_g);
+      p.ln_b = static_cast<const bf16 *>(h->dw.hln_b);
+      p.ln_eps = h->cfg.ln_eps;
+      if ((e = gemm(h, nullptr, wkv, p, s)) != cudaSuccess) return e;
+    } else if ((e = gemm(h, h->hn, wkv, p, s)) != cudaSuccess) {
+      return e;
+    }
   }
   return cudaSuccess;
 }
@@ -481,6 +525,7 @@ cudaError_t target_pass(wf_handle *h, int n_seq, int rps, const int32_t *slots, 
   ep.forced = forced;
   ep.prompt = prompt;
   ep.x = h->x;
+  ep.stats_out = h->st_x;
   ep.n_seq = n_seq;
   ep.rps = rps;
   ep.d = h->d;
@@ -495,7 +540,7 @@ cudaError_t target_pass(wf_handle *h, int n_seq, int rps, const int32_t *slots, 
   cudaError_t e = launch_embed(ep, s, kPDL);
   prof_end(h, s, WF_FAM_OTHER, 0.0);
   if (e != cudaSuccess) return e;
-  Pass ps{n_seq, rps, slots, false, h->x, taps};
+  Pass ps{n_seq, rps, slots, false, h->x, h->st_x, taps};
   for (int l = 0; l < h->nl; ++l)
     if ((e = run_block(h, ps, h->tl[l], l, s)) != cudaSuccess) return e;
   return cudaSuccess;
@@ -551,6 +596,12 @@ wf_status wf_create(const wf_config *cfg, const wf_target_weights *tw, const wf_
   if (!tw->tok_emb || !tw->pos_emb || !tw->lnf_g || !tw->lnf_b || !tw->layers) return WF_ERR_INVALID;
   if (!dw->layers || !dw->proj_w || !dw->proj_b || !dw->hln_g || !dw->hln_b || !dw->mask_emb)
     return WF_ERR_INVALID;
+  {
+    const void *ptrs[] = {tw->tok_emb, tw->pos_emb, tw->lnf_g, tw->lnf_b, dw->proj_w,
+                          dw->proj_b,  dw->hln_g,   dw->hln_b, dw->mask_emb};
+    for (const void *p : ptrs)
+      if (reinterpret_cast<uintptr_t>(p) & 15) return WF_ERR_INVALID;
+  }
   int dev = 0, major = 0, minor = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return WF_ERR_CUDA;
   if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
@@ -731,7 +782,7 @@ wf_status wf_prefill_cross_kv(wf_handle *h, int32_t n, const int32_t *d_slots, c
     WF_TRY(target_pass(h, gn, P, slots, TOK_PROMPT, d_prompt + static_cast<size_t>(i0) * P, P,
                        nullptr, true, s));
     WF_TRY(ingest(h, gn, P, slots, s));
-    WF_TRY(head(h, h->x, P, P - 1, gn, slots, 1, h->recs_t, h->hout_t, h->logits_t, sp, kTagBonus,
+    WF_TRY(head(h, h->x, h->st_x, P, P - 1, gn, slots, 1, h->recs_t, h->hout_t, h->logits_t, sp, kTagBonus,
                 nullptr, s));
     StateParams sp1 = sp0;
     sp1.op = 1;
@@ -765,6 +816,7 @@ static wf_status draft_body(wf_handle *h, const wf_sample_params *sp, cudaStream
   ep.seq_slot = h->active;
   ep.anchor = h->anchor;
   ep.x = h->xd;
+  ep.stats_out = h->st_xd;
   ep.n_seq = n;
   ep.rps = rps;
   ep.d = h->d;
@@ -777,9 +829,9 @@ static wf_status draft_body(wf_handle *h, const wf_sample_params *sp, cudaStream
   prof_begin(h, s);
   WF_TRY(launch_embed(ep, s, kPDL));
   prof_end(h, s, WF_FAM_OTHER, 0.0);
-  Pass ps{n, rps, h->active, true, h->xd, false};
+  Pass ps{n, rps, h->active, true, h->xd, h->st_xd, false};
   for (int l = 0; l < h->nd; ++l) WF_TRY(run_block(h, ps, h->dl[l], l, s));
-  WF_TRY(head(h, h->xd, 1, 0, n * rps, h->active, rps, h->recs_d, h->hout_d, h->logits_d, sp,
+  WF_TRY(head(h, h->xd, h->st_xd, 1, 0, n * rps, h->active, rps, h->recs_d, h->hout_d, h->logits_d, sp,
               kTagDraft, h->cand, s));
   return WF_OK;
 }
@@ -789,7 +841,7 @@ static wf_status verify_body(wf_handle *h, const wf_sample_params *sp, const int
   const int n = h->n_active, rps = h->K + 1;
   if (n > 0) {
     WF_TRY(target_pass(h, n, rps, h->active, TOK_VERIFY, nullptr, 0, d_forced, true, s));
-    WF_TRY(head(h, h->x, 1, 0, n * rps, h->active, rps, h->recs_t, h->hout_t, h->logits_t, sp,
+    WF_TRY(head(h, h->x, h->st_x, 1, 0, n * rps, h->active, rps, h->recs_t, h->hout_t, h->logits_t, sp,
                 kTagBonus, nullptr, s));
     WF_TRY(ingest(h, n, rps, h->active, s));
   }
@@ -831,7 +883,7 @@ static wf_status greedy_body(wf_handle *h, const wf_sample_params *sp, int32_t *
   const int n = h->n_active;
   if (n > 0) {
     WF_TRY(target_pass(h, n, 1, h->active, TOK_ANCHOR, nullptr, 0, nullptr, false, s));
-    WF_TRY(head(h, h->x, 1, 0, n, h->active, 1, h->recs_t, h->hout_t, h->logits_t, sp, kTagBonus,
+    WF_TRY(head(h, h->x, h->st_x, 1, 0, n, h->active, 1, h->recs_t, h->hout_t, h->logits_t, sp, kTagBonus,
                 nullptr, s));
   }
   AcceptParams ap = {};

@@ -190,6 +190,52 @@ __device__ __forceinline__ float dsmem_ld_f32(uint32_t cluster_addr) {
   asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(cluster_addr) : "memory");
   return v;
 }
+__device__ __forceinline__ float4 dsmem_ld_f32x4(uint32_t cluster_addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(cluster_addr)
+               : "memory");
+  return v;
+}
+
+// ------------------------------------------------ LayerNorm statistics --
+// Per-row statistics travel as (mean, M2) over 128-feature tiles; a row's
+// LayerNorm merges its tiles in order with Chan's pairwise update, which is
+// deterministic and exact up to rounding.  Merging tile i into the first i
+// tiles weighs the new mean by 1/(i+1) and the squared mean difference by
+// 128 i/(i+1); those weights are compile-time constants of the unrolled loop.
+constexpr int kMaxStatTiles = 12;  // d <= 1536
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  return v;
+}
+__device__ __forceinline__ float2 merge_tile_stats(const float2 *st, int tiles, float eps) {
+  float2 t[kMaxStatTiles];
+#pragma unroll
+  for (int i = 0; i < kMaxStatTiles; ++i)  // every load in flight before the merge
+    if (i < tiles) t[i] = st[i];
+  float mean = t[0].x, m2 = t[0].y;
+#pragma unroll
+  for (int i = 1; i < kMaxStatTiles; ++i) {
+    if (i < tiles) {
+      constexpr float kOne = 1.0f;
+      const float w_mean = kOne / static_cast<float>(i + 1);
+      const float w_m2 = 128.0f * static_cast<float>(i) / static_cast<float>(i + 1);
+      const float delta = __fsub_rn(t[i].x, mean);
+      mean = __fmaf_rn(delta, w_mean, mean);
+      m2 = __fadd_rn(__fadd_rn(m2, t[i].y), __fmul_rn(__fmul_rn(delta, delta), w_m2));
+    }
+  }
+  const float var = __fdiv_rn(m2, 128.0f * static_cast<float>(tiles));
+  return make_float2(mean, rsqrtf(__fadd_rn(var, eps)));  // (mean, rstd)
+}
+// One normalised feature, (x - mean) * rstd * g + b, with explicit rounding
+// so every kernel that applies a LayerNorm produces the same bits.
+__device__ __forceinline__ float ln_apply(float x, float2 ms, float g, float b) {
+  return __fmaf_rn(__fmul_rn(__fsub_rn(x, ms.x), ms.y), g, b);
+}
 
 // ---------------------------------------------------------- numerics ----
 __device__ __forceinline__ float bf2f(__nv_bfloat16 x) { return __bfloat162float(x); }

@@ -38,6 +38,7 @@ constexpr int kBlockN = 128;   // weight rows per tile (MMA M)
 constexpr int kBlockK = 64;    // K per pipeline stage (one 128-byte swizzle atom)
 constexpr int kStageA = kBlockN * kBlockK * 2;  // 16 KB
 constexpr int kSmemBudget = 200 * 1024;
+constexpr int kSmemBudgetLn = 220 * 1024;  // LN mode: resident token tiles + weight ring
 
 struct __align__(16) RedEntry {
   float m, s, gm;
@@ -122,39 +123,127 @@ __device__ __forceinline__ void epi_chunk(const GemmParams &p, int t0, int n, fl
   }
 }
 
-// Epilogue of one (token t, feature n) element.
+// Epilogue of four consecutive output features n..n+3 of token row t (the
+// cluster-reduced path).  fin[] returns the final values (the updated
+// residual for EPI_RESID) for the LayerNorm statistics.
 template <int EPI>
-__device__ __forceinline__ void epi_one(const GemmParams &p, int t, int n, float y,
-                                        const int2 *tok_local) {
-  const float v = y + (p.bias ? bf2f(p.bias[n]) : 0.f);
-  if constexpr (EPI == EPI_F32) {
-    p.out_f32[static_cast<size_t>(t) * p.ld_out + n] = v;
-  } else if constexpr (EPI == EPI_BF16) {
-    p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(v);
-  } else if constexpr (EPI == EPI_GELU) {
-    p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(gelu_erf(v));
-  } else if constexpr (EPI == EPI_RESID) {
-    float *r = p.resid + static_cast<size_t>(t) * p.ld_resid + n;
-    const float nr = *r + v;
+__device__ __forceinline__ void epi_quad(const GemmParams &p, int t, int n, const float4 &a,
+                                         const int2 *tok_local, float (&fin)[4]) {
+  float v[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) v[i] += (p.bias && n + i < p.N) ? bf2f(p.bias[n + i]) : 0.f;
+  if constexpr (EPI == EPI_RESID) {
+    // N % 128 == 0 and ld_resid % 4 == 0 (checked at launch): one float4
+    float4 *r = reinterpret_cast<float4 *>(p.resid + static_cast<size_t>(t) * p.ld_resid + n);
+    const float4 o = *r;
+    const float4 nr = make_float4(o.x + v[0], o.y + v[1], o.z + v[2], o.w + v[3]);
     *r = nr;
-    if (p.tap0) p.tap0[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
-    if (p.tap1) p.tap1[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
-  } else if constexpr (EPI == EPI_KV) {
-    if (n < p.q_cols) {
-      p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(v);
-      return;
+    fin[0] = nr.x;
+    fin[1] = nr.y;
+    fin[2] = nr.z;
+    fin[3] = nr.w;
+    __nv_bfloat162 h[2] = {__floats2bfloat162_rn(nr.x, nr.y), __floats2bfloat162_rn(nr.z, nr.w)};
+    if (p.tap0) *reinterpret_cast<uint2 *>(p.tap0 + static_cast<size_t>(t) * p.ld_tap + n) =
+        *reinterpret_cast<const uint2 *>(h);
+    if (p.tap1) *reinterpret_cast<uint2 *>(p.tap1 + static_cast<size_t>(t) * p.ld_tap + n) =
+        *reinterpret_cast<const uint2 *>(h);
+    return;
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    fin[i] = v[i];
+    if (n + i >= p.N) continue;
+    if constexpr (EPI == EPI_F32) {
+      p.out_f32[static_cast<size_t>(t) * p.ld_out + n + i] = v[i];
+    } else if constexpr (EPI == EPI_BF16) {
+      p.out_bf16[static_cast<size_t>(t) * p.ld_out + n + i] = __float2bfloat16(v[i]);
+    } else if constexpr (EPI == EPI_GELU) {
+      p.out_bf16[static_cast<size_t>(t) * p.ld_out + n + i] = __float2bfloat16(gelu_erf(v[i]));
+    } else if constexpr (EPI == EPI_KV) {
+      const int nn = n + i;
+      if (nn < p.q_cols) {
+        p.out_bf16[static_cast<size_t>(t) * p.ld_out + nn] = __float2bfloat16(v[i]);
+        continue;
+      }
+      const int c = nn - p.q_cols;
+      const int which = c / p.d_model;
+      const int hd = c - which * p.d_model;
+      const int2 sp = *tok_local;
+      if (sp.y >= p.ctx) {
+        set_error(p.err, WF_DEV_ERR_CAPACITY);
+        continue;
+      }
+      bf16 *dst = which == 0 ? p.kc : p.vc;
+      dst[((static_cast<size_t>(sp.x) * p.n_heads + (hd >> 6)) * p.ctx + sp.y) * 64 + (hd & 63)] =
+          __float2bfloat16(v[i]);
     }
-    const int c = n - p.q_cols;
-    const int which = c / p.d_model;
-    const int hd = c - which * p.d_model;
-    const int2 sp = *tok_local;
-    if (sp.y >= p.ctx) {
-      set_error(p.err, WF_DEV_ERR_CAPACITY);
-      return;
+  }
+}
+
+// Build the CTA's token operand for all kps k-steps from the fp32 residual:
+// B[i][r][k] = LN(x[t0 + r])[(kit0 + i) * 64 + k] as bf16, stored in the
+// 128-byte-swizzled K-major layout the TMA would have produced (16-byte
+// chunk j of row r at chunk position j ^ (r % 8)); rows past M are zero.
+__device__ __forceinline__ void ln_build_operand(const GemmParams &p, uint8_t *sB, uint32_t stageB,
+                                                 float2 *lnst, int t0, int kit0) {
+  const int BT = p.BT;
+  const int per_stage = BT * 8;
+  const int total = p.kps * per_stage;
+  constexpr int U = 4;
+  float4 xa[U], xb[U];
+  uint4 gv[U], bv[U];
+  // chunk c -> (k-step i, token row r, 16-byte chunk j of the 64-feature step)
+  auto load = [&](int c0) {
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int c = c0 + u * 128 + static_cast<int>(threadIdx.x);
+      xa[u] = xb[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      gv[u] = bv[u] = make_uint4(0u, 0u, 0u, 0u);
+      if (c < total) {
+        const int i = c / per_stage, rem = c - i * per_stage, r = rem >> 3, j = rem & 7;
+        const int t = t0 + r, f = (kit0 + i) * kBlockK + j * 8;
+        gv[u] = *reinterpret_cast<const uint4 *>(p.ln_g + f);
+        bv[u] = *reinterpret_cast<const uint4 *>(p.ln_b + f);
+        if (t < p.M) {
+          const float4 *src =
+              reinterpret_cast<const float4 *>(p.ln_x + static_cast<size_t>(t) * p.ln_ld + f);
+          xa[u] = src[0];
+          xb[u] = src[1];
+        }
+      }
     }
-    bf16 *dst = which == 0 ? p.kc : p.vc;
-    dst[((static_cast<size_t>(sp.x) * p.n_heads + (hd >> 6)) * p.ctx + sp.y) * 64 + (hd & 63)] =
-        __float2bfloat16(v);
+  };
+  load(0);  // the first rows are in flight while the statistics merge
+  for (int j = threadIdx.x; j < BT; j += blockDim.x) {
+    const int t = t0 + j;
+    lnst[j] = t < p.M ? merge_tile_stats(p.ln_stats + static_cast<size_t>(t) * p.ln_tiles,
+                                         p.ln_tiles, p.ln_eps)
+                      : make_float2(0.f, 0.f);
+  }
+  __syncthreads();
+  for (int c0 = 0; c0 < total; c0 += U * 128) {
+    if (c0) load(c0);
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int c = c0 + u * 128 + static_cast<int>(threadIdx.x);
+      if (c >= total) continue;
+      const int i = c / per_stage, rem = c - i * per_stage, r = rem >> 3, j = rem & 7;
+      uint4 o = make_uint4(0u, 0u, 0u, 0u);
+      if (t0 + r < p.M) {
+        const float2 ms = lnst[r];
+        const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gv[u]);
+        const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&bv[u]);
+        const float xs[8] = {xa[u].x, xa[u].y, xa[u].z, xa[u].w, xb[u].x, xb[u].y, xb[u].z, xb[u].w};
+        __nv_bfloat162 h[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          h[q] = __floats2bfloat162_rn(
+              ln_apply(xs[2 * q], ms, __low2float(g2[q]), __low2float(b2[q])),
+              ln_apply(xs[2 * q + 1], ms, __high2float(g2[q]), __high2float(b2[q])));
+        o = *reinterpret_cast<const uint4 *>(h);
+      }
+      *reinterpret_cast<uint4 *>(sB + static_cast<size_t>(i) * stageB + r * 128 + ((j ^ (r & 7)) << 4)) = o;
+    }
   }
 }
 
@@ -177,6 +266,8 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
   red = reinterpret_cast<RedEntry *>((reinterpret_cast<uintptr_t>(red) + 15) & ~uintptr_t(15));
   // per-token (slot, position) for EPI_KV, (slot, step) for sampling heads
   int2 *tok = reinterpret_cast<int2 *>(red + (EPI == EPI_HEAD ? 4 * BT : 0));
+  float2 *lnst = reinterpret_cast<float2 *>(tok + BT);  // per-token (mean, rstd), LN mode
+  const bool ln = p.ln_x != nullptr;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int tt = blockIdx.x, ntile = blockIdx.y, split = blockIdx.z;
@@ -200,24 +291,39 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
   const uint32_t tmem = *tmem_slot;
   pdl_launch_dependents();
 
-  if (warp == 0 && lane == 0) {
-    // ---------------- TMA producer
-    const int npre = kps < stages ? kps : stages;
-    const uint32_t tx = kStageA + stageB;
+  // Weight tiles of the first stages do not depend on the previous kernel:
+  // request them before the dependency wait.  In LN mode each stage carries
+  // only its weight tile; the token operand is built once for all k-steps.
+  const int npre = kps < stages ? kps : stages;
+  const uint32_t tx = ln ? static_cast<uint32_t>(kStageA) : kStageA + stageB;
+  if (threadIdx.x == 0) {
     for (int i = 0; i < npre; ++i) {
       mbar_arrive_expect_tx(&full[i], tx);
       tma_load_2d(sA + static_cast<size_t>(i) * kStageA, &tmW, (kit0 + i) * kBlockK, n0, &full[i]);
     }
-    pdl_wait();  // token rows come from the previous kernel
-    for (int i = 0; i < npre; ++i)
-      tma_load_2d(sB + static_cast<size_t>(i) * stageB, &tmX, (kit0 + i) * kBlockK, t0, &full[i]);
+  }
+  if (ln) {
+    pdl_wait();  // the residual rows and their statistics come from the previous kernels
+    ln_build_operand(p, sB, stageB, lnst, t0, kit0);
+    fence_proxy_async();  // generic-proxy writes -> visible to tcgen05.mma
+    __syncthreads();
+  }
+
+  if (warp == 0 && lane == 0) {
+    // ---------------- TMA producer
+    if (!ln) {
+      pdl_wait();  // token rows come from the previous kernel
+      for (int i = 0; i < npre; ++i)
+        tma_load_2d(sB + static_cast<size_t>(i) * stageB, &tmX, (kit0 + i) * kBlockK, t0, &full[i]);
+    }
     for (int it = npre; it < kps; ++it) {
       const int s = it % stages;
       const uint32_t ph = static_cast<uint32_t>((it / stages) - 1) & 1u;
       if (!mbar_wait(&empty[s], ph, p.err)) break;
       mbar_arrive_expect_tx(&full[s], tx);
       tma_load_2d(sA + static_cast<size_t>(s) * kStageA, &tmW, (kit0 + it) * kBlockK, n0, &full[s]);
-      tma_load_2d(sB + static_cast<size_t>(s) * stageB, &tmX, (kit0 + it) * kBlockK, t0, &full[s]);
+      if (!ln)
+        tma_load_2d(sB + static_cast<size_t>(s) * stageB, &tmX, (kit0 + it) * kBlockK, t0, &full[s]);
     }
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer
@@ -228,7 +334,7 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
       if (!mbar_wait(&full[s], ph, p.err)) break;
       tc_fence_after();
       const uint32_t a0 = smem_u32(sA + static_cast<size_t>(s) * kStageA);
-      const uint32_t b0 = smem_u32(sB + static_cast<size_t>(s) * stageB);
+      const uint32_t b0 = smem_u32(sB + static_cast<size_t>(ln ? it : s) * stageB);
 #pragma unroll
       for (int kk = 0; kk < kBlockK / 16; ++kk) {
         umma_bf16(tmem, umma_desc_sw128(a0 + kk * 32), umma_desc_sw128(b0 + kk * 32), idesc,
@@ -337,17 +443,19 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
     }
   } else {
     const float bn = (p.bias && n < p.N) ? bf2f(p.bias[n]) : 0.f;
-    if (p.splits == 1) {
+    if (p.splits == 1 && !p.stats_out) {
       for (int c = 0; c < BT / 16; ++c) {
         float v[16];
         tmem_ld16(trow + c * 16, v);
         if (ok) epi_chunk<EPI>(p, t0 + c * 16, n, bn, v, tok + c * 16);
       }
     } else {
-      // Split-K across the thread-block cluster of this tile: every CTA stages
-      // its fp32 partial tile [BT][128] in its own shared memory (the pipeline
-      // buffers are free once the MMAs completed), then each CTA reduces a
-      // slice of the tile by reading the S partials over DSMEM in split order.
+      // Every CTA stages its fp32 tile [BT][128] in its own shared memory
+      // (the pipeline buffers are free once the MMAs completed).  With split-K
+      // the S CTAs of the tile form a cluster and each reduces a share of the
+      // token rows by reading the S partials over DSMEM in split order.  A
+      // warp owns a token row (4 features per lane), so the row's LayerNorm
+      // statistics over this 128-feature tile are two warp reductions.
       float *tile = reinterpret_cast<float *>(smem);
       const int r = warp * 32 + lane;
       for (int c = 0; c < BT / 16; ++c) {
@@ -356,34 +464,42 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
 #pragma unroll
         for (int jj = 0; jj < 16; ++jj) tile[(c * 16 + jj) * kBlockN + r] = v[jj];
       }
-      cluster_sync();
       const int S = p.splits;
-      const int rank = static_cast<int>(cluster_ctarank());
+      if (S > 1) cluster_sync();
+      else __syncthreads();
+      const int rank = S > 1 ? static_cast<int>(cluster_ctarank()) : 0;
       const int cols = min(BT, p.M - t0);
-      const int E = cols * kBlockN;
-      const int lo = static_cast<int>((static_cast<long long>(E) * rank) / S);
-      const int hi = static_cast<int>((static_cast<long long>(E) * (rank + 1)) / S);
+      const int rlo = cols * rank / S, rhi = cols * (rank + 1) / S;
       const uint32_t tile_u32 = smem_u32(tile);
-      for (int e0 = lo; e0 < hi; e0 += 2 * 128) {
-        float acc[2] = {0.f, 0.f};
+      const int stat_tiles = p.N / kBlockN;
+      for (int tl = rlo + warp; tl < rhi; tl += 4) {
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        const int e = tl * kBlockN + 4 * lane;
+        if (S == 1) {
+          acc = *reinterpret_cast<const float4 *>(tile + e);
+        } else {
 #pragma unroll
-        for (int sp = 0; sp < 16; ++sp) {
-          if (sp < S) {
-#pragma unroll
-            for (int u = 0; u < 2; ++u) {
-              const int e = e0 + u * 128 + threadIdx.x;
-              if (e < hi) acc[u] += dsmem_ld_f32(dsmem_map(tile_u32 + 4u * e, sp));
+          for (int sp = 0; sp < 16; ++sp) {
+            if (sp < S) {
+              const float4 v = dsmem_ld_f32x4(dsmem_map(tile_u32 + 4u * e, sp));
+              acc.x += v.x;
+              acc.y += v.y;
+              acc.z += v.z;
+              acc.w += v.w;
             }
           }
         }
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          const int e = e0 + u * 128 + threadIdx.x;
-          const int tl = e >> 7, nn = n0 + (e & 127);
-          if (e < hi && ok && nn < p.N) epi_one<EPI>(p, t0 + tl, nn, acc[u], tok + tl);
+        float fin[4] = {0.f, 0.f, 0.f, 0.f};
+        if (ok) epi_quad<EPI>(p, t0 + tl, n0 + 4 * lane, acc, tok + tl, fin);
+        if (p.stats_out) {
+          const float mean = warp_sum((fin[0] + fin[1]) + (fin[2] + fin[3])) * (1.0f / 128.f);
+          const float d0 = fin[0] - mean, d1 = fin[1] - mean, d2 = fin[2] - mean, d3 = fin[3] - mean;
+          const float m2 = warp_sum((d0 * d0 + d1 * d1) + (d2 * d2 + d3 * d3));
+          if (lane == 0 && ok)
+            p.stats_out[static_cast<size_t>(t0 + tl) * stat_tiles + ntile] = make_float2(mean, m2);
         }
       }
-      cluster_sync();
+      if (S > 1) cluster_sync();
     }
   }
 
@@ -542,32 +658,82 @@ cudaError_t gemm_init() {
   return status;
 }
 
-cudaError_t launch_gemm(const void *X, const void *W, GemmParams p, cudaStream_t s, bool pdl) {
-  if (p.M <= 0 || p.N <= 0 || p.K <= 0 || p.K % kBlockK) return cudaErrorInvalidValue;
+// Tiling, split and shared-memory plan of one launch; false if it does not fit.
+static bool plan_gemm(GemmParams &p, size_t *smem_out) {
+  if (p.M <= 0 || p.N <= 0 || p.K <= 0 || p.K % kBlockK) return false;
   gemm_token_tiling(p.M, &p.BT, &p.n_tt);
   if (p.epi == EPI_HEAD) p.splits = 1;
   if (p.splits < 1) p.splits = 1;
   const int k_iters = p.K / kBlockK;
-  if (k_iters % p.splits) return cudaErrorInvalidValue;
+  if (k_iters % p.splits) return false;
   p.kps = k_iters / p.splits;
-  const size_t stage = kStageA + static_cast<size_t>(p.BT) * kBlockK * 2;
+  const bool ln = p.ln_x != nullptr;
+  const size_t stageA = kStageA, stageB = static_cast<size_t>(p.BT) * kBlockK * 2;
   const size_t red = (p.epi == EPI_HEAD ? 4 * static_cast<size_t>(p.BT) * sizeof(RedEntry) : 0) +
-                     static_cast<size_t>(p.BT) * sizeof(int2);
-  int stages = static_cast<int>((kSmemBudget - red) / stage);
-  if (stages > p.kps) stages = p.kps;
-  if (stages > 16) stages = 16;
-  if (stages < 1) return cudaErrorInvalidValue;
+                     static_cast<size_t>(p.BT) * sizeof(int2) * (ln ? 2 : 1);
+  int stages;
+  size_t pipe;
+  if (ln) {
+    // every k-step's token tile stays resident; the weight tiles cycle through a ring
+    const size_t btiles = static_cast<size_t>(p.kps) * stageB;
+    if (btiles + 2 * stageA + red > kSmemBudgetLn) return false;
+    stages = static_cast<int>((kSmemBudgetLn - red - btiles) / stageA);
+    if (stages > p.kps) stages = p.kps;
+    if (stages > 16) stages = 16;
+    pipe = stages * stageA + btiles;
+  } else {
+    stages = static_cast<int>((kSmemBudget - red) / (stageA + stageB));
+    if (stages > p.kps) stages = p.kps;
+    if (stages > 16) stages = 16;
+    if (stages < 1) return false;
+    pipe = stages * (stageA + stageB);
+  }
   p.stages = stages;
   uint32_t cols = 32;
   while (cols < static_cast<uint32_t>(p.BT)) cols <<= 1;
   p.tmem_cols = cols;
-  // the split-K cluster reduction reuses the pipeline buffers for a [BT][128] fp32 tile
-  const size_t pipe = std::max<size_t>(stages * stage, p.splits > 1 ? 512 * static_cast<size_t>(p.BT) : 0);
+  // the staged epilogue reuses the pipeline buffers for a [BT][128] fp32 tile
+  if (p.splits > 1 || p.stats_out) pipe = std::max<size_t>(pipe, 512 * static_cast<size_t>(p.BT));
   const size_t smem = 1024 + pipe + (2 * stages + 1) * 8 + 32 + 16 + red;
-  if (smem > 227 * 1024) return cudaErrorInvalidValue;
+  if (smem > 227 * 1024) return false;
   p.pipe_bytes = static_cast<int>(pipe);
+  *smem_out = smem;
+  return true;
+}
+
+bool gemm_ln_fits(int M, int N, int K, int epi) {
+  GemmParams p = {};
+  p.M = M;
+  p.N = N;
+  p.K = K;
+  p.epi = epi;
+  p.splits = gemm_splits(N, K);
+  p.ln_x = reinterpret_cast<const float *>(16);  // only tested for non-null
+  size_t smem = 0;
+  return plan_gemm(p, &smem);
+}
+
+cudaError_t launch_gemm(const void *X, const void *W, GemmParams p, cudaStream_t s, bool pdl) {
+  const bool ln = p.ln_x != nullptr;
+  const bool quad = p.splits > 1 || p.stats_out;  // the staged (four-feature) epilogue
+  if (p.epi == EPI_HEAD && (ln || p.stats_out)) return cudaErrorInvalidValue;
+  if ((p.stats_out || p.epi == EPI_RESID) && p.N % kBlockN) return cudaErrorInvalidValue;
+  if (p.epi == EPI_RESID && (p.ld_resid % 4 || (reinterpret_cast<uintptr_t>(p.resid) & 15)))
+    return cudaErrorInvalidValue;
+  if (quad && p.epi == EPI_RESID && (p.tap0 || p.tap1) && p.ld_tap % 4) return cudaErrorInvalidValue;
+  if (ln) {
+    const uintptr_t al = reinterpret_cast<uintptr_t>(p.ln_x) | reinterpret_cast<uintptr_t>(p.ln_g) |
+                         reinterpret_cast<uintptr_t>(p.ln_b);
+    if (!p.ln_stats || !p.ln_g || !p.ln_b || (al & 15) || p.ln_ld % 4 || p.ln_tiles < 1 || p.ln_tiles > kMaxStatTiles ||
+        p.K > p.ln_tiles * 128 || p.ln_ld < p.K)
+      return cudaErrorInvalidValue;
+  } else if (!X) {
+    return cudaErrorInvalidValue;
+  }
+  size_t smem = 0;
+  if (!plan_gemm(p, &smem)) return cudaErrorInvalidValue;
   const CUtensorMap *tw = tmap_bf16_2d(W, p.N, p.K, kBlockN);
-  const CUtensorMap *tx = tmap_bf16_2d(X, p.M, p.K, p.BT);
+  const CUtensorMap *tx = ln ? tw : tmap_bf16_2d(X, p.M, p.K, p.BT);
   if (!tw || !tx) return cudaErrorInvalidValue;
   switch (p.epi) {
     case EPI_F32: return launch_typed<EPI_F32>(tw, tx, p, smem, s, pdl);

@@ -64,6 +64,19 @@ struct GemmParams {
   const int32_t *step;  // per slot
   uint32_t tag;
   uint32_t *err;
+  // LayerNorm-fused token operand: when ln_x is set the CTA builds its bf16
+  // B tiles as LN(x) = (x - mean) * rstd * g + b from fp32 rows ln_x (row
+  // stride ln_ld) and per-row statistics ln_stats[t][0..ln_tiles) (mean, M2
+  // over each 128-feature tile, merged in tile order); X is then unused.
+  const float *ln_x;
+  int ln_ld, ln_tiles;
+  const float2 *ln_stats;
+  const bf16 *ln_g, *ln_b;
+  float ln_eps;
+  // Statistics of this GEMM's outputs for the next LayerNorm: per output row
+  // and 128-feature tile, (mean, M2) of the final values (the updated
+  // residual for EPI_RESID, the output for EPI_F32); [M][N/128].
+  float2 *stats_out;
 };
 
 // Cache of TMA descriptors keyed by (address, rows, cols, box rows).
@@ -77,8 +90,12 @@ int gemm_splits(int N, int K);
 
 // Opt every GEMM instantiation into large dynamic shared memory (once).
 cudaError_t gemm_init();
-// Launch one GEMM.  W is [N, K] bf16, X is [M, K] bf16 (row stride K).
+// Launch one GEMM.  W is [N, K] bf16, X is [M, K] bf16 (row stride K), or
+// X is null and the token operand is LN(p.ln_x) built inside the kernel.
 cudaError_t launch_gemm(const void *X, const void *W, GemmParams p, cudaStream_t s, bool pdl);
+// Whether the LayerNorm-fused form of a launch fits in shared memory (all of
+// the CTA's token tiles resident); otherwise run launch_layernorm first.
+bool gemm_ln_fits(int M, int N, int K, int epi);
 
 // ------------------------------------------------------------- attention --
 struct AttnParams {
@@ -107,15 +124,17 @@ struct EmbedParams {
   const int32_t *seq_slot, *L, *anchor, *cand_in, *forced, *prompt;
   int32_t *cand_out;   // effective proposals (after forcing) [slot][K]
   float *x;
+  float2 *stats_out;  // nullable: per row and 128-feature tile (mean, M2) of x
   int n_seq, rps, d, K, P, vocab, src, drafter;
   uint32_t *err;
 };
 cudaError_t launch_embed(const EmbedParams &p, cudaStream_t s, bool pdl);
 
-// y[r] = LN(x[r*in_stride + in_off]) as bf16 (fp32 statistics).
-cudaError_t launch_layernorm(const float *x, int in_stride, int in_off, const bf16 *g,
-                             const bf16 *b, bf16 *y, int rows, int d, float eps, cudaStream_t s,
-                             bool pdl);
+// y[r] = LN(x[i]) as bf16 with i = r*in_stride + in_off, using the row's
+// per-tile statistics stats[i][0..d/128) (mean, M2) written by its producer.
+cudaError_t launch_layernorm(const float *x, const float2 *stats, int in_stride, int in_off,
+                             const bf16 *g, const bf16 *b, bf16 *y, int rows, int d, float eps,
+                             cudaStream_t s, bool pdl);
 
 // Reduce head records over the vocabulary tiles of each row.
 struct HeadOut {

@@ -48,15 +48,52 @@ __global__ void embed_kernel(const EmbedParams p) {
   }
   const int pos = (p.drafter || !p.L) ? 0 : ((p.src == TOK_PROMPT ? 0 : p.L[slot]) + j);
   float *x = p.x + static_cast<size_t>(r) * p.d;
-  for (int e = threadIdx.x; e < p.d; e += blockDim.x) {
-    float v;
+  // thread tid holds feature 128k + tid of every 128-feature tile k
+  const int tiles = p.d >> 7;
+  float v[kMaxStatTiles];
+#pragma unroll
+  for (int k = 0; k < kMaxStatTiles; ++k) {
+    if (k >= tiles) continue;
+    const int e = k * 128 + threadIdx.x;
+    float val;
     if (use_mask) {
-      v = bf2f(p.mask_emb[e]);
+      val = bf2f(p.mask_emb[e]);
     } else {
-      v = bf2f(p.tok_emb[static_cast<size_t>(tok) * p.d + e]);
-      if (!p.drafter) v += bf2f(p.pos_emb[static_cast<size_t>(pos) * p.d + e]);
+      val = bf2f(p.tok_emb[static_cast<size_t>(tok) * p.d + e]);
+      if (!p.drafter) val += bf2f(p.pos_emb[static_cast<size_t>(pos) * p.d + e]);
     }
-    x[e] = v;
+    v[k] = val;
+    x[e] = val;
+  }
+  if (!p.stats_out) return;
+  // per-tile (mean, M2) of the row for the next LayerNorm
+  __shared__ float red[4][kMaxStatTiles];
+  __shared__ float mean_s[kMaxStatTiles];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+#pragma unroll
+  for (int k = 0; k < kMaxStatTiles; ++k) {
+    if (k >= tiles) continue;
+    const float sum = warp_sum(v[k]);
+    if (lane == 0) red[warp][k] = sum;
+  }
+  __syncthreads();
+  if (threadIdx.x < tiles) {
+    const int k = threadIdx.x;
+    mean_s[k] = ((red[0][k] + red[1][k]) + (red[2][k] + red[3][k])) * (1.0f / 128.f);
+  }
+  __syncthreads();
+#pragma unroll
+  for (int k = 0; k < kMaxStatTiles; ++k) {
+    if (k >= tiles) continue;
+    const float dv = v[k] - mean_s[k];
+    const float sq = warp_sum(dv * dv);
+    if (lane == 0) red[warp][k] = sq;
+  }
+  __syncthreads();
+  if (threadIdx.x < tiles) {
+    const int k = threadIdx.x;
+    p.stats_out[static_cast<size_t>(r) * tiles + k] =
+        make_float2(mean_s[k], (red[0][k] + red[1][k]) + (red[2][k] + red[3][k]));
   }
 }
 
@@ -69,12 +106,14 @@ cudaError_t launch_embed(const EmbedParams &p0, cudaStream_t s, bool pdl) {
 
 // ------------------------------------------------------------ LayerNorm --
 // One warp per row; lane l owns the float4 chunks l, l+32, ... of the row.
-// Every load (the row, the gain, the bias) is issued before any arithmetic so
-// their latencies overlap; mean, then the mean squared deviation, then
-// y = (x - mean) / sqrt(var + eps) * g + b written as bf16.
-constexpr int kLnMaxChunks = 12;  // d <= 1536 (d % 128 == 0)
-__global__ void __launch_bounds__(128) layernorm_kernel(const float *__restrict__ x, int in_stride,
-                                                        int in_off, const bf16 *__restrict__ g,
+// The row's statistics come from the kernel that wrote it (per 128-feature
+// tile, merged in tile order), so this kernel and the GEMMs that normalise
+// their own token operand produce identical bits.  Every load is issued
+// before any arithmetic so the latencies overlap.
+__global__ void __launch_bounds__(128) layernorm_kernel(const float *__restrict__ x,
+                                                        const float2 *__restrict__ stats,
+                                                        int in_stride, int in_off,
+                                                        const bf16 *__restrict__ g,
                                                         const bf16 *__restrict__ b,
                                                         bf16 *__restrict__ y, int rows, int d,
                                                         float eps) {
@@ -83,53 +122,36 @@ __global__ void __launch_bounds__(128) layernorm_kernel(const float *__restrict_
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (warp >= rows) return;
-  const float4 *xr =
-      reinterpret_cast<const float4 *>(x + static_cast<size_t>(warp * in_stride + in_off) * d);
+  const size_t row = static_cast<size_t>(warp) * in_stride + in_off;
+  const float4 *xr = reinterpret_cast<const float4 *>(x + row * d);
   const uint2 *gr = reinterpret_cast<const uint2 *>(g);
   const uint2 *br = reinterpret_cast<const uint2 *>(b);
   const int chunks = d >> 7;
-  float4 v[kLnMaxChunks];
-  uint2 gv[kLnMaxChunks], bv[kLnMaxChunks];
+  float4 v[kMaxStatTiles];
+  uint2 gv[kMaxStatTiles], bv[kMaxStatTiles];
 #pragma unroll
-  for (int k = 0; k < kLnMaxChunks; ++k) {
+  for (int k = 0; k < kMaxStatTiles; ++k) {
     if (k < chunks) {
       v[k] = xr[k * 32 + lane];
       gv[k] = gr[k * 32 + lane];
       bv[k] = br[k * 32 + lane];
     }
   }
-  float sum = 0.f;
-#pragma unroll
-  for (int k = 0; k < kLnMaxChunks; ++k)
-    if (k < chunks) sum += (v[k].x + v[k].y) + (v[k].z + v[k].w);
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-  const float mean = sum / static_cast<float>(d);
-  float sq = 0.f;
-#pragma unroll
-  for (int k = 0; k < kLnMaxChunks; ++k) {
-    if (k < chunks) {
-      const float a = v[k].x - mean, bb = v[k].y - mean, c = v[k].z - mean, e = v[k].w - mean;
-      sq += (a * a + bb * bb) + (c * c + e * e);
-    }
-  }
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
-  const float rstd = rsqrtf(sq / static_cast<float>(d) + eps);
+  const float2 ms = merge_tile_stats(stats + row * chunks, chunks, eps);
   uint2 *yr = reinterpret_cast<uint2 *>(y + static_cast<size_t>(warp) * d);
 #pragma unroll
-  for (int k = 0; k < kLnMaxChunks; ++k) {
+  for (int k = 0; k < kMaxStatTiles; ++k) {
     if (k < chunks) {
       const __nv_bfloat162 g01 = *reinterpret_cast<const __nv_bfloat162 *>(&gv[k].x);
       const __nv_bfloat162 g23 = *reinterpret_cast<const __nv_bfloat162 *>(&gv[k].y);
       const __nv_bfloat162 b01 = *reinterpret_cast<const __nv_bfloat162 *>(&bv[k].x);
       const __nv_bfloat162 b23 = *reinterpret_cast<const __nv_bfloat162 *>(&bv[k].y);
-      const __nv_bfloat162 o01 = __floats2bfloat162_rn(
-          (v[k].x - mean) * rstd * __low2float(g01) + __low2float(b01),
-          (v[k].y - mean) * rstd * __high2float(g01) + __high2float(b01));
-      const __nv_bfloat162 o23 = __floats2bfloat162_rn(
-          (v[k].z - mean) * rstd * __low2float(g23) + __low2float(b23),
-          (v[k].w - mean) * rstd * __high2float(g23) + __high2float(b23));
+      const __nv_bfloat162 o01 =
+          __floats2bfloat162_rn(ln_apply(v[k].x, ms, __low2float(g01), __low2float(b01)),
+                                ln_apply(v[k].y, ms, __high2float(g01), __high2float(b01)));
+      const __nv_bfloat162 o23 =
+          __floats2bfloat162_rn(ln_apply(v[k].z, ms, __low2float(g23), __low2float(b23)),
+                                ln_apply(v[k].w, ms, __high2float(g23), __high2float(b23)));
       uint2 o;
       o.x = *reinterpret_cast<const uint32_t *>(&o01);
       o.y = *reinterpret_cast<const uint32_t *>(&o23);
@@ -138,11 +160,11 @@ __global__ void __launch_bounds__(128) layernorm_kernel(const float *__restrict_
   }
 }
 
-cudaError_t launch_layernorm(const float *x, int in_stride, int in_off, const bf16 *g,
-                             const bf16 *b, bf16 *y, int rows, int d, float eps, cudaStream_t s,
-                             bool pdl) {
-  if (d % 128 || d / 128 > kLnMaxChunks) return cudaErrorInvalidValue;
-  void *args[] = {&x, &in_stride, &in_off, &g, &b, &y, &rows, &d, &eps};
+cudaError_t launch_layernorm(const float *x, const float2 *stats, int in_stride, int in_off,
+                             const bf16 *g, const bf16 *b, bf16 *y, int rows, int d, float eps,
+                             cudaStream_t s, bool pdl) {
+  if (d % 128 || d / 128 > kMaxStatTiles || !stats) return cudaErrorInvalidValue;
+  void *args[] = {&x, &stats, &in_stride, &in_off, &g, &b, &y, &rows, &d, &eps};
   const int threads = 128;
   const int blocks = (rows * 32 + threads - 1) / threads;
   return launch_ex(reinterpret_cast<const void *>(layernorm_kernel), dim3(blocks), dim3(threads),
