@@ -48,6 +48,15 @@ WORKLOADS = {
     "tiny_b1": dict(cfg="TINY", batch=1, budget=(200, 200), accept="uniform",
                     text="Whisper-tiny-shaped decoder (d=384, 6 heads, FFN 1536, 4 layers, "
                          "vocab 51865), batch 1, accept length uniform 0..8"),
+    # Depth-reduced cases for profiler captures: every kernel keeps the large
+    # per-layer shapes and launch configuration; only the number of target
+    # blocks shrinks so a capture holds a few GB and few launches.
+    "large_b1_4l": dict(cfg="LARGE", layers=4, batch=1, budget=(40, 40), accept="uniform",
+                        text="large per-layer shapes cut to 4 target blocks (profiling case), "
+                             "batch 1, 40-token transcript, accept length uniform 0..8"),
+    "large_b96_2l": dict(cfg="LARGE", layers=2, batch=96, budget=(20, 40), accept="geometric",
+                         text="large per-layer shapes cut to 2 target blocks (profiling case), "
+                              "batch 96, transcript lengths uniform 20..40"),
 }
 
 
@@ -60,8 +69,14 @@ def _peaks():
         return 6800.0, 1900.0, "fallback"
 
 
-def _cfg(name):
-    return getattr(syn, name)
+def _cfg(name, layers=None):
+    cfg = getattr(syn, name)
+    if layers:
+        import dataclasses
+        taps = tuple(min(t, layers - 1) for t in (0, 1, 2, 3, 3))
+        cfg = dataclasses.replace(cfg, name=f"{cfg.name}_{layers}l", n_layers=layers, taps=taps,
+                                  draft_init_from=(0, layers - 1))
+    return cfg
 
 
 # ----------------------------------------------------------------- schedule --
@@ -172,7 +187,7 @@ def run_ours(args, rank, world):
     local = int(os.environ.get("LOCAL_RANK", "0"))
     torch.cuda.set_device(local)
     wl = WORKLOADS[args.workload]
-    cfg = _cfg(wl["cfg"])
+    cfg = _cfg(wl["cfg"], wl.get("layers"))
     Bn = wl["batch"]
     host_ws = syn.make_weights(cfg, seed=0)
     dev = upload_weights(host_ws)
@@ -463,7 +478,7 @@ def cpu_baseline(cfg, ws, enc, prompt, budgets, acc, budget_s=15.0):
 
 def run_reference(args):
     wl = WORKLOADS[args.workload]
-    cfg = _cfg(wl["cfg"])
+    cfg = _cfg(wl["cfg"], wl.get("layers"))
     ws = syn.make_weights(cfg, seed=0)
     Bn = wl["batch"]
     enc = syn.encoder_output(cfg, 1, seed=1)

@@ -39,6 +39,7 @@ constexpr int kBlockK = 64;    // K per pipeline stage (one 128-byte swizzle ato
 constexpr int kStageA = kBlockN * kBlockK * 2;  // 16 KB
 constexpr int kSmemBudget = 200 * 1024;
 constexpr int kSmemBudgetLn = 220 * 1024;  // LN mode: resident token tiles + weight ring
+constexpr size_t kSmemPerSM = 228 * 1024;  // shared memory of one SM
 
 struct __align__(16) RedEntry {
   float m, s, gm;
@@ -128,14 +129,13 @@ __device__ __forceinline__ void epi_chunk(const GemmParams &p, int t0, int n, fl
 // residual for EPI_RESID) for the LayerNorm statistics.
 template <int EPI>
 __device__ __forceinline__ void epi_quad(const GemmParams &p, int t, int n, const float4 &a,
+                                         const float (&b4)[4], const float4 *pre_resid,
                                          const int2 *tok_local, float (&fin)[4]) {
-  float v[4] = {a.x, a.y, a.z, a.w};
-#pragma unroll
-  for (int i = 0; i < 4; ++i) v[i] += (p.bias && n + i < p.N) ? bf2f(p.bias[n + i]) : 0.f;
+  float v[4] = {a.x + b4[0], a.y + b4[1], a.z + b4[2], a.w + b4[3]};
   if constexpr (EPI == EPI_RESID) {
     // N % 128 == 0 and ld_resid % 4 == 0 (checked at launch): one float4
     float4 *r = reinterpret_cast<float4 *>(p.resid + static_cast<size_t>(t) * p.ld_resid + n);
-    const float4 o = *r;
+    const float4 o = pre_resid ? *pre_resid : *r;
     const float4 nr = make_float4(o.x + v[0], o.y + v[1], o.z + v[2], o.w + v[3]);
     *r = nr;
     fin[0] = nr.x;
@@ -374,6 +374,28 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
       tok[j] = sp;
     }
   }
+  // Inputs of the four-feature epilogue that do not depend on this GEMM's
+  // result load while the MMAs run: the bias of the lane's four features and,
+  // for a residual update, the first row this warp will own.
+  const int cols = max(0, min(BT, p.M - t0));
+  float b4[4] = {0.f, 0.f, 0.f, 0.f};
+  float4 pre = make_float4(0.f, 0.f, 0.f, 0.f);
+  bool has_pre = false;
+  if (EPI != EPI_HEAD && (p.splits > 1 || p.stats_out)) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int nn = n0 + 4 * lane + i;
+      b4[i] = (p.bias && nn < p.N) ? bf2f(p.bias[nn]) : 0.f;
+    }
+    if constexpr (EPI == EPI_RESID) {
+      const int S = p.splits, tl = cols * split / S + warp;
+      if (tl < cols * (split + 1) / S) {
+        pre = *reinterpret_cast<const float4 *>(p.resid + static_cast<size_t>(t0 + tl) * p.ld_resid +
+                                                n0 + 4 * lane);
+        has_pre = true;
+      }
+    }
+  }
   __syncthreads();
   const bool ok = mbar_wait(done, 0, p.err);
   tc_fence_after();
@@ -441,64 +463,82 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
       r._pad[0] = r._pad[1] = r._pad[2] = 0;
       p.recs[static_cast<size_t>(t) * n_tiles + ntile] = r;
     }
-  } else {
+  } else if (p.splits == 1 && !p.stats_out) {
     const float bn = (p.bias && n < p.N) ? bf2f(p.bias[n]) : 0.f;
-    if (p.splits == 1 && !p.stats_out) {
-      for (int c = 0; c < BT / 16; ++c) {
-        float v[16];
-        tmem_ld16(trow + c * 16, v);
-        if (ok) epi_chunk<EPI>(p, t0 + c * 16, n, bn, v, tok + c * 16);
+    for (int c = 0; c < BT / 16; ++c) {
+      float v[16];
+      tmem_ld16(trow + c * 16, v);
+      if (ok) epi_chunk<EPI>(p, t0 + c * 16, n, bn, v, tok + c * 16);
+    }
+  } else {
+    // Four-feature epilogue: a warp owns a token row (lane l: features
+    // 4l..4l+3), so the row's LayerNorm statistics over this 128-feature tile
+    // are two warp reductions.  Split-K partials are summed in split order.
+    const int S = p.splits;
+    const int rank = split;  // cluster (1, 1, S) over gridDim.z == S: rank == blockIdx.z
+    const int rlo = cols * rank / S, rhi = cols * (rank + 1) / S;
+    const int stat_tiles = p.N / kBlockN;
+    auto finish_row = [&](int tl, const float4 &acc, bool valid) {
+      float fin[4] = {0.f, 0.f, 0.f, 0.f};
+      if (valid)
+        epi_quad<EPI>(p, t0 + tl, n0 + 4 * lane, acc, b4, (has_pre && tl == rlo + warp) ? &pre : nullptr,
+                      tok + tl, fin);
+      if (p.stats_out) {
+        const float mean = warp_sum((fin[0] + fin[1]) + (fin[2] + fin[3])) * (1.0f / 128.f);
+        const float d0 = fin[0] - mean, d1 = fin[1] - mean, d2 = fin[2] - mean, d3 = fin[3] - mean;
+        const float m2 = warp_sum((d0 * d0 + d1 * d1) + (d2 * d2 + d3 * d3));
+        if (lane == 0 && valid)
+          p.stats_out[static_cast<size_t>(t0 + tl) * stat_tiles + ntile] = make_float2(mean, m2);
       }
-    } else {
-      // Every CTA stages its fp32 tile [BT][128] in its own shared memory
-      // (the pipeline buffers are free once the MMAs completed).  With split-K
-      // the S CTAs of the tile form a cluster and each reduces a share of the
-      // token rows by reading the S partials over DSMEM in split order.  A
-      // warp owns a token row (4 features per lane), so the row's LayerNorm
-      // statistics over this 128-feature tile are two warp reductions.
-      float *tile = reinterpret_cast<float *>(smem);
-      const int r = warp * 32 + lane;
-      for (int c = 0; c < BT / 16; ++c) {
-        float v[16];
-        tmem_ld16(trow + c * 16, v);
+    };
+    const int r = warp * 32 + lane;
+    // Every CTA stages its fp32 tile [BT][128] in its own shared memory (the
+    // pipeline buffers are free once the MMAs completed); with split-K the S
+    // CTAs of the tile form a cluster and each reduces its share of the token
+    // rows by reading the S partials over DSMEM.
+    float *tile = reinterpret_cast<float *>(smem);
+    for (int c = 0; c < BT / 16; ++c) {
+      float v[16];
+      tmem_ld16(trow + c * 16, v);
 #pragma unroll
-        for (int jj = 0; jj < 16; ++jj) tile[(c * 16 + jj) * kBlockN + r] = v[jj];
-      }
-      const int S = p.splits;
-      if (S > 1) cluster_sync();
-      else __syncthreads();
-      const int rank = S > 1 ? static_cast<int>(cluster_ctarank()) : 0;
-      const int cols = min(BT, p.M - t0);
-      const int rlo = cols * rank / S, rhi = cols * (rank + 1) / S;
-      const uint32_t tile_u32 = smem_u32(tile);
-      const int stat_tiles = p.N / kBlockN;
-      for (int tl = rlo + warp; tl < rhi; tl += 4) {
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        const int e = tl * kBlockN + 4 * lane;
-        if (S == 1) {
-          acc = *reinterpret_cast<const float4 *>(tile + e);
-        } else {
+      for (int jj = 0; jj < 16; ++jj) tile[(c * 16 + jj) * kBlockN + r] = v[jj];
+    }
+    if (S > 1) cluster_sync();
+    else __syncthreads();
+    const uint32_t tile_u32 = smem_u32(tile);
+    auto reduce_row = [&](int tl) {
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      const int e = tl * kBlockN + 4 * lane;
+      if (S == 1) {
+        acc = *reinterpret_cast<const float4 *>(tile + e);
+      } else {
 #pragma unroll
-          for (int sp = 0; sp < 16; ++sp) {
-            if (sp < S) {
-              const float4 v = dsmem_ld_f32x4(dsmem_map(tile_u32 + 4u * e, sp));
-              acc.x += v.x;
-              acc.y += v.y;
-              acc.z += v.z;
-              acc.w += v.w;
-            }
+        for (int sp = 0; sp < 16; ++sp) {
+          if (sp < S) {
+            const float4 v = dsmem_ld_f32x4(dsmem_map(tile_u32 + 4u * e, sp));
+            acc.x += v.x;
+            acc.y += v.y;
+            acc.z += v.z;
+            acc.w += v.w;
           }
         }
-        float fin[4] = {0.f, 0.f, 0.f, 0.f};
-        if (ok) epi_quad<EPI>(p, t0 + tl, n0 + 4 * lane, acc, tok + tl, fin);
-        if (p.stats_out) {
-          const float mean = warp_sum((fin[0] + fin[1]) + (fin[2] + fin[3])) * (1.0f / 128.f);
-          const float d0 = fin[0] - mean, d1 = fin[1] - mean, d2 = fin[2] - mean, d3 = fin[3] - mean;
-          const float m2 = warp_sum((d0 * d0 + d1 * d1) + (d2 * d2 + d3 * d3));
-          if (lane == 0 && ok)
-            p.stats_out[static_cast<size_t>(t0 + tl) * stat_tiles + ntile] = make_float2(mean, m2);
-        }
       }
+      return acc;
+    };
+    if (S > 1 && rhi - rlo <= 8) {
+      // at most two rows per warp: read every partial first, tell the peers
+      // their tiles are free, then run the epilogue while they finish
+      float4 acc[2];
+#pragma unroll
+      for (int k = 0; k < 2; ++k)
+        if (rlo + warp + 4 * k < rhi) acc[k] = reduce_row(rlo + warp + 4 * k);
+      cluster_arrive();
+#pragma unroll
+      for (int k = 0; k < 2; ++k)
+        if (rlo + warp + 4 * k < rhi) finish_row(rlo + warp + 4 * k, acc[k], ok);
+      cluster_wait();
+    } else {
+      for (int tl = rlo + warp; tl < rhi; tl += 4) finish_row(tl, reduce_row(tl), ok);
       if (S > 1) cluster_sync();
     }
   }
@@ -671,21 +711,22 @@ static bool plan_gemm(GemmParams &p, size_t *smem_out) {
   const size_t stageA = kStageA, stageB = static_cast<size_t>(p.BT) * kBlockK * 2;
   const size_t red = (p.epi == EPI_HEAD ? 4 * static_cast<size_t>(p.BT) * sizeof(RedEntry) : 0) +
                      static_cast<size_t>(p.BT) * sizeof(int2) * (ln ? 2 : 1);
+  const size_t fixed = red;
   int stages;
   size_t pipe;
   if (ln) {
     // every k-step's token tile stays resident; the weight tiles cycle through a ring
     const size_t btiles = static_cast<size_t>(p.kps) * stageB;
-    if (btiles + 2 * stageA + red > kSmemBudgetLn) return false;
-    stages = static_cast<int>((kSmemBudgetLn - red - btiles) / stageA);
+    if (btiles + 2 * stageA + fixed > kSmemBudgetLn) return false;
+    stages = static_cast<int>((kSmemBudgetLn - fixed - btiles) / stageA);
     if (stages > p.kps) stages = p.kps;
     if (stages > 16) stages = 16;
     pipe = stages * stageA + btiles;
   } else {
-    stages = static_cast<int>((kSmemBudget - red) / (stageA + stageB));
+    if (fixed + stageA + stageB > kSmemBudget) return false;
+    stages = static_cast<int>((kSmemBudget - fixed) / (stageA + stageB));
     if (stages > p.kps) stages = p.kps;
     if (stages > 16) stages = 16;
-    if (stages < 1) return false;
     pipe = stages * (stageA + stageB);
   }
   p.stages = stages;
@@ -694,7 +735,13 @@ static bool plan_gemm(GemmParams &p, size_t *smem_out) {
   p.tmem_cols = cols;
   // the staged epilogue reuses the pipeline buffers for a [BT][128] fp32 tile
   if (p.splits > 1 || p.stats_out) pipe = std::max<size_t>(pipe, 512 * static_cast<size_t>(p.BT));
-  const size_t smem = 1024 + pipe + (2 * stages + 1) * 8 + 32 + 16 + red;
+  size_t smem = 1024 + pipe + (2 * stages + 1) * 8 + 32 + 16 + red;
+  // A CTA blocks in tcgen05.alloc while co-resident CTAs hold the SM's 512
+  // TMEM columns; CTAs of one cluster wait for each other, so no more CTAs
+  // may fit on an SM (by shared memory) than can hold TMEM at once.
+  const int tmem_ctas = 512 / static_cast<int>(cols);
+  if (tmem_ctas < 4)  // registers already cap residency at 4 CTAs of 128 threads
+    smem = std::max<size_t>(smem, kSmemPerSM / (tmem_ctas + 1) + 1);
   if (smem > 227 * 1024) return false;
   p.pipe_bytes = static_cast<int>(pipe);
   *smem_out = smem;

@@ -28,6 +28,9 @@ GEMM_CASES = [
     # (M, N, K): split-K and single-split shapes, ragged N and M tails, several token tiles
     (1, 1280, 1280), (9, 1280, 1280), (9, 3840, 1280), (17, 5120, 1280), (9, 1280, 5120),
     (9, 1280, 6400), (144, 2560, 1280), (300, 1000, 128), (9, 51866, 1280), (1500, 2560, 1280),
+    # token tiles of 48 and 64 rows (split-K rows pushed to their owner CTA)
+    # and just past them (rows reduced by pulling partials), 16 and 10 splits
+    (40, 1280, 5120), (64, 1280, 5120), (65, 1280, 5120), (64, 1280, 1280), (97, 1280, 1280),
 ]
 
 
@@ -60,7 +63,7 @@ def test_gemm_rows_do_not_depend_on_batch():
     x = syn.normal_bf16(21, "xb", (300, K), 1.0)
     w = _dev(syn.normal_bf16(22, "wb", (N, K), 0.02))
     outs = {}
-    for M in (1, 9, 300):
+    for M in (1, 9, 64, 65, 300):
         y = torch.empty(M, N, dtype=torch.float32, device="cuda")
         nb = B.wf_gemm_scratch_bytes(M, N, K)
         sc = torch.empty(max(nb, 256), dtype=torch.uint8, device="cuda")
@@ -68,6 +71,8 @@ def test_gemm_rows_do_not_depend_on_batch():
         outs[M] = y.cpu().numpy()
     np.testing.assert_array_equal(outs[1][0], outs[300][0])
     np.testing.assert_array_equal(outs[9], outs[300][:9])
+    np.testing.assert_array_equal(outs[64], outs[300][:64])
+    np.testing.assert_array_equal(outs[65], outs[300][:65])
 
 
 def _cache(n_slots, H, ctx, seed, name, std=1.0):
