@@ -7,7 +7,7 @@
 // 128 weight rows fill the MMA's M side, the token tile (a multiple of 16,
 // <= 256) its N side.  Weight and token tiles stream into shared memory by
 // TMA (128-byte swizzle) through an mbarrier ring; one thread issues
-// tcgen05.mma into a TMEM accumulator; four warps read it back with
+// tcgen05.mma into a TMEM accumulator; eight warps read it back with
 // tcgen05.ld for a fused epilogue (bias, GELU, residual add, taps, key/value
 // cache scatter, or the output-head reduction).
 //
@@ -35,11 +35,13 @@
 namespace wf {
 
 constexpr int kBlockN = 128;   // weight rows per tile (MMA M)
+constexpr int kThreads = 256;  // 8 warps: two per TMEM lane quarter
 constexpr int kBlockK = 64;    // K per pipeline stage (one 128-byte swizzle atom)
 constexpr int kStageA = kBlockN * kBlockK * 2;  // 16 KB
 constexpr int kSmemBudget = 200 * 1024;
 constexpr int kSmemBudgetLn = 220 * 1024;  // LN mode: resident token tiles + weight ring
 constexpr size_t kSmemPerSM = 228 * 1024;  // shared memory of one SM
+constexpr int kLnFuseMaxM = 256;              // token rows up to which LN is fused
 
 struct __align__(16) RedEntry {
   float m, s, gm;
@@ -196,7 +198,7 @@ __device__ __forceinline__ void ln_build_operand(const GemmParams &p, uint8_t *s
   auto load = [&](int c0) {
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const int c = c0 + u * 128 + static_cast<int>(threadIdx.x);
+      const int c = c0 + u * kThreads + static_cast<int>(threadIdx.x);
       xa[u] = xb[u] = make_float4(0.f, 0.f, 0.f, 0.f);
       gv[u] = bv[u] = make_uint4(0u, 0u, 0u, 0u);
       if (c < total) {
@@ -221,11 +223,11 @@ __device__ __forceinline__ void ln_build_operand(const GemmParams &p, uint8_t *s
                       : make_float2(0.f, 0.f);
   }
   __syncthreads();
-  for (int c0 = 0; c0 < total; c0 += U * 128) {
+  for (int c0 = 0; c0 < total; c0 += U * kThreads) {
     if (c0) load(c0);
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const int c = c0 + u * 128 + static_cast<int>(threadIdx.x);
+      const int c = c0 + u * kThreads + static_cast<int>(threadIdx.x);
       if (c >= total) continue;
       const int i = c / per_stage, rem = c - i * per_stage, r = rem >> 3, j = rem & 7;
       uint4 o = make_uint4(0u, 0u, 0u, 0u);
@@ -248,7 +250,7 @@ __device__ __forceinline__ void ln_build_operand(const GemmParams &p, uint8_t *s
 }
 
 template <int EPI>
-__global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW,
+__global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW,
                                                       const __grid_constant__ CUtensorMap tmX,
                                                       const GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -400,14 +402,19 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
   const bool ok = mbar_wait(done, 0, p.err);
   tc_fence_after();
   __syncwarp();
-  const int n = n0 + warp * 32 + lane;
-  const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+  // warp w reads TMEM lane quarter w % 4 (weight rows 32 (w % 4) ..) and the
+  // token-column chunks [c_lo, c_hi) of its half of the tile
+  const int quarter = warp & 3, half = warp >> 2;
+  const int n = n0 + quarter * 32 + lane;
+  const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+  const int n_chunks = BT / 16, c_per = (n_chunks + 1) / 2;
+  const int c_lo = half * c_per, c_hi = min(n_chunks, c_lo + c_per);
 
   if constexpr (EPI == EPI_HEAD) {
     const bool sampling = p.temperature > 0.f;
     const int n_tiles = gridDim.y;
     const bool masked = n >= p.N || (p.suppress && p.suppress[n]);
-    for (int c = 0; c < BT / 16; ++c) {
+    for (int c = c_lo; c < c_hi; ++c) {
       float v[16];
       tmem_ld16(trow + c * 16, v);
 #pragma unroll
@@ -441,7 +448,7 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
           e.gm = gm;
           e.arg = arg;
           e.garg = garg;
-          red[warp * BT + c * 16 + jj] = e;
+          red[quarter * BT + c * 16 + jj] = e;
         }
       }
     }
@@ -465,7 +472,7 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
     }
   } else if (p.splits == 1 && !p.stats_out) {
     const float bn = (p.bias && n < p.N) ? bf2f(p.bias[n]) : 0.f;
-    for (int c = 0; c < BT / 16; ++c) {
+    for (int c = c_lo; c < c_hi; ++c) {
       float v[16];
       tmem_ld16(trow + c * 16, v);
       if (ok) epi_chunk<EPI>(p, t0 + c * 16, n, bn, v, tok + c * 16);
@@ -491,13 +498,13 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
           p.stats_out[static_cast<size_t>(t0 + tl) * stat_tiles + ntile] = make_float2(mean, m2);
       }
     };
-    const int r = warp * 32 + lane;
+    const int r = quarter * 32 + lane;
     // Every CTA stages its fp32 tile [BT][128] in its own shared memory (the
     // pipeline buffers are free once the MMAs completed); with split-K the S
     // CTAs of the tile form a cluster and each reduces its share of the token
     // rows by reading the S partials over DSMEM.
     float *tile = reinterpret_cast<float *>(smem);
-    for (int c = 0; c < BT / 16; ++c) {
+    for (int c = c_lo; c < c_hi; ++c) {
       float v[16];
       tmem_ld16(trow + c * 16, v);
 #pragma unroll
@@ -525,20 +532,21 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
       }
       return acc;
     };
-    if (S > 1 && rhi - rlo <= 8) {
+    constexpr int W = kThreads / 32;
+    if (S > 1 && rhi - rlo <= 2 * W) {
       // at most two rows per warp: read every partial first, tell the peers
       // their tiles are free, then run the epilogue while they finish
       float4 acc[2];
 #pragma unroll
       for (int k = 0; k < 2; ++k)
-        if (rlo + warp + 4 * k < rhi) acc[k] = reduce_row(rlo + warp + 4 * k);
+        if (rlo + warp + W * k < rhi) acc[k] = reduce_row(rlo + warp + W * k);
       cluster_arrive();
 #pragma unroll
       for (int k = 0; k < 2; ++k)
-        if (rlo + warp + 4 * k < rhi) finish_row(rlo + warp + 4 * k, acc[k], ok);
+        if (rlo + warp + W * k < rhi) finish_row(rlo + warp + W * k, acc[k], ok);
       cluster_wait();
     } else {
-      for (int tl = rlo + warp; tl < rhi; tl += 4) finish_row(tl, reduce_row(tl), ok);
+      for (int tl = rlo + warp; tl < rhi; tl += W) finish_row(tl, reduce_row(tl), ok);
       if (S > 1) cluster_sync();
     }
   }
@@ -620,7 +628,7 @@ static cudaError_t cluster_fits(int splits, size_t smem, dim3 grid) {
   if (it == seen.end()) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
-    cfg.blockDim = dim3(128, 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = smem;
     cudaLaunchAttribute attr;
     attr.id = cudaLaunchAttributeClusterDimension;
@@ -647,7 +655,7 @@ static cudaError_t launch_typed(const CUtensorMap *tw, const CUtensorMap *tx, co
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
-  cfg.blockDim = dim3(128, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
@@ -740,7 +748,7 @@ static bool plan_gemm(GemmParams &p, size_t *smem_out) {
   // TMEM columns; CTAs of one cluster wait for each other, so no more CTAs
   // may fit on an SM (by shared memory) than can hold TMEM at once.
   const int tmem_ctas = 512 / static_cast<int>(cols);
-  if (tmem_ctas < 4)  // registers already cap residency at 4 CTAs of 128 threads
+  if (tmem_ctas < 4)
     smem = std::max<size_t>(smem, kSmemPerSM / (tmem_ctas + 1) + 1);
   if (smem > 227 * 1024) return false;
   p.pipe_bytes = static_cast<int>(pipe);
@@ -749,6 +757,9 @@ static bool plan_gemm(GemmParams &p, size_t *smem_out) {
 }
 
 bool gemm_ln_fits(int M, int N, int K, int epi) {
+  // Every weight tile of the projection normalises the same token rows again;
+  // past one token tile that repeated work outweighs the launch it saves.
+  if (M > kLnFuseMaxM) return false;
   GemmParams p = {};
   p.M = M;
   p.N = N;

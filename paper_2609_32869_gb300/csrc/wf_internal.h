@@ -93,8 +93,9 @@ cudaError_t gemm_init();
 // Launch one GEMM.  W is [N, K] bf16, X is [M, K] bf16 (row stride K), or
 // X is null and the token operand is LN(p.ln_x) built inside the kernel.
 cudaError_t launch_gemm(const void *X, const void *W, GemmParams p, cudaStream_t s, bool pdl);
-// Whether the LayerNorm-fused form of a launch fits in shared memory (all of
-// the CTA's token tiles resident); otherwise run launch_layernorm first.
+// Whether to use the LayerNorm-fused form of a launch: one token tile, and
+// all of the CTA's token tiles fit in shared memory; otherwise run
+// launch_layernorm first (same bits either way).
 bool gemm_ln_fits(int M, int N, int K, int epi);
 
 // ------------------------------------------------------------- attention --
