@@ -60,6 +60,14 @@ WORKLOADS = {
 }
 
 
+# DRAM bytes (read + write) per projection launch, averaged over one step's
+# launch mix, from ncu captures of the depth-reduced profiling cases with the
+# same per-layer shapes (profiles/dram_per_kernel_large_b1_4l.md and
+# profiles/dram_per_kernel_large_b96_2l.md); None where no capture covers the
+# workload's shapes.
+GEMM_DRAM_BYTES_PER_LAUNCH = {"large_b1": 7.825e6, "large_b96": 13.16e6}
+
+
 def _peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -312,14 +320,16 @@ def run_ours(args, rank, world):
            "dev_in": torch.empty((Bn, Kc), dtype=torch.int32, device="cuda"),
            "out_tok": torch.empty((Bn, Kc + 1), dtype=torch.int32).pin_memory(),
            "out_cnt": torch.empty((Bn,), dtype=torch.int32).pin_memory()}
-    pl2 = make_plan(args.steps)
+    # the same steps as the device-timed region, after the same warm-up
+    pl2 = make_plan(n_steps)
     restart_job()
+    execute(pl2, 0, args.warmup)
     torch.cuda.synchronize()
     w0 = time.perf_counter()
-    execute(pl2, 0, args.steps, e2e=True, pin=pin)
+    execute(pl2, args.warmup, n_steps, e2e=True, pin=pin)
     torch.cuda.synchronize()
     e2e_s = time.perf_counter() - w0
-    e2e_tokens = sum(pl2["toks"])
+    e2e_tokens = sum(pl2["toks"][args.warmup:])
 
     # ---- per-family kernel time with CUDA events (roofline of the top kernel)
     n_prof = min(args.steps, 5)
@@ -383,7 +393,8 @@ def run_ours(args, rank, world):
                           "peak_source": f"{peak_src} (MEASURED_PEAKS hbm_gbs)"},
         "roofline": {"kernel": "gemm_tc_kernel (tcgen05 projections)", "bound": "hbm",
                      "achieved": gemm_gbs, "peak": hbm_peak, "unit": "GB/s",
-                     "frac": gemm_gbs / hbm_peak if gemm_gbs else None, "traffic": None,
+                     "frac": gemm_gbs / hbm_peak if gemm_gbs else None,
+                     "traffic": GEMM_DRAM_BYTES_PER_LAUNCH.get(args.workload),
                      "peak_source": peak_src,
                      "measured": f"CUDA events around each launch over {n_prof} profiled steps",
                      "share_of_kernel_time": fam_ms / step_total_prof if step_total_prof else None},
