@@ -32,15 +32,25 @@ constexpr int kQG = kAttnQGroup;      // 16 query rows per CTA
 constexpr int kPartStride = 2 + 64;   // m, l, o[64]
 constexpr int kSmemK = kKB * 128;     // bytes
 constexpr int kSmemQ = kQG * 128;
-constexpr int kSmemAttn = 2 * kSmemK + kSmemQ + 4 * kQG * (2 + 64) * 4 + 16;
+// K, V, Q, then the warps' (m, l); the warps' O partials reuse the K tile
+constexpr int kSmemAttn = 2 * kSmemK + kSmemQ + 4 * kQG * 2 * 4 + 16;
+static_assert(4 * kQG * 64 * 4 <= kSmemK, "O partials must fit in the key tile");
+// A launch with fewer CTAs than SMs asks for enough shared memory that no two
+// of its CTAs share an SM (it runs beside the neighbouring kernels' CTAs
+// under programmatic dependent launch); a larger one packs three per SM.
+constexpr int kSmemAttnSpread = 116 * 1024;
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, bool valid) {
   const int n = valid ? 16 : 0;  // zero-fill when the source row is past the cache
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(n)
                : "memory");
 }
-__device__ __forceinline__ void cp_async_wait_all() {
-  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
                                         uint32_t &r3) {
@@ -78,7 +88,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
   uint8_t *sQ = smem + 2 * kSmemK;
   float *sm = reinterpret_cast<float *>(smem + 2 * kSmemK + kSmemQ);  // [4][16]
   float *sl = sm + 4 * kQG;                                          // [4][16]
-  float *so = sl + 4 * kQG;                                          // [4][16][64]
+  float *so = reinterpret_cast<float *>(sK);  // [4][16][64], after every warp is done with K
   __shared__ int s_last;
 
   const int blk = blockIdx.x;
@@ -132,12 +142,23 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
       const bool valid = pos < n_keys;
       const size_t off = (cache_off + (valid ? pos : 0)) * 64 + ch * 8;
       cp_async16(k_u32 + swz(kr, ch), p.kc + off, valid);
+    }
+    cp_async_commit();
+#pragma unroll 4
+    for (int idx = tid; idx < kKB * 8; idx += 128) {
+      const int kr = idx >> 3, ch = idx & 7;
+      const int pos = key0 + kr;
+      if (pos >= fresh && pos < n_keys) continue;
+      const bool valid = pos < n_keys;
+      const size_t off = (cache_off + (valid ? pos : 0)) * 64 + ch * 8;
       cp_async16(v_u32 + swz(kr, ch), p.vc + off, valid);
     }
+    cp_async_commit();
   }
   pdl_wait();
   pdl_launch_dependents();
-  if (fresh < n_keys && key0 + kKB > fresh) {
+  const bool has_fresh = fresh < n_keys && key0 + kKB > fresh;
+  if (has_fresh) {
     const uint32_t k_u32 = smem_u32(sK), v_u32 = smem_u32(sV);
     for (int idx = tid; idx < kKB * 8; idx += 128) {
       const int kr = idx >> 3, ch = idx & 7;
@@ -147,6 +168,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
       cp_async16(k_u32 + swz(kr, ch), p.kc + off, true);
       cp_async16(v_u32 + swz(kr, ch), p.vc + off, true);
     }
+    cp_async_commit();
   }
   // ---- queries, pre-scaled by 1/8 = 1/sqrt(64) (exact in binary), RoPE in fp32
   {
@@ -178,7 +200,10 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
     o.w = pack_bf16(f[6], f[7]);
     *reinterpret_cast<uint4 *>(sQ + swz(r, ch)) = o;
   }
-  cp_async_wait_all();
+  // keys (and this step's rows) first; the acoustic values keep streaming
+  // while the scores are formed
+  if (has_fresh) cp_async_wait<0>();
+  else cp_async_wait<1>();
   __syncthreads();
 
   // ---- RoPE on the keys (drafter): dims i and i+32 rotate by pos * base^(-2i/64)
@@ -263,6 +288,10 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
     lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 1);
     lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 2);
   }
+  if (!has_fresh) {
+    cp_async_wait<0>();  // the values
+    __syncthreads();
+  }
   // O = P V (P rounded to bf16 as the A operand)
   float o[8][4];
 #pragma unroll
@@ -283,6 +312,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
       mma_bf16(o[2 * dp + 1], a0, a1, a2, a3, b2, b3);
     }
   }
+  __syncthreads();  // every warp is done with the key tile, which now holds O
   // stage this warp's (m, l, O) for the in-order combine
   if (c4 == 0) {
     sm[warp * kQG + g] = mrow[0];
@@ -412,7 +442,7 @@ cudaError_t attention_init() {
   static std::once_flag once;
   std::call_once(once, [] {
     status = cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  kSmemAttn);
+                                  kSmemAttnSpread);
   });
   return status;
 }
@@ -424,7 +454,15 @@ cudaError_t launch_attention(const AttnParams &p0, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.n_chunks, p.n_heads * p.qgroups, p.n_seq);
   cfg.blockDim = dim3(128, 1, 1);
-  cfg.dynamicSmemBytes = kSmemAttn;
+  static const int n_sm = [] {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return 0;
+    return n;
+  }();
+  const long long ctas = static_cast<long long>(cfg.gridDim.x) * cfg.gridDim.y * cfg.gridDim.z;
+  cfg.dynamicSmemBytes = ctas <= n_sm ? kSmemAttnSpread : kSmemAttn;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
