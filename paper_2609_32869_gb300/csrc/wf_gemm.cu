@@ -43,11 +43,6 @@ constexpr int kSmemBudgetLn = 220 * 1024;  // LN mode: resident token tiles + we
 constexpr size_t kSmemPerSM = 228 * 1024;  // shared memory of one SM
 constexpr int kLnFuseMaxM = 256;              // token rows up to which LN is fused
 
-struct __align__(16) RedEntry {
-  float m, s, gm;
-  int arg, garg;
-};
-
 __device__ __forceinline__ void head_combine(float &m, float &s, int &arg, float &gm, int &garg,
                                              float m2, float s2, int arg2, float gm2, int garg2) {
   const float M = fmaxf(m, m2);
@@ -264,10 +259,8 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
   uint64_t *empty = full + stages;
   uint64_t *done = empty + stages;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
-  RedEntry *red = reinterpret_cast<RedEntry *>(smem + p.pipe_bytes + (2 * stages + 1) * 8 + 16 + 16);
-  red = reinterpret_cast<RedEntry *>((reinterpret_cast<uintptr_t>(red) + 15) & ~uintptr_t(15));
   // per-token (slot, position) for EPI_KV, (slot, step) for sampling heads
-  int2 *tok = reinterpret_cast<int2 *>(red + (EPI == EPI_HEAD ? 4 * BT : 0));
+  int2 *tok = reinterpret_cast<int2 *>(smem + p.pipe_bytes + (2 * stages + 1) * 8 + 16 + 16);
   float2 *lnst = reinterpret_cast<float2 *>(tok + BT);  // per-token (mean, rstd), LN mode
   const bool ln = p.ln_x != nullptr;
 
@@ -411,64 +404,62 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
   const int c_lo = half * c_per, c_hi = min(n_chunks, c_lo + c_per);
 
   if constexpr (EPI == EPI_HEAD) {
+    // Stage the [BT][128] logit tile in shared memory (the pipeline buffers
+    // are free once the MMAs completed); then a warp owns a token row, lane l
+    // folds features 4l..4l+3 in order and the warp combines its lanes:
+    // running max with the lowest id on ties, sum of exp(x - max), and the
+    // Gumbel-max draw.  One record per (row, vocabulary tile).
     const bool sampling = p.temperature > 0.f;
     const int n_tiles = gridDim.y;
-    const bool masked = n >= p.N || (p.suppress && p.suppress[n]);
+    float *tile = reinterpret_cast<float *>(smem);
+    const int r = quarter * 32 + lane;
     for (int c = c_lo; c < c_hi; ++c) {
       float v[16];
       tmem_ld16(trow + c * 16, v);
 #pragma unroll
-      for (int jj = 0; jj < 16; ++jj) {
-        const int t = t0 + c * 16 + jj;
-        float z = v[jj];
-        if (ok && p.logits && t < p.M && n < p.N)
-          p.logits[static_cast<size_t>(t) * p.N + n] = z;
-        float x = masked ? -INFINITY : (sampling ? __fdiv_rn(z, p.temperature) : z);
-        float m = x, s = masked ? 0.f : 1.f, gm = -INFINITY;
-        int arg = n, garg = n;
-        if (sampling && !masked && t < p.M) {
-          const int j = t % p.rows_per_seq;
-          const int2 ss = tok[c * 16 + jj];
-          gm = x + gumbel(p.seed, static_cast<uint32_t>(ss.x), static_cast<uint32_t>(ss.y),
-                          static_cast<uint32_t>(j), p.tag, static_cast<uint32_t>(n));
-        }
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) {
-          const float m2 = __shfl_down_sync(0xffffffffu, m, off);
-          const float s2 = __shfl_down_sync(0xffffffffu, s, off);
-          const float gm2 = __shfl_down_sync(0xffffffffu, gm, off);
-          const int a2 = __shfl_down_sync(0xffffffffu, arg, off);
-          const int ga2 = __shfl_down_sync(0xffffffffu, garg, off);
-          head_combine(m, s, arg, gm, garg, m2, s2, a2, gm2, ga2);
-        }
-        if (lane == 0) {
-          RedEntry e;
-          e.m = m;
-          e.s = s;
-          e.gm = gm;
-          e.arg = arg;
-          e.garg = garg;
-          red[quarter * BT + c * 16 + jj] = e;
-        }
-      }
+      for (int jj = 0; jj < 16; ++jj) tile[(c * 16 + jj) * kBlockN + r] = v[jj];
     }
     __syncthreads();
-    for (int col = threadIdx.x; col < BT; col += blockDim.x) {
-      const int t = t0 + col;
-      if (t >= p.M) continue;
-      RedEntry e = red[col];
-      for (int w = 1; w < 4; ++w) {
-        const RedEntry f = red[w * BT + col];
-        head_combine(e.m, e.s, e.arg, e.gm, e.garg, f.m, f.s, f.arg, f.gm, f.garg);
+    constexpr int W = kThreads / 32;
+    for (int tl = warp; tl < cols; tl += W) {
+      const int t = t0 + tl;
+      const float4 z4 = *reinterpret_cast<const float4 *>(tile + tl * kBlockN + 4 * lane);
+      const float z[4] = {z4.x, z4.y, z4.z, z4.w};
+      const int2 ss = sampling ? tok[tl] : make_int2(0, 0);
+      const int j = t % p.rows_per_seq;
+      float m = -INFINITY, sum = 0.f, gm = -INFINITY;
+      int arg = 0x7fffffff, garg = 0x7fffffff;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int nn = n0 + 4 * lane + i;
+        const bool masked = nn >= p.N || (p.suppress && p.suppress[nn]);
+        if (ok && p.logits && nn < p.N) p.logits[static_cast<size_t>(t) * p.N + nn] = z[i];
+        const float x = masked ? -INFINITY : (sampling ? __fdiv_rn(z[i], p.temperature) : z[i]);
+        float g = -INFINITY;
+        if (sampling && !masked)
+          g = x + gumbel(p.seed, static_cast<uint32_t>(ss.x), static_cast<uint32_t>(ss.y),
+                         static_cast<uint32_t>(j), p.tag, static_cast<uint32_t>(nn));
+        head_combine(m, sum, arg, gm, garg, x, masked ? 0.f : 1.f, nn, g, nn);
       }
-      HeadRec r;
-      r.m = e.m;
-      r.s = e.s;
-      r.gm = e.gm;
-      r.arg = e.arg;
-      r.garg = e.garg;
-      r._pad[0] = r._pad[1] = r._pad[2] = 0;
-      p.recs[static_cast<size_t>(t) * n_tiles + ntile] = r;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        const float m2 = __shfl_down_sync(0xffffffffu, m, off);
+        const float s2 = __shfl_down_sync(0xffffffffu, sum, off);
+        const float gm2 = __shfl_down_sync(0xffffffffu, gm, off);
+        const int a2 = __shfl_down_sync(0xffffffffu, arg, off);
+        const int ga2 = __shfl_down_sync(0xffffffffu, garg, off);
+        head_combine(m, sum, arg, gm, garg, m2, s2, a2, gm2, ga2);
+      }
+      if (lane == 0 && ok) {
+        HeadRec rec;
+        rec.m = m;
+        rec.s = sum;
+        rec.gm = gm;
+        rec.arg = arg;
+        rec.garg = garg;
+        rec._pad[0] = rec._pad[1] = rec._pad[2] = 0;
+        p.recs[static_cast<size_t>(t) * n_tiles + ntile] = rec;
+      }
     }
   } else if (p.splits == 1 && !p.stats_out) {
     const float bn = (p.bias && n < p.N) ? bf2f(p.bias[n]) : 0.f;
@@ -717,8 +708,7 @@ static bool plan_gemm(GemmParams &p, size_t *smem_out) {
   p.kps = k_iters / p.splits;
   const bool ln = p.ln_x != nullptr;
   const size_t stageA = kStageA, stageB = static_cast<size_t>(p.BT) * kBlockK * 2;
-  const size_t red = (p.epi == EPI_HEAD ? 4 * static_cast<size_t>(p.BT) * sizeof(RedEntry) : 0) +
-                     static_cast<size_t>(p.BT) * sizeof(int2) * (ln ? 2 : 1);
+  const size_t red = static_cast<size_t>(p.BT) * sizeof(int2) * (ln ? 2 : 1);
   const size_t fixed = red;
   int stages;
   size_t pipe;
@@ -741,8 +731,9 @@ static bool plan_gemm(GemmParams &p, size_t *smem_out) {
   uint32_t cols = 32;
   while (cols < static_cast<uint32_t>(p.BT)) cols <<= 1;
   p.tmem_cols = cols;
-  // the staged epilogue reuses the pipeline buffers for a [BT][128] fp32 tile
-  if (p.splits > 1 || p.stats_out) pipe = std::max<size_t>(pipe, 512 * static_cast<size_t>(p.BT));
+  // the staged epilogues reuse the pipeline buffers for a [BT][128] fp32 tile
+  if (p.splits > 1 || p.stats_out || p.epi == EPI_HEAD)
+    pipe = std::max<size_t>(pipe, 512 * static_cast<size_t>(p.BT));
   size_t smem = 1024 + pipe + (2 * stages + 1) * 8 + 32 + 16 + red;
   // A CTA blocks in tcgen05.alloc while co-resident CTAs hold the SM's 512
   // TMEM columns; CTAs of one cluster wait for each other, so no more CTAs
