@@ -12,8 +12,8 @@
 //
 // A CTA takes one (sequence, head, group of <= 16 query rows, block of 256
 // keys).  Keys and values stream into XOR-swizzled shared memory with
-// cp.async (rows past the cache length are zero-filled); each of the four
-// warps multiplies the 16 query rows against its 64 keys on the tensor cores
+// cp.async (rows past the cache length are zero-filled); each of the eight
+// warps multiplies the 16 query rows against its 32 keys on the tensor cores
 // (mma.sync m16n8k16, bf16 in, fp32 accumulate), keeps the row maxima and
 // sums in fp32 and forms P V the same way.  Warps combine in order, and the
 // blocks of a (sequence, head, group) are combined by the last CTA in block
@@ -27,14 +27,21 @@
 
 namespace wf {
 
-constexpr int kKB = kAttnKeysPerCTA;  // 256 keys per CTA, 64 per warp
+constexpr int kKB = kAttnKeysPerCTA;  // 256 keys per CTA
 constexpr int kQG = kAttnQGroup;      // 16 query rows per CTA
+constexpr int kWarps = 8;             // each takes kKW consecutive keys of the block
+constexpr int kThreadsA = 32 * kWarps;
+constexpr int kKW = kKB / kWarps;     // 32 keys per warp
+constexpr int kNT = kKW / 8;          // 8-key score tiles per warp
+constexpr int kKS = kKW / 16;         // 16-key steps per warp
+constexpr int kDPT = kQG * 64 / kThreadsA;  // output dims per thread in the combine
 constexpr int kPartStride = 2 + 64;   // m, l, o[64]
 constexpr int kSmemK = kKB * 128;     // bytes
 constexpr int kSmemQ = kQG * 128;
 // K, V, Q, then the warps' (m, l); the warps' O partials reuse the K tile
-constexpr int kSmemAttn = 2 * kSmemK + kSmemQ + 4 * kQG * 2 * 4 + 16;
-static_assert(4 * kQG * 64 * 4 <= kSmemK, "O partials must fit in the key tile");
+constexpr int kSmemAttn = 2 * kSmemK + kSmemQ + kWarps * kQG * 2 * 4 + 16;
+static_assert(kWarps * kQG * 64 * 4 <= kSmemK, "O partials must fit in the key tile");
+static_assert(kQG * 8 <= kThreadsA && kDPT * kThreadsA == kQG * 64, "thread mapping");
 // A launch with fewer CTAs than SMs asks for enough shared memory that no two
 // of its CTAs share an SM (it runs beside the neighbouring kernels' CTAs
 // under programmatic dependent launch); a larger one packs three per SM.
@@ -76,19 +83,31 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<const uint32_t *>(&v);
 }
+// kDPT consecutive output dims (scaled by inv) as bf16
+__device__ __forceinline__ void store_row(bf16 *orow, const float (&v)[kDPT], float inv) {
+  uint32_t w[kDPT / 2];
+#pragma unroll
+  for (int e = 0; e < kDPT / 2; ++e) w[e] = pack_bf16(v[2 * e] * inv, v[2 * e + 1] * inv);
+  if constexpr (kDPT == 8) {
+    *reinterpret_cast<uint4 *>(orow) = make_uint4(w[0], w[1], w[2], w[3]);
+  } else {
+    static_assert(kDPT == 4, "combine width");
+    *reinterpret_cast<uint2 *>(orow) = make_uint2(w[0], w[1]);
+  }
+}
 // byte offset of 16-byte chunk `ch` of row `row` in a [rows][64] bf16 tile
 __device__ __forceinline__ uint32_t swz(int row, int ch) {
   return static_cast<uint32_t>(row * 128 + ((ch ^ (row & 7)) << 4));
 }
 
-__global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
+__global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p) {
   extern __shared__ __align__(128) uint8_t smem[];
   uint8_t *sK = smem;
   uint8_t *sV = smem + kSmemK;
   uint8_t *sQ = smem + 2 * kSmemK;
-  float *sm = reinterpret_cast<float *>(smem + 2 * kSmemK + kSmemQ);  // [4][16]
-  float *sl = sm + 4 * kQG;                                          // [4][16]
-  float *so = reinterpret_cast<float *>(sK);  // [4][16][64], after every warp is done with K
+  float *sm = reinterpret_cast<float *>(smem + 2 * kSmemK + kSmemQ);  // [kWarps][16]
+  float *sl = sm + kWarps * kQG;                                     // [kWarps][16]
+  float *so = reinterpret_cast<float *>(sK);  // [kWarps][16][64], once every warp is done with K
   __shared__ int s_last;
 
   const int blk = blockIdx.x;
@@ -135,7 +154,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
   {
     const uint32_t k_u32 = smem_u32(sK), v_u32 = smem_u32(sV);
 #pragma unroll 4
-    for (int idx = tid; idx < kKB * 8; idx += 128) {
+    for (int idx = tid; idx < kKB * 8; idx += kThreadsA) {
       const int kr = idx >> 3, ch = idx & 7;
       const int pos = key0 + kr;
       if (pos >= fresh && pos < n_keys) continue;
@@ -145,7 +164,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
     }
     cp_async_commit();
 #pragma unroll 4
-    for (int idx = tid; idx < kKB * 8; idx += 128) {
+    for (int idx = tid; idx < kKB * 8; idx += kThreadsA) {
       const int kr = idx >> 3, ch = idx & 7;
       const int pos = key0 + kr;
       if (pos >= fresh && pos < n_keys) continue;
@@ -160,7 +179,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
   const bool has_fresh = fresh < n_keys && key0 + kKB > fresh;
   if (has_fresh) {
     const uint32_t k_u32 = smem_u32(sK), v_u32 = smem_u32(sV);
-    for (int idx = tid; idx < kKB * 8; idx += 128) {
+    for (int idx = tid; idx < kKB * 8; idx += kThreadsA) {
       const int kr = idx >> 3, ch = idx & 7;
       const int pos = key0 + kr;
       if (pos < fresh || pos >= n_keys) continue;
@@ -171,7 +190,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
     cp_async_commit();
   }
   // ---- queries, pre-scaled by 1/8 = 1/sqrt(64) (exact in binary), RoPE in fp32
-  {
+  if (tid < kQG * 8) {
     const int r = tid >> 3, ch = tid & 7;
     uint4 raw = make_uint4(0, 0, 0, 0), par = make_uint4(0, 0, 0, 0);
     if (r < nq) {
@@ -208,7 +227,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
 
   // ---- RoPE on the keys (drafter): dims i and i+32 rotate by pos * base^(-2i/64)
   if (p.rope_tab) {
-    for (int idx = tid; idx < kKB * 4; idx += 128) {
+    for (int idx = tid; idx < kKB * 4; idx += kThreadsA) {
       const int kr = idx >> 2, c = idx & 3;  // chunk c (dims 8c..8c+7) pairs with chunk c+4
       const int pos = key0 + kr;
       if (pos >= n_keys) continue;
@@ -230,13 +249,13 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
     __syncthreads();
   }
 
-  // ---- per warp: 16 query rows x 64 keys on the tensor cores
+  // ---- per warp: 16 query rows x kKW keys on the tensor cores
   const int g = lane >> 2, c4 = lane & 3;
-  const int kw = warp * 64;  // first key of this warp within the block
+  const int kw = warp * kKW;  // first key of this warp within the block
   const uint32_t q_u32 = smem_u32(sQ), k_u32 = smem_u32(sK), v_u32 = smem_u32(sV);
-  float s[8][4];
+  float s[kNT][4];
 #pragma unroll
-  for (int nt = 0; nt < 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+  for (int nt = 0; nt < kNT; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
 #pragma unroll
   for (int ks = 0; ks < 4; ++ks) {
     uint32_t a0, a1, a2, a3;
@@ -245,7 +264,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
       ldsm_x4(q_u32 + swz((mi & 1) * 8 + (lane & 7), 2 * ks + (mi >> 1)), a0, a1, a2, a3);
     }
 #pragma unroll
-    for (int np = 0; np < 4; ++np) {
+    for (int np = 0; np < kKS; ++np) {
       uint32_t b0, b1, b2, b3;
       const int mi = lane >> 3;
       ldsm_x4(k_u32 + swz(kw + np * 16 + (mi >> 1) * 8 + (lane & 7), 2 * ks + (mi & 1)), b0, b1, b2,
@@ -257,7 +276,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
   // masks, row maxima and exponentials (rows g and g+8 of the group)
   float mrow[2] = {-INFINITY, -INFINITY};
 #pragma unroll
-  for (int nt = 0; nt < 8; ++nt) {
+  for (int nt = 0; nt < kNT; ++nt) {
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
       const int row = g + (e >> 1) * 8;
@@ -275,7 +294,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
   }
   float lrow[2] = {0.f, 0.f};
 #pragma unroll
-  for (int nt = 0; nt < 8; ++nt) {
+  for (int nt = 0; nt < kNT; ++nt) {
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
       const float v = s[nt][e] == -INFINITY ? 0.f : expf(s[nt][e] - mrow[e >> 1]);
@@ -297,7 +316,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
 #pragma unroll
   for (int nd = 0; nd < 8; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
 #pragma unroll
-  for (int kk = 0; kk < 4; ++kk) {
+  for (int kk = 0; kk < kKS; ++kk) {
     const uint32_t a0 = pack_bf16(s[2 * kk][0], s[2 * kk][1]);
     const uint32_t a1 = pack_bf16(s[2 * kk][2], s[2 * kk][3]);
     const uint32_t a2 = pack_bf16(s[2 * kk + 1][0], s[2 * kk + 1][1]);
@@ -331,33 +350,28 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
   }
   __syncthreads();
 
-  // ---- combine the four warps in order: thread -> (row qi, dims d0..d0+7)
-  const int qi = tid >> 3, d0 = (tid & 7) * 8;
+  // ---- combine the warps in order: thread -> (row qi, dims d0..d0+kDPT-1)
+  const int qi = tid / (64 / kDPT), d0 = (tid % (64 / kDPT)) * kDPT;
   float M = -INFINITY;
 #pragma unroll
-  for (int w = 0; w < 4; ++w) M = fmaxf(M, sm[w * kQG + qi]);
-  float L = 0.f, acc[8];
+  for (int w = 0; w < kWarps; ++w) M = fmaxf(M, sm[w * kQG + qi]);
+  float L = 0.f, acc[kDPT];
 #pragma unroll
-  for (int e = 0; e < 8; ++e) acc[e] = 0.f;
+  for (int e = 0; e < kDPT; ++e) acc[e] = 0.f;
 #pragma unroll
-  for (int w = 0; w < 4; ++w) {
+  for (int w = 0; w < kWarps; ++w) {
     const float mw = sm[w * kQG + qi];
     const float wt = (mw == -INFINITY) ? 0.f : expf(mw - M);
     L += sl[w * kQG + qi] * wt;
 #pragma unroll
-    for (int e = 0; e < 8; ++e) acc[e] += so[(w * kQG + qi) * 64 + d0 + e] * wt;
+    for (int e = 0; e < kDPT; ++e) acc[e] += so[(w * kQG + qi) * 64 + d0 + e] * wt;
   }
 
   if (n_blocks == 1) {
     if (qi < nq) {
       const float inv = 1.0f / L;
       bf16 *orow = p.out + static_cast<size_t>(i * p.rps + q0 + qi) * d_model + h * 64 + d0;
-      uint4 ov;
-      ov.x = pack_bf16(acc[0] * inv, acc[1] * inv);
-      ov.y = pack_bf16(acc[2] * inv, acc[3] * inv);
-      ov.z = pack_bf16(acc[4] * inv, acc[5] * inv);
-      ov.w = pack_bf16(acc[6] * inv, acc[7] * inv);
-      *reinterpret_cast<uint4 *>(orow) = ov;
+      store_row(orow, acc, inv);
     }
     return;
   }
@@ -372,7 +386,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
       pe[1] = L;
     }
 #pragma unroll
-    for (int e = 0; e < 8; ++e) pe[2 + d0 + e] = acc[e];
+    for (int e = 0; e < kDPT; ++e) pe[2 + d0 + e] = acc[e];
   }
   __threadfence();
   __syncthreads();
@@ -389,29 +403,24 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
     const float *pg = p.part + static_cast<size_t>(group_id) * p.n_chunks * kQG * kPartStride;
     float MM = -INFINITY;
     for (int u = 0; u < n_blocks; ++u) MM = fmaxf(MM, __ldcg(pg + (u * kQG + qi) * kPartStride));
-    float LL = 0.f, oo[8];
+    float LL = 0.f, oo[kDPT];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) oo[e] = 0.f;
+    for (int e = 0; e < kDPT; ++e) oo[e] = 0.f;
     for (int u = 0; u < n_blocks; ++u) {
       const float *pe = pg + (u * kQG + qi) * kPartStride;
       const float mc = __ldcg(pe);
       const float lc = __ldcg(pe + 1);
-      float ov[8];
+      float ov[kDPT];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) ov[e] = __ldcg(pe + 2 + d0 + e);
+      for (int e = 0; e < kDPT; ++e) ov[e] = __ldcg(pe + 2 + d0 + e);
       const float wt = (mc == -INFINITY) ? 0.f : expf(mc - MM);
       LL += lc * wt;
 #pragma unroll
-      for (int e = 0; e < 8; ++e) oo[e] += ov[e] * wt;
+      for (int e = 0; e < kDPT; ++e) oo[e] += ov[e] * wt;
     }
     const float inv = 1.0f / LL;
     bf16 *orow = p.out + static_cast<size_t>(i * p.rps + q0 + qi) * d_model + h * 64 + d0;
-    uint4 ov;
-    ov.x = pack_bf16(oo[0] * inv, oo[1] * inv);
-    ov.y = pack_bf16(oo[2] * inv, oo[3] * inv);
-    ov.z = pack_bf16(oo[4] * inv, oo[5] * inv);
-    ov.w = pack_bf16(oo[6] * inv, oo[7] * inv);
-    *reinterpret_cast<uint4 *>(orow) = ov;
+    store_row(orow, oo, inv);
   }
   if (tid == 0) p.counters[group_id] = 0;
 }
@@ -453,7 +462,7 @@ cudaError_t launch_attention(const AttnParams &p0, cudaStream_t s, bool pdl) {
   p.n_chunks = (p.ctx + kKB - 1) / kKB;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.n_chunks, p.n_heads * p.qgroups, p.n_seq);
-  cfg.blockDim = dim3(128, 1, 1);
+  cfg.blockDim = dim3(kThreadsA, 1, 1);
   static const int n_sm = [] {
     int dev = 0, n = 0;
     if (cudaGetDevice(&dev) != cudaSuccess ||
