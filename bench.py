@@ -48,6 +48,16 @@ WORKLOADS = {
     "tiny_b1": dict(cfg="TINY", batch=1, budget=(200, 200), accept="uniform",
                     text="Whisper-tiny-shaped decoder (d=384, 6 heads, FFN 1536, 4 layers, "
                          "vocab 51865), batch 1, accept length uniform 0..8"),
+    # Temperature sampling (App. A.4): the drafter draws its own proposals and
+    # the target applies the rejection rule with seeded Philox streams; no
+    # teacher forcing, so the accepted lengths are whatever the random weights
+    # give (reported in the line).
+    "large_b32_t07": dict(cfg="LARGE", batch=32, budget=(220, 220), temperature=0.7,
+                          text="large shapes, batch 32, temperature 0.7 speculative sampling "
+                               "(drafter's own proposals, rejection rule), 220-token budget"),
+    "large_b32_t10": dict(cfg="LARGE", batch=32, budget=(220, 220), temperature=1.0,
+                          text="large shapes, batch 32, temperature 1.0 speculative sampling "
+                               "(drafter's own proposals, rejection rule), 220-token budget"),
     # Depth-reduced cases for profiler captures: every kernel keeps the large
     # per-layer shapes and launch configuration; only the number of target
     # blocks shrinks so a capture holds a few GB and few launches.
@@ -415,6 +425,154 @@ def run_ours(args, rank, world):
     return result
 
 
+def run_sampling(args, rank, world):
+    """Speculative sampling steps: tokens/s from the counts the step itself
+    returns (written per step into a device array, read after the region)."""
+    import torch
+    import torch.distributed as dist
+    from paper_2609_32869_gb300 import binding as B
+    from paper_2609_32869_gb300.session import Session, upload_weights
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    wl = WORKLOADS[args.workload]
+    cfg = _cfg(wl["cfg"], wl.get("layers"))
+    Bn, Kc = wl["batch"], cfg.block_k
+    dev = upload_weights(syn.make_weights(cfg, seed=0))
+    enc = syn.encoder_output(cfg, Bn, seed=1)
+    prompt = syn.prompts(cfg, Bn, length=4, seed=1)
+    budgets = np.full(Bn, wl["budget"][0], np.int32)
+    sess = Session(cfg, dev, max_batch=Bn, max_ctx=cfg.max_pos)
+    stream = sess.stream
+    sp = B.sample_params(wl["temperature"], 4 + rank)
+    sess.prefill(np.arange(Bn, dtype=np.int32), enc, prompt, budgets, sp=sp)
+    n_steps = args.warmup + args.steps
+    counts = torch.zeros(n_steps, Bn, dtype=torch.int32, device="cuda")
+    toks = torch.zeros(n_steps, Bn, Kc + 1, dtype=torch.int32, device="cuda")
+
+    def run(lo, hi):
+        n = 0
+        for i in range(lo, hi):
+            B.wf_step(sess.h, sp, None, toks[i], counts[i], stream)
+            n += B.wf_last_launch_count(sess.h)
+        return n
+
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(local).uuid)
+        if uuid and not uuid.startswith("GPU-"):
+            uuid = "GPU-" + uuid
+    except Exception:
+        uuid = None
+    sampler, clock_path = _clock_sampler(uuid)
+    run(0, args.warmup)
+    torch.cuda.synchronize()
+    len0 = sess.state()["len"].astype(np.float64)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if args.profile_region:
+        torch.cuda.profiler.start()
+    e0.record(stream)
+    launches = run(args.warmup, n_steps)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if args.profile_region:
+        torch.cuda.profiler.stop()
+    if world > 1:
+        dist.barrier()
+    dev_ms = e0.elapsed_time(e1)
+    len1 = sess.state()["len"].astype(np.float64)
+    c = counts[args.warmup:].cpu().numpy()
+    tokens = float(c.sum())
+    live = c > 0
+    accepted = float((c[live] - 1).mean()) if live.any() else 0.0
+
+    # end to end: the same call with the step's outputs read back to pinned
+    # host memory every step (the step takes no per-step input)
+    h_tok = torch.empty((Bn, Kc + 1), dtype=torch.int32).pin_memory()
+    h_cnt = torch.empty((Bn,), dtype=torch.int32).pin_memory()
+    e2e_tokens = 0
+    torch.cuda.synchronize()
+    w0 = time.perf_counter()
+    for i in range(args.warmup, n_steps):
+        B.wf_step(sess.h, sp, None, toks[i], counts[i], stream)
+        h_tok.copy_(toks[i], non_blocking=True)
+        h_cnt.copy_(counts[i], non_blocking=True)
+        stream.synchronize()
+        e2e_tokens += int(h_cnt.sum())
+    e2e_s = time.perf_counter() - w0
+
+    n_prof = min(args.steps, 3)
+    B.wf_set_option(sess.h, B.WF_OPT_PROFILE, 1)
+    run(0, n_prof)
+    prof = B.wf_profile_read(sess.h, stream)
+    B.wf_set_option(sess.h, B.WF_OPT_PROFILE, 0)
+    if sampler is not None:
+        sampler.terminate()
+        sampler.wait()
+    clocks = _clock_summary(clock_path)
+    try:
+        os.unlink(clock_path)
+    except OSError:
+        pass
+
+    t_dev = torch.tensor([dev_ms, e2e_s], dtype=torch.float64, device="cuda")
+    t_tok = torch.tensor([tokens, e2e_tokens], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(t_dev, op=dist.ReduceOp.MAX)
+        dist.all_reduce(t_tok, op=dist.ReduceOp.SUM)
+    dev_ms, e2e_s = float(t_dev[0]), float(t_dev[1])
+    tokens, e2e_tokens = float(t_tok[0]), float(t_tok[1])
+    hbm_peak, _, peak_src = _peaks()
+    step_ms = dev_ms / args.steps
+    mean_len = list((len0 + len1) / 2.0)
+    wbytes, kvbytes = step_weight_kv_bytes(cfg, Bn, [int(x) for x in mean_len])
+    fam_ms = prof["gemm"]["ms"]
+    gemm_gbs = prof["gemm"]["bytes"] / (fam_ms * 1e-3) / 1e9 if fam_ms > 0 else None
+    return {
+        "metric": METRIC,
+        "value": tokens / (dev_ms * 1e-3),
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": step_ms,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded random weights and encoder outputs; the drafter's own "
+                "sampled proposals)",
+        "config": {"workload": args.workload, "description": wl["text"], "batch": Bn,
+                   "block": Kc + 1, "temperature": wl["temperature"],
+                   "parallelism": f"replicas x{world}",
+                   "l2": "inputs larger than L2 (every step streams "
+                         f"{(wbytes + kvbytes) / 1e9:.2f} GB of weights and K/V > 129 MB L2)"},
+        "step_us": step_ms * 1e3,
+        "tokens_per_step": tokens / args.steps / world,
+        "accepted_drafts_per_sequence_step": accepted,
+        "step_roofline": {"bytes": wbytes + kvbytes, "weights": wbytes, "kv": kvbytes,
+                          "achieved_gbs": (wbytes + kvbytes) / (step_ms * 1e-3) / 1e9,
+                          "peak_gbs": hbm_peak,
+                          "frac": (wbytes + kvbytes) / (step_ms * 1e-3) / 1e9 / hbm_peak,
+                          "peak_source": f"{peak_src} (MEASURED_PEAKS hbm_gbs)"},
+        "roofline": {"kernel": "gemm_tc_kernel (tcgen05 projections)", "bound": "hbm",
+                     "achieved": gemm_gbs, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": gemm_gbs / hbm_peak if gemm_gbs else None,
+                     "traffic": GEMM_DRAM_BYTES_PER_LAUNCH.get(args.workload),
+                     "peak_source": peak_src,
+                     "measured": f"CUDA events around each launch over {n_prof} profiled steps"},
+        "kernel_families_ms_per_step": {k: v["ms"] / n_prof for k, v in prof.items()},
+        "e2e": {"value": e2e_tokens / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": Bn * (Kc + 1) * 4 + Bn * 4},
+        "gpu_launches": launches,
+        "clocks": clocks,
+        "device_error": sess.error(),
+    }
+
+
 # ------------------------------------------------------------ CPU oracle ----
 def _oracle_setup(cfg, ws, enc, prompt, budgets):
     from oracle.decoder import WhisperFlashOracle
@@ -487,6 +645,27 @@ def cpu_baseline(cfg, ws, enc, prompt, budgets, acc, budget_s=15.0):
             "ms_per_step": secs / steps * 1e3}
 
 
+def _oracle_sampling_run(cfg, ws, enc, prompt, budget, T, n_warm, n_steps, time_cap_s):
+    """The oracle's own speculative sampling of sequence 0 (drafter proposals,
+    rejection rule) with the same Philox streams as the GPU run."""
+    o, encf = _oracle_setup(cfg, ws, enc, prompt, [budget])
+    seq = o.prefill(encf, prompt[0], budget, seq_id=0, temperature=T, seed=4)
+    tokens, secs, done_steps = 0, 0.0, 0
+    for i in range(n_warm + n_steps):
+        if seq.done:
+            break
+        t0 = time.perf_counter()
+        rec = o.spec_step(seq, temperature=T, seed=4)
+        dt = time.perf_counter() - t0
+        if i >= n_warm:
+            tokens += len(rec.emitted)
+            secs += dt
+            done_steps += 1
+            if secs >= time_cap_s:
+                break
+    return tokens, secs, done_steps
+
+
 def run_reference(args):
     wl = WORKLOADS[args.workload]
     cfg = _cfg(wl["cfg"], wl.get("layers"))
@@ -496,6 +675,23 @@ def run_reference(args):
     prompt = syn.prompts(cfg, 1, length=4, seed=1)
     lo, hi = wl["budget"]
     budgets = np.full(Bn, lo, np.int32) if lo == hi else syn.budgets(Bn, lo, hi, seed=2)
+    if wl.get("temperature"):
+        tokens, secs, steps = _oracle_sampling_run(cfg, ws, enc, prompt, int(budgets[0]),
+                                                   wl["temperature"], min(args.warmup, 3),
+                                                   args.steps, args.cpu_seconds * 4)
+        v = tokens / secs
+        return {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s",
+                "n_gpus": 1, "steps": steps, "warmup": args.warmup,
+                "ms_per_step": secs / steps * 1e3, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                "config": {"workload": args.workload, "description": wl["text"], "batch": 1,
+                           "block": cfg.block_k + 1, "temperature": wl["temperature"]},
+                "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": _cores(),
+                                 "kind": "oracle",
+                                 "sample": f"{steps} speculative sampling steps of one sequence "
+                                           f"(float64 numpy oracle; prefill untimed)"},
+                "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
     if wl["accept"] == "uniform":
         acc = syn.accept_uniform(max(args.warmup + args.steps, 64), Bn, k=cfg.block_k, seed=3)
     else:
@@ -542,7 +738,10 @@ def main():
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl")
-    res = run_ours(args, rank, world)
+    if WORKLOADS[args.workload].get("temperature"):
+        res = run_sampling(args, rank, world)
+    else:
+        res = run_ours(args, rank, world)
     if rank == 0:
         print(json.dumps(res), flush=True)
     if world > 1:
