@@ -122,58 +122,77 @@ __device__ __forceinline__ void epi_chunk(const GemmParams &p, int t0, int n, fl
 }
 
 // Epilogue of four consecutive output features n..n+3 of token row t (the
-// cluster-reduced path).  fin[] returns the final values (the updated
-// residual for EPI_RESID) for the LayerNorm statistics.
+// staged path).  `old` is the residual row's current value (EPI_RESID).
+// fin[] returns the final values (the updated residual for EPI_RESID) for the
+// LayerNorm statistics.  Four consecutive features never straddle a head or
+// the key/value boundary (multiples of 4), so each store is one vector.
+__device__ __forceinline__ uint2 pack4_bf16(const float (&v)[4]) {
+  __nv_bfloat162 h[2] = {__floats2bfloat162_rn(v[0], v[1]), __floats2bfloat162_rn(v[2], v[3])};
+  return *reinterpret_cast<const uint2 *>(h);
+}
 template <int EPI>
 __device__ __forceinline__ void epi_quad(const GemmParams &p, int t, int n, const float4 &a,
-                                         const float (&b4)[4], const float4 *pre_resid,
+                                         const float (&b4)[4], const float4 &old,
                                          const int2 *tok_local, float (&fin)[4]) {
   float v[4] = {a.x + b4[0], a.y + b4[1], a.z + b4[2], a.w + b4[3]};
   if constexpr (EPI == EPI_RESID) {
     // N % 128 == 0 and ld_resid % 4 == 0 (checked at launch): one float4
     float4 *r = reinterpret_cast<float4 *>(p.resid + static_cast<size_t>(t) * p.ld_resid + n);
-    const float4 o = pre_resid ? *pre_resid : *r;
-    const float4 nr = make_float4(o.x + v[0], o.y + v[1], o.z + v[2], o.w + v[3]);
+    const float4 nr = make_float4(old.x + v[0], old.y + v[1], old.z + v[2], old.w + v[3]);
     *r = nr;
     fin[0] = nr.x;
     fin[1] = nr.y;
     fin[2] = nr.z;
     fin[3] = nr.w;
-    __nv_bfloat162 h[2] = {__floats2bfloat162_rn(nr.x, nr.y), __floats2bfloat162_rn(nr.z, nr.w)};
-    if (p.tap0) *reinterpret_cast<uint2 *>(p.tap0 + static_cast<size_t>(t) * p.ld_tap + n) =
-        *reinterpret_cast<const uint2 *>(h);
-    if (p.tap1) *reinterpret_cast<uint2 *>(p.tap1 + static_cast<size_t>(t) * p.ld_tap + n) =
-        *reinterpret_cast<const uint2 *>(h);
+    const uint2 h = pack4_bf16(fin);
+    if (p.tap0) *reinterpret_cast<uint2 *>(p.tap0 + static_cast<size_t>(t) * p.ld_tap + n) = h;
+    if (p.tap1) *reinterpret_cast<uint2 *>(p.tap1 + static_cast<size_t>(t) * p.ld_tap + n) = h;
     return;
   }
+  if constexpr (EPI == EPI_GELU) {
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    fin[i] = v[i];
-    if (n + i >= p.N) continue;
-    if constexpr (EPI == EPI_F32) {
-      p.out_f32[static_cast<size_t>(t) * p.ld_out + n + i] = v[i];
-    } else if constexpr (EPI == EPI_BF16) {
-      p.out_bf16[static_cast<size_t>(t) * p.ld_out + n + i] = __float2bfloat16(v[i]);
-    } else if constexpr (EPI == EPI_GELU) {
-      p.out_bf16[static_cast<size_t>(t) * p.ld_out + n + i] = __float2bfloat16(gelu_erf(v[i]));
-    } else if constexpr (EPI == EPI_KV) {
-      const int nn = n + i;
-      if (nn < p.q_cols) {
-        p.out_bf16[static_cast<size_t>(t) * p.ld_out + nn] = __float2bfloat16(v[i]);
-        continue;
-      }
-      const int c = nn - p.q_cols;
-      const int which = c / p.d_model;
-      const int hd = c - which * p.d_model;
-      const int2 sp = *tok_local;
-      if (sp.y >= p.ctx) {
-        set_error(p.err, WF_DEV_ERR_CAPACITY);
-        continue;
-      }
-      bf16 *dst = which == 0 ? p.kc : p.vc;
-      dst[((static_cast<size_t>(sp.x) * p.n_heads + (hd >> 6)) * p.ctx + sp.y) * 64 + (hd & 63)] =
-          __float2bfloat16(v[i]);
+    for (int i = 0; i < 4; ++i) v[i] = gelu_erf(v[i]);
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) fin[i] = v[i];
+  const bool whole = n + 3 < p.N && (p.ld_out & 3) == 0;
+  if constexpr (EPI == EPI_F32) {
+    float *o = p.out_f32 + static_cast<size_t>(t) * p.ld_out + n;
+    if (whole) {
+      *reinterpret_cast<float4 *>(o) = make_float4(v[0], v[1], v[2], v[3]);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (n + i < p.N) o[i] = v[i];
     }
+  } else if constexpr (EPI == EPI_BF16 || EPI == EPI_GELU) {
+    bf16 *o = p.out_bf16 + static_cast<size_t>(t) * p.ld_out + n;
+    if (whole) {
+      *reinterpret_cast<uint2 *>(o) = pack4_bf16(v);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (n + i < p.N) o[i] = __float2bfloat16(v[i]);
+    }
+  } else if constexpr (EPI == EPI_KV) {
+    // N, q_cols and d_model are multiples of 4 (checked at launch)
+    if (n >= p.N) return;
+    if (n < p.q_cols) {
+      *reinterpret_cast<uint2 *>(p.out_bf16 + static_cast<size_t>(t) * p.ld_out + n) = pack4_bf16(v);
+      return;
+    }
+    const int c = n - p.q_cols;
+    const int which = c / p.d_model;
+    const int hd = c - which * p.d_model;
+    const int2 sp = *tok_local;
+    if (sp.y >= p.ctx) {
+      set_error(p.err, WF_DEV_ERR_CAPACITY);
+      return;
+    }
+    bf16 *dst = which == 0 ? p.kc : p.vc;
+    *reinterpret_cast<uint2 *>(
+        dst + ((static_cast<size_t>(sp.x) * p.n_heads + (hd >> 6)) * p.ctx + sp.y) * 64 + (hd & 63)) =
+        pack4_bf16(v);
   }
 }
 
@@ -476,11 +495,21 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
     const int rank = split;  // cluster (1, 1, S) over gridDim.z == S: rank == blockIdx.z
     const int rlo = cols * rank / S, rhi = cols * (rank + 1) / S;
     const int stat_tiles = p.N / kBlockN;
-    auto finish_row = [&](int tl, const float4 &acc, bool valid) {
+    // the residual row a warp updates next (EPI_RESID; the first one was
+    // loaded under the MMAs)
+    auto load_old = [&](int tl) {
+      float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+      if constexpr (EPI == EPI_RESID) {
+        o = (has_pre && tl == rlo + warp)
+                ? pre
+                : *reinterpret_cast<const float4 *>(p.resid + static_cast<size_t>(t0 + tl) * p.ld_resid +
+                                                    n0 + 4 * lane);
+      }
+      return o;
+    };
+    auto finish_row = [&](int tl, const float4 &acc, bool valid, const float4 &old) {
       float fin[4] = {0.f, 0.f, 0.f, 0.f};
-      if (valid)
-        epi_quad<EPI>(p, t0 + tl, n0 + 4 * lane, acc, b4, (has_pre && tl == rlo + warp) ? &pre : nullptr,
-                      tok + tl, fin);
+      if (valid) epi_quad<EPI>(p, t0 + tl, n0 + 4 * lane, acc, b4, old, tok + tl, fin);
       if (p.stats_out) {
         const float mean = warp_sum((fin[0] + fin[1]) + (fin[2] + fin[3])) * (1.0f / 128.f);
         const float d0 = fin[0] - mean, d1 = fin[1] - mean, d2 = fin[2] - mean, d3 = fin[3] - mean;
@@ -527,17 +556,31 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
     if (S > 1 && rhi - rlo <= 2 * W) {
       // at most two rows per warp: read every partial first, tell the peers
       // their tiles are free, then run the epilogue while they finish
-      float4 acc[2];
+      float4 acc[2], old[2];
 #pragma unroll
-      for (int k = 0; k < 2; ++k)
-        if (rlo + warp + W * k < rhi) acc[k] = reduce_row(rlo + warp + W * k);
+      for (int k = 0; k < 2; ++k) {
+        if (rlo + warp + W * k < rhi) {
+          old[k] = load_old(rlo + warp + W * k);
+          acc[k] = reduce_row(rlo + warp + W * k);
+        }
+      }
       cluster_arrive();
 #pragma unroll
       for (int k = 0; k < 2; ++k)
-        if (rlo + warp + W * k < rhi) finish_row(rlo + warp + W * k, acc[k], ok);
+        if (rlo + warp + W * k < rhi) finish_row(rlo + warp + W * k, acc[k], ok, old[k]);
       cluster_wait();
     } else {
-      for (int tl = rlo + warp; tl < rhi; tl += W) finish_row(tl, reduce_row(tl), ok);
+      // two rows per warp at a time, so their loads overlap
+      for (int tl = rlo + warp; tl < rhi; tl += 2 * W) {
+        const int tl2 = tl + W;
+        const bool two = tl2 < rhi;
+        const float4 old1 = load_old(tl);
+        const float4 old2 = two ? load_old(tl2) : make_float4(0.f, 0.f, 0.f, 0.f);
+        const float4 acc1 = reduce_row(tl);
+        const float4 acc2 = two ? reduce_row(tl2) : make_float4(0.f, 0.f, 0.f, 0.f);
+        finish_row(tl, acc1, ok, old1);
+        if (two) finish_row(tl2, acc2, ok, old2);
+      }
       if (S > 1) cluster_sync();
     }
   }
@@ -768,6 +811,8 @@ cudaError_t launch_gemm(const void *X, const void *W, GemmParams p, cudaStream_t
   if (p.epi == EPI_HEAD && (ln || p.stats_out)) return cudaErrorInvalidValue;
   if ((p.stats_out || p.epi == EPI_RESID) && p.N % kBlockN) return cudaErrorInvalidValue;
   if (p.epi == EPI_RESID && (p.ld_resid % 4 || (reinterpret_cast<uintptr_t>(p.resid) & 15)))
+    return cudaErrorInvalidValue;
+  if (quad && p.epi == EPI_KV && (p.N % 4 || p.q_cols % 4 || p.d_model % 4 || p.ld_out % 4))
     return cudaErrorInvalidValue;
   if (quad && p.epi == EPI_RESID && (p.tap0 || p.tap1) && p.ld_tap % 4) return cudaErrorInvalidValue;
   if (ln) {
