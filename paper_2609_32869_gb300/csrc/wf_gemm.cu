@@ -5,7 +5,7 @@
 // large weight matrix, so the weights stream from HBM once and set the time.
 // The kernel computes a 128 x BT tile of D = W_tile X_tile^T ("swap-AB"): the
 // 128 weight rows fill the MMA's M side, the token tile (a multiple of 16,
-// <= 256) its N side.  Weight and token tiles stream into shared memory by
+// <= 128) its N side.  Weight and token tiles stream into shared memory by
 // TMA (128-byte swizzle) through an mbarrier ring; one thread issues
 // tcgen05.mma into a TMEM accumulator; eight warps read it back with
 // tcgen05.ld for a fused epilogue (bias, GELU, residual add, taps, key/value
@@ -38,8 +38,11 @@ constexpr int kBlockN = 128;   // weight rows per tile (MMA M)
 constexpr int kThreads = 256;  // 8 warps: two per TMEM lane quarter
 constexpr int kBlockK = 64;    // K per pipeline stage (one 128-byte swizzle atom)
 constexpr int kStageA = kBlockN * kBlockK * 2;  // 16 KB
-constexpr int kSmemBudget = 200 * 1024;
-constexpr int kSmemBudgetLn = 220 * 1024;  // LN mode: resident token tiles + weight ring
+// Shared memory a CTA plans for: two CTAs fit on an SM, so one CTA's
+// epilogue overlaps the other's weight stream.
+constexpr int kSmemBudget = 110 * 1024;
+constexpr int kSmemBudgetLn = 110 * 1024;  // LN mode: resident token tiles + weight ring
+constexpr int kMaxBT = 128;                // token rows per tile (MMA N)
 constexpr size_t kSmemPerSM = 228 * 1024;  // shared memory of one SM
 constexpr int kLnFuseMaxM = 256;              // token rows up to which LN is fused
 
@@ -633,7 +636,7 @@ const CUtensorMap *tmap_bf16_2d(const void *ptr, uint64_t rows, uint64_t cols, u
 }
 
 void gemm_token_tiling(int M, int *BT, int *n_tt) {
-  const int nt = (M + 255) / 256;
+  const int nt = (M + kMaxBT - 1) / kMaxBT;
   const int per = (M + nt - 1) / nt;
   *n_tt = nt;
   *BT = ((per + 15) / 16) * 16;

@@ -82,7 +82,7 @@ struct GemmParams {
 // Cache of TMA descriptors keyed by (address, rows, cols, box rows).
 const CUtensorMap *tmap_bf16_2d(const void *ptr, uint64_t rows, uint64_t cols, uint32_t box_rows);
 
-// Token tile for M rows: a multiple of 16, at most 256.
+// Token tile for M rows: a multiple of 16, at most 128.
 void gemm_token_tiling(int M, int *BT, int *n_tt);
 // Split-K count for a projection of N outputs over K inputs (a function of
 // the shape only, so a row's result never depends on how many rows run).
