@@ -141,7 +141,10 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
     return;
   }
   const int n_blocks = (n_keys + kKB - 1) / kKB;
-  if (blk >= n_blocks) return;
+  // In a cluster launch every CTA of a multi-block group takes part in the
+  // merge; a block past the keys computes over masked keys only and yields
+  // the exact empty partial (m = -inf, l = 0, o = 0).
+  if (blk >= n_blocks && !(p.cluster && n_blocks > 1)) return;
 
   const int d_model = p.n_heads * 64;
   const size_t cache_off = (static_cast<size_t>(slot) * p.n_heads + h) * p.ctx;
@@ -376,6 +379,45 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
     return;
   }
 
+  if (p.cluster) {
+    // ---- several key blocks in one cluster: each CTA leaves its partial in
+    // its shared memory ([16][68]: m, l, -, -, o[64]); CTA 0 combines them in
+    // block order over DSMEM with the same arithmetic as the global path.
+    float *pb = reinterpret_cast<float *>(sV);
+    if (d0 == 0) {
+      pb[qi * 68] = M;
+      pb[qi * 68 + 1] = L;
+    }
+#pragma unroll
+    for (int e = 0; e < kDPT; ++e) pb[qi * 68 + 4 + d0 + e] = acc[e];
+    cluster_sync();
+    float MM = -INFINITY, LL = 0.f, oo[kDPT];
+    if (blk == 0) {
+      const uint32_t pb_u32 = smem_u32(pb);
+      for (int u = 0; u < p.n_chunks; ++u)
+        MM = fmaxf(MM, dsmem_ld_f32(dsmem_map(pb_u32 + 4u * (qi * 68), u)));
+#pragma unroll
+      for (int e = 0; e < kDPT; ++e) oo[e] = 0.f;
+      for (int u = 0; u < p.n_chunks; ++u) {
+        const float mc = dsmem_ld_f32(dsmem_map(pb_u32 + 4u * (qi * 68), u));
+        const float lc = dsmem_ld_f32(dsmem_map(pb_u32 + 4u * (qi * 68 + 1), u));
+        const float4 o4 = dsmem_ld_f32x4(dsmem_map(pb_u32 + 4u * (qi * 68 + 4 + d0), u));
+        const float ov[4] = {o4.x, o4.y, o4.z, o4.w};
+        const float wt = (mc == -INFINITY) ? 0.f : expf(mc - MM);
+        LL = __fmaf_rn(lc, wt, LL);
+#pragma unroll
+        for (int e = 0; e < kDPT; ++e) oo[e] = __fmaf_rn(ov[e], wt, oo[e]);
+      }
+    }
+    cluster_arrive();  // CTA 0 has read every partial; peers may exit
+    cluster_wait();
+    if (blk == 0 && qi < nq) {
+      bf16 *orow = p.out + static_cast<size_t>(i * p.rps + q0 + qi) * d_model + h * 64 + d0;
+      store_row(orow, oo, 1.0f / LL);
+    }
+    return;
+  }
+
   // ---- several key blocks: partials to global, the last CTA combines in order
   const int group_id = (i * p.n_heads + h) * p.qgroups + qg;
   float *part = p.part + (static_cast<size_t>(group_id) * p.n_chunks + blk) * kQG * kPartStride;
@@ -414,9 +456,9 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
 #pragma unroll
       for (int e = 0; e < kDPT; ++e) ov[e] = __ldcg(pe + 2 + d0 + e);
       const float wt = (mc == -INFINITY) ? 0.f : expf(mc - MM);
-      LL += lc * wt;
+      LL = __fmaf_rn(lc, wt, LL);
 #pragma unroll
-      for (int e = 0; e < kDPT; ++e) oo[e] += ov[e] * wt;
+      for (int e = 0; e < kDPT; ++e) oo[e] = __fmaf_rn(ov[e], wt, oo[e]);
     }
     const float inv = 1.0f / LL;
     bf16 *orow = p.out + static_cast<size_t>(i * p.rps + q0 + qi) * d_model + h * 64 + d0;
@@ -472,12 +514,27 @@ cudaError_t launch_attention(const AttnParams &p0, cudaStream_t s, bool pdl) {
   }();
   const long long ctas = static_cast<long long>(cfg.gridDim.x) * cfg.gridDim.y * cfg.gridDim.z;
   cfg.dynamicSmemBytes = ctas <= n_sm ? kSmemAttnSpread : kSmemAttn;
+  // small launches merge their blocks over DSMEM (no global round trip);
+  // large ones keep the global partials, where cluster placement costs more
+  // than it saves.  Both paths do the same arithmetic in the same order.
+  p.cluster = (p.n_chunks > 1 && p.n_chunks <= 8 && ctas <= n_sm) ? 1 : 0;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[2];
+  int na = 0;
+  if (p.cluster) {
+    attr[na].id = cudaLaunchAttributeClusterDimension;
+    attr[na].val.clusterDim.x = p.n_chunks;
+    attr[na].val.clusterDim.y = 1;
+    attr[na].val.clusterDim.z = 1;
+    ++na;
+  }
+  if (pdl) {
+    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
+  cfg.numAttrs = na;
   return cudaLaunchKernelEx(&cfg, attention_kernel, p);
 }
 

@@ -109,8 +109,9 @@ struct AttnParams {
   int32_t *counters;
   uint32_t *err;
   int n_seq, rps, n_heads, ctx, mode, n_chunks, qgroups;
+  int cluster;  // the n_chunks blocks of a (sequence, head, group) form a cluster
 };
-constexpr int kAttnKeysPerCTA = 256;  // keys per CTA (64 per warp), aligned to absolute positions
+constexpr int kAttnKeysPerCTA = 256;  // keys per CTA (32 per warp), aligned to absolute positions
 constexpr int kAttnQGroup = 16;       // query rows per CTA
 cudaError_t attention_init();
 size_t attn_partial_floats(int n_seq, int rps, int n_heads, int ctx);
