@@ -215,6 +215,13 @@ int32_t wf_last_launch_count(const wf_handle *h);
 #define WF_OPT_GRAPHS 3      /* 1 (default): wf_step / wf_greedy_step replay a CUDA graph
                                 captured on first use per (active count, forcing, sampling
                                 parameters); 0: launch kernel by kernel */
+#define WF_OPT_PERSIST 5     /* 1 (off by default; accepted where supported): the blocks of every drafter,
+                                verify and greedy pass run in one persistent cooperative
+                                launch; supported when max_batch * (block_k + 1) <= 16,
+                                d_model <= 1280 and d_ff a multiple of 512 with
+                                d_ff / 4 <= 1280.  0: one launch per projection and
+                                attention.  Both give results within the tolerances of
+                                the method, not bit-identical ones. */
 #define WF_VIEW_TARGET_LOGITS 1
 #define WF_VIEW_DRAFT_LOGITS 2
 #define WF_VIEW_TAPS 3
@@ -228,7 +235,9 @@ wf_status wf_set_option(wf_handle *h, int32_t option, int32_t value);
 #define WF_FAM_ATTN_CROSS 3 /* cross-attention over the encoder frames */
 #define WF_FAM_LAYERNORM 4
 #define WF_FAM_OTHER 5      /* embeddings, head reduction, accept, slot state */
-#define WF_PROF_FAMILIES 6
+#define WF_FAM_PERSIST 6    /* persistent small-batch pass: every block of a drafter,
+                               verify or greedy pass in one launch (WF_OPT_PERSIST) */
+#define WF_PROF_FAMILIES 7
 /* With WF_OPT_PROFILE on: synchronise `stream`, then return per family the
  * summed kernel time (ms, CUDA events on the launching stream), the number of
  * launches and, for the GEMM and head families, the algorithmic bytes those

@@ -78,6 +78,15 @@ struct wf_handle {
   bool use_graphs = true;
   cudaStream_t cap_stream = nullptr;
   int32_t *forced_buf = nullptr, *tok_buf = nullptr, *cnt_buf = nullptr;
+  // persistent small-batch passes (wf_persist.cu)
+  bool mk_ok = false;   // the shapes and limits allow it (fixed at create)
+  bool mk_on = false;   // in use (WF_OPT_PERSIST)
+  MkParams mkp = {};    // fields shared by every pass; the rest are set per launch
+  MkLayer *mkl = nullptr;        // device [nl + nd]: target blocks, then drafter blocks
+  char *mk_cnt_begin = nullptr;  // the persistent pass's counters, contiguous
+  size_t mk_cnt_bytes = 0;
+  CUtensorMap *tmaps = nullptr;  // device table
+  int tm_self_k = 0, tm_hist_k = 0, tm_cross_k = 0;
 };
 
 namespace {
@@ -176,6 +185,27 @@ size_t layout(wf_handle *h, const wf_config *c, int Bmax, int ctx, char *base) {
   o->logits_t = cv.take<float>(M * V);
   o->logits_d = cv.take<float>(M * V);
   o->rope = cv.take<float2>(static_cast<size_t>(c->max_pos) * 32);
+  o->mk_ok = persist_supported(d, H, F, T, Bmax * (K + 1));
+  if (o->mk_ok) {
+    MkParams &p = o->mkp;
+    const size_t R = kMkRows;
+    p.x = cv.take<float>(R * d);
+    p.q_x = cv.take<bf16>(R * d);
+    p.att_x = cv.take<bf16>(R * d);
+    p.xq_x = cv.take<bf16>(R * d);
+    p.xatt_x = cv.take<bf16>(R * d);
+    p.h_x = cv.take<bf16>(R * F);
+    p.part2 = cv.take<float>(static_cast<size_t>(d / 8) * 3 * R * 8);
+    p.xpart = cv.take<float>(mk_xpart_words(Bmax, H, T));
+    p.cnt = cv.take<uint32_t>(kMkCounters);
+    o->mk_cnt_begin = reinterpret_cast<char *>(p.cnt);
+    p.cnt2 = cv.take<uint32_t>(d / 8);
+    p.cntx = cv.take<uint32_t>(static_cast<size_t>(Bmax) * H);
+    p.sync = cv.take<uint32_t>(2);
+    o->mk_cnt_bytes = reinterpret_cast<char *>(p.sync + 2) - o->mk_cnt_begin;
+    o->mkl = cv.take<MkLayer>(nl + nd);
+    o->tmaps = cv.take<CUtensorMap>(static_cast<size_t>(6) * (nl + nd) + 6);
+  }
   return cv.off + kAlign;
 }
 
@@ -426,12 +456,13 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
 }
 
 // Final LayerNorm (the target's, shared with the drafter) and the tied head.
+// x == nullptr: h->xn already holds the normalised rows (persistent pass).
 cudaError_t head(wf_handle *h, const float *x, const float2 *st, int stride, int off, int rows,
                  const int32_t *slots,
                  int rps, HeadRec *recs, HeadOut *out, float *logits, const wf_sample_params *sp,
                  uint32_t tag, int32_t *cand, cudaStream_t s) {
   cudaError_t e;
-  if ((e = layernorm(h, x, st, stride, off, h->tw.lnf_g, h->tw.lnf_b, h->xn, rows, s)) != cudaSuccess)
+  if (x && (e = layernorm(h, x, st, stride, off, h->tw.lnf_g, h->tw.lnf_b, h->xn, rows, s)) != cudaSuccess)
     return e;
   const bool sampling = sp && sp->temperature > 0.f;
   GemmParams p = gemm_base(h, rows, h->V, h->d, EPI_HEAD);
@@ -546,6 +577,143 @@ cudaError_t target_pass(wf_handle *h, int n_seq, int rps, const int32_t *slots, 
   return cudaSuccess;
 }
 
+// Tensor maps and per-block tables of the persistent passes: every weight
+// matrix as [rows][cols] bf16 with [8][64] boxes (one unit of 8 output rows,
+// one 128-byte swizzle atom), every cache as [rows][64] with [32][64] boxes.
+cudaError_t persist_setup(wf_handle *h, cudaStream_t s) {
+  int G = 0;
+  cudaError_t e = persist_init(&G);
+  if (e != cudaSuccess) return e;
+  if (G > kMkMaxG) G = kMkMaxG;
+  if (G < 4 * kMkRows) return cudaErrorInvalidConfiguration;
+  const int d = h->d, F = h->F, H = h->H, T = h->cfg.enc_frames;
+  const int nl = h->nl, nd = h->nd;
+  std::vector<CUtensorMap> maps;
+  std::vector<MkLayer> lys;
+  auto add_map = [&](const void *ptr, uint64_t rows, uint64_t cols, uint32_t box) -> int {
+    const CUtensorMap *m = tmap_bf16_2d(ptr, rows, cols, box);
+    if (!m) return -1;
+    maps.push_back(*m);
+    return static_cast<int>(maps.size()) - 1;
+  };
+  // one copy per projection unit: 8 rows by the unit's whole K range
+  auto add_units = [&](const void *ptr, uint64_t rows, uint64_t cols, uint32_t kblocks) -> int {
+    CUtensorMap m;
+    if (!tmap_bf16_units(&m, ptr, rows, cols, kblocks)) return -1;
+    maps.push_back(m);
+    return static_cast<int>(maps.size()) - 1;
+  };
+  for (int l = 0; l < nl + nd; ++l) {
+    const wf_layer_weights &w = l < nl ? h->tl[l] : h->dl[l - nl];
+    MkLayer ly = {};
+    ly.ln1_g = static_cast<const bf16 *>(w.ln1_g);
+    ly.ln1_b = static_cast<const bf16 *>(w.ln1_b);
+    ly.qkv_b = static_cast<const bf16 *>(w.qkv_b);
+    ly.out_b = static_cast<const bf16 *>(w.out_b);
+    ly.ln2_g = static_cast<const bf16 *>(w.ln2_g);
+    ly.ln2_b = static_cast<const bf16 *>(w.ln2_b);
+    ly.xq_b = static_cast<const bf16 *>(w.xq_b);
+    ly.xout_b = static_cast<const bf16 *>(w.xout_b);
+    ly.ln3_g = static_cast<const bf16 *>(w.ln3_g);
+    ly.ln3_b = static_cast<const bf16 *>(w.ln3_b);
+    ly.fc1_b = static_cast<const bf16 *>(w.fc1_b);
+    ly.fc2_b = static_cast<const bf16 *>(w.fc2_b);
+    ly.tm[0] = add_units(w.qkv_w, 3 * d, d, d / 64);
+    ly.tm[1] = add_units(w.out_w, d, d, d / 64);
+    ly.tm[2] = add_units(w.xq_w, d, d, d / 64);
+    ly.tm[3] = add_units(w.xout_w, d, d, d / 64);
+    ly.tm[4] = add_units(w.fc1_w, F, d, d / 64);
+    ly.tm[5] = add_units(w.fc2_w, d, F, F / 4 / 64);  // one quarter of K per copy
+    for (int k = 0; k < 6; ++k)
+      if (ly.tm[k] < 0) return cudaErrorInvalidValue;
+    ly.self_layer = l < nl ? l : l - nl;
+    ly.cross_layer = l;
+    ly.tap[0] = ly.tap[1] = -1;
+    if (l < nl) {
+      int found = 0;
+      for (int t = 0; t < h->cfg.n_taps && found < 2; ++t)
+        if (h->cfg.taps[t] == l) ly.tap[found++] = t;
+    }
+    lys.push_back(ly);
+  }
+  const uint64_t self_rows = static_cast<uint64_t>(nl) * h->Bmax * H * h->ctx;
+  const uint64_t hist_rows = static_cast<uint64_t>(nd) * h->Bmax * H * h->ctx;
+  const uint64_t cross_rows = static_cast<uint64_t>(nl + nd) * h->Bmax * H * T;
+  // one copy per 128 keys (or values) of one head
+  h->tm_self_k = add_map(h->self_k, self_rows, 64, 128);
+  const int sv = add_map(h->self_v, self_rows, 64, 128);
+  h->tm_hist_k = add_map(h->hist_k, hist_rows, 64, 128);
+  const int hv = add_map(h->hist_v, hist_rows, 64, 128);
+  h->tm_cross_k = add_map(h->cross_k, cross_rows, 64, 128);
+  const int cv2 = add_map(h->cross_v, cross_rows, 64, 128);
+  if (h->tm_self_k < 0 || sv != h->tm_self_k + 1 || h->tm_hist_k < 0 || hv != h->tm_hist_k + 1 ||
+      h->tm_cross_k < 0 || cv2 != h->tm_cross_k + 1)
+    return cudaErrorInvalidValue;
+  // synchronous copies: the host vectors die with this call
+  if ((e = cudaMemcpy(h->tmaps, maps.data(), maps.size() * sizeof(CUtensorMap), cudaMemcpyHostToDevice)) !=
+      cudaSuccess)
+    return e;
+  if ((e = cudaMemcpy(h->mkl, lys.data(), lys.size() * sizeof(MkLayer), cudaMemcpyHostToDevice)) != cudaSuccess)
+    return e;
+  // every counter starts at zero; each pass leaves them at zero
+  if ((e = cudaMemsetAsync(h->mk_cnt_begin, 0, h->mk_cnt_bytes, s)) != cudaSuccess) return e;
+  MkParams &p = h->mkp;
+  p.tmaps = h->tmaps;
+  p.G = G;
+  p.d = d;
+  p.H = H;
+  p.F = F;
+  p.T = T;
+  p.ctx = h->ctx;
+  p.Bmax = h->Bmax;
+  p.K = h->K;
+  p.vocab = h->V;
+  p.tm_xk = h->tm_cross_k;
+  p.tm_xv = h->tm_cross_k + 1;
+  p.L = h->L;
+  p.anchor = h->anchor;
+  p.cand_in = h->cand;
+  p.tok_emb = static_cast<const bf16 *>(h->tw.tok_emb);
+  p.pos_emb = static_cast<const bf16 *>(h->tw.pos_emb);
+  p.mask_emb = static_cast<const bf16 *>(h->dw.mask_emb);
+  p.lnf_g = static_cast<const bf16 *>(h->tw.lnf_g);
+  p.lnf_b = static_cast<const bf16 *>(h->tw.lnf_b);
+  p.rope_tab = h->rope;
+  p.eps = h->cfg.ln_eps;
+  p.taps = h->taps;
+  p.ld_tap = h->cfg.n_taps * d;
+  p.xn = h->xn;
+  p.err = h->err;
+  h->mk_on = false;
+  return cudaSuccess;
+}
+
+// Every block of one pass in a single persistent launch; the final
+// LayerNorm's output is left in h->xn for the head.
+cudaError_t persist_pass(wf_handle *h, bool drafter, int n_seq, int rps, const int32_t *slots,
+                         const int32_t *forced, bool taps, cudaStream_t s) {
+  MkParams p = h->mkp;
+  p.layers = drafter ? h->mkl + h->nl : h->mkl;
+  p.nl = drafter ? h->nd : h->nl;
+  p.drafter = drafter ? 1 : 0;
+  p.write_taps = taps ? 1 : 0;
+  p.n_seq = n_seq;
+  p.rps = rps;
+  p.M = n_seq * rps;
+  p.seq_slot = slots;
+  p.forced = forced;
+  p.cand_out = (drafter || rps == 1) ? nullptr : h->cand;
+  p.kc = drafter ? h->hist_k : h->self_k;
+  p.vc = drafter ? h->hist_v : h->self_v;
+  p.tm_kc = drafter ? h->tm_hist_k : h->tm_self_k;
+  p.tm_vc = p.tm_kc + 1;
+  h->launches++;
+  prof_begin(h, s);
+  cudaError_t e = launch_persist(p, s);
+  prof_end(h, s, WF_FAM_PERSIST, 0.0);
+  return e;
+}
+
 wf_status check_weights(const wf_layer_weights &w) {
   const void *ptrs[] = {w.ln1_g, w.ln1_b, w.qkv_w, w.qkv_b, w.out_w, w.out_b, w.ln2_g,
                         w.ln2_b, w.xq_w,  w.xq_b,  w.xkv_w, w.xkv_b, w.xout_w, w.xout_b,
@@ -647,6 +815,7 @@ wf_status wf_create(const wf_config *cfg, const wf_target_weights *tw, const wf_
             launch_rope_table(h->rope, cfg->max_pos, cfg->rope_base, s) == cudaSuccess;
   ok = ok && gemm_init() == cudaSuccess && attention_init() == cudaSuccess &&
        cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) == cudaSuccess;
+  if (ok && h->mk_ok) ok = persist_setup(h, s) == cudaSuccess;
   if (!ok) {
     if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
     delete h;
@@ -681,6 +850,13 @@ wf_status wf_set_option(wf_handle *h, int32_t option, int32_t value) {
   }
   if (option == WF_OPT_GRAPHS) {
     h->use_graphs = value != 0;
+    return WF_OK;
+  }
+  if (option == WF_OPT_PERSIST) {
+    if (value && !h->mk_ok) return WF_ERR_UNSUPPORTED;
+    h->mk_on = value != 0;
+    for (auto &kv : h->graphs) cudaGraphExecDestroy(kv.second.exec);
+    h->graphs.clear();
     return WF_OK;
   }
   if (option == WF_OPT_PROFILE) {
@@ -810,6 +986,12 @@ wf_status wf_prefill_cross_kv(wf_handle *h, int32_t n, const int32_t *d_slots, c
 static wf_status draft_body(wf_handle *h, const wf_sample_params *sp, cudaStream_t s) {
   if (h->n_active == 0) return WF_OK;
   const int n = h->n_active, rps = h->K + 1;
+  if (h->mk_on) {
+    WF_TRY(persist_pass(h, true, n, rps, h->active, nullptr, false, s));
+    WF_TRY(head(h, nullptr, nullptr, 1, 0, n * rps, h->active, rps, h->recs_d, h->hout_d, h->logits_d, sp,
+                kTagDraft, h->cand, s));
+    return WF_OK;
+  }
   EmbedParams ep = {};
   ep.tok_emb = static_cast<const bf16 *>(h->tw.tok_emb);
   ep.mask_emb = static_cast<const bf16 *>(h->dw.mask_emb);
@@ -840,9 +1022,15 @@ static wf_status verify_body(wf_handle *h, const wf_sample_params *sp, const int
                              int32_t *d_out_tokens, int32_t *d_out_count, cudaStream_t s) {
   const int n = h->n_active, rps = h->K + 1;
   if (n > 0) {
-    WF_TRY(target_pass(h, n, rps, h->active, TOK_VERIFY, nullptr, 0, d_forced, true, s));
-    WF_TRY(head(h, h->x, h->st_x, 1, 0, n * rps, h->active, rps, h->recs_t, h->hout_t, h->logits_t, sp,
-                kTagBonus, nullptr, s));
+    if (h->mk_on) {
+      WF_TRY(persist_pass(h, false, n, rps, h->active, d_forced, true, s));
+      WF_TRY(head(h, nullptr, nullptr, 1, 0, n * rps, h->active, rps, h->recs_t, h->hout_t, h->logits_t,
+                  sp, kTagBonus, nullptr, s));
+    } else {
+      WF_TRY(target_pass(h, n, rps, h->active, TOK_VERIFY, nullptr, 0, d_forced, true, s));
+      WF_TRY(head(h, h->x, h->st_x, 1, 0, n * rps, h->active, rps, h->recs_t, h->hout_t, h->logits_t, sp,
+                  kTagBonus, nullptr, s));
+    }
     WF_TRY(ingest(h, n, rps, h->active, s));
   }
   AcceptParams ap = {};
@@ -882,9 +1070,15 @@ static wf_status greedy_body(wf_handle *h, const wf_sample_params *sp, int32_t *
                              int32_t *d_out_count, cudaStream_t s) {
   const int n = h->n_active;
   if (n > 0) {
-    WF_TRY(target_pass(h, n, 1, h->active, TOK_ANCHOR, nullptr, 0, nullptr, false, s));
-    WF_TRY(head(h, h->x, h->st_x, 1, 0, n, h->active, 1, h->recs_t, h->hout_t, h->logits_t, sp, kTagBonus,
-                nullptr, s));
+    if (h->mk_on) {
+      WF_TRY(persist_pass(h, false, n, 1, h->active, nullptr, false, s));
+      WF_TRY(head(h, nullptr, nullptr, 1, 0, n, h->active, 1, h->recs_t, h->hout_t, h->logits_t, sp,
+                  kTagBonus, nullptr, s));
+    } else {
+      WF_TRY(target_pass(h, n, 1, h->active, TOK_ANCHOR, nullptr, 0, nullptr, false, s));
+      WF_TRY(head(h, h->x, h->st_x, 1, 0, n, h->active, 1, h->recs_t, h->hout_t, h->logits_t, sp, kTagBonus,
+                  nullptr, s));
+    }
   }
   AcceptParams ap = {};
   ap.seq_slot = h->active;

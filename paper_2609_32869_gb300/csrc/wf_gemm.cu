@@ -635,6 +635,25 @@ const CUtensorMap *tmap_bf16_2d(const void *ptr, uint64_t rows, uint64_t cols, u
   return m;
 }
 
+// 3-D view of a row-major [rows][cols] bf16 matrix as (64 columns, row,
+// 64-column block) with strides (cols * 2 bytes, 128 bytes): a box of
+// {64, 8, kblocks} is 8 consecutive rows by kblocks * 64 columns, landing in
+// shared memory as [kblock][8 rows][128 B] with 128-byte swizzling (one
+// swizzle atom per k-block), in a single copy.
+bool tmap_bf16_units(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint32_t kblocks) {
+  auto fn = encode_fn();
+  if (!fn || (reinterpret_cast<uintptr_t>(ptr) & 15) || cols % 64 || kblocks == 0 || kblocks > 256 ||
+      kblocks > cols / 64)
+    return false;
+  cuuint64_t gdim[3] = {64, rows, cols / 64};
+  cuuint64_t gstride[2] = {cols * 2, 128};
+  cuuint32_t box[3] = {64, 8, kblocks};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), gdim, gstride, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 void gemm_token_tiling(int M, int *BT, int *n_tt) {
   const int nt = (M + kMaxBT - 1) / kMaxBT;
   const int per = (M + nt - 1) / nt;

@@ -81,6 +81,8 @@ struct GemmParams {
 
 // Cache of TMA descriptors keyed by (address, rows, cols, box rows).
 const CUtensorMap *tmap_bf16_2d(const void *ptr, uint64_t rows, uint64_t cols, uint32_t box_rows);
+// A whole 8-row unit of a [rows][cols] matrix per copy: box {64, 8, kblocks}.
+bool tmap_bf16_units(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint32_t kblocks);
 
 // Token tile for M rows: a multiple of 16, at most 128.
 void gemm_token_tiling(int M, int *BT, int *n_tt);
@@ -188,5 +190,54 @@ struct StateParams {
 cudaError_t launch_state(const StateParams &p, cudaStream_t s, bool pdl);
 cudaError_t launch_compact(const int32_t *done, int max_batch, int32_t *active,
                            int32_t *n_active_dev, cudaStream_t s);
+
+// ------------------------------------------------- persistent decode pass --
+// One cooperative launch runs every block of a small-batch pass (M <= 16
+// token rows).  See wf_persist.cu.
+constexpr int kMkRows = 16;       // token rows a persistent pass supports
+constexpr int kMkMaxSeq = 16;     // sequences per persistent pass
+constexpr int kMkPhases = 8;      // QKV, self-attn, out, cross-query, cross-attn, cross-out, fc1, fc2
+constexpr int kMkMaxG = 256;      // CTAs a persistent pass may use
+constexpr int kMkCounters = 8 * 64 + 2;  // phase counters: embedding + 8 phases x 64 blocks
+struct MkLayer {
+  const bf16 *ln1_g, *ln1_b, *qkv_b, *out_b, *ln2_g, *ln2_b, *xq_b, *xout_b;
+  const bf16 *ln3_g, *ln3_b, *fc1_b, *fc2_b;
+  int32_t tm[6];        // tensor-map index of qkv_w, out_w, xq_w, xout_w, fc1_w, fc2_w
+  int32_t self_layer;   // layer of the self (target) or history (drafter) cache
+  int32_t cross_layer;  // layer of the acoustic cache
+  int32_t tap[2];       // tap column blocks written after the block (-1: none)
+};
+struct MkParams {
+  const CUtensorMap *tmaps;  // device table: weight maps, then the cache maps below
+  const MkLayer *layers;     // device array [nl]
+  int nl, drafter, src, write_taps;
+  int G, n_seq, rps, M;
+  int d, H, F, T, ctx, Bmax, K, vocab;
+  int tm_kc, tm_vc, tm_xk, tm_xv;
+  const int32_t *seq_slot, *L, *anchor, *cand_in, *forced;
+  int32_t *cand_out;
+  const bf16 *tok_emb, *pos_emb, *mask_emb, *lnf_g, *lnf_b;
+  bf16 *kc, *vc;             // self or history cache, layer 0
+  const float2 *rope_tab;
+  float eps;
+  // buffers between CTAs (rows: token rows of the pass)
+  float *x;                    // [kMkRows][d]    residual stream
+  bf16 *q_x, *att_x, *xq_x, *xatt_x;  // [kMkRows][d]
+  bf16 *h_x;                   // [kMkRows][F]    fc1 output
+  float *part2;                // [d/8][3][kMkRows][8] fc2 split-K partials
+  float *xpart;                // [n_seq*H*nch][kMkRows][68] cross-attention partials
+  uint32_t *cnt;               // [kMkCounters] CTAs that finished each phase
+  uint32_t *cnt2;              // [d/8] fc2 partials published per output unit (cumulative)
+  uint32_t *cntx;              // [max_batch*H] cross-attention partials published per head
+  bf16 *taps;
+  int ld_tap;
+  bf16 *xn;                    // [M][d] final LayerNorm output (plain bf16)
+  uint32_t *sync;              // [1] CTAs finished (reset by the last)
+  uint32_t *err;
+};
+size_t mk_xpart_words(int M, int H, int T);
+cudaError_t persist_init(int *G);
+bool persist_supported(int d, int H, int F, int T, int rows);
+cudaError_t launch_persist(const MkParams &p, cudaStream_t s);
 
 }  // namespace wf

@@ -1,0 +1,238 @@
+"""Parity of the persistent small-batch pass (one cooperative launch per
+drafter, verify or greedy pass; wf_persist.cu) on the GPU.
+
+A handle with max_batch * (K + 1) <= 16 runs its passes persistently once
+WF_OPT_PERSIST is set.  Bars as everywhere else: logits max-abs <= 3e-2 against the
+oracle, hidden states (taps) relative L2 <= 1e-2, tokens and cache lengths
+equal wherever the deciding top-2 margins exceed 0.05; speculative greedy
+equals plain greedy token for token (Sec. 3.1)."""
+import numpy as np
+import pytest
+
+from oracle.decoder import WhisperFlashOracle
+from paper_2609_32869_gb300 import synthetic as syn
+
+pytestmark = pytest.mark.gpu
+
+LOGIT_ATOL = 3e-2
+HIDDEN_REL = 1e-2
+MARGIN = 0.05
+
+
+def _margin(row):
+    top = np.partition(np.asarray(row, np.float64), -2)[-2:]
+    return float(top[1] - top[0])
+
+
+def _forced(g, t, a, K, V):
+    cand = [g[t + j] if t + j < len(g) else 0 for j in range(K)]
+    if a < K and t + a < len(g):
+        cand[a] = (g[t + a] + 1) % V
+    return cand
+
+
+@pytest.fixture(scope="module")
+def tiny():
+    import torch
+    from paper_2609_32869_gb300.session import upload_weights
+    cfg = syn.TINY
+    ws = syn.make_weights(cfg, seed=0)
+    dev = upload_weights(ws)
+    enc = syn.encoder_output(cfg, 1, seed=1)
+    torch.cuda.synchronize()
+    return cfg, ws, dev, enc
+
+
+def _session(cfg, dev, persist=True, keep_logits=False):
+    from paper_2609_32869_gb300 import binding as B
+    from paper_2609_32869_gb300.session import Session
+    s = Session(cfg, dev, max_batch=1, keep_logits=keep_logits)
+    B.wf_set_option(s.h, B.WF_OPT_PERSIST, 1 if persist else 0)
+    return s
+
+
+def test_persistent_path_is_a_few_launches_at_batch_one(tiny):
+    """The whole step is a handful of launches, not one per projection."""
+    from paper_2609_32869_gb300 import binding as B
+    cfg, ws, dev, enc = tiny
+    prompt = syn.prompts(cfg, 1, length=4, seed=1)
+    s = _session(cfg, dev)
+    s.prefill([0], enc, prompt, np.array([40], np.int32))
+    B.wf_set_option(s.h, B.WF_OPT_GRAPHS, 0)
+    s.step()
+    assert s.launches() <= 12
+    s.greedy_step()
+    assert s.launches() <= 4
+    assert s.error() == 0
+    s.close()
+    from paper_2609_32869_gb300.session import Session
+    s4 = Session(cfg, dev, max_batch=4)
+    with pytest.raises(B.WfError):
+        B.wf_set_option(s4.h, B.WF_OPT_PERSIST, 1)
+    s4.close()
+
+
+def test_persistent_steps_match_oracle(tiny):
+    import torch
+    from paper_2609_32869_gb300 import binding as B
+    cfg, ws, dev, enc = tiny
+    K, V, d = cfg.block_k, cfg.vocab, cfg.d_model
+    P, budget = 6, 60
+    prompt = syn.prompts(cfg, 1, length=P, seed=7)
+    o = WhisperFlashOracle(syn.weights_as_float(ws), cfg)
+    encf = syn.bf16_bits_to_f32(enc[0]).astype(np.float64)
+    greedy = o.greedy_decode(encf, prompt[0], 40, seq_id=0)
+    seq = o.prefill(encf, prompt[0], budget, seq_id=0)
+    s = _session(cfg, dev, keep_logits=True)
+    first = int(s.prefill([0], enc, prompt, np.array([budget], np.int32)).cpu()[0])
+    if first != seq.emitted[0]:
+        assert _margin(seq._prefill_logits[-1]) <= MARGIN
+        pytest.skip("near tie at the first token")
+    decisions = 0
+    for step, acc in enumerate((8, 2, 5)):
+        forced = np.array([_forced(greedy, len(seq.emitted), acc, K, V)], np.int32)
+        toks, cnt = s.step(forced=forced)
+        torch.cuda.synchronize()
+        dl = s.view(B.WF_VIEW_DRAFT_LOGITS, torch.float32, (K + 1, V)).cpu().numpy()
+        vl = s.view(B.WF_VIEW_TARGET_LOGITS, torch.float32, (K + 1, V)).cpu().numpy()
+        taps = s.view(B.WF_VIEW_TAPS, torch.bfloat16, (K + 1, cfg.n_taps * d)).float().cpu().numpy()
+        rec = o.spec_step(seq, forced=forced[0])
+        assert np.abs(dl[1:1 + K] - rec.draft_logits).max() <= LOGIT_ATOL
+        assert np.abs(vl[:rec.k + 1] - rec.verify_logits).max() <= LOGIT_ATOL
+        rel = (np.linalg.norm(taps[:rec.k + 1] - rec.verify_taps, axis=1)
+               / np.linalg.norm(rec.verify_taps, axis=1))
+        assert rel.max() <= HIDDEN_REL
+        for gpu_rows, ora_rows in ((dl[1:1 + K], rec.draft_logits), (vl[:rec.k + 1], rec.verify_logits)):
+            for gr, orow in zip(gpu_rows, ora_rows):
+                if _margin(orow) > MARGIN:
+                    assert int(np.argmax(gr)) == int(np.argmax(orow))
+                    decisions += 1
+        deciding = [_margin(rec.verify_logits[j]) for j in range(min(rec.accepted + 1, rec.k + 1))]
+        if min(deciding) > MARGIN:
+            got = [int(x) for x in toks.cpu().numpy()[0, :int(cnt.cpu()[0])]]
+            assert got == rec.emitted
+            assert s.state()["len"][0] == seq.L
+            assert rec.accepted == acc
+        else:
+            break
+    assert decisions >= 8
+    assert s.error() == 0
+    s.close()
+
+
+def test_persistent_speculative_equals_plain_greedy(tiny):
+    """Sec. 3.1: the persistent speculative step (9 rows) and the persistent
+    plain greedy step (1 row) produce the same transcript token for token."""
+    cfg, ws, dev, enc = tiny
+    K, V = cfg.block_k, cfg.vocab
+    prompt = syn.prompts(cfg, 1, length=4, seed=3)
+    budget = np.array([48], np.int32)
+    g = _session(cfg, dev)
+    ref = [int(g.prefill([0], enc, prompt, budget).cpu()[0])]
+    while True:
+        toks, cnt = g.greedy_step()
+        c = int(cnt.cpu()[0])
+        if c == 0:
+            break
+        ref.extend(int(x) for x in toks.cpu().numpy()[0, :c])
+    assert g.error() == 0
+    g.close()
+    assert len(ref) == budget[0] or ref[-1] == cfg.eos_id
+    for mode in ("forced", "drafter"):
+        s = _session(cfg, dev)
+        got = [int(s.prefill([0], enc, prompt, budget).cpu()[0])]
+        sched = syn.accept_uniform(64, 1, k=K, seed=11)
+        it = 0
+        while True:
+            forced = None
+            if mode == "forced":
+                forced = np.array([_forced(ref, len(got), int(sched[it, 0]), K, V)], np.int32)
+            toks, cnt = s.step(forced=forced)
+            c = int(cnt.cpu()[0])
+            if c == 0:
+                break
+            got.extend(int(x) for x in toks.cpu().numpy()[0, :c])
+            it += 1
+            assert it < 100
+        assert got == ref, mode
+        assert s.error() == 0
+        s.close()
+
+
+def test_persistent_and_launch_by_launch_paths_agree(tiny):
+    """Both implementations of the same step stay within the logit tolerance
+    of each other (they round differently, so bits may differ)."""
+    import torch
+    from paper_2609_32869_gb300 import binding as B
+    cfg, ws, dev, enc = tiny
+    K, V = cfg.block_k, cfg.vocab
+    prompt = syn.prompts(cfg, 1, length=5, seed=2)
+    forced = syn.random_tokens(cfg, (1, K), seed=5).astype(np.int32)
+    out = {}
+    for persist in (True, False):
+        s = _session(cfg, dev, persist=persist, keep_logits=True)
+        s.prefill([0], enc, prompt, np.array([30], np.int32))
+        s.step(forced=forced)
+        torch.cuda.synchronize()
+        out[persist] = (s.view(B.WF_VIEW_DRAFT_LOGITS, torch.float32, (K + 1, V)).cpu().numpy().copy(),
+                        s.view(B.WF_VIEW_TARGET_LOGITS, torch.float32, (K + 1, V)).cpu().numpy().copy())
+        assert s.error() == 0
+        s.close()
+    for a, b in zip(out[True], out[False]):
+        assert np.abs(a - b).max() <= LOGIT_ATOL
+
+
+@pytest.mark.slow
+def test_persistent_large_shapes_match_oracle():
+    """Whisper-large shapes (d=1280, 20 heads, FFN 5120, 32 layers,
+    vocabulary 51866, 1500 frames) at batch 1, the benchmark's configuration."""
+    import torch
+    from paper_2609_32869_gb300 import binding as B
+    from paper_2609_32869_gb300.session import Session
+    cfg = syn.LARGE
+    K, V, d = cfg.block_k, cfg.vocab, cfg.d_model
+    ws = syn.make_weights(cfg, seed=0)
+    enc = syn.encoder_output(cfg, 1, seed=1)
+    prompt = syn.prompts(cfg, 1, length=4, seed=1)
+    budget = 60
+    s = Session(cfg, ws, max_batch=1, keep_logits=True)
+    first = int(s.prefill([0], enc, prompt, np.array([budget], np.int32)).cpu()[0])
+    o = WhisperFlashOracle(syn.weights_as_float(ws, np.float64), cfg)
+    encf = syn.bf16_bits_to_f32(enc[0]).astype(np.float64)
+    seq = o.prefill(encf, prompt[0], budget, seq_id=0)
+    gseq = o.prefill(encf, prompt[0], budget, seq_id=0)
+    while len(gseq.emitted) < 24 and not gseq.done:
+        o.greedy_step(gseq)
+    greedy = gseq.emitted
+    if first != seq.emitted[0]:
+        assert _margin(seq._prefill_logits[-1]) <= MARGIN
+        pytest.skip("near tie at the first token")
+    decisions = 0
+    for step, acc in enumerate((8, 3)):
+        forced = np.array([_forced(greedy, len(seq.emitted), acc, K, V)], np.int32)
+        toks, cnt = s.step(forced=forced)
+        torch.cuda.synchronize()
+        dl = s.view(B.WF_VIEW_DRAFT_LOGITS, torch.float32, (K + 1, V)).cpu().numpy()
+        vl = s.view(B.WF_VIEW_TARGET_LOGITS, torch.float32, (K + 1, V)).cpu().numpy()
+        taps = s.view(B.WF_VIEW_TAPS, torch.bfloat16, (K + 1, cfg.n_taps * d)).float().cpu().numpy()
+        rec = o.spec_step(seq, forced=forced[0])
+        assert np.abs(dl[1:1 + K] - rec.draft_logits).max() <= LOGIT_ATOL
+        assert np.abs(vl[:rec.k + 1] - rec.verify_logits).max() <= LOGIT_ATOL
+        rel = (np.linalg.norm(taps[:rec.k + 1] - rec.verify_taps, axis=1)
+               / np.linalg.norm(rec.verify_taps, axis=1))
+        assert rel.max() <= HIDDEN_REL
+        for gpu_rows, ora_rows in ((dl[1:1 + K], rec.draft_logits), (vl[:rec.k + 1], rec.verify_logits)):
+            for gr, orow in zip(gpu_rows, ora_rows):
+                if _margin(orow) > MARGIN:
+                    assert int(np.argmax(gr)) == int(np.argmax(orow))
+                    decisions += 1
+        deciding = [_margin(rec.verify_logits[j]) for j in range(min(rec.accepted + 1, rec.k + 1))]
+        got = [int(x) for x in toks.cpu().numpy()[0, :int(cnt.cpu()[0])]]
+        if min(deciding) > MARGIN:
+            assert got == rec.emitted
+            assert s.state()["len"][0] == seq.L
+        else:
+            break
+    assert decisions >= 8
+    assert s.error() == 0
+    s.close()
