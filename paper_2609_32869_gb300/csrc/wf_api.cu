@@ -579,7 +579,7 @@ cudaError_t target_pass(wf_handle *h, int n_seq, int rps, const int32_t *slots, 
 
 // Tensor maps and per-block tables of the persistent passes: every weight
 // matrix as [rows][cols] bf16 with [8][64] boxes (one unit of 8 output rows,
-// one 128-byte swizzle atom), every cache as [rows][64] with [32][64] boxes.
+// one 128-byte swizzle atom), every cache as [rows][64] with [128][64] boxes.
 cudaError_t persist_setup(wf_handle *h, cudaStream_t s) {
   int G = 0;
   cudaError_t e = persist_init(&G);
@@ -587,6 +587,10 @@ cudaError_t persist_setup(wf_handle *h, cudaStream_t s) {
   if (G > kMkMaxG) G = kMkMaxG;
   if (G < 4 * kMkRows) return cudaErrorInvalidConfiguration;
   const int d = h->d, F = h->F, H = h->H, T = h->cfg.enc_frames;
+  if (!persist_grid_fits(d, F, G)) {  // too few SMs for these widths: launch by launch only
+    h->mk_ok = false;
+    return cudaSuccess;
+  }
   const int nl = h->nl, nd = h->nd;
   std::vector<CUtensorMap> maps;
   std::vector<MkLayer> lys;

@@ -238,6 +238,9 @@ struct MkParams {
 size_t mk_xpart_words(int M, int H, int T);
 cudaError_t persist_init(int *G);
 bool persist_supported(int d, int H, int F, int T, int rows);
+// Whether a grid of G CTAs leaves at most five projection units per CTA and
+// phase (the persistent pass reduces one CTA's units in one batch).
+bool persist_grid_fits(int d, int F, int G);
 cudaError_t launch_persist(const MkParams &p, cudaStream_t s);
 
 }  // namespace wf

@@ -54,12 +54,13 @@ constexpr int kSlot = 20 * 1024;          // bytes per slot: one projection unit
                                           // K <= 1280) or 128 keys (or values) of one head
 constexpr int kKeysPerSlot = 128;
 constexpr int kScratch = 42 * 1024;       // operand tile, reductions, attention staging
-constexpr int kUB = 4;                    // projection units reduced together
+constexpr int kUB = 5;                    // projection units per CTA and phase (at most)
 constexpr int kKS = 10;                   // k16-steps per warp: operand width <= 1280
 constexpr int kQ2 = 4;                    // fc2 split-K factor (partials add in order)
 constexpr int kPS = 68;                   // attention partial: m, l, -, -, o[64] (o 16-byte aligned)
 constexpr long long kMkSpin = 400000000LL;  // cycles before a wait gives up (~0.2 s)
-constexpr int kSmemMk = 1024 + kNS * kSlot + kScratch + 2 * kNS * 8 + 2048;
+constexpr int kLnGB = 2 * 1280 * 2;        // LayerNorm gain and bias (bf16, d <= 1280)
+constexpr int kSmemMk = 1024 + kNS * kSlot + kScratch + kLnGB + 2 * kNS * 8 + 2048;
 
 enum : int { PH_QKV = 0, PH_SATT, PH_OUT, PH_XQ, PH_XATT, PH_XOUT, PH_FC1, PH_FC2 };
 
@@ -84,9 +85,37 @@ __device__ __forceinline__ void add_release(uint32_t *ptr, uint32_t v) {
   cuda::atomic_ref<uint32_t, cuda::thread_scope_device> r(*ptr);
   r.fetch_add(v, cuda::memory_order_release);
 }
-__device__ __forceinline__ uint32_t ldcg_u32(const void *ptr) { return __ldcg(static_cast<const unsigned int *>(ptr)); }
-__device__ __forceinline__ float ldcg_f32(const float *ptr) { return __ldcg(ptr); }
 __device__ __forceinline__ uint4 ldcg_u128(const void *ptr) { return __ldcg(static_cast<const uint4 *>(ptr)); }
+__device__ __forceinline__ void ldcg_f32x4x5(float4 *v, const float4 *p0, const float4 *p1, const float4 *p2,
+                                             const float4 *p3, const float4 *p4) {
+  asm volatile(
+      "ld.global.cg.v4.f32 {%0, %1, %2, %3}, [%20];\n\t"
+      "ld.global.cg.v4.f32 {%4, %5, %6, %7}, [%21];\n\t"
+      "ld.global.cg.v4.f32 {%8, %9, %10, %11}, [%22];\n\t"
+      "ld.global.cg.v4.f32 {%12, %13, %14, %15}, [%23];\n\t"
+      "ld.global.cg.v4.f32 {%16, %17, %18, %19}, [%24];"
+      : "=f"(v[0].x), "=f"(v[0].y), "=f"(v[0].z), "=f"(v[0].w), "=f"(v[1].x), "=f"(v[1].y), "=f"(v[1].z),
+        "=f"(v[1].w), "=f"(v[2].x), "=f"(v[2].y), "=f"(v[2].z), "=f"(v[2].w), "=f"(v[3].x), "=f"(v[3].y),
+        "=f"(v[3].z), "=f"(v[3].w), "=f"(v[4].x), "=f"(v[4].y), "=f"(v[4].z), "=f"(v[4].w)
+      : "l"(p0), "l"(p1), "l"(p2), "l"(p3), "l"(p4)
+      : "memory");
+}
+// Five 16-byte loads (L2, not L1) in one statement, so that they issue back
+// to back: the scheduler may not put a use of the first between them.
+__device__ __forceinline__ void ldcg_u128x5(uint4 (&v)[5], const void *p0, const void *p1, const void *p2,
+                                            const void *p3, const void *p4) {
+  asm volatile(
+      "ld.global.cg.v4.u32 {%0, %1, %2, %3}, [%20];\n\t"
+      "ld.global.cg.v4.u32 {%4, %5, %6, %7}, [%21];\n\t"
+      "ld.global.cg.v4.u32 {%8, %9, %10, %11}, [%22];\n\t"
+      "ld.global.cg.v4.u32 {%12, %13, %14, %15}, [%23];\n\t"
+      "ld.global.cg.v4.u32 {%16, %17, %18, %19}, [%24];"
+      : "=r"(v[0].x), "=r"(v[0].y), "=r"(v[0].z), "=r"(v[0].w), "=r"(v[1].x), "=r"(v[1].y), "=r"(v[1].z),
+        "=r"(v[1].w), "=r"(v[2].x), "=r"(v[2].y), "=r"(v[2].z), "=r"(v[2].w), "=r"(v[3].x), "=r"(v[3].y),
+        "=r"(v[3].z), "=r"(v[3].w), "=r"(v[4].x), "=r"(v[4].y), "=r"(v[4].z), "=r"(v[4].w)
+      : "l"(p0), "l"(p1), "l"(p2), "l"(p3), "l"(p4)
+      : "memory");
+}
 __device__ __forceinline__ int seq_of(int b, int ph) { return 1 + b * kMkPhases + ph; }
 
 // Bounded spin: gives up (recording WF_DEV_ERR_TIMEOUT) after kMkSpin cycles,
@@ -117,6 +146,17 @@ __device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, uint32_
   Spin sp;
   while (!mbar_try_wait(bar, parity))
     if (!sp.again(err)) return false;
+  return true;
+}
+// The producer's wait for a free slot backs off between tries: it shares a
+// scheduler with two compute warps and must not take their issue slots.
+__device__ __forceinline__ bool wait_bar_idle(uint64_t *bar, uint32_t parity, uint32_t *err) {
+  if (mbar_try_wait(bar, parity)) return true;
+  Spin sp;
+  while (!mbar_try_wait(bar, parity)) {
+    if (!sp.again(err)) return false;
+    __nanosleep(64);
+  }
   return true;
 }
 // 3-D tiled bulk-tensor load (a whole projection unit) into shared memory.
@@ -168,17 +208,14 @@ __device__ __forceinline__ bool is_gemm(int ph) { return ph != PH_SATT && ph != 
 // Shared memory: the ring, the scratch area, the ring's mbarriers and a few
 // per-CTA values, at fixed offsets from one 1024-aligned base.
 constexpr int kOffScratch = kNS * kSlot;
-constexpr int kOffFull = kOffScratch + kScratch;
+constexpr int kOffLnGB = kOffScratch + kScratch;
+constexpr int kOffFull = kOffLnGB + kLnGB;
 constexpr int kOffEmpty = kOffFull + kNS * 8;
 constexpr int kOffNk = kOffEmpty + kNS * 8;                 // int[kMkMaxSeq]
 constexpr int kOffSlot = kOffNk + kMkMaxSeq * 4;            // int[kMkMaxSeq]
-constexpr int kLnRedW = 32;                                 // floats per warp in lnred
-constexpr int kOffLnRed = kOffSlot + kMkMaxSeq * 4;         // float[kW][kLnRedW]
-constexpr int kOffLnM = kOffLnRed + kW * kLnRedW * 4;       // float[kMkRows]
-constexpr int kOffLnR = kOffLnM + kMkRows * 4;              // float[kMkRows]
-constexpr int kOffEpoch = kOffLnR + kMkRows * 4;            // uint32
-constexpr int kOffZero = (kOffEpoch + 16 + 15) / 16 * 16;   // 16 zero bytes (operand rows >= M)
-constexpr int kSmemUsed = kOffZero + 16;
+constexpr int kOffZero = (kOffSlot + kMkMaxSeq * 4 + 15) / 16 * 16;  // 16 zero bytes (operand rows >= M)
+constexpr int kOffParams = kOffZero + 16;                  // MkParams (a copy of the launch's)
+constexpr int kSmemUsed = kOffParams + (static_cast<int>(sizeof(MkParams)) + 15) / 16 * 16;
 static_assert(kSmemUsed + 1024 <= kSmemMk, "shared-memory plan");
 struct Smem {
   uint8_t *base;
@@ -188,10 +225,9 @@ struct Smem {
   __device__ __forceinline__ uint64_t *empty(int s) const { return reinterpret_cast<uint64_t *>(base + kOffEmpty) + s; }
   __device__ __forceinline__ int *nk() const { return reinterpret_cast<int *>(base + kOffNk); }
   __device__ __forceinline__ int *slot() const { return reinterpret_cast<int *>(base + kOffSlot); }
-  __device__ __forceinline__ float *lnred() const { return reinterpret_cast<float *>(base + kOffLnRed); }
-  __device__ __forceinline__ float *lnm() const { return reinterpret_cast<float *>(base + kOffLnM); }
-  __device__ __forceinline__ float *lnr() const { return reinterpret_cast<float *>(base + kOffLnR); }
   __device__ __forceinline__ uint8_t *zero16() const { return base + kOffZero; }
+  __device__ __forceinline__ bf16 *lngb() const { return reinterpret_cast<bf16 *>(base + kOffLnGB); }
+  __device__ __forceinline__ MkParams *params() const { return reinterpret_cast<MkParams *>(base + kOffParams); }
 };
 
 // ------------------------------------------------------------ producer ----
@@ -200,7 +236,7 @@ __device__ void producer(const MkParams &p, const Smem sm, int c) {
   bool ok = true;
   auto acquire = [&](uint32_t bytes, uint8_t *&dst, uint64_t *&bar) {
     const uint32_t s = sc % kNS, n = sc / kNS;
-    if (n > 0 && !wait_bar(sm.empty(s), (n - 1) & 1u, p.err)) {
+    if (n > 0 && !wait_bar_idle(sm.empty(s), (n - 1) & 1u, p.err)) {
       ok = false;
       return;
     }
@@ -388,91 +424,120 @@ struct Cons {
   // Warp w owns k16-steps s = w, w + 8, ... of the operand; lane (g, c4)
   // holds rows g and g + 8, columns 16s + 2c4 (+1, +8, +9) as in the
   // m16n8k16 A fragment.
-  // LayerNorm operand: rows of the residual (x_ln), statistics per row in a
-  // fixed order (lanes, then warps), then (x - mean) * rstd * g + b as bf16.
-  // LayerNorm operand: the bf16 tile LN(x)[t][k] for t < M is built in
-  // shared memory, then every warp reads its A fragments with ldmatrix.
-  // Thread tid owns elements k = tid + 256 e of every row, so each row's
-  // statistics reduce in one fixed order (elements, warp tree, warps in
-  // order) whatever M is: a row's result never depends on the other rows.
-  static constexpr int kLnRows = 9;   // rows normalised per pass
-  static constexpr int kLnElems = 5;  // elements per thread and row (d <= 1280)
-  __device__ __forceinline__ int tile_ld() const { return p.d + 8; }  // bf16 row stride (conflict-free ldmatrix)
-  __device__ __forceinline__ void ln_rows(int r_lo, int nr, const bf16 *lg, const bf16 *lb) {
-    bf16 *tile = reinterpret_cast<bf16 *>(sm.scratch());
-    const int ld = tile_ld();
-    float x[kLnRows][kLnElems];
-    // every load is unconditional (outside the rows: element tid of row
-    // r_lo) so all of them are in flight before any is used
+  // LayerNorm operand: LN(x) as a bf16 tile [M][d] in shared memory (rows
+  // >= M read zeros), from which every warp reads its A fragments with
+  // ldmatrix.  Warp w normalises rows w and w + 8; lane l holds float4s
+  // l + 32 j of a row, so a row's sums run in one fixed order (the lane's
+  // elements, then the shuffle tree, whose result is the same in every lane)
+  // whatever M is: a row's result never depends on the other rows.
+  static constexpr int kLnJ = 10;  // float4s per lane and row (d <= 1280)
+  // The LayerNorm's gain and bias go to shared memory before the phase
+  // waits: they do not depend on the previous phase.
+  __device__ __forceinline__ void stage_ln(const bf16 *lg, const bf16 *lb) {
+    uint4 *dst = reinterpret_cast<uint4 *>(sm.lngb());
+    const int n = p.d / 8;
+    for (int i = tid; i < 2 * n; i += kCThr)
+      dst[i] = i < n ? __ldg(reinterpret_cast<const uint4 *>(lg) + i)
+                     : __ldg(reinterpret_cast<const uint4 *>(lb) + (i - n));
+  }
+  // Four independent running sums (one per float4 component), added in a
+  // fixed order: short dependency chains, same result for any M.
+  __device__ __forceinline__ float2 row_stats(const float4 (&v)[kLnJ], int nj, float inv_d, float eps) const {
+    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
 #pragma unroll
-    for (int r = 0; r < kLnRows; ++r) {
-#pragma unroll
-      for (int e = 0; e < kLnElems; ++e) {
-        const int k = tid + kCThr * e;
-        const bool valid = r < nr && k < p.d;
-        x[r][e] = ldcg_f32(p.x + (valid ? (r_lo + r) * p.d + k : r_lo * p.d + tid % p.d));
+    for (int j = 0; j < kLnJ; ++j) {
+      if (j < nj) {
+        s0 += v[j].x;
+        s1 += v[j].y;
+        s2 += v[j].z;
+        s3 += v[j].w;
       }
     }
+    const float mean = warp_sum((s0 + s1) + (s2 + s3)) * inv_d;
+    float q0 = 0.f, q1 = 0.f, q2 = 0.f, q3 = 0.f;
 #pragma unroll
-    for (int r = 0; r < kLnRows; ++r) {
-#pragma unroll
-      for (int e = 0; e < kLnElems; ++e)
-        if (!(r < nr && tid + kCThr * e < p.d)) x[r][e] = 0.f;
-    }
-    const float inv_d = 1.0f / static_cast<float>(p.d);
-#pragma unroll
-    for (int r = 0; r < kLnRows; ++r) {
-      float s = 0.f;
-#pragma unroll
-      for (int e = 0; e < kLnElems; ++e) s += x[r][e];
-      s = warp_sum(s);
-      if (lane == 0) sm.lnred()[warp * kLnRedW + r] = s;
-    }
-    cbar();
-    if (tid < nr) {
-      float s = 0.f;
-#pragma unroll
-      for (int w = 0; w < kW; ++w) s += sm.lnred()[w * kLnRedW + tid];
-      sm.lnm()[tid] = s * inv_d;
-    }
-    cbar();
-    float mean[kLnRows];
-#pragma unroll
-    for (int r = 0; r < kLnRows; ++r) {
-      mean[r] = sm.lnm()[r];
-      float q = 0.f;
-#pragma unroll
-      for (int e = 0; e < kLnElems; ++e) {
-        const int k = tid + kCThr * e;
-        const float dv = (k < p.d) ? x[r][e] - mean[r] : 0.f;
-        q += dv * dv;
+    for (int j = 0; j < kLnJ; ++j) {
+      if (j < nj) {
+        const float a = v[j].x - mean, b = v[j].y - mean, c2 = v[j].z - mean, d2 = v[j].w - mean;
+        q0 = __fmaf_rn(a, a, q0);
+        q1 = __fmaf_rn(b, b, q1);
+        q2 = __fmaf_rn(c2, c2, q2);
+        q3 = __fmaf_rn(d2, d2, q3);
       }
-      q = warp_sum(q);
-      if (lane == 0) sm.lnred()[warp * kLnRedW + kLnRows + r] = q;
     }
-    cbar();
-    if (tid < nr) {
-      float s = 0.f;
+    return make_float2(mean, rsqrtf(__fadd_rn(warp_sum((q0 + q1) + (q2 + q3)) * inv_d, eps)));
+  }
+  __device__ __forceinline__ void row_out(bf16 *trow, const float4 (&v)[kLnJ], int nj, float2 ms) const {
+    const bf16 *g = sm.lngb(), *bb = sm.lngb() + p.d;
 #pragma unroll
-      for (int w = 0; w < kW; ++w) s += sm.lnred()[w * kLnRedW + kLnRows + tid];
-      sm.lnr()[tid] = rsqrtf(__fadd_rn(s * inv_d, p.eps));
-    }
-    cbar();
-#pragma unroll
-    for (int e = 0; e < kLnElems; ++e) {
-      const int k = tid + kCThr * e;
-      if (k >= p.d) continue;
-      const float gk = bf2f(lg[k]), bk = bf2f(lb[k]);
-#pragma unroll
-      for (int r = 0; r < kLnRows; ++r)
-        if (r < nr)
-          tile[(r_lo + r) * ld + k] = __float2bfloat16(ln_apply(x[r][e], make_float2(mean[r], sm.lnr()[r]), gk, bk));
+    for (int j = 0; j < kLnJ; ++j) {
+      if (j < nj) {
+        const int col = 4 * (lane + 32 * j);
+        const uint2 gr = *reinterpret_cast<const uint2 *>(g + col);
+        const uint2 br = *reinterpret_cast<const uint2 *>(bb + col);
+        const bf16 *ge = reinterpret_cast<const bf16 *>(&gr);
+        const bf16 *be = reinterpret_cast<const bf16 *>(&br);
+        uint2 o;
+        o.x = pack_bf16(ln_apply(v[j].x, ms, bf2f(ge[0]), bf2f(be[0])), ln_apply(v[j].y, ms, bf2f(ge[1]), bf2f(be[1])));
+        o.y = pack_bf16(ln_apply(v[j].z, ms, bf2f(ge[2]), bf2f(be[2])), ln_apply(v[j].w, ms, bf2f(ge[3]), bf2f(be[3])));
+        *reinterpret_cast<uint2 *>(trow + col) = o;
+      }
     }
   }
-  // A fragments of k-steps s = w + 8 j from the shared tile (rows >= M read zeros).
-  __device__ __forceinline__ void tile_frags(uint32_t (&a)[kKS][4], int nks) {
+  // Row t of the residual: lane l's float4s l + 32 j, j < nj (those past the
+  // row repeat its last and are never used), all ten loads in flight at once.
+  __device__ __forceinline__ void load_row(float4 (&v)[kLnJ], int t, int nj) const {
+    static_assert(kLnJ == 10, "two groups of five loads");
+    const float4 *xr = reinterpret_cast<const float4 *>(p.x + static_cast<size_t>(t) * p.d) + lane;
+    auto at = [&](int j) { return xr + 32 * min(j, nj - 1); };
+    ldcg_f32x4x5(v, at(0), at(1), at(2), at(3), at(4));
+    ldcg_f32x4x5(v + 5, at(5), at(6), at(7), at(8), at(9));
+  }
+  __device__ __forceinline__ void ln_tile() {
+    static_assert(kMkRows <= 2 * kW, "two rows per warp at most");
+    if (warp >= p.M) return;
+    bf16 *tile = reinterpret_cast<bf16 *>(sm.scratch());
+    const int nj = p.d / 128, ld = p.d + 8, t1 = warp + kW;
+    const float inv_d = 1.0f / static_cast<float>(p.d), eps = p.eps;
+    float4 v0[kLnJ], v1[kLnJ];
+    load_row(v0, warp, nj);
+    // both rows in flight together (a lone row loads itself twice), and
+    // both statistics computed side by side
+    load_row(v1, t1 < p.M ? t1 : warp, nj);
+    const float2 ms0 = row_stats(v0, nj, inv_d, eps), ms1 = row_stats(v1, nj, inv_d, eps);
+    row_out(tile + warp * ld, v0, nj, ms0);
+    if (t1 < p.M) row_out(tile + t1 * ld, v1, nj, ms1);
+  }
+  // bf16 operand: rows [0, M), columns [k0, k0 + Kp) of buf (row stride
+  // cols) copied into the tile with 16-byte loads, warp w taking rows w and
+  // w + 8, every load in flight before the first store.
+  static constexpr int kPlainJ = 5;  // uint4 per lane and row (Kp <= 1280)
+  __device__ __forceinline__ void plain_tile(const bf16 *buf, int cols, int k0, int Kp) {
+    if (warp >= p.M) return;
+    bf16 *tile = reinterpret_cast<bf16 *>(sm.scratch());
+    const int ld = Kp + 8, per = Kp / 8;
+    const int r1 = warp + 8 < p.M ? warp + 8 : warp;
+    const bf16 *s0 = buf + static_cast<size_t>(warp) * cols + k0;
+    const bf16 *s1 = buf + static_cast<size_t>(r1) * cols + k0;
+    static_assert(kPlainJ == 5, "five loads per row");
+    // columns past the row read its last chunk (valid) and are not stored
+    auto col = [&](int j) { return 8 * min(lane + 32 * j, per - 1); };
+    uint4 v0[kPlainJ], v1[kPlainJ];
+    ldcg_u128x5(v0, s0 + col(0), s0 + col(1), s0 + col(2), s0 + col(3), s0 + col(4));
+    ldcg_u128x5(v1, s1 + col(0), s1 + col(1), s1 + col(2), s1 + col(3), s1 + col(4));
+#pragma unroll
+    for (int j = 0; j < kPlainJ; ++j) {
+      const int q = lane + 32 * j;
+      if (q < per) {
+        *reinterpret_cast<uint4 *>(tile + warp * ld + 8 * q) = v0[j];
+        if (r1 != warp) *reinterpret_cast<uint4 *>(tile + r1 * ld + 8 * q) = v1[j];
+      }
+    }
+  }
+  // A fragments of k-steps s = w + 8 j from the shared tile of row stride ld
+  // (rows >= M read zeros).
+  __device__ __forceinline__ void tile_frags(uint32_t (&a)[kKS][4], int nks, int ld) {
     const bf16 *tile = reinterpret_cast<const bf16 *>(sm.scratch());
-    const int ld = tile_ld();
     const int row = lane & 15, koff = (lane >> 4) * 8;
     const uint32_t rbase = row < p.M ? smem_u32(tile + row * ld + 16 * warp + koff) : smem_u32(sm.zero16());
     const uint32_t rstep = row < p.M ? 256u : 0u;  // 128 bf16 per j
@@ -482,46 +547,11 @@ struct Cons {
       ldsm_x4(rbase + rstep * j, a[j][0], a[j][1], a[j][2], a[j][3]);
     }
   }
-  __device__ __forceinline__ void ln_frags(uint32_t (&a)[kKS][4], int nks, const bf16 *lg, const bf16 *lb) {
-    for (int r0 = 0; r0 < p.M; r0 += kLnRows) {
-      ln_rows(r0, min(kLnRows, p.M - r0), lg, lb);
-      cbar();  // the statistics scratch is reused by the next group of rows
-    }
-    tile_frags(a, nks);
-    cbar();  // the reduction buffer of the projection overlaps the tile
-  }
-
-  // bf16 operand X[t][k] (row stride cols), columns [k0, k0 + Kp): each
-  // lane loads its m16n8k16 A fragments (bf16 pairs) directly from L2.
-  __device__ __forceinline__ void plain_frags(uint32_t (&a)[kKS][4], int nks, const bf16 *buf, int cols,
-                                              int k0) {
-    const int gr = lane >> 2, c4 = lane & 3;
-    const int r0 = gr, r1 = gr + 8;
-    const bool v0 = r0 < p.M, v1 = r1 < p.M;
-    // rows past M read row 0 (always valid) and are zeroed afterwards, so
-    // every load is in flight before any is used
-    const bf16 *b0 = buf + (v0 ? r0 : 0) * cols + k0 + 16 * warp + 2 * c4;
-    const bf16 *b1 = buf + (v1 ? r1 : 0) * cols + k0 + 16 * warp + 2 * c4;
-#pragma unroll
-    for (int j = 0; j < kKS; ++j) {
-      if (j >= nks) continue;
-      a[j][0] = ldcg_u32(b0 + 128 * j);
-      a[j][1] = ldcg_u32(b1 + 128 * j);
-      a[j][2] = ldcg_u32(b0 + 128 * j + 8);
-      a[j][3] = ldcg_u32(b1 + 128 * j + 8);
-    }
-#pragma unroll
-    for (int j = 0; j < kKS; ++j) {
-      if (!v0) a[j][0] = a[j][2] = 0u;
-      if (!v1) a[j][1] = a[j][3] = 0u;
-    }
-  }
 
   // ------------------------------------------------------- projections ----
   // Phases are separate (non-inlined) functions: inlined into the block loop
   // their live ranges add up past the register budget of a 288-thread CTA.
-  template <int PH>
-  __device__ __noinline__ void gemm_phase(int b) {
+  __device__ __noinline__ void gemm_phase(int b, const int PH) {
     refresh();
     const int U = units_of(p, PH);
     const int u0 = first_unit(p, b, PH, c);
@@ -530,21 +560,46 @@ struct Cons {
       arrive(s);
       return;
     }
-    wait_phase(s - 1);
     const MkLayer &ly = p.layers[b];
+    const bool ln = PH == PH_QKV || PH == PH_XQ || PH == PH_FC1;
+    if (ln)
+      stage_ln(PH == PH_QKV ? ly.ln1_g : PH == PH_XQ ? ly.ln2_g : ly.ln3_g,
+               PH == PH_QKV ? ly.ln1_b : PH == PH_XQ ? ly.ln2_b : ly.ln3_b);
+    // Thread tid finishes unit u0 + (tid / 32) G (if any): its bias pair is
+    // loaded before the wait, the residual it updates right after it, both
+    // in the shadow of the operand loads.
+    const int eu = u0 + (tid >> 5) * p.G;
+    const bool epi = (tid >> 5) < kUB && eu < U;
+    const int en0 = 8 * (PH == PH_FC2 ? eu / kQ2 : eu) + 2 * (lane & 3);
+    const bool resid = PH == PH_OUT || PH == PH_XOUT || (PH == PH_FC2 && u0 % kQ2 == 0);
+    uint32_t bias2 = 0u;
+    if (epi && (PH != PH_FC2 || resid)) {
+      const bf16 *bias = PH == PH_QKV ? ly.qkv_b : PH == PH_OUT ? ly.out_b : PH == PH_XQ ? ly.xq_b
+                       : PH == PH_XOUT ? ly.xout_b : PH == PH_FC1 ? ly.fc1_b : ly.fc2_b;
+      bias2 = __ldg(reinterpret_cast<const unsigned int *>(bias + en0));
+    }
+    wait_phase(s - 1);  // its barrier also publishes the staged gain and bias
+    float2 old[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+    if (epi && resid) {
+#pragma unroll
+      for (int hr = 0; hr < 2; ++hr) {
+        const int t = (lane >> 2) + 8 * hr;
+        if (t < p.M) old[hr] = __ldcg(reinterpret_cast<const float2 *>(p.x + static_cast<size_t>(t) * p.d + en0));
+      }
+    }
     const int Kp = PH == PH_FC2 ? fc2_k(p) : p.d;
     const int nks = Kp / 128;  // k16-steps per warp
     const int nslot = (Kp + 255) / 256;
     uint32_t a[kKS][4];
-    if constexpr (PH == PH_QKV) ln_frags(a, nks, ly.ln1_g, ly.ln1_b);
-    if constexpr (PH == PH_XQ) ln_frags(a, nks, ly.ln2_g, ly.ln2_b);
-    if constexpr (PH == PH_FC1) ln_frags(a, nks, ly.ln3_g, ly.ln3_b);
-    if constexpr (PH == PH_OUT) plain_frags(a, nks, p.att_x, p.d, 0);
-    if constexpr (PH == PH_XOUT) plain_frags(a, nks, p.xatt_x, p.d, 0);
-    // G is a multiple of the split (checked at launch), so every fc2 unit of
-    // this CTA reads the same quarter of the fc1 output
-    if constexpr (PH == PH_FC2)
-      plain_frags(a, nks, p.h_x, p.F, (u0 % kQ2) * fc2_k(p));
+    if (ln)
+      ln_tile();
+    else  // G is a multiple of the fc2 split (checked at launch), so every fc2
+          // unit of this CTA reads the same quarter of the fc1 output
+      plain_tile(PH == PH_OUT ? p.att_x : PH == PH_XOUT ? p.xatt_x : p.h_x, PH == PH_FC2 ? p.F : p.d,
+                 PH == PH_FC2 ? (u0 % kQ2) * Kp : 0, Kp);
+    cbar();
+    tile_frags(a, nks, Kp + 8);
+    cbar();  // the reduction buffer of the projection overlaps the tile
     // ldmatrix addressing inside a unit: k-block atoms of [8 rows][64] bf16,
     // 128-byte swizzled; warp w's k-steps 16m + w and 16m + w + 8 sit in the
     // 4 KB (four k-blocks) at 4096 m
@@ -553,7 +608,8 @@ struct Cons {
     const int ch = 2 * (warp & 3) + (mi & 1);
     const uint32_t ld_off = static_cast<uint32_t>(kb * 1024 + lr * 128 + ((ch ^ lr) << 4));
     float4 *red = reinterpret_cast<float4 *>(sm.scratch());
-    for (int ub = u0; ub < U; ub += kUB * p.G) {
+    {  // every unit of the CTA in one batch (at most kUB, checked at launch)
+      const int ub = u0;
       float acc[kUB][4];
       int nb = 0;
 #pragma unroll
@@ -579,7 +635,7 @@ struct Cons {
       for (int k = 0; k < kUB; ++k)
         if (k < nb) red[(k * kW + warp) * 32 + lane] = make_float4(acc[k][0], acc[k][1], acc[k][2], acc[k][3]);
       cbar();
-      if constexpr (PH == PH_FC2) {
+      if (PH == PH_FC2) {
         // a quarter-0 unit owns the output: wait for the other quarters'
         // partials (every fc2 unit of this CTA has the same quarter)
         if (u0 % kQ2 == 0) {
@@ -600,10 +656,10 @@ struct Cons {
           v.z += o.z;
           v.w += o.w;
         }
-        epilogue<PH>(b, ly, ub + k * p.G, ln, v);
+        epilogue(PH, b, ly, ub + k * p.G, ln, v, bias2, old);
       }
       cbar();
-      if constexpr (PH == PH_FC2) {  // partials of quarters 1..3 are published
+      if (PH == PH_FC2) {  // partials of quarters 1..3 are published
         if (u0 % kQ2 != 0 && tid == 0)
           for (int k = 0; k < nb; ++k) add_release(p.cnt2 + (ub + k * p.G) / kQ2, 1u);
       }
@@ -612,8 +668,9 @@ struct Cons {
   }
 
   // D fragment of one unit: rows g, g+8; columns n0, n0+1 (n0 = 8 ru + 2 c4).
-  template <int PH>
-  __device__ __forceinline__ void epilogue(int b, const MkLayer &ly, int u, int ln, float4 v) {
+  __device__ __forceinline__ void epilogue(const int PH, int b, const MkLayer &ly, int u, int ln, float4 v,
+                                          uint32_t bias2, const float2 (&old)[2]) {
+    const float bias0 = __uint_as_float(bias2 << 16), bias1 = __uint_as_float(bias2 & 0xffff0000u);
     const int gr = ln >> 2, c4 = ln & 3;
     const int ru = PH == PH_FC2 ? u / kQ2 : u;
     const int n0 = 8 * ru + 2 * c4;
@@ -623,9 +680,9 @@ struct Cons {
       const int t = gr + 8 * hr;
       if (t >= p.M) continue;
       float y0 = vals[hr][0], y1 = vals[hr][1];
-      if constexpr (PH == PH_QKV) {
-        y0 += bf2f(ly.qkv_b[n0]);
-        y1 += bf2f(ly.qkv_b[n0 + 1]);
+      if (PH == PH_QKV) {
+        y0 += bias0;
+        y1 += bias1;
         const uint32_t pr = pack_bf16(y0, y1);
         if (n0 < p.d) {
           *reinterpret_cast<uint32_t *>(p.q_x + t * p.d + n0) = pr;
@@ -645,18 +702,17 @@ struct Cons {
             set_error(p.err, WF_DEV_ERR_CAPACITY);
           }
         }
-      } else if constexpr (PH == PH_XQ) {
-        y0 += bf2f(ly.xq_b[n0]);
-        y1 += bf2f(ly.xq_b[n0 + 1]);
+      } else if (PH == PH_XQ) {
+        y0 += bias0;
+        y1 += bias1;
         *reinterpret_cast<uint32_t *>(p.xq_x + t * p.d + n0) = pack_bf16(y0, y1);
-      } else if constexpr (PH == PH_FC1) {
-        y0 = gelu_erf(y0 + bf2f(ly.fc1_b[n0]));
-        y1 = gelu_erf(y1 + bf2f(ly.fc1_b[n0 + 1]));
+      } else if (PH == PH_FC1) {
+        y0 = gelu_erf(y0 + bias0);
+        y1 = gelu_erf(y1 + bias1);
         *reinterpret_cast<uint32_t *>(p.h_x + t * p.F + n0) = pack_bf16(y0, y1);
       } else {
         // residual updates: OUT, XOUT, FC2
-        const bf16 *bias = PH == PH_OUT ? ly.out_b : PH == PH_XOUT ? ly.xout_b : ly.fc2_b;
-        if constexpr (PH == PH_FC2) {
+        if (PH == PH_FC2) {
           const int q = u % kQ2;
           float *pp = p.part2 + (static_cast<size_t>(ru) * (kQ2 - 1) * kMkRows) * 8;
           if (q != 0) {
@@ -672,11 +728,10 @@ struct Cons {
           }
         }
         float *xo = p.x + static_cast<size_t>(t) * p.d + n0;
-        const float2 old = __ldcg(reinterpret_cast<const float2 *>(xo));
-        const float x0 = old.x + (y0 + bf2f(bias[n0]));
-        const float x1 = old.y + (y1 + bf2f(bias[n0 + 1]));
+        const float x0 = old[hr].x + (y0 + bias0);
+        const float x1 = old[hr].y + (y1 + bias1);
         *reinterpret_cast<float2 *>(xo) = make_float2(x0, x1);
-        if constexpr (PH == PH_FC2) {
+        if (PH == PH_FC2) {
           if (p.write_taps) {
             const uint32_t pr = pack_bf16(x0, x1);
 #pragma unroll
@@ -695,11 +750,18 @@ struct Cons {
   __device__ __forceinline__ uint8_t *sQ() const { return sm.scratch(); }
   __device__ __forceinline__ float *sMax() const { return reinterpret_cast<float *>(sm.scratch() + 2048); }
   __device__ __forceinline__ float *sSum() const { return reinterpret_cast<float *>(sm.scratch() + 2560); }
+  // per-warp O partials, rows padded to 72 floats: the fragment stores of
+  // one half-warp fall in distinct banks
+  static constexpr int kOLd = 72;
+  static_assert(3072 + kW * 16 * kOLd * 4 <= kScratch, "attention scratch");
+  // Scores are kept in base-2 units (times log2 e), so every weight of the
+  // softmax, and of the merges of partial results, is one exp2.
+  static constexpr float kLog2e = 1.4426950408889634f;
   __device__ __forceinline__ float *sO() const { return reinterpret_cast<float *>(sm.scratch() + 3072); }
 
   // Query rows of unit (sequence i, head h) of buf [rows][d], scaled by
   // 1/8 = 1/sqrt(64) after RoPE (drafter) in fp32.
-  __device__ __forceinline__ void load_q(const bf16 *buf, int i, int h, int base, bool rope) {
+  __device__ __noinline__ void load_q(const bf16 *buf, int i, int h, int base, bool rope) {
     if (tid < 16 * 8) {
       const int r = tid >> 3, chq = tid & 7;
       uint4 raw = make_uint4(0u, 0u, 0u, 0u), par = make_uint4(0u, 0u, 0u, 0u);
@@ -735,7 +797,7 @@ struct Cons {
   // at absolute positions key0 .. key0 + 31; a key is visible when
   // pos < nk and, for causal rows, pos <= cbase + row.  Leaves the warp's
   // (m, l, O) in scratch.
-  __device__ __forceinline__ void attn_warp(bool active, uint32_t k_u32, uint32_t v_u32, int key0, int nk, int nq,
+  __device__ __noinline__ void attn_warp(bool active, uint32_t k_u32, uint32_t v_u32, int key0, int nk, int nq,
                             int cbase) {
     float *smx = sMax(), *ssm = sSum(), *so = sO();
     const int gq = lane >> 2, c4 = lane & 3;
@@ -748,9 +810,10 @@ struct Cons {
       }
 #pragma unroll
       for (int nd = 0; nd < 8; ++nd) {
-        float *o0 = so + (warp * 16 + gq) * 64 + nd * 8 + c4 * 2;
-        float *o1 = so + (warp * 16 + gq + 8) * 64 + nd * 8 + c4 * 2;
-        o0[0] = o0[1] = o1[0] = o1[1] = 0.f;
+        float *o0 = so + (warp * 16 + gq) * kOLd + nd * 8 + c4 * 2;
+        float *o1 = so + (warp * 16 + gq + 8) * kOLd + nd * 8 + c4 * 2;
+        *reinterpret_cast<float2 *>(o0) = make_float2(0.f, 0.f);
+        *reinterpret_cast<float2 *>(o1) = make_float2(0.f, 0.f);
       }
       return;
     }
@@ -780,7 +843,7 @@ struct Cons {
         const int pos = key0 + nt * 8 + c4 * 2 + (e & 1);
         bool vis = row < nq && pos < nk;
         if (cbase >= 0) vis = vis && pos <= cbase + row;
-        s[nt][e] = vis ? s[nt][e] : -INFINITY;
+        s[nt][e] = vis ? s[nt][e] * kLog2e : -INFINITY;  // base-2 logits
         mrow[e >> 1] = fmaxf(mrow[e >> 1], s[nt][e]);
       }
     }
@@ -794,7 +857,7 @@ struct Cons {
     for (int nt = 0; nt < 4; ++nt) {
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
-        const float v = s[nt][e] == -INFINITY ? 0.f : expf(s[nt][e] - mrow[e >> 1]);
+        const float v = s[nt][e] == -INFINITY ? 0.f : exp2f(s[nt][e] - mrow[e >> 1]);
         s[nt][e] = v;
         lrow[e >> 1] += v;
       }
@@ -830,12 +893,10 @@ struct Cons {
     }
 #pragma unroll
     for (int nd = 0; nd < 8; ++nd) {
-      float *o0 = so + (warp * 16 + gq) * 64 + nd * 8 + c4 * 2;
-      float *o1 = so + (warp * 16 + gq + 8) * 64 + nd * 8 + c4 * 2;
-      o0[0] = o[nd][0];
-      o0[1] = o[nd][1];
-      o1[0] = o[nd][2];
-      o1[1] = o[nd][3];
+      float *o0 = so + (warp * 16 + gq) * kOLd + nd * 8 + c4 * 2;
+      float *o1 = so + (warp * 16 + gq + 8) * kOLd + nd * 8 + c4 * 2;
+      *reinterpret_cast<float2 *>(o0) = make_float2(o[nd][0], o[nd][1]);
+      *reinterpret_cast<float2 *>(o1) = make_float2(o[nd][2], o[nd][3]);
     }
   }
 
@@ -852,18 +913,18 @@ struct Cons {
 #pragma unroll
     for (int w = 0; w < kW; ++w) {
       const float mw = smx[w * 16 + qi];
-      const float wt = (mw == -INFINITY) ? 0.f : expf(mw - M);
+      const float wt = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
       L += ssm[w * 16 + qi] * wt;
 #pragma unroll
-      for (int e = 0; e < 4; ++e) acc[e] += so[(w * 16 + qi) * 64 + d0 + e] * wt;
+      for (int e = 0; e < 4; ++e) acc[e] += so[(w * 16 + qi) * kOLd + d0 + e] * wt;
     }
   }
   // (Mr, Lr, ar) <- merge with (M, L, a), earlier block first.
   __device__ __forceinline__ static void merge(float &Mr, float &Lr, float (&ar)[4], float M, float L,
                                                const float (&a)[4]) {
     const float MM = fmaxf(Mr, M);
-    const float wr = (Mr == -INFINITY) ? 0.f : expf(Mr - MM);
-    const float wc = (M == -INFINITY) ? 0.f : expf(M - MM);
+    const float wr = (Mr == -INFINITY) ? 0.f : exp2f(Mr - MM);
+    const float wc = (M == -INFINITY) ? 0.f : exp2f(M - MM);
     Lr = __fmaf_rn(L, wc, Lr * wr);
 #pragma unroll
     for (int e = 0; e < 4; ++e) ar[e] = __fmaf_rn(a[e], wc, ar[e] * wr);
@@ -899,22 +960,36 @@ struct Cons {
       const int nk = sm.nk()[i];
       const int base = nk - p.rps;
       float Mr = -INFINITY, Lr = 0.f, ar[4] = {0.f, 0.f, 0.f, 0.f};
-      if (nk > 0) load_q(p.q_x, i, h, base, rope);
       const bf16 *kcache = p.kc + (static_cast<size_t>(p.layers[b].self_layer * p.Bmax + sm.slot()[i]) * p.H + h) * p.ctx * 64;
       const bf16 *vcache = p.vc + (kcache - p.kc);
+      // This step's rows (positions base .. nk-1) were written by the
+      // projection in this pass (the prefetched slots hold stale copies):
+      // item tid + 256 r is (row jr, keys or values, 16-byte chunk chv),
+      // fetched together with the queries.
+      static_assert(kMkRows * 16 <= 2 * kCThr, "two fresh-row items per thread");
+      uint4 fresh[2];
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        const int idx = tid + r * kCThr;
+        if (nk > 0 && idx < p.rps * 16) {
+          const int jr = idx >> 4, kv = (idx >> 3) & 1, chv = idx & 7;
+          fresh[r] = ldcg_u128((kv ? vcache : kcache) + static_cast<size_t>(base + jr) * 64 + chv * 8);
+        }
+      }
+      if (nk > 0) load_q(p.q_x, i, h, base, rope);
       for (int ch = 0; ch * 256 < nk; ++ch) {
         const int ng = min(8, (nk - ch * 256 + 31) / 32);
         const int nh = (ng + 3) / 4;  // 128-key halves holding visible keys
         for (int m = 0; m < 2 * nh; ++m) wait_slot(m);
-        // this step's rows (positions base .. nk-1) come from the projection
-        for (int idx = tid; idx < p.rps * 2 * 8; idx += kCThr) {
+#pragma unroll
+        for (int r2 = 0; r2 < 2; ++r2) {
+          const int idx = tid + r2 * kCThr;
+          if (idx >= p.rps * 16) continue;
           const int jr = idx >> 4, kv = (idx >> 3) & 1, chv = idx & 7;
           const int pos = base + jr;
           if (pos < ch * 256 || pos >= ch * 256 + 256) continue;
-          // written this phase by the projection; the prefetched copy is stale
-          const uint4 wv = ldcg_u128((kv ? vcache : kcache) + static_cast<size_t>(pos) * 64 + chv * 8);
           const int gi = (pos - ch * 256) >> 5, r = pos & 31;
-          *reinterpret_cast<uint4 *>((kv ? vgroup(gi, nh) : kgroup(gi)) + swz(r, chv)) = wv;
+          *reinterpret_cast<uint4 *>((kv ? vgroup(gi, nh) : kgroup(gi)) + swz(r, chv)) = fresh[r2];
         }
         if ((nk & 31) && nk <= ch * 256 + 256) zero_rows(vgroup(ng - 1, nh), nk & 31);
         cbar();
@@ -1040,48 +1115,13 @@ struct Cons {
   __device__ __noinline__ void final_ln() {
     const int t = c;
     if (t >= p.M) return;
-    wait_phase(seq_of(p.nl - 1, PH_FC2));
-    const int per = (p.d + kCThr - 1) / kCThr;  // <= 6 for d <= 1536
-    float xv[6];
-    float s = 0.f;
-#pragma unroll
-    for (int k = 0; k < 6; ++k) {
-      const int e = tid + k * kCThr;
-      xv[k] = (k < per && e < p.d) ? ldcg_f32(p.x + static_cast<size_t>(t) * p.d + e) : 0.f;
-      s += xv[k];
-    }
-    float *red = reinterpret_cast<float *>(sm.scratch());
-    s = warp_sum(s);
-    if (lane == 0) red[warp] = s;
-    cbar();
-    float tot = 0.f;
-#pragma unroll
-    for (int w = 0; w < kW; ++w) tot += red[w];
-    const float mean = tot / static_cast<float>(p.d);
-    cbar();
-    float q = 0.f;
-#pragma unroll
-    for (int k = 0; k < 6; ++k) {
-      const int e = tid + k * kCThr;
-      if (k < per && e < p.d) {
-        const float dv = xv[k] - mean;
-        q += dv * dv;
-      }
-    }
-    q = warp_sum(q);
-    if (lane == 0) red[warp] = q;
-    cbar();
-    float m2 = 0.f;
-#pragma unroll
-    for (int w = 0; w < kW; ++w) m2 += red[w];
-    const float2 ms = make_float2(mean, rsqrtf(__fadd_rn(m2 / static_cast<float>(p.d), p.eps)));
-#pragma unroll
-    for (int k = 0; k < 6; ++k) {
-      const int e = tid + k * kCThr;
-      if (k < per && e < p.d)
-        p.xn[static_cast<size_t>(t) * p.d + e] =
-            __float2bfloat16(ln_apply(xv[k], ms, bf2f(p.lnf_g[e]), bf2f(p.lnf_b[e])));
-    }
+    stage_ln(p.lnf_g, p.lnf_b);
+    wait_phase(seq_of(p.nl - 1, PH_FC2));  // its barrier also publishes the staged gain and bias
+    if (warp != 0) return;
+    const int nj = p.d / 128;
+    float4 v[kLnJ];
+    load_row(v, t, nj);
+    row_out(p.xn + static_cast<size_t>(t) * p.d, v, nj, row_stats(v, nj, 1.0f / static_cast<float>(p.d), p.eps));
   }
 
   __device__ void run() {
@@ -1089,14 +1129,14 @@ struct Cons {
     arrive(0);
 #pragma unroll 1
     for (int b = 0; b < p.nl; ++b) {
-      gemm_phase<PH_QKV>(b);
+      gemm_phase(b, PH_QKV);
       satt_phase(b);
-      gemm_phase<PH_OUT>(b);
-      gemm_phase<PH_XQ>(b);
+      gemm_phase(b, PH_OUT);
+      gemm_phase(b, PH_XQ);
       xatt_phase(b);
-      gemm_phase<PH_XOUT>(b);
-      gemm_phase<PH_FC1>(b);
-      gemm_phase<PH_FC2>(b);
+      gemm_phase(b, PH_XOUT);
+      gemm_phase(b, PH_FC1);
+      gemm_phase(b, PH_FC2);
     }
     final_ln();
   }
@@ -1111,6 +1151,11 @@ __global__ void __launch_bounds__(kThr, 1) persist_kernel(const __grid_constant_
   sm.base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
   const int c = blockIdx.x;
   const int tid = threadIdx.x;
+  // The phases read the parameters through a reference; pointing it at a
+  // shared-memory copy keeps those reads out of local memory.
+  static_assert(sizeof(MkParams) % 4 == 0, "parameter copy in words");
+  for (int w = tid; w < static_cast<int>(sizeof(MkParams) / 4); w += kThr)
+    reinterpret_cast<uint32_t *>(sm.params())[w] = reinterpret_cast<const uint32_t *>(&p)[w];
   if (tid == 0) {
     for (int s = 0; s < kNS; ++s) {
       mbar_init(sm.full(s), 1);
@@ -1129,9 +1174,9 @@ __global__ void __launch_bounds__(kThr, 1) persist_kernel(const __grid_constant_
   }
   __syncthreads();
   if (tid >= kCThr) {
-    if (tid == kCThr) producer(p, sm, c);
+    if (tid == kCThr) producer(*sm.params(), sm, c);
   } else {
-    Cons cons(p, sm);
+    Cons cons(*sm.params(), sm);
     cons.run();
   }
   __syncthreads();
@@ -1160,6 +1205,12 @@ bool persist_supported(int d, int H, int F, int T, int rows) {
          F / kQ2 <= 1280 && T <= 8 * 256;
 }
 
+bool persist_grid_fits(int d, int F, int G) {
+  auto per_cta = [G](int units) { return (units + G - 1) / G; };
+  return G > 0 && per_cta(3 * d / 8) <= kUB && per_cta(F / 8) <= kUB && per_cta(d / 8 * kQ2) <= kUB &&
+         per_cta(d / 8) <= kUB;
+}
+
 cudaError_t persist_init(int *G) {
   static cudaError_t status = cudaErrorNotReady;
   static int grid = 0;
@@ -1181,7 +1232,9 @@ cudaError_t persist_init(int *G) {
 }
 
 cudaError_t launch_persist(const MkParams &p, cudaStream_t s) {
-  if (p.M > kMkRows || p.n_seq > kMkMaxSeq || p.rps > 16 || p.G < p.M || p.G % kQ2) return cudaErrorInvalidValue;
+  if (p.M > kMkRows || p.n_seq > kMkMaxSeq || p.rps > 16 || p.G < p.M || p.G % kQ2 ||
+      !persist_grid_fits(p.d, p.F, p.G))
+    return cudaErrorInvalidValue;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.G, 1, 1);
   cfg.blockDim = dim3(kThr, 1, 1);
