@@ -219,6 +219,8 @@ def run_ours(args, rank, world):
         lo = hi = args.budget
     budgets = np.full(Bn, lo, np.int32) if lo == hi else syn.budgets(Bn, lo, hi, seed=2)
     sess = Session(cfg, dev, max_batch=Bn, max_ctx=cfg.max_pos)
+    if args.persist:
+        B.wf_set_option(sess.h, B.WF_OPT_PERSIST, 1)
     slots = np.arange(Bn, dtype=np.int32)
     stream = sess.stream
 
@@ -372,9 +374,10 @@ def run_ours(args, rank, world):
     step_ms = dev_ms / args.steps
     wbytes = step_weight_kv_bytes(cfg, 0, [])[0]
     kvbytes = float(np.mean(pl["kv"][args.warmup:]))
-    fam = max(("gemm", "head", "attn_cross", "attn_self"), key=lambda f: prof[f]["ms"])
-    fam_ms = prof["gemm"]["ms"]
-    gemm_gbs = prof["gemm"]["bytes"] / (fam_ms * 1e-3) / 1e9 if fam_ms > 0 else None
+    fam = max(("gemm", "head", "attn_cross", "attn_self", "persist"), key=lambda f: prof[f]["ms"])
+    roof_fam = "persist" if args.persist else "gemm"
+    fam_ms = prof[roof_fam]["ms"]
+    gemm_gbs = prof[roof_fam]["bytes"] / (fam_ms * 1e-3) / 1e9 if fam_ms > 0 else None
     step_total_prof = sum(v["ms"] for v in prof.values())
     result = {
         "metric": METRIC,
@@ -392,6 +395,7 @@ def run_ours(args, rank, world):
                 "from the target's own greedy continuation)",
         "config": {"workload": args.workload, "description": wl["text"], "batch": Bn,
                    "block": cfg.block_k + 1, "parallelism": f"replicas x{world}",
+                   "path": "persistent passes" if args.persist else "launch by launch",
                    "l2": "inputs larger than L2 (every step streams "
                          f"{(wbytes + kvbytes) / 1e9:.2f} GB of weights and K/V > 129 MB L2)"},
         "step_us": step_ms * 1e3,
@@ -401,10 +405,12 @@ def run_ours(args, rank, world):
                           "peak_gbs": hbm_peak,
                           "frac": (wbytes + kvbytes) / (step_ms * 1e-3) / 1e9 / hbm_peak,
                           "peak_source": f"{peak_src} (MEASURED_PEAKS hbm_gbs)"},
-        "roofline": {"kernel": "gemm_tc_kernel (tcgen05 projections)", "bound": "hbm",
+        "roofline": {"kernel": ("persist_kernel (every block of a pass in one launch; bytes = weights "
+                                "and acoustic K/V)") if args.persist else "gemm_tc_kernel (tcgen05 projections)",
+                     "bound": "hbm",
                      "achieved": gemm_gbs, "peak": hbm_peak, "unit": "GB/s",
                      "frac": gemm_gbs / hbm_peak if gemm_gbs else None,
-                     "traffic": GEMM_DRAM_BYTES_PER_LAUNCH.get(args.workload),
+                     "traffic": None if args.persist else GEMM_DRAM_BYTES_PER_LAUNCH.get(args.workload),
                      "peak_source": peak_src,
                      "measured": f"CUDA events around each launch over {n_prof} profiled steps",
                      "share_of_kernel_time": fam_ms / step_total_prof if step_total_prof else None},
@@ -726,6 +732,9 @@ def main():
                     help="cudaProfilerStart/Stop around the timed steps (for ncu)")
     ap.add_argument("--budget", type=int, default=0,
                     help="override every transcript budget (short profiling runs)")
+    ap.add_argument("--persist", action="store_true",
+                    help="run every drafter, verify and greedy pass as one persistent launch "
+                         "(WF_OPT_PERSIST; batch * 9 <= 16 only)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     world = int(os.environ.get("WORLD_SIZE", "1"))

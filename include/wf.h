@@ -242,7 +242,8 @@ wf_status wf_set_option(wf_handle *h, int32_t option, int32_t value);
  * summed kernel time (ms, CUDA events on the launching stream), the number of
  * launches and, for the GEMM and head families, the algorithmic bytes those
  * launches move (weights + token rows in + results out; split-K scratch is
- * not counted).  Each array has WF_PROF_FAMILIES entries; accumulators reset. */
+ * not counted); for the persistent family the blocks' projection weights and
+ * acoustic keys/values.  Each array has WF_PROF_FAMILIES entries; accumulators reset. */
 wf_status wf_profile_read(wf_handle *h, void *stream, double *h_ms, int32_t *h_launches,
                           double *h_bytes);
 wf_status wf_debug_view(wf_handle *h, int32_t which, void **d_ptr, size_t *bytes);

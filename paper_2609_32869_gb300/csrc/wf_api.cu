@@ -714,7 +714,12 @@ cudaError_t persist_pass(wf_handle *h, bool drafter, int n_seq, int rps, const i
   h->launches++;
   prof_begin(h, s);
   cudaError_t e = launch_persist(p, s);
-  prof_end(h, s, WF_FAM_PERSIST, 0.0);
+  // algorithmic bytes: every block's six projection matrices and each
+  // sequence's acoustic keys and values (self/history K/V, a few percent at
+  // these lengths, and the activations are not counted)
+  const double d = h->d, F = h->F;
+  const double block_bytes = 2.0 * (6.0 * d * d + 2.0 * d * F) + 2.0 * 2.0 * n_seq * h->cfg.enc_frames * d;
+  prof_end(h, s, WF_FAM_PERSIST, p.nl * block_bytes);
   return e;
 }
 

@@ -36,6 +36,9 @@ constexpr int kNT = kKW / 8;          // 8-key score tiles per warp
 constexpr int kKS = kKW / 16;         // 16-key steps per warp
 constexpr int kDPT = kQG * 64 / kThreadsA;  // output dims per thread in the combine
 constexpr int kPartStride = 2 + 64;   // m, l, o[64]
+// Scores are kept in base-2 units (times log2 e): every softmax weight, and
+// every weight of the merges of partial results, is one exp2.
+constexpr float kLog2e = 1.4426950408889634f;
 constexpr int kSmemK = kKB * 128;     // bytes
 constexpr int kSmemQ = kQG * 128;
 // K, V, Q, then the warps' (m, l); the warps' O partials reuse the K tile
@@ -257,7 +260,7 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
       const int pos = key0 + kw + nt * 8 + c4 * 2 + (e & 1);
       bool vis = row < nq && pos < n_keys;
       if (p.mode == 0) vis = vis && pos <= base + q0 + row;
-      s[nt][e] = vis ? s[nt][e] : -INFINITY;
+      s[nt][e] = vis ? s[nt][e] * kLog2e : -INFINITY;  // base-2 logits
       mrow[e >> 1] = fmaxf(mrow[e >> 1], s[nt][e]);
     }
   }
@@ -271,7 +274,7 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
   for (int nt = 0; nt < kNT; ++nt) {
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
-      const float v = s[nt][e] == -INFINITY ? 0.f : expf(s[nt][e] - mrow[e >> 1]);
+      const float v = s[nt][e] == -INFINITY ? 0.f : exp2f(s[nt][e] - mrow[e >> 1]);
       s[nt][e] = v;
       lrow[e >> 1] += v;
     }
@@ -313,14 +316,13 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
     sl[warp * kQG + g] = lrow[0];
     sl[warp * kQG + g + 8] = lrow[1];
   }
+  // O rows of 64 floats, 8-float column groups XOR-swizzled by the row's
+  // low two bits: a half-warp's fragment stores fall in distinct banks
 #pragma unroll
   for (int nd = 0; nd < 8; ++nd) {
-    float *o0 = so + (warp * kQG + g) * 64 + nd * 8 + c4 * 2;
-    float *o1 = so + (warp * kQG + g + 8) * 64 + nd * 8 + c4 * 2;
-    o0[0] = o[nd][0];
-    o0[1] = o[nd][1];
-    o1[0] = o[nd][2];
-    o1[1] = o[nd][3];
+    const int col = (nd ^ (g & 3)) * 8 + c4 * 2;
+    *reinterpret_cast<float2 *>(so + (warp * kQG + g) * 64 + col) = make_float2(o[nd][0], o[nd][1]);
+    *reinterpret_cast<float2 *>(so + (warp * kQG + g + 8) * 64 + col) = make_float2(o[nd][2], o[nd][3]);
   }
   __syncthreads();
 
@@ -335,10 +337,10 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
 #pragma unroll
   for (int w = 0; w < kWarps; ++w) {
     const float mw = sm[w * kQG + qi];
-    const float wt = (mw == -INFINITY) ? 0.f : expf(mw - M);
+    const float wt = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
     L += sl[w * kQG + qi] * wt;
 #pragma unroll
-    for (int e = 0; e < kDPT; ++e) acc[e] += so[(w * kQG + qi) * 64 + d0 + e] * wt;
+    for (int e = 0; e < kDPT; ++e) acc[e] += so[(w * kQG + qi) * 64 + ((d0 + e) ^ ((qi & 3) << 3))] * wt;
   }
 
   if (n_blocks == 1) {
@@ -374,7 +376,7 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
         const float lc = dsmem_ld_f32(dsmem_map(pb_u32 + 4u * (qi * 68 + 1), u));
         const float4 o4 = dsmem_ld_f32x4(dsmem_map(pb_u32 + 4u * (qi * 68 + 4 + d0), u));
         const float ov[4] = {o4.x, o4.y, o4.z, o4.w};
-        const float wt = (mc == -INFINITY) ? 0.f : expf(mc - MM);
+        const float wt = (mc == -INFINITY) ? 0.f : exp2f(mc - MM);
         LL = __fmaf_rn(lc, wt, LL);
 #pragma unroll
         for (int e = 0; e < kDPT; ++e) oo[e] = __fmaf_rn(ov[e], wt, oo[e]);
@@ -426,7 +428,7 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
       float ov[kDPT];
 #pragma unroll
       for (int e = 0; e < kDPT; ++e) ov[e] = __ldcg(pe + 2 + d0 + e);
-      const float wt = (mc == -INFINITY) ? 0.f : expf(mc - MM);
+      const float wt = (mc == -INFINITY) ? 0.f : exp2f(mc - MM);
       LL = __fmaf_rn(lc, wt, LL);
 #pragma unroll
       for (int e = 0; e < kDPT; ++e) oo[e] = __fmaf_rn(ov[e], wt, oo[e]);
