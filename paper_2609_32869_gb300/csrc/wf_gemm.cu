@@ -350,13 +350,15 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
       const uint32_t ph = static_cast<uint32_t>(it / stages) & 1u;
       if (!mbar_wait(&full[s], ph, p.err)) break;
       tc_fence_after();
-      const uint32_t a0 = smem_u32(sA + static_cast<size_t>(s) * kStageA);
-      const uint32_t b0 = smem_u32(sB + static_cast<size_t>(ln ? it : s) * stageB);
+      // One descriptor per operand and stage: a 16-deep K step is 32 bytes,
+      // +2 in the descriptor's start-address field (address >> 4, 14 bits;
+      // no carry within a 16 KB stage).  Building each descriptor afresh
+      // made the single issuing thread the MMA's bottleneck at small N.
+      const uint64_t ad = umma_desc_sw128(smem_u32(sA + static_cast<size_t>(s) * kStageA));
+      const uint64_t bd = umma_desc_sw128(smem_u32(sB + static_cast<size_t>(ln ? it : s) * stageB));
 #pragma unroll
-      for (int kk = 0; kk < kBlockK / 16; ++kk) {
-        umma_bf16(tmem, umma_desc_sw128(a0 + kk * 32), umma_desc_sw128(b0 + kk * 32), idesc,
-                  (it | kk) != 0 ? 1u : 0u);
-      }
+      for (int kk = 0; kk < kBlockK / 16; ++kk)
+        umma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (it | kk) != 0 ? 1u : 0u);
       umma_commit(&empty[s]);
     }
     umma_commit(done);
