@@ -1,20 +1,23 @@
 // Persistent decode pass for small batches (M <= 16 token rows: one
 // speculative sequence of K + 1 = 9 rows, or plain greedy steps).
 //
-// At batch 1 a decoder block is a chain of dependent, tiny computations over
-// 46 MB of weights: LN1 -> QKV -> self-attention -> out + residual -> LN2 ->
-// cross-query -> cross-attention -> cross-out + residual -> LN3 -> fc1 ->
-// fc2 + residual (the Whisper decoder block, pre-LayerNorm).  Launched kernel
-// by kernel, each link pays a launch edge and a cold start, so the step is
-// bound by latency, not by HBM.  Here one cooperative launch runs every block
-// of the pass with one CTA per SM:
+// The verification pass of Sec. 3.1 (and the drafter pass of Sec. 3.2, and
+// plain greedy steps) at small batch.  At batch 1 a decoder block is a chain
+// of dependent, tiny computations over 46 MB of weights: LN1 -> QKV ->
+// self-attention -> out + residual -> LN2 -> cross-query -> cross-attention
+// -> cross-out + residual -> LN3 -> fc1 -> fc2 + residual (the Whisper
+// decoder block, pre-LayerNorm).  Launched kernel by kernel, each link pays a
+// launch edge and a cold start, so the step is bound by latency, not by HBM.
+// Here one cooperative launch runs every block of the pass with one CTA per
+// SM:
 //
 //  - A producer thread streams everything that does not depend on the
-//    activations through a ring of 32 KB shared-memory slots with TMA,
+//    activations through a ring of eight 20 KB shared-memory slots with TMA,
 //    running ahead of the dependency chain across phases and blocks: each
 //    projection unit (8 weight rows by the unit's whole K range) is one
-//    copy, each 256-key block of cached keys or values another.  Large copies
-//    matter: a TMA instruction costs about the same for 1 KB as for 20 KB.
+//    copy, each 128 cached keys (or values) of one head another.  Large
+//    copies matter: a TMA instruction costs about the same for 1 KB as for
+//    20 KB.
 //  - Eight compute warps follow the chain.  Work is cut into units: 8 weight
 //    rows of a projection (the n = 8 side of mma.sync m16n8k16; the <= 16
 //    token rows fill the m side), a (sequence, head) of self-attention, a
