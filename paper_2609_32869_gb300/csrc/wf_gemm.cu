@@ -344,22 +344,41 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
     }
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer
+    // Descriptors are built once and stepped: a 16-deep K step is 32 bytes,
+    // +2 in the descriptor's start-address field (shared address >> 4, 14
+    // bits; shared memory is below 256 KB, so the field never carries).  At
+    // small N the single issuing thread, not the tensor pipe, sets the MMA
+    // rate, so the loop keeps everything but the MMAs out of the way.
     const uint32_t idesc = umma_idesc_bf16(kBlockN, BT);
-    for (int it = 0; it < kps; ++it) {
-      const int s = it % stages;
-      const uint32_t ph = static_cast<uint32_t>(it / stages) & 1u;
-      if (!mbar_wait(&full[s], ph, p.err)) break;
-      tc_fence_after();
-      // One descriptor per operand and stage: a 16-deep K step is 32 bytes,
-      // +2 in the descriptor's start-address field (address >> 4, 14 bits;
-      // no carry within a 16 KB stage).  Building each descriptor afresh
-      // made the single issuing thread the MMA's bottleneck at small N.
-      const uint64_t ad = umma_desc_sw128(smem_u32(sA + static_cast<size_t>(s) * kStageA));
-      const uint64_t bd = umma_desc_sw128(smem_u32(sB + static_cast<size_t>(ln ? it : s) * stageB));
+    const uint64_t a_base = umma_desc_sw128(smem_u32(sA)), b_base = umma_desc_sw128(smem_u32(sB));
+    if (kps <= stages) {
+      // every k-step has its own stage and none is refilled: wait for all
+      // of them, then issue the MMAs back to back (no per-stage commit)
+      bool landed = true;
+      for (int it = 0; it < kps && landed; ++it) landed = mbar_wait(&full[it], 0u, p.err);
+      if (landed) {
+        tc_fence_after();
+        for (int it = 0; it < kps; ++it) {
+          const uint64_t ad = a_base + static_cast<uint64_t>((it * kStageA) >> 4);
+          const uint64_t bd = b_base + static_cast<uint64_t>((it * stageB) >> 4);
 #pragma unroll
-      for (int kk = 0; kk < kBlockK / 16; ++kk)
-        umma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (it | kk) != 0 ? 1u : 0u);
-      umma_commit(&empty[s]);
+          for (int kk = 0; kk < kBlockK / 16; ++kk)
+            umma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (it | kk) != 0 ? 1u : 0u);
+        }
+      }
+    } else {
+      for (int it = 0; it < kps; ++it) {
+        const int s = it % stages;
+        const uint32_t ph = static_cast<uint32_t>(it / stages) & 1u;
+        if (!mbar_wait(&full[s], ph, p.err)) break;
+        tc_fence_after();
+        const uint64_t ad = a_base + static_cast<uint64_t>((s * kStageA) >> 4);
+        const uint64_t bd = b_base + static_cast<uint64_t>(((ln ? it : s) * stageB) >> 4);
+#pragma unroll
+        for (int kk = 0; kk < kBlockK / 16; ++kk)
+          umma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (it | kk) != 0 ? 1u : 0u);
+        umma_commit(&empty[s]);
+      }
     }
     umma_commit(done);
   }
