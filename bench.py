@@ -75,7 +75,7 @@ WORKLOADS = {
 # same per-layer shapes (profiles/dram_per_kernel_large_b1_4l.md and
 # profiles/dram_per_kernel_large_b96_2l.md); None where no capture covers the
 # workload's shapes.
-GEMM_DRAM_BYTES_PER_LAUNCH = {"large_b1": 7.824e6, "large_b96": 13.16e6}
+GEMM_DRAM_BYTES_PER_LAUNCH = {"large_b1": 7.826e6, "large_b96": 13.17e6}
 
 
 def _peaks():
