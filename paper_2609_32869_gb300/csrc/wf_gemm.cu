@@ -124,34 +124,16 @@ __device__ __forceinline__ void epi_chunk(const GemmParams &p, int t0, int n, fl
   }
 }
 
-// Epilogue of four consecutive output features n..n+3 of token row t (the
-// staged path).  `old` is the residual row's current value (EPI_RESID).
-// fin[] returns the final values (the updated residual for EPI_RESID) for the
-// LayerNorm statistics.  Four consecutive features never straddle a head or
-// the key/value boundary (multiples of 4), so each store is one vector.
+// Four floats as four bf16 (round to nearest even) in one 8-byte word.
 __device__ __forceinline__ uint2 pack4_bf16(const float (&v)[4]) {
   __nv_bfloat162 h[2] = {__floats2bfloat162_rn(v[0], v[1]), __floats2bfloat162_rn(v[2], v[3])};
   return *reinterpret_cast<const uint2 *>(h);
 }
+// Non-residual epilogues of four features: GELU, then fp32, bf16 or the
+// query / key / value split with the cache scatter.
 template <int EPI>
-__device__ __forceinline__ void epi_quad(const GemmParams &p, int t, int n, const float4 &a,
-                                         const float (&b4)[4], const float4 &old,
-                                         const int2 *tok_local, float (&fin)[4]) {
-  float v[4] = {a.x + b4[0], a.y + b4[1], a.z + b4[2], a.w + b4[3]};
-  if constexpr (EPI == EPI_RESID) {
-    // N % 128 == 0 and ld_resid % 4 == 0 (checked at launch): one float4
-    float4 *r = reinterpret_cast<float4 *>(p.resid + static_cast<size_t>(t) * p.ld_resid + n);
-    const float4 nr = make_float4(old.x + v[0], old.y + v[1], old.z + v[2], old.w + v[3]);
-    *r = nr;
-    fin[0] = nr.x;
-    fin[1] = nr.y;
-    fin[2] = nr.z;
-    fin[3] = nr.w;
-    const uint2 h = pack4_bf16(fin);
-    if (p.tap0) *reinterpret_cast<uint2 *>(p.tap0 + static_cast<size_t>(t) * p.ld_tap + n) = h;
-    if (p.tap1) *reinterpret_cast<uint2 *>(p.tap1 + static_cast<size_t>(t) * p.ld_tap + n) = h;
-    return;
-  }
+__device__ __forceinline__ void epi_quad_out(const GemmParams &p, int t, int n, float (&v)[4],
+                                             const int2 *tok_local, float (&fin)[4]) {
   if constexpr (EPI == EPI_GELU) {
 #pragma unroll
     for (int i = 0; i < 4; ++i) v[i] = gelu_erf(v[i]);
@@ -196,6 +178,33 @@ __device__ __forceinline__ void epi_quad(const GemmParams &p, int t, int n, cons
     *reinterpret_cast<uint2 *>(
         dst + ((static_cast<size_t>(sp.x) * p.n_heads + (hd >> 6)) * p.ctx + sp.y) * 64 + (hd & 63)) =
         pack4_bf16(v);
+  }
+}
+
+// Epilogue of four consecutive output features n..n+3 of token row t (the
+// staged path).  `old` is the residual row's current value (EPI_RESID).
+// fin[] returns the final values (the updated residual for EPI_RESID) for the
+// LayerNorm statistics.  Four consecutive features never straddle a head or
+// the key/value boundary (multiples of 4), so each store is one vector.
+template <int EPI>
+__device__ __forceinline__ void epi_quad(const GemmParams &p, int t, int n, const float4 &a,
+                                         const float (&b4)[4], const float4 &old,
+                                         const int2 *tok_local, float (&fin)[4]) {
+  float v[4] = {a.x + b4[0], a.y + b4[1], a.z + b4[2], a.w + b4[3]};
+  if constexpr (EPI == EPI_RESID) {
+    // N % 128 == 0 and ld_resid % 4 == 0 (checked at launch): one float4
+    float4 *r = reinterpret_cast<float4 *>(p.resid + static_cast<size_t>(t) * p.ld_resid + n);
+    const float4 nr = make_float4(old.x + v[0], old.y + v[1], old.z + v[2], old.w + v[3]);
+    *r = nr;
+    fin[0] = nr.x;
+    fin[1] = nr.y;
+    fin[2] = nr.z;
+    fin[3] = nr.w;
+    const uint2 h = pack4_bf16(fin);
+    if (p.tap0) *reinterpret_cast<uint2 *>(p.tap0 + static_cast<size_t>(t) * p.ld_tap + n) = h;
+    if (p.tap1) *reinterpret_cast<uint2 *>(p.tap1 + static_cast<size_t>(t) * p.ld_tap + n) = h;
+  } else {
+    epi_quad_out<EPI>(p, t, n, v, tok_local, fin);
   }
 }
 
