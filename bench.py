@@ -78,6 +78,21 @@ WORKLOADS = {
 GEMM_DRAM_BYTES_PER_LAUNCH = {"large_b1": 7.826e6, "large_b96": 13.17e6}
 
 
+def aggregate_ranks(times, counts, world, device):
+    """Whole-job figures over `world` replica ranks: each time is the maximum
+    over ranks (the slowest rank bounds the job), each count the sum (every
+    rank decodes its own sequences).  With world == 1 the values come back
+    unchanged; otherwise every rank must call this with the same lengths."""
+    import torch
+    t = torch.tensor([float(x) for x in times], dtype=torch.float64, device=device)
+    c = torch.tensor([float(x) for x in counts], dtype=torch.float64, device=device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        dist.all_reduce(c, op=dist.ReduceOp.SUM)
+    return [float(x) for x in t.cpu()], [float(x) for x in c.cpu()]
+
+
 def _peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -362,13 +377,7 @@ def run_ours(args, rank, world):
         pass
 
     # ---- aggregate over ranks
-    t_dev = torch.tensor([dev_ms, e2e_s], dtype=torch.float64, device="cuda")
-    t_tok = torch.tensor([tokens, e2e_tokens], dtype=torch.float64, device="cuda")
-    if world > 1:
-        dist.all_reduce(t_dev, op=dist.ReduceOp.MAX)
-        dist.all_reduce(t_tok, op=dist.ReduceOp.SUM)
-    dev_ms, e2e_s = float(t_dev[0]), float(t_dev[1])
-    tokens, e2e_tokens = float(t_tok[0]), float(t_tok[1])
+    (dev_ms, e2e_s), (tokens, e2e_tokens) = aggregate_ranks([dev_ms, e2e_s], [tokens, e2e_tokens], world, "cuda")
 
     hbm_peak, bf16_peak, peak_src = _peaks()
     step_ms = dev_ms / args.steps
@@ -524,13 +533,7 @@ def run_sampling(args, rank, world):
     except OSError:
         pass
 
-    t_dev = torch.tensor([dev_ms, e2e_s], dtype=torch.float64, device="cuda")
-    t_tok = torch.tensor([tokens, e2e_tokens], dtype=torch.float64, device="cuda")
-    if world > 1:
-        dist.all_reduce(t_dev, op=dist.ReduceOp.MAX)
-        dist.all_reduce(t_tok, op=dist.ReduceOp.SUM)
-    dev_ms, e2e_s = float(t_dev[0]), float(t_dev[1])
-    tokens, e2e_tokens = float(t_tok[0]), float(t_tok[1])
+    (dev_ms, e2e_s), (tokens, e2e_tokens) = aggregate_ranks([dev_ms, e2e_s], [tokens, e2e_tokens], world, "cuda")
     hbm_peak, _, peak_src = _peaks()
     step_ms = dev_ms / args.steps
     mean_len = list((len0 + len1) / 2.0)
