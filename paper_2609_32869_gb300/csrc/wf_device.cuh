@@ -61,6 +61,14 @@ __device__ __forceinline__ uint32_t mbar_try_wait(uint64_t *bar, uint32_t parity
 }
 // Bounded wait on a phase of an mbarrier.  Returns false (and sets the error
 // word) if the phase did not complete within kSpinLimitCycles.
+// Before a CTA exits: wait (bounded, whatever the error word says) for a
+// copy this thread issued into the CTA's shared memory to land, so that no
+// bulk copy is still writing there once the CTA is gone.
+__device__ __forceinline__ void mbar_drain(uint64_t *bar, uint32_t parity) {
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity) && clock64() - t0 < kSpinLimitCycles) {
+  }
+}
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint32_t *err) {
   if (mbar_try_wait(bar, parity)) return true;
   long long t0 = clock64();

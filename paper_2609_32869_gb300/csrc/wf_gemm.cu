@@ -294,12 +294,16 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
   int2 *tok = reinterpret_cast<int2 *>(smem + p.pipe_bytes + (2 * stages + 1) * 8 + 16 + 16);
   float2 *lnst = reinterpret_cast<float2 *>(tok + BT);  // per-token (mean, rstd), LN mode
   const bool ln = p.ln_x != nullptr;
+  // a bounded wait of this CTA gave up (in the 32 bytes reserved after the
+  // barriers, beside the TMEM address; the kernel has no static shared memory)
+  volatile int &s_timed_out = *reinterpret_cast<int *>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int tt = blockIdx.x, ntile = blockIdx.y, split = blockIdx.z;
   const int n0 = ntile * kBlockN, t0 = tt * BT, kit0 = split * kps;
 
   if (threadIdx.x == 0) {
+    s_timed_out = 0;
     tma_prefetch_desc(&tmW);
     tma_prefetch_desc(&tmX);
     for (int s = 0; s < stages; ++s) {
@@ -335,6 +339,7 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
     __syncthreads();
   }
 
+  int issued = npre;  // k-steps whose tiles the producer (thread 0) has requested
   if (warp == 0 && lane == 0) {
     // ---------------- TMA producer
     if (!ln) {
@@ -345,7 +350,11 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
     for (int it = npre; it < kps; ++it) {
       const int s = it % stages;
       const uint32_t ph = static_cast<uint32_t>((it / stages) - 1) & 1u;
-      if (!mbar_wait(&empty[s], ph, p.err)) break;
+      if (!mbar_wait(&empty[s], ph, p.err)) {
+        s_timed_out = 1;
+        break;
+      }
+      issued = it + 1;
       mbar_arrive_expect_tx(&full[s], tx);
       tma_load_2d(sA + static_cast<size_t>(s) * kStageA, &tmW, (kit0 + it) * kBlockK, n0, &full[s]);
       if (!ln)
@@ -365,6 +374,7 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
       // of them, then issue the MMAs back to back (no per-stage commit)
       bool landed = true;
       for (int it = 0; it < kps && landed; ++it) landed = mbar_wait(&full[it], 0u, p.err);
+      if (!landed) s_timed_out = 1;
       if (landed) {
         tc_fence_after();
         for (int it = 0; it < kps; ++it) {
@@ -379,7 +389,10 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
       for (int it = 0; it < kps; ++it) {
         const int s = it % stages;
         const uint32_t ph = static_cast<uint32_t>(it / stages) & 1u;
-        if (!mbar_wait(&full[s], ph, p.err)) break;
+        if (!mbar_wait(&full[s], ph, p.err)) {
+          s_timed_out = 1;
+          break;
+        }
         tc_fence_after();
         const uint64_t ad = a_base + static_cast<uint64_t>((s * kStageA) >> 4);
         const uint64_t bd = b_base + static_cast<uint64_t>(((ln ? it : s) * stageB) >> 4);
@@ -618,6 +631,12 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
     }
   }
 
+  // After a timeout, copies this CTA requested may still be landing: wait for
+  // them (bounded) before the CTA leaves.  Otherwise every one was consumed
+  // by the MMA thread before the MMAs completed.
+  if (threadIdx.x == 0 && (!ok || s_timed_out))
+    for (int q = max(0, issued - stages); q < issued; ++q)
+      mbar_drain(&full[q % stages], static_cast<uint32_t>(q / stages) & 1u);
   tc_fence_before();
   __syncthreads();
   if (warp == 2) tmem_dealloc(tmem, p.tmem_cols);

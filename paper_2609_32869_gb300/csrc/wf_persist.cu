@@ -89,6 +89,10 @@ __device__ __forceinline__ void add_release(uint32_t *ptr, uint32_t v) {
   r.fetch_add(v, cuda::memory_order_release);
 }
 __device__ __forceinline__ uint4 ldcg_u128(const void *ptr) { return __ldcg(static_cast<const uint4 *>(ptr)); }
+// Five 16-byte loads (L2, not L1) in one statement, so that they issue back
+// to back: under the kernel's register budget the compiler otherwise places
+// uses (or stores) of the first loads between them and serialises the round
+// trips.
 __device__ __forceinline__ void ldcg_f32x4x5(float4 *v, const float4 *p0, const float4 *p1, const float4 *p2,
                                              const float4 *p3, const float4 *p4) {
   asm volatile(
@@ -103,8 +107,6 @@ __device__ __forceinline__ void ldcg_f32x4x5(float4 *v, const float4 *p0, const 
       : "l"(p0), "l"(p1), "l"(p2), "l"(p3), "l"(p4)
       : "memory");
 }
-// Five 16-byte loads (L2, not L1) in one statement, so that they issue back
-// to back: the scheduler may not put a use of the first between them.
 __device__ __forceinline__ void ldcg_u128x5(uint4 (&v)[5], const void *p0, const void *p1, const void *p2,
                                             const void *p3, const void *p4) {
   asm volatile(
@@ -151,8 +153,8 @@ __device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, uint32_
     if (!sp.again(err)) return false;
   return true;
 }
-// The producer's wait for a free slot backs off between tries: it shares a
-// scheduler with two compute warps and must not take their issue slots.
+// The producer's wait for a free slot backs off between tries, leaving the
+// issue slots of its scheduler to the two compute warps that share it.
 __device__ __forceinline__ bool wait_bar_idle(uint64_t *bar, uint32_t parity, uint32_t *err) {
   if (mbar_try_wait(bar, parity)) return true;
   Spin sp;
@@ -217,7 +219,8 @@ constexpr int kOffEmpty = kOffFull + kNS * 8;
 constexpr int kOffNk = kOffEmpty + kNS * 8;                 // int[kMkMaxSeq]
 constexpr int kOffSlot = kOffNk + kMkMaxSeq * 4;            // int[kMkMaxSeq]
 constexpr int kOffZero = (kOffSlot + kMkMaxSeq * 4 + 15) / 16 * 16;  // 16 zero bytes (operand rows >= M)
-constexpr int kOffParams = kOffZero + 16;                  // MkParams (a copy of the launch's)
+constexpr int kOffIssued = kOffZero + 16;                  // uint32: ring copies the producer requested
+constexpr int kOffParams = kOffIssued + 16;                // MkParams (a copy of the launch's)
 constexpr int kSmemUsed = kOffParams + (static_cast<int>(sizeof(MkParams)) + 15) / 16 * 16;
 static_assert(kSmemUsed + 1024 <= kSmemMk, "shared-memory plan");
 struct Smem {
@@ -231,6 +234,7 @@ struct Smem {
   __device__ __forceinline__ uint8_t *zero16() const { return base + kOffZero; }
   __device__ __forceinline__ bf16 *lngb() const { return reinterpret_cast<bf16 *>(base + kOffLnGB); }
   __device__ __forceinline__ MkParams *params() const { return reinterpret_cast<MkParams *>(base + kOffParams); }
+  __device__ __forceinline__ uint32_t *issued() const { return reinterpret_cast<uint32_t *>(base + kOffIssued); }
 };
 
 // ------------------------------------------------------------ producer ----
@@ -315,7 +319,9 @@ __device__ void producer(const MkParams &p, const Smem sm, int c) {
       }
     }
   }
+  *sm.issued() = sc;  // copies requested, for the drain at the end of the kernel
 }
+
 
 // ------------------------------------------------------------ consumer ----
 struct Cons {
@@ -1166,6 +1172,7 @@ __global__ void __launch_bounds__(kThr, 1) persist_kernel(const __grid_constant_
     }
     fence_barrier_init();
     *reinterpret_cast<uint4 *>(sm.zero16()) = make_uint4(0u, 0u, 0u, 0u);
+    *sm.issued() = 0u;
   }
   if (tid < p.n_seq) {
     const int slot = p.seq_slot[tid];
@@ -1183,6 +1190,14 @@ __global__ void __launch_bounds__(kThr, 1) persist_kernel(const __grid_constant_
     cons.run();
   }
   __syncthreads();
+  if (tid == 0 && (ld_relaxed(p.err) & WF_DEV_ERR_TIMEOUT)) {
+    // After a timeout the compute warps may have left ring slots unconsumed:
+    // wait (bounded) for the copies still landing before the CTA leaves.
+    // Otherwise every copy was consumed before the barrier above.
+    const uint32_t sc = *sm.issued();
+    for (uint32_t q = sc > static_cast<uint32_t>(kNS) ? sc - kNS : 0u; q < sc; ++q)
+      mbar_drain(sm.full(q % kNS), (q / kNS) & 1u);
+  }
   if (tid == 0) {
     // The last CTA to finish resets the counters for the next pass: no CTA
     // reads them any more once all have finished.
