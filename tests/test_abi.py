@@ -53,3 +53,51 @@ def test_host_validation_without_gpu():
     except B.WfError as e:
         assert e.status == B.WF_ERR_INVALID
     assert B.wf_gemm_scratch_bytes(9, 1280, 1000) == 0   # K not a multiple of 64
+
+
+def test_null_handle_is_rejected_on_the_host():
+    """Every call that takes a handle checks it before touching the device."""
+    from paper_2609_32869_gb300 import binding as B
+    lib = B.lib()
+    sp = B.WfSampleParams()
+    calls = {
+        "wf_destroy": (None,),
+        "wf_prefill_cross_kv": (None, 1, None, None, None, 4, None, None, None, None),
+        "wf_draft": (None, None, None),
+        "wf_verify_accept": (None, None, None, None, None, None),
+        "wf_step": (None, None, None, None, None, None),
+        "wf_greedy_step": (None, None, None, None, None),
+        "wf_compact": (None, None, None),
+        "wf_reset_slots": (None, 1, None, None),
+        "wf_get_state": (None, None, None, None, None, None),
+        "wf_get_error": (None, None, 0, None),
+        "wf_set_option": (None, B.WF_OPT_PERSIST, 1),
+        "wf_debug_view": (None, 1, None, None),
+        "wf_profile_read": (None, None, None, None, None),
+    }
+    for name, args in calls.items():
+        assert getattr(lib, name)(*args) == B.WF_ERR_INVALID, name
+    # with a (non-null) sampling-parameter block the answer is the same
+    assert lib.wf_draft(None, ctypes.byref(sp), None) == B.WF_ERR_INVALID
+
+
+def test_status_strings_are_distinct():
+    from paper_2609_32869_gb300 import binding as B
+    lib = B.lib()
+    codes = (B.WF_OK, B.WF_ERR_INVALID, B.WF_ERR_CAPACITY, B.WF_ERR_CUDA, B.WF_ERR_UNSUPPORTED,
+             B.WF_ERR_DEVICE)
+    texts = [lib.wf_status_str(c) for c in codes]
+    assert all(t for t in texts) and len(set(texts)) == len(codes)
+
+
+def test_workspace_grows_with_batch_and_context():
+    """The caller-owned workspace holds per-slot caches: a second slot adds at
+    least one slot's target key/value cache and acoustic keys/values."""
+    from paper_2609_32869_gb300 import binding as B
+    from paper_2609_32869_gb300 import synthetic as syn
+    cfg = B.make_config(syn.LARGE)
+    one, two = B.wf_workspace_bytes(cfg, 1, 448), B.wf_workspace_bytes(cfg, 2, 448)
+    d, layers, frames = 1280, 32, 1500
+    per_slot = 2 * layers * 448 * d * 2 + 2 * layers * frames * d * 2
+    assert two - one >= per_slot
+    assert B.wf_workspace_bytes(cfg, 1, 200) < one
