@@ -215,13 +215,17 @@ int32_t wf_last_launch_count(const wf_handle *h);
 #define WF_OPT_GRAPHS 3      /* 1 (default): wf_step / wf_greedy_step replay a CUDA graph
                                 captured on first use per (active count, forcing, sampling
                                 parameters); 0: launch kernel by kernel */
-#define WF_OPT_PERSIST 5     /* 1 (off by default; accepted where supported): the blocks of every drafter,
-                                verify and greedy pass run in one persistent cooperative
-                                launch; supported when max_batch * (block_k + 1) <= 16,
-                                d_model <= 1280 and d_ff a multiple of 512 with
-                                d_ff / 4 <= 1280.  0: one launch per projection and
-                                attention.  Both give results within the tolerances of
-                                the method, not bit-identical ones. */
+#define WF_OPT_PERSIST 5     /* 1: the blocks of every drafter, verify and greedy pass run
+                                in one persistent cooperative launch (one CTA per SM, so
+                                no other kernel may hold SMs meanwhile).  Off by default:
+                                on GB300 it is slower than launch by launch.  Supported
+                                when max_batch * (block_k + 1) <= 16, 64-wide heads,
+                                d_model <= 1280, d_ff a multiple of 512 with
+                                d_ff / 4 <= 1280, at most 2048 encoder frames and enough
+                                SMs for at most five projection units per CTA; otherwise
+                                setting it returns WF_ERR_UNSUPPORTED.  0: one launch per
+                                projection and attention.  Both give results within the
+                                tolerances of the method, not bit-identical ones. */
 #define WF_VIEW_TARGET_LOGITS 1
 #define WF_VIEW_DRAFT_LOGITS 2
 #define WF_VIEW_TAPS 3
