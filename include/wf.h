@@ -226,6 +226,14 @@ int32_t wf_last_launch_count(const wf_handle *h);
                                 setting it returns WF_ERR_UNSUPPORTED.  0: one launch per
                                 projection and attention.  Both give results within the
                                 tolerances of the method, not bit-identical ones. */
+#define WF_OPT_SPIN_LIMIT 6  /* clock cycles a bounded wait in the projection kernels and the
+                                persistent pass spins before it gives up (records
+                                WF_DEV_ERR_TIMEOUT in the error word and returns; the kernel
+                                still waits, with the default limit, for its own copies and
+                                tensor-core work in flight before it exits).  0 (default)
+                                restores about 1 s (projections) and 0.2 s (persistent pass).
+                                Meant for tests of the failure path: a limit below a wait's
+                                normal duration makes the results of that call invalid. */
 #define WF_VIEW_TARGET_LOGITS 1
 #define WF_VIEW_DRAFT_LOGITS 2
 #define WF_VIEW_TAPS 3

@@ -46,6 +46,7 @@ struct wf_handle {
   float2 *rope;
   int n_vtiles = 0;
   int n_active = 0;
+  long long spin = 0;  // bounded-wait limit in clock cycles (WF_OPT_SPIN_LIMIT; 0: default)
   int launches = 0;
   bool keep_logits = false;
   // profiling (WF_OPT_PROFILE)
@@ -276,6 +277,7 @@ GemmParams gemm_base(wf_handle *h, int M, int N, int K, int epi) {
   p.epi = epi;
   p.splits = gemm_splits(N, K);
   p.err = h->err;
+  p.spin = h->spin;
   p.d_model = h->d;
   p.n_heads = h->H;
   return p;
@@ -688,6 +690,7 @@ cudaError_t persist_setup(wf_handle *h, cudaStream_t s) {
   p.ld_tap = h->cfg.n_taps * d;
   p.xn = h->xn;
   p.err = h->err;
+  p.spin = kMkSpinCycles;
   h->mk_on = false;
   return cudaSuccess;
 }
@@ -697,6 +700,7 @@ cudaError_t persist_setup(wf_handle *h, cudaStream_t s) {
 cudaError_t persist_pass(wf_handle *h, bool drafter, int n_seq, int rps, const int32_t *slots,
                          const int32_t *forced, bool taps, cudaStream_t s) {
   MkParams p = h->mkp;
+  if (h->spin > 0) p.spin = h->spin;
   p.layers = drafter ? h->mkl + h->nl : h->mkl;
   p.nl = drafter ? h->nd : h->nl;
   p.drafter = drafter ? 1 : 0;
@@ -864,6 +868,13 @@ wf_status wf_set_option(wf_handle *h, int32_t option, int32_t value) {
   if (option == WF_OPT_PERSIST) {
     if (value && !h->mk_ok) return WF_ERR_UNSUPPORTED;
     h->mk_on = value != 0;
+    for (auto &kv : h->graphs) cudaGraphExecDestroy(kv.second.exec);
+    h->graphs.clear();
+    return WF_OK;
+  }
+  if (option == WF_OPT_SPIN_LIMIT) {
+    if (value < 0) return WF_ERR_INVALID;
+    h->spin = value;
     for (auto &kv : h->graphs) cudaGraphExecDestroy(kv.second.exec);
     h->graphs.clear();
     return WF_OK;

@@ -14,6 +14,8 @@ namespace wf {
 
 // A spin-wait gives up after this many clock cycles (about a second at the
 // GB300 clock) and records WF_DEV_ERR_TIMEOUT instead of hanging the GPU.
+// Kernels take their limit as a parameter (this is the default); the drain
+// of a CTA's own copies after a timeout always uses this one.
 constexpr long long kSpinLimitCycles = 2000000000LL;
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -59,21 +61,23 @@ __device__ __forceinline__ uint32_t mbar_try_wait(uint64_t *bar, uint32_t parity
       : "memory");
   return ok;
 }
-// Bounded wait on a phase of an mbarrier.  Returns false (and sets the error
-// word) if the phase did not complete within kSpinLimitCycles.
 // Before a CTA exits: wait (bounded, whatever the error word says) for a
-// copy this thread issued into the CTA's shared memory to land, so that no
-// bulk copy is still writing there once the CTA is gone.
+// copy this thread issued into the CTA's shared memory to land, or for the
+// tensor-core work it issued to complete, so that nothing asynchronous still
+// writes into the CTA's shared memory or TMEM once it is released.
 __device__ __forceinline__ void mbar_drain(uint64_t *bar, uint32_t parity) {
   const long long t0 = clock64();
   while (!mbar_try_wait(bar, parity) && clock64() - t0 < kSpinLimitCycles) {
   }
 }
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint32_t *err) {
+// Bounded wait on a phase of an mbarrier.  Returns false (and sets the error
+// word) if the phase did not complete within `limit` clock cycles.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint32_t *err,
+                                          long long limit) {
   if (mbar_try_wait(bar, parity)) return true;
   long long t0 = clock64();
   while (!mbar_try_wait(bar, parity)) {
-    if (clock64() - t0 > kSpinLimitCycles) {
+    if (clock64() - t0 > limit) {
       set_error(err, WF_DEV_ERR_TIMEOUT);
       return false;
     }

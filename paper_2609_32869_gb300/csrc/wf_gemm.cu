@@ -350,7 +350,7 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
     for (int it = npre; it < kps; ++it) {
       const int s = it % stages;
       const uint32_t ph = static_cast<uint32_t>((it / stages) - 1) & 1u;
-      if (!mbar_wait(&empty[s], ph, p.err)) {
+      if (!mbar_wait(&empty[s], ph, p.err, p.spin)) {
         s_timed_out = 1;
         break;
       }
@@ -373,7 +373,7 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
       // every k-step has its own stage and none is refilled: wait for all
       // of them, then issue the MMAs back to back (no per-stage commit)
       bool landed = true;
-      for (int it = 0; it < kps && landed; ++it) landed = mbar_wait(&full[it], 0u, p.err);
+      for (int it = 0; it < kps && landed; ++it) landed = mbar_wait(&full[it], 0u, p.err, p.spin);
       if (!landed) s_timed_out = 1;
       if (landed) {
         tc_fence_after();
@@ -389,7 +389,7 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
       for (int it = 0; it < kps; ++it) {
         const int s = it % stages;
         const uint32_t ph = static_cast<uint32_t>(it / stages) & 1u;
-        if (!mbar_wait(&full[s], ph, p.err)) {
+        if (!mbar_wait(&full[s], ph, p.err, p.spin)) {
           s_timed_out = 1;
           break;
         }
@@ -457,7 +457,8 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
     }
   }
   __syncthreads();
-  const bool ok = mbar_wait(done, 0, p.err);
+  const bool ok = mbar_wait(done, 0, p.err, p.spin);
+  if (!ok) s_timed_out = 1;
   tc_fence_after();
   __syncwarp();
   // warp w reads TMEM lane quarter w % 4 (weight rows 32 (w % 4) ..) and the
@@ -631,12 +632,16 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
     }
   }
 
-  // After a timeout, copies this CTA requested may still be landing: wait for
-  // them (bounded) before the CTA leaves.  Otherwise every one was consumed
-  // by the MMA thread before the MMAs completed.
-  if (threadIdx.x == 0 && (!ok || s_timed_out))
+  // After a timeout, copies this CTA requested may still be landing and
+  // MMAs it issued may still be running: wait for both (bounded) before the
+  // CTA frees its TMEM and leaves.  Otherwise every copy was consumed by the
+  // MMA thread and the MMAs completed before the epilogue read TMEM.
+  __syncthreads();
+  if (threadIdx.x == 0 && s_timed_out) {
     for (int q = max(0, issued - stages); q < issued; ++q)
       mbar_drain(&full[q % stages], static_cast<uint32_t>(q / stages) & 1u);
+    mbar_drain(done, 0u);
+  }
   tc_fence_before();
   __syncthreads();
   if (warp == 2) tmem_dealloc(tmem, p.tmem_cols);
@@ -878,6 +883,7 @@ bool gemm_ln_fits(int M, int N, int K, int epi) {
 
 cudaError_t launch_gemm(const void *X, const void *W, GemmParams p, cudaStream_t s, bool pdl) {
   const bool ln = p.ln_x != nullptr;
+  if (p.spin <= 0) p.spin = kSpinLimitCycles;
   const bool quad = p.splits > 1 || p.stats_out;  // the staged (four-feature) epilogue
   if (p.epi == EPI_HEAD && (ln || p.stats_out)) return cudaErrorInvalidValue;
   if ((p.stats_out || p.epi == EPI_RESID) && p.N % kBlockN) return cudaErrorInvalidValue;

@@ -64,6 +64,7 @@ struct GemmParams {
   const int32_t *step;  // per slot
   uint32_t tag;
   uint32_t *err;
+  long long spin;  // clock cycles a bounded wait spins before it gives up
   // LayerNorm-fused token operand: when ln_x is set the CTA builds its bf16
   // B tiles as LN(x) = (x - mean) * rstd * g + b from fp32 rows ln_x (row
   // stride ln_ld) and per-row statistics ln_stats[t][0..ln_tiles) (mean, M2
@@ -199,6 +200,7 @@ constexpr int kMkMaxSeq = 16;     // sequences per persistent pass
 constexpr int kMkPhases = 8;      // QKV, self-attn, out, cross-query, cross-attn, cross-out, fc1, fc2
 constexpr int kMkMaxG = 256;      // CTAs a persistent pass may use
 constexpr int kMkCounters = 8 * 64 + 2;  // phase counters: embedding + 8 phases x 64 blocks
+constexpr long long kMkSpinCycles = 400000000LL;  // default bounded-wait limit (~0.2 s)
 struct MkLayer {
   const bf16 *ln1_g, *ln1_b, *qkv_b, *out_b, *ln2_g, *ln2_b, *xq_b, *xout_b;
   const bf16 *ln3_g, *ln3_b, *fc1_b, *fc2_b;
@@ -234,6 +236,7 @@ struct MkParams {
   bf16 *xn;                    // [M][d] final LayerNorm output (plain bf16)
   uint32_t *sync;              // [1] CTAs finished (reset by the last)
   uint32_t *err;
+  long long spin;              // clock cycles a bounded wait spins before it gives up
 };
 size_t mk_xpart_words(int M, int H, int T);
 cudaError_t persist_init(int *G);

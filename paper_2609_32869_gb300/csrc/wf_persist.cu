@@ -61,7 +61,6 @@ constexpr int kUB = 5;                    // projection units per CTA and phase 
 constexpr int kKS = 10;                   // k16-steps per warp: operand width <= 1280
 constexpr int kQ2 = 4;                    // fc2 split-K factor (partials add in order)
 constexpr int kPS = 68;                   // attention partial: m, l, -, -, o[64] (o 16-byte aligned)
-constexpr long long kMkSpin = 400000000LL;  // cycles before a wait gives up (~0.2 s)
 constexpr int kLnGB = 2 * 1280 * 2;        // LayerNorm gain and bias (bf16, d <= 1280)
 constexpr int kSmemMk = 1024 + kNS * kSlot + kScratch + kLnGB + 2 * kNS * 8 + 2048;
 
@@ -123,17 +122,20 @@ __device__ __forceinline__ void ldcg_u128x5(uint4 (&v)[5], const void *p0, const
 }
 __device__ __forceinline__ int seq_of(int b, int ph) { return 1 + b * kMkPhases + ph; }
 
-// Bounded spin: gives up (recording WF_DEV_ERR_TIMEOUT) after kMkSpin cycles,
-// or at once when another thread of the grid has already given up.
+// Bounded spin: gives up (recording WF_DEV_ERR_TIMEOUT) after `limit` cycles
+// (MkParams::spin), or at once when another thread of the grid has already
+// given up.
 struct Spin {
+  long long limit;
   long long t0 = 0;
   int it = 0;
+  __device__ __forceinline__ explicit Spin(long long lim) : limit(lim) {}
   __device__ __forceinline__ bool again(uint32_t *err) {
     if (it == 0) t0 = clock64();
     ++it;
     if ((it & 31) == 0) {
       if (ld_relaxed(err) & WF_DEV_ERR_TIMEOUT) return false;
-      if (clock64() - t0 > kMkSpin) {
+      if (clock64() - t0 > limit) {
         set_error(err, WF_DEV_ERR_TIMEOUT);
         return false;
       }
@@ -142,22 +144,24 @@ struct Spin {
   }
 };
 // One thread waits (acquire) until *ctr >= target.
-__device__ __forceinline__ void wait_ge(const uint32_t *ctr, uint32_t target, uint32_t *err) {
-  Spin sp;
+__device__ __forceinline__ void wait_ge(const uint32_t *ctr, uint32_t target, uint32_t *err,
+                                        long long limit) {
+  Spin sp(limit);
   while (ld_acquire(ctr) < target && sp.again(err)) __nanosleep(100);
 }
-__device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, uint32_t *err) {
+__device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, uint32_t *err, long long limit) {
   if (mbar_try_wait(bar, parity)) return true;
-  Spin sp;
+  Spin sp(limit);
   while (!mbar_try_wait(bar, parity))
     if (!sp.again(err)) return false;
   return true;
 }
 // The producer's wait for a free slot backs off between tries, leaving the
 // issue slots of its scheduler to the two compute warps that share it.
-__device__ __forceinline__ bool wait_bar_idle(uint64_t *bar, uint32_t parity, uint32_t *err) {
+__device__ __forceinline__ bool wait_bar_idle(uint64_t *bar, uint32_t parity, uint32_t *err,
+                                              long long limit) {
   if (mbar_try_wait(bar, parity)) return true;
-  Spin sp;
+  Spin sp(limit);
   while (!mbar_try_wait(bar, parity)) {
     if (!sp.again(err)) return false;
     __nanosleep(64);
@@ -243,7 +247,7 @@ __device__ void producer(const MkParams &p, const Smem sm, int c) {
   bool ok = true;
   auto acquire = [&](uint32_t bytes, uint8_t *&dst, uint64_t *&bar) {
     const uint32_t s = sc % kNS, n = sc / kNS;
-    if (n > 0 && !wait_bar_idle(sm.empty(s), (n - 1) & 1u, p.err)) {
+    if (n > 0 && !wait_bar_idle(sm.empty(s), (n - 1) & 1u, p.err, p.spin)) {
       ok = false;
       return;
     }
@@ -358,7 +362,7 @@ struct Cons {
   __device__ __forceinline__ uint8_t *slot_ptr(int m) const {
     return sm.ring() + static_cast<size_t>(ahead(m)) * kSlot;
   }
-  __device__ __forceinline__ void wait_slot(int m) const { wait_bar(sm.full(ahead(m)), ahead_par(m), p.err); }
+  __device__ __forceinline__ void wait_slot(int m) const { wait_bar(sm.full(ahead(m)), ahead_par(m), p.err, p.spin); }
   // The 32-key group gi (0..7) of a 256-key block whose keys fill the first
   // nh slots at the cursor and whose values the next nh.
   __device__ __forceinline__ uint8_t *kgroup(int gi) const { return slot_ptr(gi >> 2) + (gi & 3) * 4096; }
@@ -386,7 +390,7 @@ struct Cons {
   }
   // Wait until every CTA has finished phase s.
   __device__ __forceinline__ void wait_phase(int s) {
-    if (tid == 0) wait_ge(p.cnt + s, static_cast<uint32_t>(p.G), p.err);
+    if (tid == 0) wait_ge(p.cnt + s, static_cast<uint32_t>(p.G), p.err, p.spin);
     cbar();
   }
 
@@ -650,7 +654,7 @@ struct Cons {
         if (u0 % kQ2 == 0) {
           if (tid == 0)
             for (int k = 0; k < nb; ++k)
-              wait_ge(p.cnt2 + (ub + k * p.G) / kQ2, static_cast<uint32_t>((kQ2 - 1) * (b + 1)), p.err);
+              wait_ge(p.cnt2 + (ub + k * p.G) / kQ2, static_cast<uint32_t>((kQ2 - 1) * (b + 1)), p.err, p.spin);
           cbar();
         }
       }
@@ -1091,7 +1095,7 @@ struct Cons {
         if (tid == 0) add_release(p.cntx + hu, 1u);
       } else {
         // merge the other blocks' partials in block order
-        if (tid == 0) wait_ge(p.cntx + hu, static_cast<uint32_t>((n_chunks(p) - 1) * (b + 1)), p.err);
+        if (tid == 0) wait_ge(p.cntx + hu, static_cast<uint32_t>((n_chunks(p) - 1) * (b + 1)), p.err, p.spin);
         cbar();
         if (qi < p.rps) {
           constexpr int kMaxCh = 8;  // T <= 2048 frames
@@ -1229,24 +1233,33 @@ bool persist_grid_fits(int d, int F, int G) {
          per_cta(d / 8) <= kUB;
 }
 
+// Per device: the shared-memory opt-in and the grid (one CTA per SM, rounded
+// down to a multiple of the fc2 split), set up the first time a handle on
+// that device asks.  A cooperative launch needs every CTA resident at once,
+// so the grid must come from the device the pass runs on.
 cudaError_t persist_init(int *G) {
-  static cudaError_t status = cudaErrorNotReady;
-  static int grid = 0;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    status = cudaFuncSetAttribute(persist_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMk);
-    if (status != cudaSuccess) return;
-    int dev = 0, n_sm = 0, per_sm = 0;
-    status = cudaGetDevice(&dev);
-    if (status == cudaSuccess) status = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
-    if (status == cudaSuccess)
-      status = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, persist_kernel, kThr, kSmemMk);
-    if (status == cudaSuccess && per_sm < 1) status = cudaErrorInvalidConfiguration;
-    // a multiple of the fc2 split so every CTA's fc2 units share one input quarter
-    grid = (n_sm / kQ2) * kQ2;
-  });
-  if (G) *G = grid;
-  return status;
+  constexpr int kMaxDev = 64;
+  static std::mutex mu;
+  static cudaError_t status[kMaxDev];
+  static int grid[kMaxDev];
+  static bool ready[kMaxDev] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDev) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!ready[dev]) {
+    int n_sm = 0, per_sm = 0;
+    e = cudaFuncSetAttribute(persist_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMk);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, persist_kernel, kThr, kSmemMk);
+    if (e == cudaSuccess && per_sm < 1) e = cudaErrorInvalidConfiguration;
+    status[dev] = e;
+    grid[dev] = (n_sm / kQ2) * kQ2;
+    ready[dev] = true;
+  }
+  if (G) *G = grid[dev];
+  return status[dev];
 }
 
 cudaError_t launch_persist(const MkParams &p, cudaStream_t s) {

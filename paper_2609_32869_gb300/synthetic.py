@@ -17,7 +17,9 @@ Workload shapes follow the paper's setting: a Whisper-large-shaped decoder
 positions) and 1500 encoder frames per 30 s window (Sec. 4, Sec. 5.1,
 App. A.2); the tiny shape is Whisper-tiny's (d=384, 6 heads, FFN 1536,
 4 layers, vocabulary 51865).  Weights are N(0, 0.02) bf16, LayerNorm gains 1
-and biases 0; encoder outputs are N(0, 1) bf16.
+and biases 0; encoder outputs are N(0, 1) bf16.  With `ln_noise` every
+LayerNorm gain is drawn from N(1, 0.1) and every LayerNorm bias from
+N(0, 0.05) instead (bf16), so that a test can tell the LayerNorms apart.
 """
 from __future__ import annotations
 
@@ -184,12 +186,20 @@ LAYER_KEYS = ("ln1_g", "ln1_b", "qkv_w", "qkv_b", "out_w", "out_b",
               "ln3_g", "ln3_b", "fc1_w", "fc1_b", "fc2_w", "fc2_b")
 
 
-def _layer(seed: int, prefix: str, cfg: ModelConfig, std: float) -> dict:
+def _ln_pair(seed: int, name: str, d: int, noise: bool):
+    """LayerNorm gain and bias: 1 and 0, or N(1, 0.1) and N(0, 0.05) draws."""
+    if not noise:
+        return _const_bf16((d,), 1.0), _const_bf16((d,), 0.0)
+    dev = bf16_bits_to_f32(normal_bf16(seed, name + "_g", (d,), 0.1))
+    g = f32_to_bf16_bits((dev + np.float32(1.0)).astype(np.float32))
+    return g, normal_bf16(seed, name + "_b", (d,), 0.05)
+
+
+def _layer(seed: int, prefix: str, cfg: ModelConfig, std: float, ln_noise: bool = False) -> dict:
     d, f = cfg.d_model, cfg.d_ff
     w = {}
     for nm in ("ln1", "ln2", "ln3"):
-        w[nm + "_g"] = _const_bf16((d,), 1.0)
-        w[nm + "_b"] = _const_bf16((d,), 0.0)
+        w[nm + "_g"], w[nm + "_b"] = _ln_pair(seed, prefix + nm, d, ln_noise)
     w["qkv_w"] = normal_bf16(seed, prefix + "qkv_w", (3 * d, d), std)
     qkv_b = normal_bf16(seed, prefix + "qkv_b", (3 * d,), std)
     qkv_b[d:2 * d] = 0          # the key projection carries no bias in Whisper
@@ -225,23 +235,25 @@ class WeightSet:
     drafter_layers: list = field(default_factory=list)
 
 
-def make_weights(cfg: ModelConfig, seed: int = 0, std: float = 0.02) -> WeightSet:
+def make_weights(cfg: ModelConfig, seed: int = 0, std: float = 0.02,
+                 ln_noise: bool = False) -> WeightSet:
+    """Seeded parameters.  ln_noise: LayerNorm gains N(1, 0.1) and biases
+    N(0, 0.05) (every LayerNorm its own draw) instead of 1 and 0."""
     d = cfg.d_model
     ws = WeightSet(cfg=cfg)
     ws.target["tok_emb"] = normal_bf16(seed, "tok_emb", (cfg.vocab, d), std)
     ws.target["pos_emb"] = normal_bf16(seed, "pos_emb", (cfg.max_pos, d), std)
-    ws.target["lnf_g"] = _const_bf16((d,), 1.0)
-    ws.target["lnf_b"] = _const_bf16((d,), 0.0)
-    ws.target_layers = [_layer(seed, f"t{i}.", cfg, std) for i in range(cfg.n_layers)]
+    ws.target["lnf_g"], ws.target["lnf_b"] = _ln_pair(seed, "lnf", d, ln_noise)
+    ws.target_layers = [_layer(seed, f"t{i}.", cfg, std, ln_noise) for i in range(cfg.n_layers)]
     if cfg.draft_init_from is not None:
         ws.drafter_layers = [{k: v.copy() for k, v in ws.target_layers[i].items()}
                              for i in cfg.draft_init_from]
     else:
-        ws.drafter_layers = [_layer(seed, f"d{i}.", cfg, std) for i in range(cfg.n_draft_layers)]
+        ws.drafter_layers = [_layer(seed, f"d{i}.", cfg, std, ln_noise)
+                             for i in range(cfg.n_draft_layers)]
     ws.drafter["proj_w"] = normal_bf16(seed, "d.proj_w", (d, cfg.n_taps * d), std)
     ws.drafter["proj_b"] = normal_bf16(seed, "d.proj_b", (d,), std)
-    ws.drafter["hln_g"] = _const_bf16((d,), 1.0)
-    ws.drafter["hln_b"] = _const_bf16((d,), 0.0)
+    ws.drafter["hln_g"], ws.drafter["hln_b"] = _ln_pair(seed, "d.hln", d, ln_noise)
     ws.drafter["mask_emb"] = normal_bf16(seed, "d.mask_emb", (d,), std)
     return ws
 

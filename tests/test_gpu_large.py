@@ -28,13 +28,14 @@ def _forced(g, t, a, K, V):
     return cand
 
 
-def test_large_shapes_two_steps_match_oracle():
+@pytest.mark.parametrize("ln_noise", [False, True], ids=["ln-unit", "ln-noise"])
+def test_large_shapes_two_steps_match_oracle(ln_noise):
     import torch
     from paper_2609_32869_gb300 import binding as B
     from paper_2609_32869_gb300.session import Session
     cfg = syn.LARGE
     K, V, d = cfg.block_k, cfg.vocab, cfg.d_model
-    ws = syn.make_weights(cfg, seed=0)
+    ws = syn.make_weights(cfg, seed=0, ln_noise=ln_noise)
     n = 4
     enc = syn.encoder_output(cfg, n, seed=1)
     prompt = syn.prompts(cfg, n, length=4, seed=1)

@@ -31,12 +31,12 @@ def _forced(g, t, a, K, V):
     return cand
 
 
-@pytest.fixture(scope="module")
-def tiny():
+@pytest.fixture(scope="module", params=[False, True], ids=["ln-unit", "ln-noise"])
+def tiny(request):
     import torch
     from paper_2609_32869_gb300.session import upload_weights
     cfg = syn.TINY
-    ws = syn.make_weights(cfg, seed=0)
+    ws = syn.make_weights(cfg, seed=0, ln_noise=request.param)
     dev = upload_weights(ws)
     enc = syn.encoder_output(cfg, 1, seed=1)
     torch.cuda.synchronize()

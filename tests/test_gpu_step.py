@@ -24,12 +24,15 @@ def _margin(row):
     return float(top[1] - top[0])
 
 
-@pytest.fixture(scope="module")
-def tiny():
+@pytest.fixture(scope="module", params=[False, True], ids=["ln-unit", "ln-noise"])
+def tiny(request):
+    """Tiny weights with LayerNorm gains 1 / biases 0, and with every
+    LayerNorm's gain and bias drawn on its own (so a LayerNorm applied in the
+    wrong place, or a dropped gain or bias, changes the logits)."""
     import torch
     from paper_2609_32869_gb300.session import upload_weights
     cfg = syn.TINY
-    ws = syn.make_weights(cfg, seed=0)
+    ws = syn.make_weights(cfg, seed=0, ln_noise=request.param)
     wf = syn.weights_as_float(ws)
     dev = upload_weights(ws)
     enc = syn.encoder_output(cfg, 3, seed=1)
