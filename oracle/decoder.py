@@ -284,11 +284,14 @@ class WhisperFlashOracle:
         return logits[0]
 
     def spec_step(self, seq: Sequence, forced=None, temperature: float = 0.0,
-                  seed: int = 0, suppress=None) -> StepRecord | None:
+                  seed: int = 0, suppress=None, forced_q=None) -> StepRecord | None:
         """One propose-verify-advance round (Sec. 3.1, App. A.1, A.4).
 
         forced: optional K proposals that replace the drafter's (teacher
-        forcing); the drafter still runs and its logits are returned."""
+        forcing); the drafter still runs and its logits are returned.
+        forced_q: optional [K, V] logits of the distributions the forced
+        proposals were drawn from; the rejection rule then takes q from them
+        (Sec. 3.1: q_i is the distribution the candidate was sampled from)."""
         if seq.done:
             return None
         cfg = self.cfg
@@ -308,8 +311,9 @@ class WhisperFlashOracle:
                                                         cfg.eos_id)
         else:
             xt = np.stack([acceptance.scaled_logits_fp32(r, temperature, suppress) for r in zt])
+            zq = zd if forced_q is None else np.asarray(forced_q, dtype=np.float64)
             xd = np.stack([acceptance.scaled_logits_fp32(r, temperature, suppress)
-                           for r in zd[:k]]) if k else np.zeros((0, cfg.vocab), np.float32)
+                           for r in zq[:k]]) if k else np.zeros((0, cfg.vocab), np.float32)
             coins = [philox.accept_uniform(seed, seq.seq_id, seq.step, i + 1) for i in range(k)]
             rnoise = [philox.gumbel_noise(seed, seq.seq_id, seq.step, i + 1,
                                           philox.TAG_RESIDUAL, cfg.vocab) for i in range(k)]
