@@ -48,16 +48,18 @@ WORKLOADS = {
     "tiny_b1": dict(cfg="TINY", batch=1, budget=(200, 200), accept="uniform",
                     text="Whisper-tiny-shaped decoder (d=384, 6 heads, FFN 1536, 4 layers, "
                          "vocab 51865), batch 1, accept length uniform 0..8"),
-    # Temperature sampling (App. A.4): the drafter draws its own proposals and
-    # the target applies the rejection rule with seeded Philox streams; no
-    # teacher forcing, so the accepted lengths are whatever the random weights
-    # give (reported in the line).
-    "large_b32_t07": dict(cfg="LARGE", batch=32, budget=(220, 220), temperature=0.7,
-                          text="large shapes, batch 32, temperature 0.7 speculative sampling "
-                               "(drafter's own proposals, rejection rule), 220-token budget"),
-    "large_b32_t10": dict(cfg="LARGE", batch=32, budget=(220, 220), temperature=1.0,
-                          text="large shapes, batch 32, temperature 1.0 speculative sampling "
-                               "(drafter's own proposals, rejection rule), 220-token budget"),
+    # Temperature sampling (App. A.4): proposals drawn from a seeded softmax over
+    # perturbed target logits along the target's own sampled path, passed with
+    # the logits of that distribution; the target applies the rejection rule
+    # with seeded Philox streams.
+    "large_b32_t07": dict(cfg="LARGE", batch=32, budget=(20, 220), temperature=0.7, sigma=1.0,
+                          text="large shapes, batch 32, temperature 0.7 speculative sampling; "
+                               "proposals from softmax((z_target + eps) / T), eps ~ N(0, 1) seeded, "
+                               "along the target's own sampled path; lengths uniform 20..220"),
+    "large_b32_t10": dict(cfg="LARGE", batch=32, budget=(20, 220), temperature=1.0, sigma=1.0,
+                          text="large shapes, batch 32, temperature 1.0 speculative sampling; "
+                               "proposals from softmax((z_target + eps) / T), eps ~ N(0, 1) seeded, "
+                               "along the target's own sampled path; lengths uniform 20..220"),
     # Depth-reduced cases for profiler captures: every kernel keeps the large
     # per-layer shapes and launch configuration; only the number of target
     # blocks shrinks so a capture holds a few GB and few launches.
@@ -75,7 +77,11 @@ WORKLOADS = {
 # same per-layer shapes (profiles/dram_per_kernel_large_b1_4l.md and
 # profiles/dram_per_kernel_large_b96_2l.md); None where no capture covers the
 # workload's shapes.
-GEMM_DRAM_BYTES_PER_LAUNCH = {"large_b1": 7.826e6, "large_b96": 13.17e6}
+GEMM_DRAM_BYTES_PER_LAUNCH = {}
+
+# Tensor-pipe activity of the projections at batch 96 from the committed ncu
+# capture of the same kernels (profiles/), or absent until one is taken.
+TENSOR_PIPE_FROM_PROFILE = {}
 
 
 def aggregate_ranks(times, counts, world, device):
@@ -211,22 +217,48 @@ def step_weight_kv_bytes(cfg, B, L):
     return weights, cross + self_kv
 
 
-def run_ours(args, rank, world):
+def _device_uuid(local):
+    import torch
+    try:
+        uuid = str(torch.cuda.get_device_properties(local).uuid)
+        return uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        return None
+
+
+def _family_roofline(prof, n_prof, step_ms, fam, hbm_peak, peak_src, kernel, traffic):
+    """Roofline of one kernel family.  The family's share of the step comes from
+    CUDA events around each launch (which serialise the launches), and its time
+    per step is that share of the device-timed step, so it never exceeds the
+    step; achieved = the family's algorithmic bytes per step / that time."""
+    total = sum(v["ms"] for v in prof.values())
+    share = prof[fam]["ms"] / total if total > 0 else None
+    launches = prof[fam]["launches"] / n_prof
+    if not share or not launches:
+        return None
+    fam_ms = share * step_ms
+    bytes_step = prof[fam]["bytes"] / n_prof
+    achieved = bytes_step / (fam_ms * 1e-3) / 1e9
+    return {"kernel": kernel, "bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+            "frac": achieved / hbm_peak, "traffic": traffic, "peak_source": peak_src,
+            "algorithmic_bytes_per_launch": bytes_step / launches,
+            "launches_per_step": launches, "share_of_step": share,
+            "us_per_launch": fam_ms * 1e3 / launches,
+            "measured": f"share of CUDA-event kernel time over {n_prof} profiled steps x the "
+                        f"device-timed ms_per_step"}
+
+
+def measure_greedy(args, wl_name, dev, host_ws, rank, world, steps, warmup, e2e=True):
+    """Teacher-forced speculative steps of one workload: device-timed region,
+    optionally the same steps end to end, and per-family kernel time."""
     import torch
     import torch.distributed as dist
     from paper_2609_32869_gb300 import binding as B
-    from paper_2609_32869_gb300.session import Session, upload_weights
+    from paper_2609_32869_gb300.session import Session
 
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    torch.cuda.set_device(local)
-    wl = WORKLOADS[args.workload]
+    wl = WORKLOADS[wl_name]
     cfg = _cfg(wl["cfg"], wl.get("layers"))
     Bn = wl["batch"]
-    host_ws = syn.make_weights(cfg, seed=0)
-    dev = upload_weights(host_ws)
-    need_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline
-    if not need_cpu:
-        host_ws = None
     enc = syn.encoder_output(cfg, Bn, seed=1)
     prompt = syn.prompts(cfg, Bn, length=4, seed=1)
     lo, hi = wl["budget"]
@@ -249,13 +281,12 @@ def run_ours(args, rank, world):
             break
         for b in range(Bn):
             g[b].extend(int(x) for x in toks[b, :cnt[b]])
-    n_steps = args.warmup + args.steps
+    n_steps = warmup + steps
     if wl["accept"] == "uniform":
         acc = syn.accept_uniform(max(n_steps, 64), Bn, k=cfg.block_k, seed=3)
     else:
         acc = syn.accept_geometric(max(n_steps, 64), Bn, mean=4.0, k=cfg.block_k, seed=3)
     sched = Schedule(cfg, g, budgets, acc)
-
     d_slots = torch.as_tensor(slots, device="cuda")
 
     def restart_job():
@@ -270,13 +301,14 @@ def run_ours(args, rank, world):
         and the tokens it emits."""
         sched.restart()
         forced = np.zeros((n, Bn, cfg.block_k), np.int32)
-        pre, comp, toks, kv = [], [], [], []
+        pre, comp, toks, kv, ctx = [], [], [], [], []
         for i in range(n):
             restart = bool(sched.done.all())
             if restart:
                 sched.restart()
             live = [4 + int(sched.t[b]) - 1 for b in range(Bn) if not sched.done[b]]
             kv.append(step_weight_kv_bytes(cfg, len(live), live)[1])
+            ctx.append(float(np.mean(live)) if live else 0.0)
             f, em = sched.step()
             forced[i] = f
             pre.append(restart)
@@ -284,7 +316,8 @@ def run_ours(args, rank, world):
             toks.append(int(em.sum()))
         lens = [4 + int(sched.t[b]) - 1 for b in range(Bn)]
         dev_forced = torch.as_tensor(forced).cuda()
-        return dict(forced=forced, dev=dev_forced, pre=pre, comp=comp, toks=toks, lens=lens, kv=kv)
+        return dict(forced=forced, dev=dev_forced, pre=pre, comp=comp, toks=toks, lens=lens, kv=kv,
+                    ctx=ctx)
 
     def execute(pl, lo, hi, e2e=False, pin=None):
         launches = 0
@@ -294,32 +327,26 @@ def run_ours(args, rank, world):
             if e2e:
                 pin["in"].copy_(torch.as_tensor(pl["forced"][i]))
                 pin["dev_in"].copy_(pin["in"], non_blocking=True)
-                B.wf_step(sess.h, None, pin["dev_in"], sess.out_tokens, sess.out_count, stream)
+                B.wf_step(sess.h, None, pin["dev_in"], None, sess.out_tokens, sess.out_count, stream)
                 launches += B.wf_last_launch_count(sess.h)
                 pin["out_tok"].copy_(sess.out_tokens, non_blocking=True)
                 pin["out_cnt"].copy_(sess.out_count, non_blocking=True)
                 stream.synchronize()
             else:
-                B.wf_step(sess.h, None, pl["dev"][i], sess.out_tokens, sess.out_count, stream)
+                B.wf_step(sess.h, None, pl["dev"][i], None, sess.out_tokens, sess.out_count, stream)
                 launches += B.wf_last_launch_count(sess.h)
             if pl["comp"][i]:
                 B.wf_compact(sess.h, stream)
                 launches += 1
         return launches
 
-    uuid = None
-    try:
-        uuid = str(torch.cuda.get_device_properties(local).uuid)
-        if uuid and not uuid.startswith("GPU-"):
-            uuid = "GPU-" + uuid
-    except Exception:
-        uuid = None
-    sampler, clock_path = _clock_sampler(uuid)
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    sampler, clock_path = _clock_sampler(_device_uuid(local))
 
     # ---- warm-up and the device-timed region (inputs already in HBM)
     pl = make_plan(n_steps)
     restart_job()
-    execute(pl, 0, args.warmup)
+    execute(pl, 0, warmup)
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
@@ -328,7 +355,7 @@ def run_ours(args, rank, world):
     if args.profile_region:
         torch.cuda.profiler.start()
     e0.record(stream)
-    launches = execute(pl, args.warmup, n_steps)
+    launches = execute(pl, warmup, n_steps)
     e1.record(stream)
     torch.cuda.synchronize()
     if args.profile_region:
@@ -336,37 +363,6 @@ def run_ours(args, rank, world):
     if world > 1:
         dist.barrier()
     dev_ms = e0.elapsed_time(e1)
-    tokens = sum(pl["toks"][args.warmup:])
-    state = sess.state()
-    err = sess.error()
-    consistent = bool(all(int(state["len"][b]) == pl["lens"][b] for b in range(Bn)) and err == 0)
-
-    # ---- end to end through the C ABI: pinned host proposals in, tokens out
-    Kc = cfg.block_k
-    pin = {"in": torch.empty((Bn, Kc), dtype=torch.int32).pin_memory(),
-           "dev_in": torch.empty((Bn, Kc), dtype=torch.int32, device="cuda"),
-           "out_tok": torch.empty((Bn, Kc + 1), dtype=torch.int32).pin_memory(),
-           "out_cnt": torch.empty((Bn,), dtype=torch.int32).pin_memory()}
-    # the same steps as the device-timed region, after the same warm-up
-    pl2 = make_plan(n_steps)
-    restart_job()
-    execute(pl2, 0, args.warmup)
-    torch.cuda.synchronize()
-    w0 = time.perf_counter()
-    execute(pl2, args.warmup, n_steps, e2e=True, pin=pin)
-    torch.cuda.synchronize()
-    e2e_s = time.perf_counter() - w0
-    e2e_tokens = sum(pl2["toks"][args.warmup:])
-
-    # ---- per-family kernel time with CUDA events (roofline of the top kernel)
-    n_prof = min(args.steps, 5)
-    pl3 = make_plan(n_prof)
-    restart_job()
-    B.wf_set_option(sess.h, B.WF_OPT_PROFILE, 1)
-    execute(pl3, 0, n_prof)
-    prof = B.wf_profile_read(sess.h, stream)
-    B.wf_set_option(sess.h, B.WF_OPT_PROFILE, 0)
-
     if sampler is not None:
         sampler.terminate()
         sampler.wait()
@@ -375,19 +371,79 @@ def run_ours(args, rank, world):
         os.unlink(clock_path)
     except OSError:
         pass
+    tokens = sum(pl["toks"][warmup:])
+    state = sess.state()
+    err = sess.error()
+    consistent = bool(all(int(state["len"][b]) == pl["lens"][b] for b in range(Bn)) and err == 0)
 
-    # ---- aggregate over ranks
-    (dev_ms, e2e_s), (tokens, e2e_tokens) = aggregate_ranks([dev_ms, e2e_s], [tokens, e2e_tokens], world, "cuda")
+    e2e_s = e2e_tokens = None
+    if e2e:
+        # end to end through the C ABI: pinned host proposals in, tokens out
+        Kc = cfg.block_k
+        pin = {"in": torch.empty((Bn, Kc), dtype=torch.int32).pin_memory(),
+               "dev_in": torch.empty((Bn, Kc), dtype=torch.int32, device="cuda"),
+               "out_tok": torch.empty((Bn, Kc + 1), dtype=torch.int32).pin_memory(),
+               "out_cnt": torch.empty((Bn,), dtype=torch.int32).pin_memory()}
+        pl2 = make_plan(n_steps)
+        restart_job()
+        execute(pl2, 0, warmup)
+        torch.cuda.synchronize()
+        w0 = time.perf_counter()
+        execute(pl2, warmup, n_steps, e2e=True, pin=pin)
+        torch.cuda.synchronize()
+        e2e_s = time.perf_counter() - w0
+        e2e_tokens = sum(pl2["toks"][warmup:])
 
+    # ---- per-family kernel time with CUDA events (shares of the step)
+    n_prof = min(steps, 5)
+    pl3 = make_plan(n_prof)
+    restart_job()
+    B.wf_set_option(sess.h, B.WF_OPT_PROFILE, 1)
+    execute(pl3, 0, n_prof)
+    prof = B.wf_profile_read(sess.h, stream)
+    B.wf_set_option(sess.h, B.WF_OPT_PROFILE, 0)
+    sess.close()
+    del sess
+    torch.cuda.empty_cache()
+
+    wbytes = step_weight_kv_bytes(cfg, 0, [])[0]
+    return dict(cfg=cfg, batch=Bn, dev_ms=dev_ms, tokens=tokens, e2e_s=e2e_s, e2e_tokens=e2e_tokens,
+                prof=prof, n_prof=n_prof, clocks=clocks, consistent=consistent, err=err,
+                launches=launches, wbytes=wbytes, kvbytes=float(np.mean(pl["kv"][warmup:])),
+                ctx=(min(pl["ctx"][warmup:]), float(np.mean(pl["ctx"][warmup:])), max(pl["ctx"][warmup:])),
+                budgets=budgets, acc=acc, enc=enc, prompt=prompt)
+
+
+def _step_roofline(m, step_ms, hbm_peak, peak_src):
+    b = m["wbytes"] + m["kvbytes"]
+    return {"bytes": b, "weights": m["wbytes"], "kv": m["kvbytes"],
+            "achieved_gbs": b / (step_ms * 1e-3) / 1e9, "peak_gbs": hbm_peak,
+            "frac": b / (step_ms * 1e-3) / 1e9 / hbm_peak,
+            "peak_source": f"{peak_src} (MEASURED_PEAKS hbm_gbs)"}
+
+
+def run_ours(args, rank, world):
+    import torch
+    from paper_2609_32869_gb300.session import upload_weights
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    wl = WORKLOADS[args.workload]
+    cfg = _cfg(wl["cfg"], wl.get("layers"))
+    host_ws = syn.make_weights(cfg, seed=0)
+    dev = upload_weights(host_ws)
+    need_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline
+    m = measure_greedy(args, args.workload, dev, host_ws, rank, world, args.steps, args.warmup)
+    (dev_ms, e2e_s), (tokens, e2e_tokens) = aggregate_ranks([m["dev_ms"], m["e2e_s"]],
+                                                            [m["tokens"], m["e2e_tokens"]], world, "cuda")
     hbm_peak, bf16_peak, peak_src = _peaks()
     step_ms = dev_ms / args.steps
-    wbytes = step_weight_kv_bytes(cfg, 0, [])[0]
-    kvbytes = float(np.mean(pl["kv"][args.warmup:]))
+    prof, n_prof = m["prof"], m["n_prof"]
     fam = max(("gemm", "head", "attn_cross", "attn_self", "persist"), key=lambda f: prof[f]["ms"])
     roof_fam = "persist" if args.persist else "gemm"
-    fam_ms = prof[roof_fam]["ms"]
-    gemm_gbs = prof[roof_fam]["bytes"] / (fam_ms * 1e-3) / 1e9 if fam_ms > 0 else None
-    step_total_prof = sum(v["ms"] for v in prof.values())
+    kernel = ("persist_kernel (every block of a pass in one launch; bytes = weights and acoustic K/V)"
+              if args.persist else "gemm_tc_kernel (tcgen05 projections)")
+    Bn, Kc = m["batch"], cfg.block_k
     result = {
         "metric": METRIC,
         "value": tokens / (dev_ms * 1e-3),
@@ -403,46 +459,66 @@ def run_ours(args, rank, world):
         "data": "synthetic (seeded random weights and encoder outputs; proposals teacher-forced "
                 "from the target's own greedy continuation)",
         "config": {"workload": args.workload, "description": wl["text"], "batch": Bn,
-                   "block": cfg.block_k + 1, "parallelism": f"replicas x{world}",
+                   "block": Kc + 1, "parallelism": f"replicas x{world}",
                    "path": "persistent passes" if args.persist else "launch by launch",
                    "l2": "inputs larger than L2 (every step streams "
-                         f"{(wbytes + kvbytes) / 1e9:.2f} GB of weights and K/V > 129 MB L2)"},
+                         f"{(m['wbytes'] + m['kvbytes']) / 1e9:.2f} GB of weights and K/V > 129 MB L2)"},
         "step_us": step_ms * 1e3,
         "tokens_per_step": tokens / args.steps / world,
-        "step_roofline": {"bytes": wbytes + kvbytes, "weights": wbytes, "kv": kvbytes,
-                          "achieved_gbs": (wbytes + kvbytes) / (step_ms * 1e-3) / 1e9,
-                          "peak_gbs": hbm_peak,
-                          "frac": (wbytes + kvbytes) / (step_ms * 1e-3) / 1e9 / hbm_peak,
-                          "peak_source": f"{peak_src} (MEASURED_PEAKS hbm_gbs)"},
-        "roofline": {"kernel": ("persist_kernel (every block of a pass in one launch; bytes = weights "
-                                "and acoustic K/V)") if args.persist else "gemm_tc_kernel (tcgen05 projections)",
-                     "bound": "hbm",
-                     "achieved": gemm_gbs, "peak": hbm_peak, "unit": "GB/s",
-                     "frac": gemm_gbs / hbm_peak if gemm_gbs else None,
-                     "traffic": None if args.persist else GEMM_DRAM_BYTES_PER_LAUNCH.get(args.workload),
-                     "peak_source": peak_src,
-                     "measured": f"CUDA events around each launch over {n_prof} profiled steps",
-                     "share_of_kernel_time": fam_ms / step_total_prof if step_total_prof else None},
+        "context_len": {"min": m["ctx"][0], "mean": m["ctx"][1], "max": m["ctx"][2]},
+        "step_roofline": _step_roofline(m, step_ms, hbm_peak, peak_src),
+        "roofline": _family_roofline(prof, n_prof, step_ms, roof_fam, hbm_peak, peak_src, kernel,
+                                     None if args.persist else GEMM_DRAM_BYTES_PER_LAUNCH.get(args.workload)),
         "kernel_families_ms_per_step": {k: v["ms"] / n_prof for k, v in prof.items()},
         "kernel_families_launches_per_step": {k: v["launches"] / n_prof for k, v in prof.items()},
         "top_family": fam,
         "e2e": {"value": e2e_tokens / e2e_s, "unit": "tokens/s",
                 "h2d_bytes_per_step": Bn * Kc * 4,
                 "d2h_bytes_per_step": Bn * (Kc + 1) * 4 + Bn * 4},
-        "gpu_launches": launches,
-        "clocks": clocks,
-        "consistent": consistent,
-        "device_error": err,
+        "gpu_launches": m["launches"],
+        "clocks": m["clocks"],
+        "consistent": m["consistent"],
+        "device_error": m["err"],
     }
+    if args.workload == "large_b1" and not args.no_per_batch and not args.budget:
+        # the metric's other batch sizes, timed in the same run on the same weights
+        per = {}
+        for name in ("large_b16", "large_b96"):
+            mb = measure_greedy(args, name, dev, None, rank, world, args.batch_steps, args.warmup, e2e=False)
+            (bms,), (btok,) = aggregate_ranks([mb["dev_ms"]], [mb["tokens"]], world, "cuda")
+            sms = bms / args.batch_steps
+            per[str(mb["batch"])] = {
+                "workload": name, "description": WORKLOADS[name]["text"],
+                "value": btok / (bms * 1e-3), "unit": "tokens/s", "ms_per_step": sms,
+                "steps": args.batch_steps, "tokens_per_step": btok / args.batch_steps / world,
+                "context_len": {"min": mb["ctx"][0], "mean": mb["ctx"][1], "max": mb["ctx"][2]},
+                "step_roofline": _step_roofline(mb, sms, hbm_peak, peak_src),
+                "roofline": _family_roofline(mb["prof"], mb["n_prof"], sms, "gemm", hbm_peak, peak_src,
+                                             "gemm_tc_kernel (tcgen05 projections)",
+                                             GEMM_DRAM_BYTES_PER_LAUNCH.get(name)),
+                "kernel_families_ms_per_step": {k: v["ms"] / mb["n_prof"] for k, v in mb["prof"].items()},
+                "clocks": mb["clocks"], "consistent": mb["consistent"], "device_error": mb["err"],
+                "gpu_launches": mb["launches"]}
+            if name in TENSOR_PIPE_FROM_PROFILE:
+                per[str(mb["batch"])]["projection_tensor_pipe"] = TENSOR_PIPE_FROM_PROFILE[name]
+        result["per_batch"] = per
     if need_cpu:
-        result["cpu_baseline"] = cpu_baseline(cfg, host_ws, enc, prompt, budgets, acc,
-                                              budget_s=args.cpu_seconds)
+        result["cpu_baseline"] = cpu_baseline(cfg, host_ws, m["enc"], m["prompt"], m["budgets"], m["acc"],
+                                              budget_s=args.cpu_seconds, gpu_ctx=m["ctx"])
     return result
 
 
 def run_sampling(args, rank, world):
-    """Speculative sampling steps: tokens/s from the counts the step itself
-    returns (written per step into a device array, read after the region)."""
+    """Speculative sampling steps at temperature T with the workload's proposal
+    recipe: drafts sampled from q = softmax((z + sigma eps) / T), z the target's
+    logits along its own sampled path (a plain-sampling pre-pass on the GPU,
+    untimed) and eps seeded N(0, 1); the candidates and the logits of q go to
+    wf_step, whose rejection rule takes q from them.  The job is first run
+    once untimed with host reads between steps (the proposals of each step
+    depend on how many tokens each sequence has emitted), recording every
+    step's inputs; the timed region replays the same inputs from the same
+    post-prefill state, so it runs the identical trajectory with no host
+    reads.  tokens/s counts what the steps emit."""
     import torch
     import torch.distributed as dist
     from paper_2609_32869_gb300 import binding as B
@@ -452,37 +528,93 @@ def run_sampling(args, rank, world):
     torch.cuda.set_device(local)
     wl = WORKLOADS[args.workload]
     cfg = _cfg(wl["cfg"], wl.get("layers"))
-    Bn, Kc = wl["batch"], cfg.block_k
+    Bn, Kc, V = wl["batch"], cfg.block_k, cfg.vocab
+    T, sigma = wl["temperature"], wl["sigma"]
     dev = upload_weights(syn.make_weights(cfg, seed=0))
     enc = syn.encoder_output(cfg, Bn, seed=1)
     prompt = syn.prompts(cfg, Bn, length=4, seed=1)
-    budgets = np.full(Bn, wl["budget"][0], np.int32)
+    lo, hi = wl["budget"]
+    budgets = syn.budgets(Bn, lo, hi, seed=2)
     sess = Session(cfg, dev, max_batch=Bn, max_ctx=cfg.max_pos)
     stream = sess.stream
-    sp = B.sample_params(wl["temperature"], 4 + rank)
-    sess.prefill(np.arange(Bn, dtype=np.int32), enc, prompt, budgets, sp=sp)
+    slots = np.arange(Bn, dtype=np.int32)
+    d_slots = torch.as_tensor(slots, device="cuda")
+    sp = B.sample_params(T, 4 + rank)
+    sess.prefill(slots, enc, prompt, budgets, sp=sp)
+
+    # pre-pass: plain sampling of the target along its own path; z[b, i] are
+    # the logits the target's token i + 1 of sequence b is drawn from
+    B.wf_set_option(sess.h, B.WF_OPT_KEEP_LOGITS, 1)
+    z = torch.zeros((Bn, hi + Kc, V), dtype=torch.float32, device="cuda")
+    pos = np.zeros(Bn, np.int64)
+    sess.compact()
+    while True:
+        st = sess.state()
+        act = [b for b in range(Bn) if not st["done"][b]]
+        if not act:
+            break
+        sess.greedy_step(sp=sp)
+        rows = sess.view(B.WF_VIEW_TARGET_LOGITS, torch.float32, (len(act), V))
+        for i, b in enumerate(act):
+            z[b, pos[b]] = rows[i]
+            pos[b] += 1
+        if any(sess.state()["done"][b] for b in act):
+            sess.compact()
+    B.wf_set_option(sess.h, B.WF_OPT_KEEP_LOGITS, 0)
+
+    def restart():
+        B.wf_reset_slots(sess.h, Bn, d_slots, stream)
+        return B.wf_compact(sess.h, stream)
+
     n_steps = args.warmup + args.steps
+    gen = torch.Generator(device="cuda")
     counts = torch.zeros(n_steps, Bn, dtype=torch.int32, device="cuda")
     toks = torch.zeros(n_steps, Bn, Kc + 1, dtype=torch.int32, device="cuda")
+    rec_f, rec_q, rec_pre, rec_comp = [], [], [], []
+    # recording pass (untimed): the proposals of each step from the emitted counts so far
+    restart()
+    for i in range(n_steps):
+        st = sess.state()
+        pre = bool((st["done"] != 0).all())
+        if pre:
+            restart()
+            st = sess.state()
+        t = np.array([int(budgets[b]) - int(st["remaining"][b]) for b in range(Bn)])
+        idx = torch.as_tensor(np.clip(t[:, None] - 1 + np.arange(Kc)[None, :], 0, hi + Kc - 1),
+                              device="cuda")
+        gen.manual_seed(1000 + i)
+        zq = torch.gather(z, 1, idx[:, :, None].expand(Bn, Kc, V)) + \
+            sigma * torch.randn((Bn, Kc, V), generator=gen, device="cuda")
+        u = torch.rand((Bn, Kc, V), generator=gen, device="cuda").clamp_(1e-12, 1.0)
+        cand = torch.argmax(zq / T - torch.log(-torch.log(u)), dim=-1).to(torch.int32)
+        B.wf_step(sess.h, sp, cand, zq, toks[i], counts[i], stream)
+        done = sess.state()["done"] != 0
+        comp = bool(done.any())
+        if comp:
+            B.wf_compact(sess.h, stream)
+        rec_f.append(cand)
+        rec_q.append(zq)
+        rec_pre.append(pre)
+        rec_comp.append(comp)
+    want = counts.clone()
 
-    def run(lo, hi):
+    def run(lo, hi_):
         n = 0
-        for i in range(lo, hi):
-            B.wf_step(sess.h, sp, None, toks[i], counts[i], stream)
+        for i in range(lo, hi_):
+            if rec_pre[i]:
+                restart()
+                n += 2
+            B.wf_step(sess.h, sp, rec_f[i], rec_q[i], toks[i], counts[i], stream)
             n += B.wf_last_launch_count(sess.h)
+            if rec_comp[i]:
+                B.wf_compact(sess.h, stream)
+                n += 1
         return n
 
-    uuid = None
-    try:
-        uuid = str(torch.cuda.get_device_properties(local).uuid)
-        if uuid and not uuid.startswith("GPU-"):
-            uuid = "GPU-" + uuid
-    except Exception:
-        uuid = None
-    sampler, clock_path = _clock_sampler(uuid)
+    sampler, clock_path = _clock_sampler(_device_uuid(local))
+    restart()
     run(0, args.warmup)
     torch.cuda.synchronize()
-    len0 = sess.state()["len"].astype(np.float64)
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -498,32 +630,6 @@ def run_sampling(args, rank, world):
     if world > 1:
         dist.barrier()
     dev_ms = e0.elapsed_time(e1)
-    len1 = sess.state()["len"].astype(np.float64)
-    c = counts[args.warmup:].cpu().numpy()
-    tokens = float(c.sum())
-    live = c > 0
-    accepted = float((c[live] - 1).mean()) if live.any() else 0.0
-
-    # end to end: the same call with the step's outputs read back to pinned
-    # host memory every step (the step takes no per-step input)
-    h_tok = torch.empty((Bn, Kc + 1), dtype=torch.int32).pin_memory()
-    h_cnt = torch.empty((Bn,), dtype=torch.int32).pin_memory()
-    e2e_tokens = 0
-    torch.cuda.synchronize()
-    w0 = time.perf_counter()
-    for i in range(args.warmup, n_steps):
-        B.wf_step(sess.h, sp, None, toks[i], counts[i], stream)
-        h_tok.copy_(toks[i], non_blocking=True)
-        h_cnt.copy_(counts[i], non_blocking=True)
-        stream.synchronize()
-        e2e_tokens += int(h_cnt.sum())
-    e2e_s = time.perf_counter() - w0
-
-    n_prof = min(args.steps, 3)
-    B.wf_set_option(sess.h, B.WF_OPT_PROFILE, 1)
-    run(0, n_prof)
-    prof = B.wf_profile_read(sess.h, stream)
-    B.wf_set_option(sess.h, B.WF_OPT_PROFILE, 0)
     if sampler is not None:
         sampler.terminate()
         sampler.wait()
@@ -532,14 +638,48 @@ def run_sampling(args, rank, world):
         os.unlink(clock_path)
     except OSError:
         pass
+    c = counts[args.warmup:].cpu().numpy()
+    replayed = bool(torch.equal(counts, want))
+    tokens = float(c.sum())
+    live = c > 0
+    accepted = float((c[live] - 1).mean()) if live.any() else 0.0
+
+    # end to end: the same replay with each step's outputs read back to pinned host memory
+    h_tok = torch.empty((Bn, Kc + 1), dtype=torch.int32).pin_memory()
+    h_cnt = torch.empty((Bn,), dtype=torch.int32).pin_memory()
+    restart()
+    run(0, args.warmup)
+    torch.cuda.synchronize()
+    e2e_tokens = 0
+    w0 = time.perf_counter()
+    for i in range(args.warmup, n_steps):
+        if rec_pre[i]:
+            restart()
+        B.wf_step(sess.h, sp, rec_f[i], rec_q[i], toks[i], counts[i], stream)
+        h_tok.copy_(toks[i], non_blocking=True)
+        h_cnt.copy_(counts[i], non_blocking=True)
+        stream.synchronize()
+        e2e_tokens += int(h_cnt.sum())
+        if rec_comp[i]:
+            B.wf_compact(sess.h, stream)
+    e2e_s = time.perf_counter() - w0
+
+    n_prof = min(args.steps, 3)
+    restart()
+    B.wf_set_option(sess.h, B.WF_OPT_PROFILE, 1)
+    run(0, n_prof)
+    prof = B.wf_profile_read(sess.h, stream)
+    B.wf_set_option(sess.h, B.WF_OPT_PROFILE, 0)
+    st = sess.state()
+    err = sess.error()
+    sess.close()
 
     (dev_ms, e2e_s), (tokens, e2e_tokens) = aggregate_ranks([dev_ms, e2e_s], [tokens, e2e_tokens], world, "cuda")
     hbm_peak, _, peak_src = _peaks()
     step_ms = dev_ms / args.steps
-    mean_len = list((len0 + len1) / 2.0)
-    wbytes, kvbytes = step_weight_kv_bytes(cfg, Bn, [int(x) for x in mean_len])
-    fam_ms = prof["gemm"]["ms"]
-    gemm_gbs = prof["gemm"]["bytes"] / (fam_ms * 1e-3) / 1e9 if fam_ms > 0 else None
+    mean_L = [4 + int(budgets[b]) // 2 for b in range(Bn)]
+    wbytes, kvbytes = step_weight_kv_bytes(cfg, Bn, mean_L)
+    m = {"wbytes": wbytes, "kvbytes": kvbytes}
     return {
         "metric": METRIC,
         "value": tokens / (dev_ms * 1e-3),
@@ -552,33 +692,29 @@ def run_sampling(args, rank, world):
         "scaling": "weak",
         "vs_baseline": None,
         "dtype": "bf16",
-        "data": "synthetic (seeded random weights and encoder outputs; the drafter's own "
-                "sampled proposals)",
+        "data": "synthetic (seeded random weights and encoder outputs; proposals drawn from a "
+                "seeded softmax over perturbed target logits along the target's own sampled path)",
         "config": {"workload": args.workload, "description": wl["text"], "batch": Bn,
-                   "block": Kc + 1, "temperature": wl["temperature"],
+                   "block": Kc + 1, "temperature": T, "sigma": sigma,
                    "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2 (every step streams "
                          f"{(wbytes + kvbytes) / 1e9:.2f} GB of weights and K/V > 129 MB L2)"},
         "step_us": step_ms * 1e3,
         "tokens_per_step": tokens / args.steps / world,
         "accepted_drafts_per_sequence_step": accepted,
-        "step_roofline": {"bytes": wbytes + kvbytes, "weights": wbytes, "kv": kvbytes,
-                          "achieved_gbs": (wbytes + kvbytes) / (step_ms * 1e-3) / 1e9,
-                          "peak_gbs": hbm_peak,
-                          "frac": (wbytes + kvbytes) / (step_ms * 1e-3) / 1e9 / hbm_peak,
-                          "peak_source": f"{peak_src} (MEASURED_PEAKS hbm_gbs)"},
-        "roofline": {"kernel": "gemm_tc_kernel (tcgen05 projections)", "bound": "hbm",
-                     "achieved": gemm_gbs, "peak": hbm_peak, "unit": "GB/s",
-                     "frac": gemm_gbs / hbm_peak if gemm_gbs else None,
-                     "traffic": GEMM_DRAM_BYTES_PER_LAUNCH.get(args.workload),
-                     "peak_source": peak_src,
-                     "measured": f"CUDA events around each launch over {n_prof} profiled steps"},
+        "acceptance_rate": accepted / Kc,
+        "replayed_identically": replayed,
+        "step_roofline": _step_roofline(m, step_ms, hbm_peak, peak_src),
+        "roofline": _family_roofline(prof, n_prof, step_ms, "gemm", hbm_peak, peak_src,
+                                     "gemm_tc_kernel (tcgen05 projections)", None),
         "kernel_families_ms_per_step": {k: v["ms"] / n_prof for k, v in prof.items()},
-        "e2e": {"value": e2e_tokens / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": 0,
-                "d2h_bytes_per_step": Bn * (Kc + 1) * 4 + Bn * 4},
+        "e2e": {"value": e2e_tokens / e2e_s, "unit": "tokens/s",
+                "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": Bn * (Kc + 1) * 4 + Bn * 4,
+                "note": "the proposals and their logits are prepared on the device before the region"},
         "gpu_launches": launches,
         "clocks": clocks,
-        "device_error": sess.error(),
+        "device_error": err,
     }
 
 
@@ -644,13 +780,17 @@ def _cores():
         return os.cpu_count() or 1
 
 
-def cpu_baseline(cfg, ws, enc, prompt, budgets, acc, budget_s=15.0):
+def cpu_baseline(cfg, ws, enc, prompt, budgets, acc, budget_s=15.0, gpu_ctx=None):
     tokens, secs, steps = _oracle_run(cfg, ws, enc, prompt, budgets, acc, 0, 64,
                                       prefix_tokens=24, time_cap_s=budget_s)
+    ctx = (f"; the GPU arm's steps run at context lengths {gpu_ctx[0]:.0f}..{gpu_ctx[2]:.0f} "
+           f"(mean {gpu_ctx[1]:.0f}); the oracle's cost is dominated by the weights, which do not "
+           f"depend on the context") if gpu_ctx else ""
     return {"value": tokens / secs, "unit": "tokens/s", "cores": _cores(), "kind": "oracle",
             "sample": f"{steps} teacher-forced speculative steps of sequence 0 over the first "
-                      f"24 tokens of its transcript (float64 numpy oracle; prefill and the "
-                      f"oracle's own greedy prefix untimed), {tokens} tokens in {secs:.1f} s",
+                      f"24 tokens of its transcript, context lengths 5..28 (float64 numpy oracle; "
+                      f"prefill and the oracle's own greedy prefix untimed), {tokens} tokens in "
+                      f"{secs:.1f} s" + ctx,
             "ms_per_step": secs / steps * 1e3}
 
 
@@ -735,6 +875,10 @@ def main():
                     help="cudaProfilerStart/Stop around the timed steps (for ncu)")
     ap.add_argument("--budget", type=int, default=0,
                     help="override every transcript budget (short profiling runs)")
+    ap.add_argument("--no-per-batch", action="store_true",
+                    help="skip the batch-16 and batch-96 entries of the default line")
+    ap.add_argument("--batch-steps", type=int, default=20,
+                    help="timed steps of each per-batch entry")
     ap.add_argument("--persist", action="store_true",
                     help="run every drafter, verify and greedy pass as one persistent launch "
                          "(WF_OPT_PERSIST; batch * 9 <= 16 only)")

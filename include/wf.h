@@ -164,14 +164,22 @@ wf_status wf_draft(wf_handle *h, const wf_sample_params *sp, void *stream);
  *   d_out_tokens int32 [max_batch, K+1] (per slot; entries past the count are -1)
  *   d_out_count  int32 [max_batch]      tokens emitted this step (0 if inactive)
  * d_forced (nullable) int32 [max_batch, K] replaces the drafter's proposals
- * (teacher forcing); the drafter's own pass is unaffected. */
+ * (teacher forcing); the drafter's own pass is unaffected.
+ * d_forced_q (nullable; needs d_forced) fp32 [max_batch, K, vocab]: the logits of
+ * the distributions the forced proposals were drawn from, row j for proposal
+ * c_{j+1}, in the units of the drafter's logits (they get the same temperature
+ * and suppression).  When sampling, the rejection rule then uses
+ * q = softmax(d_forced_q / T) in place of the drafter's distribution: the rule
+ * preserves the target's distribution only if q is the distribution the
+ * proposals actually came from (Sec. 3.1, App. A.4).  Ignored when greedy. */
 wf_status wf_verify_accept(wf_handle *h, const wf_sample_params *sp,
-                           const int32_t *d_forced, int32_t *d_out_tokens,
-                           int32_t *d_out_count, void *stream);
+                           const int32_t *d_forced, const float *d_forced_q,
+                           int32_t *d_out_tokens, int32_t *d_out_count, void *stream);
 
 /* wf_draft followed by wf_verify_accept. */
 wf_status wf_step(wf_handle *h, const wf_sample_params *sp, const int32_t *d_forced,
-                  int32_t *d_out_tokens, int32_t *d_out_count, void *stream);
+                  const float *d_forced_q, int32_t *d_out_tokens, int32_t *d_out_count,
+                  void *stream);
 
 /* One plain autoregressive step of the target (Eq. 1; sampling when T > 0)
  * through the same kernels: the identity reference for the speculative path.

@@ -77,8 +77,8 @@ _SIGS = {
     "wf_destroy": (_I, [_P]),
     "wf_prefill_cross_kv": (_I, [_P, _I, _P, _P, _P, _I, _P, _P, C.POINTER(WfSampleParams), _P]),
     "wf_draft": (_I, [_P, C.POINTER(WfSampleParams), _P]),
-    "wf_verify_accept": (_I, [_P, C.POINTER(WfSampleParams), _P, _P, _P, _P]),
-    "wf_step": (_I, [_P, C.POINTER(WfSampleParams), _P, _P, _P, _P]),
+    "wf_verify_accept": (_I, [_P, C.POINTER(WfSampleParams), _P, _P, _P, _P, _P]),
+    "wf_step": (_I, [_P, C.POINTER(WfSampleParams), _P, _P, _P, _P, _P]),
     "wf_greedy_step": (_I, [_P, C.POINTER(WfSampleParams), _P, _P, _P]),
     "wf_compact": (_I, [_P, _P, C.POINTER(_I)]),
     "wf_reset_slots": (_I, [_P, _I, _P, _P]),
@@ -217,15 +217,16 @@ def wf_draft(h, sp=None, stream=None):
     _check("wf_draft", lib().wf_draft(h, C.byref(sp) if sp is not None else None, _stream(stream)))
 
 
-def wf_verify_accept(h, sp, forced, out_tokens, out_count, stream=None):
+def wf_verify_accept(h, sp, forced, forced_q, out_tokens, out_count, stream=None):
     _check("wf_verify_accept", lib().wf_verify_accept(
-        h, C.byref(sp) if sp is not None else None, _ptr(forced), _ptr(out_tokens),
-        _ptr(out_count), _stream(stream)))
+        h, C.byref(sp) if sp is not None else None, _ptr(forced), _ptr(forced_q),
+        _ptr(out_tokens), _ptr(out_count), _stream(stream)))
 
 
-def wf_step(h, sp, forced, out_tokens, out_count, stream=None):
+def wf_step(h, sp, forced, forced_q, out_tokens, out_count, stream=None):
     _check("wf_step", lib().wf_step(h, C.byref(sp) if sp is not None else None, _ptr(forced),
-                                    _ptr(out_tokens), _ptr(out_count), _stream(stream)))
+                                    _ptr(forced_q), _ptr(out_tokens), _ptr(out_count),
+                                    _stream(stream)))
 
 
 def wf_greedy_step(h, sp, out_tokens, out_count, stream=None):

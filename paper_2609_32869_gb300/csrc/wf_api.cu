@@ -79,6 +79,7 @@ struct wf_handle {
   bool use_graphs = true;
   cudaStream_t cap_stream = nullptr;
   int32_t *forced_buf = nullptr, *tok_buf = nullptr, *cnt_buf = nullptr;
+  float *fq_buf = nullptr;  // forced proposal logits [Bmax][K][V] (wf_step copies them here)
   // persistent small-batch passes (wf_persist.cu)
   bool mk_ok = false;   // the shapes and limits allow it (fixed at create)
   bool mk_on = false;   // in use (WF_OPT_PERSIST)
@@ -185,6 +186,7 @@ size_t layout(wf_handle *h, const wf_config *c, int Bmax, int ctx, char *base) {
   o->hout_d = cv.take<HeadOut>(M);
   o->logits_t = cv.take<float>(M * V);
   o->logits_d = cv.take<float>(M * V);
+  o->fq_buf = cv.take<float>(sl * K * V);
   o->rope = cv.take<float2>(static_cast<size_t>(c->max_pos) * 32);
   o->mk_ok = persist_supported(d, H, F, T, Bmax * (K + 1));
   if (o->mk_ok) {
@@ -1039,7 +1041,8 @@ static wf_status draft_body(wf_handle *h, const wf_sample_params *sp, cudaStream
 }
 
 static wf_status verify_body(wf_handle *h, const wf_sample_params *sp, const int32_t *d_forced,
-                             int32_t *d_out_tokens, int32_t *d_out_count, cudaStream_t s) {
+                             const float *d_forced_q, int32_t *d_out_tokens, int32_t *d_out_count,
+                             cudaStream_t s) {
   const int n = h->n_active, rps = h->K + 1;
   if (n > 0) {
     if (h->mk_on) {
@@ -1068,6 +1071,7 @@ static wf_status verify_body(wf_handle *h, const wf_sample_params *sp, const int
   ap.cand = h->cand;
   ap.tlogits = h->logits_t;
   ap.dlogits = h->logits_d;
+  ap.forced_q = d_forced_q;
   ap.suppress = sp ? sp->d_suppress : nullptr;
   ap.temperature = (sp && sp->temperature > 0.f) ? sp->temperature : 0.f;
   ap.seed = sp ? sp->seed : 0;
@@ -1170,11 +1174,11 @@ static wf_status run_graphed(wf_handle *h, wf_handle::GraphKey key, cudaStream_t
 }
 
 static wf_handle::GraphKey graph_key(wf_handle *h, int kind, const wf_sample_params *sp,
-                                     bool forced) {
+                                     bool forced, bool forced_q = false) {
   wf_handle::GraphKey k;
   k.kind = kind;
   k.n_active = h->n_active;
-  k.forced = forced ? 1 : 0;
+  k.forced = (forced ? 1 : 0) | (forced_q ? 2 : 0);
   const bool sampling = sp && sp->temperature > 0.f;
   k.temperature = sampling ? sp->temperature : 0.f;
   k.seed = sampling ? sp->seed : 0;
@@ -1191,24 +1195,33 @@ wf_status wf_draft(wf_handle *h, const wf_sample_params *sp, void *stream) {
 }
 
 wf_status wf_verify_accept(wf_handle *h, const wf_sample_params *sp, const int32_t *d_forced,
-                           int32_t *d_out_tokens, int32_t *d_out_count, void *stream) {
-  if (!h || !d_out_tokens || !d_out_count) return WF_ERR_INVALID;
+                           const float *d_forced_q, int32_t *d_out_tokens, int32_t *d_out_count,
+                           void *stream) {
+  if (!h || !d_out_tokens || !d_out_count || (d_forced_q && !d_forced)) return WF_ERR_INVALID;
   h->launches = 0;
-  return verify_body(h, sp, d_forced, d_out_tokens, d_out_count, S(stream));
+  const bool sampling = sp && sp->temperature > 0.f;
+  return verify_body(h, sp, d_forced, sampling ? d_forced_q : nullptr, d_out_tokens, d_out_count,
+                     S(stream));
 }
 
 wf_status wf_step(wf_handle *h, const wf_sample_params *sp, const int32_t *d_forced,
-                  int32_t *d_out_tokens, int32_t *d_out_count, void *stream) {
-  if (!h || !d_out_tokens || !d_out_count) return WF_ERR_INVALID;
+                  const float *d_forced_q, int32_t *d_out_tokens, int32_t *d_out_count, void *stream) {
+  if (!h || !d_out_tokens || !d_out_count || (d_forced_q && !d_forced)) return WF_ERR_INVALID;
   cudaStream_t s = S(stream);
   const size_t kb = static_cast<size_t>(h->Bmax) * h->K * sizeof(int32_t);
   if (d_forced) WF_TRY(cudaMemcpyAsync(h->forced_buf, d_forced, kb, cudaMemcpyDeviceToDevice, s));
   const int32_t *forced = d_forced ? h->forced_buf : nullptr;
-  wf_status st = run_graphed(h, graph_key(h, 1, sp, d_forced != nullptr), s,
+  const bool use_q = d_forced_q && sp && sp->temperature > 0.f;
+  if (use_q)
+    WF_TRY(cudaMemcpyAsync(h->fq_buf, d_forced_q,
+                           static_cast<size_t>(h->Bmax) * h->K * h->V * sizeof(float),
+                           cudaMemcpyDeviceToDevice, s));
+  const float *fq = use_q ? h->fq_buf : nullptr;
+  wf_status st = run_graphed(h, graph_key(h, 1, sp, d_forced != nullptr, use_q), s,
                              [&](cudaStream_t cs) -> wf_status {
                                wf_status r = draft_body(h, sp, cs);
                                if (r != WF_OK) return r;
-                               return verify_body(h, sp, forced, h->tok_buf, h->cnt_buf, cs);
+                               return verify_body(h, sp, forced, fq, h->tok_buf, h->cnt_buf, cs);
                              });
   if (st != WF_OK) return st;
   WF_TRY(cudaMemcpyAsync(d_out_tokens, h->tok_buf, kb / h->K * (h->K + 1), cudaMemcpyDeviceToDevice, s));

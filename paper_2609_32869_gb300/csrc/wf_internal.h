@@ -166,6 +166,7 @@ struct AcceptParams {
   const HeadOut *tout, *dout;
   const int32_t *cand;  // effective proposals [slot][K]
   const float *tlogits, *dlogits;  // sampling: raw logits [rows][V]
+  const float *forced_q;  // nullable [max_batch][K][V]: logits of the forced proposals' distributions
   const uint8_t *suppress;
   float temperature;
   uint64_t seed;

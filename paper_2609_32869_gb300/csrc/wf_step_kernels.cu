@@ -232,79 +232,126 @@ cudaError_t launch_head_reduce(const HeadReduceParams &p0, cudaStream_t s, bool 
 }
 
 // --------------------------------------------------------------- accept --
-// One warp per active sequence.  Greedy (Sec. 3.1): keep proposals while they
+// One CTA per active sequence.  Greedy (Sec. 3.1): keep proposals while they
 // equal the target's argmax, then emit the target's token (correction, or
 // bonus after K agreements).  Sampling (Sec. 3.1, App. A.4): accept c_i when
 // u_i < p_i(c_i)/q_i(c_i) in FP32; at the first rejection draw from the
 // normalised residual (p_i - q_i)_+ by Gumbel-max; after a full block emit
 // the bonus drawn from the target.  An accepted EOS ends the transcript
 // without a bonus; with R tokens left at most R-1 proposals are live; the
-// cache keeps L+1+a positions (App. A.1).
-__device__ int residual_draw(const AcceptParams &p, int slot, int step, int i, const float *xt,
-                             float lse_t, const float *xd, float lse_d, int lane) {
-  // i: 1-based candidate index; xt/xd: raw logit rows
-  float best = -INFINITY;
-  int barg = 0x7fffffff;
-  bool any = false;
-  for (int v = lane; v < p.vocab; v += 32) {
-    if (p.suppress && p.suppress[v]) continue;
-    const float pt = expf(__fdiv_rn(xt[v], p.temperature) - lse_t);
-    const float qd = expf(__fdiv_rn(xd[v], p.temperature) - lse_d);
-    const float r = fmaxf(pt - qd, 0.f);
-    if (r > 0.f) {
-      any = true;
-      const float sc = logf(r) + gumbel(p.seed, slot, step, i, kTagResidual, v);
-      if (sc > best) {
-        best = sc;
-        barg = v;
-      }
-    }
-  }
-  any = __any_sync(0xffffffffu, any);
-  if (!any) {  // empty residual (rounding only): draw from the target itself
-    for (int v = lane; v < p.vocab; v += 32) {
-      if (p.suppress && p.suppress[v]) continue;
-      const float sc = __fdiv_rn(xt[v], p.temperature) + gumbel(p.seed, slot, step, i, kTagResidual, v);
-      if (sc > best) {
-        best = sc;
-        barg = v;
-      }
-    }
-  }
-  for (int off = 16; off > 0; off >>= 1) {
-    const float b2 = __shfl_xor_sync(0xffffffffu, best, off);
-    const int a2 = __shfl_xor_sync(0xffffffffu, barg, off);
-    if (b2 > best || (b2 == best && a2 < barg)) {
-      best = b2;
-      barg = a2;
-    }
-  }
-  return barg;
-}
+// cache keeps L+1+a positions (App. A.1).  The decisions are sequential and
+// taken by one thread; the residual draw and the normalisers of forced
+// proposal distributions reduce over the vocabulary with the whole CTA.
+constexpr int kAccThreads = 256;
 
-__global__ void __launch_bounds__(512) accept_kernel(const AcceptParams p) {
-  pdl_wait();
-  pdl_launch_dependents();
-  const int Kp1 = p.K + 1;
-  for (int sidx = threadIdx.x; sidx < p.max_batch; sidx += blockDim.x) {
-    p.out_count[sidx] = 0;
-    for (int j = 0; j < Kp1; ++j) p.out_tokens[sidx * Kp1 + j] = -1;
+// The CTA's maximum (value, lowest id on ties) of (v, arg) over its threads.
+__device__ __forceinline__ void block_argmax(float &v, int &arg, float *sv, int *sa) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const float v2 = __shfl_xor_sync(0xffffffffu, v, off);
+    const int a2 = __shfl_xor_sync(0xffffffffu, arg, off);
+    if (v2 > v || (v2 == v && a2 < arg)) {
+      v = v2;
+      arg = a2;
+    }
   }
   __syncthreads();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int nwarps = blockDim.x >> 5;
+  if (lane == 0) {
+    sv[warp] = v;
+    sa[warp] = arg;
+  }
+  __syncthreads();
+  v = sv[0];
+  arg = sa[0];
+  for (int w = 1; w < kAccThreads / 32; ++w)
+    if (sv[w] > v || (sv[w] == v && sa[w] < arg)) {
+      v = sv[w];
+      arg = sa[w];
+    }
+}
+// log sum exp over the CTA of per-thread (max, sum of exp(x - max)).
+__device__ __forceinline__ float block_lse(float m, float sum, float *sm, float *ss) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+    const float s2 = __shfl_xor_sync(0xffffffffu, sum, off);
+    const float M = fmaxf(m, m2);
+    sum = (M == -INFINITY) ? 0.f : sum * expf(m - M) + s2 * expf(m2 - M);
+    m = M;
+  }
+  __syncthreads();
+  if (lane == 0) {
+    sm[warp] = m;
+    ss[warp] = sum;
+  }
+  __syncthreads();
+  float M = -INFINITY, S = 0.f;
+  for (int w = 0; w < kAccThreads / 32; ++w) {
+    const float M2 = fmaxf(M, sm[w]);
+    S = (M2 == -INFINITY) ? 0.f : S * expf(M - M2) + ss[w] * expf(sm[w] - M2);
+    M = M2;
+  }
+  return M + logf(S);
+}
+
+__global__ void __launch_bounds__(kAccThreads) accept_kernel(const AcceptParams p) {
+  pdl_wait();
+  pdl_launch_dependents();
+  __shared__ float s_v[kAccThreads / 32], s_w[kAccThreads / 32];
+  __shared__ int s_a[kAccThreads / 32];
+  __shared__ float s_qlse[8];
+  __shared__ int s_em[16];
+  __shared__ int s_state[4];  // emitted count, accepted a, stopped, rejected row (0: none)
+  const int Kp1 = p.K + 1;
+  const int tid = threadIdx.x;
+  // slots outside the active list emit nothing this step
+  for (int sl = blockIdx.x; sl < p.max_batch; sl += gridDim.x) {
+    bool active = false;
+    for (int i = 0; i < p.n_seq; ++i) active = active || p.seq_slot[i] == sl;
+    if (!active) {
+      for (int j = tid; j < Kp1; j += kAccThreads) p.out_tokens[sl * Kp1 + j] = -1;
+      if (tid == 0) p.out_count[sl] = 0;
+    }
+  }
+  const int i = blockIdx.x;
+  if (i >= p.n_seq) return;
+  const int slot = p.seq_slot[i];
+  if (p.done[slot]) {
+    for (int j = tid; j < Kp1; j += kAccThreads) p.out_tokens[slot * Kp1 + j] = -1;
+    if (tid == 0) p.out_count[slot] = 0;
+    return;
+  }
   const bool sampling = p.temperature > 0.f;
-  for (int i = warp; i < p.n_seq; i += nwarps) {
-    const int slot = p.seq_slot[i];
-    if (p.done[slot]) continue;
-    const int R = p.remaining[slot];
-    const int step = p.step[slot];
-    int k = p.greedy_step ? 0 : min(p.K, R - 1);
-    if (k < 0) k = 0;
-    const int r0 = i * p.rps;
-    int emitted[16];
-    int n_em = 0, a = 0;
-    bool stop = false;
+  const int R = p.remaining[slot];
+  const int step = p.step[slot];
+  int k = p.greedy_step ? 0 : min(p.K, R - 1);
+  if (k < 0) k = 0;
+  const int r0 = i * p.rps;
+  const float *fq = p.forced_q ? p.forced_q + static_cast<size_t>(slot) * p.K * p.vocab : nullptr;
+  // normalisers of the forced proposal distributions softmax(q / T)
+  if (sampling && fq) {
+    for (int c = 0; c < k; ++c) {
+      const float *row = fq + static_cast<size_t>(c) * p.vocab;
+      float m = -INFINITY, sum = 0.f;
+      for (int v = tid; v < p.vocab; v += kAccThreads) {
+        if (p.suppress && p.suppress[v]) continue;
+        const float x = __fdiv_rn(row[v], p.temperature);
+        if (x > m) {
+          sum = sum * expf(m - x) + 1.f;
+          m = x;
+        } else {
+          sum += expf(x - m);
+        }
+      }
+      const float l = block_lse(m, sum, s_v, s_w);
+      if (tid == 0) s_qlse[c] = l;
+    }
+  }
+  if (tid == 0) {
+    int n_em = 0, a = 0, stop = 0, rej = 0;
+    bool finished = false;
     for (int c = 1; c <= k; ++c) {
       const int cand = p.cand[slot * p.K + c - 1];
       bool acc;
@@ -312,9 +359,12 @@ __global__ void __launch_bounds__(512) accept_kernel(const AcceptParams p) {
         acc = cand == p.tout[r0 + c - 1].arg;
       } else {
         const int rt = r0 + c - 1, rd = r0 + c;  // drafter row c holds mask position c
-        const float lse_t = p.tout[rt].lse, lse_d = p.dout[rd].lse;
+        const float lse_t = p.tout[rt].lse;
+        const float lse_d = fq ? s_qlse[c - 1] : p.dout[rd].lse;
+        const float zd = fq ? fq[static_cast<size_t>(c - 1) * p.vocab + cand]
+                            : p.dlogits[static_cast<size_t>(rd) * p.vocab + cand];
         const float xt = __fdiv_rn(p.tlogits[static_cast<size_t>(rt) * p.vocab + cand], p.temperature);
-        const float xd = __fdiv_rn(p.dlogits[static_cast<size_t>(rd) * p.vocab + cand], p.temperature);
+        const float xd = __fdiv_rn(zd, p.temperature);
         const bool sup = p.suppress && p.suppress[cand];
         const float pc = sup ? 0.f : expf(xt - lse_t);
         const float qc = sup ? 0.f : expf(xd - lse_d);
@@ -323,55 +373,102 @@ __global__ void __launch_bounds__(512) accept_kernel(const AcceptParams p) {
         const float u = word_to_uniform(o.x[0]);
         acc = u < __fdiv_rn(pc, qc);
         if (!acc) {
-          const int t = residual_draw(p, slot, step, c,
-                                      p.tlogits + static_cast<size_t>(rt) * p.vocab, lse_t,
-                                      p.dlogits + static_cast<size_t>(rd) * p.vocab, lse_d, lane);
-          emitted[n_em++] = t;
-          stop = (t == p.eos);
+          rej = c;  // the residual draw below supplies the token
           a = c - 1;
-          k = -1;  // mark: finished by a rejection
+          finished = true;
           break;
         }
       }
       if (!acc) break;
-      emitted[n_em++] = cand;
+      s_em[n_em++] = cand;
       a = c;
       if (cand == p.eos) {
-        stop = true;
-        k = -1;
+        stop = 1;
+        finished = true;
         break;
       }
     }
-    if (k >= 0) {  // correction (greedy mismatch) or bonus
+    if (!finished) {  // correction (greedy mismatch) or bonus
       const HeadOut &ho = p.tout[r0 + a];
       const int t = sampling ? ho.garg : ho.arg;
-      emitted[n_em++] = t;
-      stop = (t == p.eos);
+      s_em[n_em++] = t;
+      stop = t == p.eos;
     }
-    if (lane == 0) {
-      for (int e = 0; e < n_em; ++e) p.out_tokens[slot * Kp1 + e] = emitted[e];
-      p.out_count[slot] = n_em;
-      const int newL = p.L[slot] + 1 + a;
-      p.L[slot] = newL;
-      p.anchor[slot] = emitted[n_em - 1];
-      const int left = R - n_em;
-      p.remaining[slot] = left;
-      p.step[slot] = step + 1;
-      bool done = stop || left <= 0;
-      if (!done && newL + Kp1 > p.max_ctx) {
-        set_error(p.err, WF_DEV_ERR_CAPACITY);
-        done = true;
+    s_state[0] = n_em;
+    s_state[1] = a;
+    s_state[2] = stop;
+    s_state[3] = rej;
+  }
+  __syncthreads();
+  const int rej = s_state[3];
+  if (rej) {
+    // residual (p - q)_+ of row rej by Gumbel-max over log r; if it is empty
+    // (rounding only) the token is drawn from the target itself
+    const int rt = r0 + rej - 1, rd = r0 + rej;
+    const float *xt = p.tlogits + static_cast<size_t>(rt) * p.vocab;
+    const float *xd = fq ? fq + static_cast<size_t>(rej - 1) * p.vocab
+                         : p.dlogits + static_cast<size_t>(rd) * p.vocab;
+    const float lse_t = p.tout[rt].lse;
+    const float lse_d = fq ? s_qlse[rej - 1] : p.dout[rd].lse;
+    float best = -INFINITY;
+    int barg = 0x7fffffff;
+    bool any = false;
+    for (int v = tid; v < p.vocab; v += kAccThreads) {
+      if (p.suppress && p.suppress[v]) continue;
+      const float pt = expf(__fdiv_rn(xt[v], p.temperature) - lse_t);
+      const float qd = expf(__fdiv_rn(xd[v], p.temperature) - lse_d);
+      const float r = fmaxf(pt - qd, 0.f);
+      if (r > 0.f) {
+        any = true;
+        const float sc = logf(r) + gumbel(p.seed, slot, step, rej, kTagResidual, v);
+        if (sc > best || (sc == best && v < barg)) {
+          best = sc;
+          barg = v;
+        }
       }
-      p.done[slot] = done ? 1 : 0;
     }
-    __syncwarp();
+    if (!__syncthreads_or(any)) {
+      for (int v = tid; v < p.vocab; v += kAccThreads) {
+        if (p.suppress && p.suppress[v]) continue;
+        const float sc = __fdiv_rn(xt[v], p.temperature) + gumbel(p.seed, slot, step, rej, kTagResidual, v);
+        if (sc > best || (sc == best && v < barg)) {
+          best = sc;
+          barg = v;
+        }
+      }
+    }
+    block_argmax(best, barg, s_v, s_a);
+    if (tid == 0) {
+      s_em[s_state[0]++] = barg;
+      s_state[2] = barg == p.eos;
+    }
+  }
+  __syncthreads();
+  const int n_em = s_state[0], a = s_state[1];
+  for (int j = tid; j < Kp1; j += kAccThreads) p.out_tokens[slot * Kp1 + j] = j < n_em ? s_em[j] : -1;
+  if (tid == 0) {
+    p.out_count[slot] = n_em;
+    const int newL = p.L[slot] + 1 + a;
+    p.L[slot] = newL;
+    p.anchor[slot] = s_em[n_em - 1];
+    const int left = R - n_em;
+    p.remaining[slot] = left;
+    p.step[slot] = step + 1;
+    bool done = s_state[2] || left <= 0;
+    if (!done && newL + Kp1 > p.max_ctx) {
+      set_error(p.err, WF_DEV_ERR_CAPACITY);
+      done = true;
+    }
+    p.done[slot] = done ? 1 : 0;
   }
 }
 
 cudaError_t launch_accept(const AcceptParams &p0, cudaStream_t s, bool pdl) {
   AcceptParams p = p0;
+  if (p.K > 8) return cudaErrorInvalidValue;
   void *args[] = {&p};
-  return launch_ex(reinterpret_cast<const void *>(accept_kernel), dim3(1), dim3(512), args, s, pdl);
+  return launch_ex(reinterpret_cast<const void *>(accept_kernel), dim3(p.n_seq > 0 ? p.n_seq : 1),
+                   dim3(kAccThreads), args, s, pdl);
 }
 
 // ---------------------------------------------------------------- state --

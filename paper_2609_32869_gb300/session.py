@@ -79,19 +79,21 @@ class Session:
         self._keep = (d_slots, d_prompt, d_budget, enc)
         return first
 
-    def step(self, forced=None, sp=None):
+    def step(self, forced=None, sp=None, forced_q=None):
+        """forced: proposals [max_batch, K]; forced_q: a device fp32 tensor
+        [max_batch, K, vocab] of the logits they were drawn from (sampling)."""
         f = None if forced is None else (forced if not isinstance(forced, np.ndarray) else self._i32(forced))
-        B.wf_step(self.h, sp, f, self.out_tokens, self.out_count, self.stream)
-        self._keep_forced = f
+        B.wf_step(self.h, sp, f, forced_q, self.out_tokens, self.out_count, self.stream)
+        self._keep_forced = (f, forced_q)
         return self.out_tokens, self.out_count
 
     def draft(self, sp=None):
         B.wf_draft(self.h, sp, self.stream)
 
-    def verify_accept(self, forced=None, sp=None):
+    def verify_accept(self, forced=None, sp=None, forced_q=None):
         f = None if forced is None else (forced if not isinstance(forced, np.ndarray) else self._i32(forced))
-        B.wf_verify_accept(self.h, sp, f, self.out_tokens, self.out_count, self.stream)
-        self._keep_forced = f
+        B.wf_verify_accept(self.h, sp, f, forced_q, self.out_tokens, self.out_count, self.stream)
+        self._keep_forced = (f, forced_q)
         return self.out_tokens, self.out_count
 
     def greedy_step(self, sp=None):

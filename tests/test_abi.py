@@ -64,8 +64,8 @@ def test_null_handle_is_rejected_on_the_host():
         "wf_destroy": (None,),
         "wf_prefill_cross_kv": (None, 1, None, None, None, 4, None, None, None, None),
         "wf_draft": (None, None, None),
-        "wf_verify_accept": (None, None, None, None, None, None),
-        "wf_step": (None, None, None, None, None, None),
+        "wf_verify_accept": (None, None, None, None, None, None, None),
+        "wf_step": (None, None, None, None, None, None, None),
         "wf_greedy_step": (None, None, None, None, None),
         "wf_compact": (None, None, None),
         "wf_reset_slots": (None, 1, None, None),

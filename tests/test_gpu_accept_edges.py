@@ -8,8 +8,13 @@ that one transcript emits, so that within two steps:
   - slot 2 reaches its budget inside a block (k = R - 1 < K live proposals);
   - the batch compacts around the finished slots while slot 3 continues.
 Every emitted token, count, cache length and done flag must equal the
-oracle's wherever the deciding top-2 margins exceed 0.05 (they all do on
-these seeds; a closer call would only exempt that sequence)."""
+oracle's wherever the deciding top-2 margins are clear.  The weights are
+drawn wider than the workloads' N(0, 0.02) so that transcripts do not repeat
+one token; the logits grow with them, so "clear" means above both 0.05 and
+twice the largest difference between the GPU's and the oracle's logits on
+that sequence's rows (then both sides must take the same argmax).  They are
+clear for every event below on these seeds; a closer call only exempts that
+sequence from the remaining comparisons."""
 import numpy as np
 import pytest
 
@@ -35,6 +40,7 @@ def _forced(g, t, a, K, V):
 
 def test_eos_budget_and_compaction_match_oracle():
     import torch
+    from paper_2609_32869_gb300 import binding as B
     from paper_2609_32869_gb300.session import Session
     cfg0 = syn.toy_config()
     ws = syn.make_weights(cfg0, seed=3, std=0.2, ln_noise=True)
@@ -59,21 +65,24 @@ def test_eos_budget_and_compaction_match_oracle():
     seqs = [o.prefill(encf[b], prompt[b], int(budgets[b]), seq_id=b) for b in range(4)]
     assert greedy[0][5] == eos and eos not in greedy[2] + greedy[0][:5]
 
-    s = Session(cfg, ws, max_batch=4)
+    s = Session(cfg, ws, max_batch=4, keep_logits=True)
     first = s.prefill(np.arange(4, dtype=np.int32), enc, prompt, budgets).cpu().numpy()
     assert list(first) == [sq.emitted[0] for sq in seqs]
 
     live = set(range(4))                        # sequences still compared token for token
     events = set()
     gpu_done = np.zeros(4, bool)
+    max_err = 0.0                               # logit difference relative to the logits' range
     n_active, step = 4, 0
     while n_active:
         forced = np.zeros((4, K), np.int32)
         for b in range(4):
             a = sched[b][step % len(sched[b])]
             forced[b] = _forced(greedy[b], len(seqs[b].emitted), a, K, V)
+        active = [b for b in range(4) if not gpu_done[b]]   # ascending after compaction
         toks, cnt = s.step(forced=forced)
         toks, cnt = toks.cpu().numpy(), cnt.cpu().numpy()
+        vl = s.view(B.WF_VIEW_TARGET_LOGITS, torch.float32, (4 * (K + 1), V)).cpu().numpy()
         st = s.state()
         for b in range(4):
             if gpu_done[b]:                     # finished and compacted away: emits nothing
@@ -83,8 +92,11 @@ def test_eos_budget_and_compaction_match_oracle():
             if b not in live:
                 continue
             rec = o.spec_step(seqs[b], forced=forced[b])
+            r0 = active.index(b) * (K + 1)
+            err = float(np.abs(vl[r0:r0 + rec.k + 1] - rec.verify_logits).max())
+            max_err = max(max_err, err / float(np.abs(rec.verify_logits).max()))
             deciding = [_margin(rec.verify_logits[j]) for j in range(min(rec.accepted + 1, rec.k + 1))]
-            if min(deciding) <= MARGIN:
+            if min(deciding) <= max(MARGIN, 2 * err):
                 live.discard(b)
                 continue
             assert list(toks[b, :cnt[b]]) == rec.emitted, (step, b)
@@ -109,5 +121,6 @@ def test_eos_budget_and_compaction_match_oracle():
     assert seqs[0].emitted == greedy[0] and seqs[1].emitted == greedy[1]
     assert events == {"accepted EOS, no bonus", "EOS as correction", "budget ends inside a block",
                       "compacted with sequences left"}, events
+    assert max_err <= 1e-2, max_err
     assert s.error() == 0
     s.close()

@@ -147,3 +147,84 @@ def test_speculative_sampler_preserves_target_distribution():
     accepted_any = (cnt >= 2).mean()
     assert 0.02 < accepted_any < 0.98
     s.close()
+
+
+def test_forced_proposal_distribution_matches_oracle():
+    """Teacher-forced sampling (the benchmark's recipe): proposals drawn on the
+    host from q = softmax((z + 0.5 eps) / T), with z the target's logits at
+    the anchor row and eps seeded N(0, 1), are passed with the logits of q;
+    the GPU's rejection rule must then take q from them, as the oracle does
+    (Sec. 3.1: q is the distribution the candidate came from)."""
+    import torch
+    from paper_2609_32869_gb300 import binding as B
+    from paper_2609_32869_gb300.session import Session
+    cfg = syn.TINY
+    T, seed = 0.7, 4242
+    ws = syn.make_weights(cfg, seed=0, ln_noise=True)
+    wf = syn.weights_as_float(ws)
+    o = WhisperFlashOracle(wf, cfg)
+    slots = np.array([0, 1], np.int32)
+    enc = syn.encoder_output(cfg, 2, seed=1)
+    prompt = syn.prompts(cfg, 2, length=8, seed=6)
+    budget = 40
+    encf = syn.bf16_bits_to_f32(enc).astype(np.float64)
+    sp = B.sample_params(T, seed)
+    seqs = [o.prefill(encf[b], prompt[b], budget, seq_id=int(slots[b]), temperature=T, seed=seed)
+            for b in range(2)]
+    s = Session(cfg, ws, max_batch=2, keep_logits=True)
+    first = s.prefill(slots, enc, prompt, np.full(2, budget, np.int32), sp=sp).cpu().numpy()
+    K, V = cfg.block_k, cfg.vocab
+    live = [b for b in range(2) if first[b] == seqs[b].emitted[0]]
+    rng = np.random.default_rng(5)
+    compared = accepted = 0
+    for step in range(4):
+        zq = np.zeros((2, K, V), np.float32)
+        cands = np.zeros((2, K), np.int32)
+        for b in range(2):
+            z0, _, _, _ = o.target_pass(seqs[b], [seqs[b].anchor], [seqs[b].L])
+            zq[b] = (z0[0][None, :] + 0.5 * rng.standard_normal((K, V))).astype(np.float32)
+            for j in range(K):
+                cands[b, j] = int(np.argmax(zq[b, j] / np.float32(T) + rng.gumbel(size=V)))
+        toks, cnt = s.step(forced=cands, sp=sp, forced_q=torch.as_tensor(zq, device="cuda"))
+        torch.cuda.synchronize()
+        vl = s.view(B.WF_VIEW_TARGET_LOGITS, torch.float32, (2 * (K + 1), V)).cpu().numpy()
+        toks, cnt = toks.cpu().numpy(), cnt.cpu().numpy()
+        for b in list(live):
+            sl = int(slots[b])
+            seq = seqs[b]
+            step_id = seq.step
+            rec = o.spec_step(seq, forced=cands[b], temperature=T, seed=seed, forced_q=zq[b])
+            r0 = b * (K + 1)
+            assert np.abs(vl[r0:r0 + rec.k + 1] - rec.verify_logits).max() <= LOGIT_ATOL
+            k = rec.k
+            xt = np.stack([acceptance.scaled_logits_fp32(r, T) for r in rec.verify_logits])
+            xd = np.stack([acceptance.scaled_logits_fp32(r, T) for r in zq[b][:k]]) if k else None
+            margin_ok = True
+            for i in range(min(rec.accepted + 1, k)):
+                c = int(cands[b, i])
+                p = acceptance.probs_fp32(xt[i])[c]
+                q = acceptance.probs_fp32(xd[i])[c]
+                u = philox.accept_uniform(seed, sl, step_id, i + 1)
+                margin_ok &= abs(float(u) - float(p / q)) > 2e-2 * max(1.0, float(p / q))
+            last = rec.accepted
+            if last == k:
+                g = philox.gumbel_noise(seed, sl, step_id, k, philox.TAG_BONUS, V)
+                margin_ok &= _gap(xt[k] + g) > 0.1
+            elif last < k:
+                r = np.maximum(acceptance.probs_fp32(xt[last]) - acceptance.probs_fp32(xd[last]), 0)
+                with np.errstate(divide="ignore"):
+                    score = np.where(r > 0, np.log(r), -np.inf)
+                g = philox.gumbel_noise(seed, sl, step_id, last + 1, philox.TAG_RESIDUAL, V)
+                margin_ok &= _gap(np.where(np.isfinite(score), score + g, -1e30)) > 0.1
+            if margin_ok:
+                got = list(toks[sl, :cnt[sl]])
+                assert got == rec.emitted, (step, b, got, rec.emitted)
+                compared += 1
+                accepted += rec.accepted
+            else:
+                live.remove(b)
+        if not live:
+            break
+    assert compared >= 2 and accepted >= 1
+    assert s.error() == 0
+    s.close()
