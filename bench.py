@@ -52,13 +52,13 @@ WORKLOADS = {
     # perturbed target logits along the target's own sampled path, passed with
     # the logits of that distribution; the target applies the rejection rule
     # with seeded Philox streams.
-    "large_b32_t07": dict(cfg="LARGE", batch=32, budget=(20, 220), temperature=0.7, sigma=1.0,
+    "large_b32_t07": dict(cfg="LARGE", batch=32, budget=(20, 220), temperature=0.7, sigma=0.3,
                           text="large shapes, batch 32, temperature 0.7 speculative sampling; "
-                               "proposals from softmax((z_target + eps) / T), eps ~ N(0, 1) seeded, "
+                               "proposals from softmax((z_target + 0.3 eps) / T), eps ~ N(0, 1) seeded, "
                                "along the target's own sampled path; lengths uniform 20..220"),
-    "large_b32_t10": dict(cfg="LARGE", batch=32, budget=(20, 220), temperature=1.0, sigma=1.0,
+    "large_b32_t10": dict(cfg="LARGE", batch=32, budget=(20, 220), temperature=1.0, sigma=0.3,
                           text="large shapes, batch 32, temperature 1.0 speculative sampling; "
-                               "proposals from softmax((z_target + eps) / T), eps ~ N(0, 1) seeded, "
+                               "proposals from softmax((z_target + 0.3 eps) / T), eps ~ N(0, 1) seeded, "
                                "along the target's own sampled path; lengths uniform 20..220"),
     # Depth-reduced cases for profiler captures: every kernel keeps the large
     # per-layer shapes and launch configuration; only the number of target

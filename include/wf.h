@@ -242,6 +242,14 @@ int32_t wf_last_launch_count(const wf_handle *h);
                                 restores about 1 s (projections) and 0.2 s (persistent pass).
                                 Meant for tests of the failure path: a limit below a wait's
                                 normal duration makes the results of that call invalid. */
+#define WF_OPT_SKINNY 7      /* 1 (default when max_batch * (block_k + 1) <= 16): passes of at
+                                most 16 token rows run their projections as low-latency
+                                kernels that hold a CTA's whole weight slab in shared memory
+                                and reduce K in a fixed order; 0: the tcgen05 projections.
+                                Setting 1 on a larger handle returns WF_ERR_UNSUPPORTED.
+                                The two forms agree within the method's tolerances, not bit
+                                for bit; a handle's speculative and plain greedy steps
+                                always take the same form. */
 #define WF_VIEW_TARGET_LOGITS 1
 #define WF_VIEW_DRAFT_LOGITS 2
 #define WF_VIEW_TAPS 3

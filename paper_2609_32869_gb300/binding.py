@@ -24,6 +24,7 @@ WF_OPT_GRAPHS = 3
 WF_OPT_PDL = 4
 WF_OPT_PERSIST = 5
 WF_OPT_SPIN_LIMIT = 6
+WF_OPT_SKINNY = 7
 WF_FAMILIES = ("gemm", "head", "attn_self", "attn_cross", "layernorm", "other", "persist")
 WF_VIEW_TARGET_LOGITS, WF_VIEW_DRAFT_LOGITS, WF_VIEW_TAPS, WF_VIEW_CANDIDATES = 1, 2, 3, 4
 

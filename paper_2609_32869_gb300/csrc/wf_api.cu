@@ -49,6 +49,12 @@ struct wf_handle {
   long long spin = 0;  // bounded-wait limit in clock cycles (WF_OPT_SPIN_LIMIT; 0: default)
   int launches = 0;
   bool keep_logits = false;
+  // skinny projections (wf_skinny.cu) for passes of at most kSkMaxRows rows;
+  // used when every pass of the handle fits (max_batch * (K + 1) rows), so
+  // speculative and plain greedy steps take the same arithmetic
+  bool skinny = false;
+  bool skinny_ok = false;  // the handle's shapes and max_batch allow it
+  int sk_rows = 0;         // rows of its largest step pass (max_batch * (K + 1))
   // profiling (WF_OPT_PROFILE)
   bool profile = false;
   std::vector<cudaEvent_t> ev_pool;
@@ -271,6 +277,35 @@ double gemm_bytes(const GemmParams &p) {
 }
 
 // ---------------------------------------------------------------- GEMMs --
+// The skinny form of a projection's parameters (same epilogue fields).
+SkinnyParams skinny_of(const GemmParams &g) {
+  SkinnyParams p = {};
+  p.M = g.M;
+  p.N = g.N;
+  p.K = g.K;
+  p.epi = g.epi;
+  p.bias = g.bias;
+  p.out_f32 = g.out_f32;
+  p.out_bf16 = g.out_bf16;
+  p.ld_out = g.ld_out;
+  p.resid = g.resid;
+  p.ld_resid = g.ld_resid;
+  p.tap0 = g.tap0;
+  p.tap1 = g.tap1;
+  p.ld_tap = g.ld_tap;
+  p.q_cols = g.q_cols;
+  p.d_model = g.d_model;
+  p.n_heads = g.n_heads;
+  p.ctx = g.ctx;
+  p.rows_per_seq = g.rows_per_seq;
+  p.kc = g.kc;
+  p.vc = g.vc;
+  p.seq_slot = g.seq_slot;
+  p.pos_base = g.pos_base;
+  p.err = g.err;
+  p.spin = g.spin;
+  return p;
+}
 GemmParams gemm_base(wf_handle *h, int M, int N, int K, int epi) {
   GemmParams p = {};
   p.M = M;
@@ -292,6 +327,38 @@ cudaError_t gemm(wf_handle *h, const void *X, const void *W, GemmParams p, cudaS
   prof_end(h, s, p.epi == EPI_HEAD ? WF_FAM_HEAD : WF_FAM_GEMM, gemm_bytes(p));
   return e;
 }
+
+// A skinny projection: operand LN(ln_x) (g, b) when ln_x is set, else bf16 rows X.
+cudaError_t skinny(wf_handle *h, const void *X, const float *ln_x, const void *g, const void *b,
+                   const void *W, const GemmParams &gp, cudaStream_t s) {
+  SkinnyParams p = skinny_of(gp);
+  if (ln_x) {
+    p.ln_x = ln_x;
+    p.ln_ld = h->d;
+    p.ln_g = static_cast<const bf16 *>(g);
+    p.ln_b = static_cast<const bf16 *>(b);
+    p.ln_eps = h->cfg.ln_eps;
+  } else {
+    p.x = static_cast<const bf16 *>(X);
+    p.ld_x = gp.K;
+  }
+  h->launches++;
+  prof_begin(h, s);
+  cudaError_t e = launch_skinny(W, p, s, kPDL);
+  prof_end(h, s, WF_FAM_GEMM, gemm_bytes(gp));
+  return e;
+}
+
+// Whether every projection of a pass of up to M rows has a skinny plan.
+bool skinny_shapes_fit(int d, int F, int M) {
+  int U = 0, S = 0;
+  return M <= kSkMaxRows && skinny_plan(M, 3 * d, d, true, &U, &S) && skinny_plan(M, d, d, false, &U, &S) &&
+         skinny_plan(M, d, d, true, &U, &S) && skinny_plan(M, F, d, true, &U, &S) &&
+         skinny_plan(M, d, F, false, &U, &S) && skinny_plan(M, 2 * d, d, true, &U, &S);
+}
+
+// Whether a pass of M rows takes the skinny projections.
+bool use_skinny(const wf_handle *h, int M) { return h->skinny && M <= h->sk_rows; }
 
 cudaError_t layernorm(wf_handle *h, const float *x, const float2 *st, int stride, int off,
                       const void *g, const void *b, bf16 *y, int rows, cudaStream_t s) {
@@ -362,8 +429,9 @@ struct Pass {
   const int32_t *slots;
   bool drafter;
   float *x;
-  float2 *st;  // LayerNorm statistics of x
+  float2 *st;  // LayerNorm statistics of x (tcgen05 path)
   bool taps;
+  bool sk;     // skinny projections (no statistics travel)
 };
 
 // One pre-LayerNorm Whisper block over the pass's rows.
@@ -396,7 +464,9 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.rows_per_seq = ps.rps;
     p.seq_slot = ps.slots;
     p.pos_base = h->L;
-    if ((e = ln_gemm(h, ps.x, ps.st, lw.ln1_g, lw.ln1_b, lw.qkv_w, p, s)) != cudaSuccess) return e;
+    e = ps.sk ? skinny(h, nullptr, ps.x, lw.ln1_g, lw.ln1_b, lw.qkv_w, p, s)
+              : ln_gemm(h, ps.x, ps.st, lw.ln1_g, lw.ln1_b, lw.qkv_w, p, s);
+    if (e != cudaSuccess) return e;
   }
   if ((e = attention(h, h->q, kc, vc, ps.slots, ps.n_seq, ps.rps, h->ctx, ps.drafter ? 1 : 0,
                      ps.drafter, s)) != cudaSuccess)
@@ -407,7 +477,8 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.resid = ps.x;
     p.ld_resid = d;
     p.stats_out = ps.st;
-    if ((e = gemm(h, h->att, lw.out_w, p, s)) != cudaSuccess) return e;
+    e = ps.sk ? skinny(h, h->att, nullptr, nullptr, nullptr, lw.out_w, p, s) : gemm(h, h->att, lw.out_w, p, s);
+    if (e != cudaSuccess) return e;
   }
   // cross-attention
   {
@@ -415,7 +486,9 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.bias = static_cast<const bf16 *>(lw.xq_b);
     p.out_bf16 = h->q;
     p.ld_out = d;
-    if ((e = ln_gemm(h, ps.x, ps.st, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s)) != cudaSuccess) return e;
+    e = ps.sk ? skinny(h, nullptr, ps.x, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s)
+              : ln_gemm(h, ps.x, ps.st, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s);
+    if (e != cudaSuccess) return e;
   }
   if ((e = attention(h, h->q, xkc, xvc, ps.slots, ps.n_seq, ps.rps, h->cfg.enc_frames, 2, false,
                      s)) != cudaSuccess)
@@ -426,7 +499,8 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.resid = ps.x;
     p.ld_resid = d;
     p.stats_out = ps.st;
-    if ((e = gemm(h, h->att, lw.xout_w, p, s)) != cudaSuccess) return e;
+    e = ps.sk ? skinny(h, h->att, nullptr, nullptr, nullptr, lw.xout_w, p, s) : gemm(h, h->att, lw.xout_w, p, s);
+    if (e != cudaSuccess) return e;
   }
   // feed-forward
   {
@@ -434,7 +508,9 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.bias = static_cast<const bf16 *>(lw.fc1_b);
     p.out_bf16 = h->h1;
     p.ld_out = h->F;
-    if ((e = ln_gemm(h, ps.x, ps.st, lw.ln3_g, lw.ln3_b, lw.fc1_w, p, s)) != cudaSuccess) return e;
+    e = ps.sk ? skinny(h, nullptr, ps.x, lw.ln3_g, lw.ln3_b, lw.fc1_w, p, s)
+              : ln_gemm(h, ps.x, ps.st, lw.ln3_g, lw.ln3_b, lw.fc1_w, p, s);
+    if (e != cudaSuccess) return e;
   }
   {
     GemmParams p = gemm_base(h, M, d, h->F, EPI_RESID);
@@ -454,7 +530,8 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
       }
       p.ld_tap = h->cfg.n_taps * d;
     }
-    if ((e = gemm(h, h->h1, lw.fc2_w, p, s)) != cudaSuccess) return e;
+    e = ps.sk ? skinny(h, h->h1, nullptr, nullptr, nullptr, lw.fc2_w, p, s) : gemm(h, h->h1, lw.fc2_w, p, s);
+    if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
 }
@@ -514,7 +591,8 @@ cudaError_t ingest(wf_handle *h, int n_seq, int rps, const int32_t *slots, cudaS
   }
   // LN_h is applied inside each drafter block's key/value projection (or by
   // one LayerNorm kernel ahead of them when their tiles do not fit)
-  const bool fused = gemm_ln_fits(M, 2 * d, d, EPI_KV);
+  const bool sk = use_skinny(h, M);
+  const bool fused = sk || gemm_ln_fits(M, 2 * d, d, EPI_KV);
   if (!fused &&
       (e = layernorm(h, h->hproj, h->st_hp, 1, 0, h->dw.hln_g, h->dw.hln_b, h->hn, M, s)) != cudaSuccess)
     return e;
@@ -530,7 +608,9 @@ cudaError_t ingest(wf_handle *h, int n_seq, int rps, const int32_t *slots, cudaS
     p.seq_slot = slots;
     p.pos_base = h->L;
     const bf16 *wkv = static_cast<const bf16 *>(lw.qkv_w) + static_cast<size_t>(d) * d;
-    if (fused) {
+    if (sk) {
+      if ((e = skinny(h, nullptr, h->hproj, h->dw.hln_g, h->dw.hln_b, wkv, p, s)) != cudaSuccess) return e;
+    } else if (fused) {
       p.ln_x = h->hproj;
       p.ln_ld = d;
       p.ln_tiles = d / 128;
@@ -575,7 +655,7 @@ cudaError_t target_pass(wf_handle *h, int n_seq, int rps, const int32_t *slots, 
   cudaError_t e = launch_embed(ep, s, kPDL);
   prof_end(h, s, WF_FAM_OTHER, 0.0);
   if (e != cudaSuccess) return e;
-  Pass ps{n_seq, rps, slots, false, h->x, h->st_x, taps};
+  Pass ps{n_seq, rps, slots, false, h->x, h->st_x, taps, use_skinny(h, n_seq * rps)};
   for (int l = 0; l < h->nl; ++l)
     if ((e = run_block(h, ps, h->tl[l], l, s)) != cudaSuccess) return e;
   return cudaSuccess;
@@ -828,7 +908,10 @@ wf_status wf_create(const wf_config *cfg, const wf_target_weights *tw, const wf_
             cudaMemsetAsync(h->err, 0, sizeof(uint32_t), s) == cudaSuccess &&
             cudaMemsetAsync(h->attn_counters, 0, h->attn_counter_cap * sizeof(int32_t), s) == cudaSuccess &&
             launch_rope_table(h->rope, cfg->max_pos, cfg->rope_base, s) == cudaSuccess;
-  ok = ok && gemm_init() == cudaSuccess && attention_init() == cudaSuccess &&
+  h->sk_rows = max_batch * (cfg->block_k + 1);
+  h->skinny_ok = skinny_shapes_fit(h->d, h->F, h->sk_rows);
+  h->skinny = h->skinny_ok;
+  ok = ok && gemm_init() == cudaSuccess && skinny_init() == cudaSuccess && attention_init() == cudaSuccess &&
        cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) == cudaSuccess;
   if (ok && h->mk_ok) ok = persist_setup(h, s) == cudaSuccess;
   if (!ok) {
@@ -870,6 +953,13 @@ wf_status wf_set_option(wf_handle *h, int32_t option, int32_t value) {
   if (option == WF_OPT_PERSIST) {
     if (value && !h->mk_ok) return WF_ERR_UNSUPPORTED;
     h->mk_on = value != 0;
+    for (auto &kv : h->graphs) cudaGraphExecDestroy(kv.second.exec);
+    h->graphs.clear();
+    return WF_OK;
+  }
+  if (option == WF_OPT_SKINNY) {
+    if (value && !h->skinny_ok) return WF_ERR_UNSUPPORTED;
+    h->skinny = value != 0;
     for (auto &kv : h->graphs) cudaGraphExecDestroy(kv.second.exec);
     h->graphs.clear();
     return WF_OK;
@@ -980,8 +1070,8 @@ wf_status wf_prefill_cross_kv(wf_handle *h, int32_t n, const int32_t *d_slots, c
     WF_TRY(target_pass(h, gn, P, slots, TOK_PROMPT, d_prompt + static_cast<size_t>(i0) * P, P,
                        nullptr, true, s));
     WF_TRY(ingest(h, gn, P, slots, s));
-    WF_TRY(head(h, h->x, h->st_x, P, P - 1, gn, slots, 1, h->recs_t, h->hout_t, h->logits_t, sp, kTagBonus,
-                nullptr, s));
+    WF_TRY(head(h, h->x, use_skinny(h, gn * P) ? nullptr : h->st_x, P, P - 1, gn, slots, 1, h->recs_t,
+                h->hout_t, h->logits_t, sp, kTagBonus, nullptr, s));
     StateParams sp1 = sp0;
     sp1.op = 1;
     sp1.n = gn;
@@ -1033,10 +1123,10 @@ static wf_status draft_body(wf_handle *h, const wf_sample_params *sp, cudaStream
   prof_begin(h, s);
   WF_TRY(launch_embed(ep, s, kPDL));
   prof_end(h, s, WF_FAM_OTHER, 0.0);
-  Pass ps{n, rps, h->active, true, h->xd, h->st_xd, false};
+  Pass ps{n, rps, h->active, true, h->xd, h->st_xd, false, use_skinny(h, n * rps)};
   for (int l = 0; l < h->nd; ++l) WF_TRY(run_block(h, ps, h->dl[l], l, s));
-  WF_TRY(head(h, h->xd, h->st_xd, 1, 0, n * rps, h->active, rps, h->recs_d, h->hout_d, h->logits_d, sp,
-              kTagDraft, h->cand, s));
+  WF_TRY(head(h, h->xd, ps.sk ? nullptr : h->st_xd, 1, 0, n * rps, h->active, rps, h->recs_d, h->hout_d,
+              h->logits_d, sp, kTagDraft, h->cand, s));
   return WF_OK;
 }
 
@@ -1051,8 +1141,8 @@ static wf_status verify_body(wf_handle *h, const wf_sample_params *sp, const int
                   sp, kTagBonus, nullptr, s));
     } else {
       WF_TRY(target_pass(h, n, rps, h->active, TOK_VERIFY, nullptr, 0, d_forced, true, s));
-      WF_TRY(head(h, h->x, h->st_x, 1, 0, n * rps, h->active, rps, h->recs_t, h->hout_t, h->logits_t, sp,
-                  kTagBonus, nullptr, s));
+      WF_TRY(head(h, h->x, use_skinny(h, n * rps) ? nullptr : h->st_x, 1, 0, n * rps, h->active, rps,
+                  h->recs_t, h->hout_t, h->logits_t, sp, kTagBonus, nullptr, s));
     }
     WF_TRY(ingest(h, n, rps, h->active, s));
   }
@@ -1100,8 +1190,8 @@ static wf_status greedy_body(wf_handle *h, const wf_sample_params *sp, int32_t *
                   kTagBonus, nullptr, s));
     } else {
       WF_TRY(target_pass(h, n, 1, h->active, TOK_ANCHOR, nullptr, 0, nullptr, false, s));
-      WF_TRY(head(h, h->x, h->st_x, 1, 0, n, h->active, 1, h->recs_t, h->hout_t, h->logits_t, sp, kTagBonus,
-                  nullptr, s));
+      WF_TRY(head(h, h->x, use_skinny(h, n) ? nullptr : h->st_x, 1, 0, n, h->active, 1, h->recs_t, h->hout_t,
+                  h->logits_t, sp, kTagBonus, nullptr, s));
     }
   }
   AcceptParams ap = {};

@@ -101,6 +101,43 @@ cudaError_t launch_gemm(const void *X, const void *W, GemmParams p, cudaStream_t
 // launch_layernorm first (same bits either way).
 bool gemm_ln_fits(int M, int N, int K, int epi);
 
+// ------------------------------------------------------ skinny projections --
+// Y = X W^T for M <= 16 token rows (wf_skinny.cu): each CTA prefetches its
+// whole weight slab (U units of 8 rows over K / S) with TMA before the
+// dependency wait and reduces K in a fixed order.  The operand is LN(ln_x)
+// computed in the kernel (row statistics included) or bf16 rows x.  Epilogues
+// as EpiMode (no EPI_HEAD; EPI_RESID writes no statistics).
+constexpr int kSkMaxRows = 16;
+struct SkinnyParams {
+  int M, N, K;
+  int U, S;  // set by launch_skinny
+  int epi;
+  const bf16 *x;
+  int ld_x;
+  const float *ln_x;
+  int ln_ld;
+  const bf16 *ln_g, *ln_b;
+  float ln_eps;
+  const bf16 *bias;
+  float *out_f32;
+  bf16 *out_bf16;
+  int ld_out;
+  float *resid;
+  int ld_resid;
+  bf16 *tap0, *tap1;
+  int ld_tap;
+  int q_cols, d_model, n_heads, ctx, rows_per_seq;
+  bf16 *kc, *vc;
+  const int32_t *seq_slot, *pos_base;
+  uint32_t *err;
+  long long spin;
+};
+// Whether a projection of M rows, N outputs and K inputs has a skinny plan
+// (units per CTA U, K split S); LN operands need S == 1.
+bool skinny_plan(int M, int N, int K, bool ln, int *U, int *S);
+cudaError_t skinny_init();
+cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pdl);
+
 // ------------------------------------------------------------- attention --
 struct AttnParams {
   const bf16 *q;
@@ -136,7 +173,8 @@ struct EmbedParams {
 cudaError_t launch_embed(const EmbedParams &p, cudaStream_t s, bool pdl);
 
 // y[r] = LN(x[i]) as bf16 with i = r*in_stride + in_off, using the row's
-// per-tile statistics stats[i][0..d/128) (mean, M2) written by its producer.
+// per-tile statistics stats[i][0..d/128) (mean, M2) written by its producer,
+// or (stats == nullptr) the row's mean and variance computed here.
 cudaError_t launch_layernorm(const float *x, const float2 *stats, int in_stride, int in_off,
                              const bf16 *g, const bf16 *b, bf16 *y, int rows, int d, float eps,
                              cudaStream_t s, bool pdl);

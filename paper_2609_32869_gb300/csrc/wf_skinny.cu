@@ -1,0 +1,408 @@
+// Low-latency projections for a handful of token rows (M <= 16: one
+// speculative block of K + 1 = 9 rows, a plain greedy step, a short prompt).
+//
+// At batch 1 a decoder block is a chain of eight dependent steps over 46 MB
+// of weights (Sec. 3.1: one verify pass; Sec. 3.2: one drafter pass), so each
+// projection's time after its dependency wait, not its weight stream, sets
+// the step time.  This kernel is shaped for that:
+//  - every CTA owns U units of 8 weight rows over a K range (the whole K, or
+//    1/S of it inside a cluster of S CTAs) and requests its entire weight slab
+//    with TMA before griddepcontrol.wait, one 3-D tensor copy per unit that
+//    lands 128-byte swizzled ([k-block][8 rows][64 features]); the slab
+//    streams while the previous kernels run;
+//  - after the wait the token operand is built in shared memory: LN(x) from
+//    the fp32 residual rows (each warp computes its rows' mean and variance
+//    itself, so no statistics travel between kernels), or plain bf16 rows;
+//  - all eight warps issue mma.sync m16n8k16 at once (tokens on the 16-row
+//    side, weight rows on the 8-column side), each over its own slice of K;
+//    the slices are summed in warp order, then (S > 1) the S CTAs' sums in
+//    rank order over distributed shared memory, so a row's result never
+//    depends on how many rows run with it;
+//  - the epilogue adds the bias and applies GELU, the residual update with
+//    the history taps, or the key/value cache scatter.
+// At these shapes tcgen05.mma would be issued by one thread per CTA, 64 or
+// more rows wide, for 9 useful rows; the warp-level MMA issues from every
+// warp at once, and the tensor pipe is idle either way: the weights bound it.
+#include <map>
+#include <mutex>
+#include <tuple>
+
+#include "wf_device.cuh"
+#include "wf_internal.h"
+
+namespace wf {
+
+namespace {
+
+constexpr int kSkThreads = 256;
+constexpr int kSkWarps = kSkThreads / 32;
+
+__device__ __forceinline__ void tma_load_3d(void *smem_dst, const CUtensorMap *m, int32_t x, int32_t y,
+                                            int32_t z, uint64_t *bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// Shared-memory layout of one CTA (offsets from the 1024-aligned base).  The
+// warps' partial sums reuse the weight slab once every MMA has read it.
+struct SkLayout {
+  int unit_bytes, w_bytes, a_off, a_bytes, sum_off, bias_off, bar_off, zero_off, flag_off, total;
+  __host__ __device__ SkLayout(int M, int Ks, int U) {
+    const int kb = Ks / 64;
+    unit_bytes = kb * 1024;
+    w_bytes = U * unit_bytes;
+    a_off = w_bytes;
+    a_bytes = kb * M * 128;
+    sum_off = (a_off + a_bytes + 15) & ~15;
+    bias_off = sum_off + U * 128 * 4;
+    bar_off = (bias_off + U * 8 * 4 + 15) & ~15;
+    zero_off = bar_off + 16;
+    flag_off = zero_off + 16;
+    total = flag_off + 16;
+  }
+};
+
+// byte offset of element k of token row r in the operand tile: [k-block][M rows][128 B],
+// 16-byte chunk j of a row stored at chunk j ^ (r & 7) (the TMA's 128-byte swizzle)
+__device__ __forceinline__ uint32_t a_off(int M, int r, int k) {
+  return static_cast<uint32_t>(((k >> 6) * M + r) * 128 + ((((k >> 3) & 7) ^ (r & 7)) << 4) + (k & 7) * 2);
+}
+
+}  // namespace
+
+__global__ void __launch_bounds__(kSkThreads, 1) skinny_kernel(const __grid_constant__ CUtensorMap tmW,
+                                                               const SkinnyParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  uint8_t *smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+  const int M = p.M, U = p.U, S = p.S;
+  const int Ks = p.K / S;  // K range of this CTA
+  const int kb = Ks / 64;  // 64-wide k-blocks
+  const SkLayout L(M, Ks, U);
+  const int unit_bytes = L.unit_bytes;             // one unit: [kb][8 rows][128 B]
+  uint8_t *sW = smem;
+  uint8_t *sA = smem + L.a_off;                    // [kb][M][128 B]
+  float *sPart = reinterpret_cast<float *>(smem);  // [warps][U][16][8], over the slab after the MMAs
+  float *sSum = reinterpret_cast<float *>(smem + L.sum_off);    // [U][16][8]
+  float *sBias = reinterpret_cast<float *>(smem + L.bias_off);  // [U * 8]
+  uint64_t *bar = reinterpret_cast<uint64_t *>(smem + L.bar_off);
+  uint4 *sZero = reinterpret_cast<uint4 *>(smem + L.zero_off);
+  int *s_flag = reinterpret_cast<int *>(smem + L.flag_off);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int cta = blockIdx.x, split = blockIdx.z;
+  const int unit0 = cta * U;  // first 8-row unit of this CTA
+  const int n_base = unit0 * 8;
+
+  if (tid == 0) {
+    *s_flag = 0;
+    tma_prefetch_desc(&tmW);
+    mbar_init(bar, 1);
+    fence_barrier_init();
+    *sZero = make_uint4(0u, 0u, 0u, 0u);
+    // the whole weight slab: one copy per unit, before the dependency wait
+    mbar_arrive_expect_tx(bar, static_cast<uint32_t>(U * unit_bytes));
+    for (int u = 0; u < U; ++u)
+      tma_load_3d(sW + static_cast<size_t>(u) * unit_bytes, &tmW, 0, (unit0 + u) * 8, split * kb, bar);
+  }
+  for (int i = tid; i < U * 8; i += kSkThreads) {
+    const int n = n_base + i;
+    sBias[i] = (p.bias && n < p.N) ? bf2f(p.bias[n]) : 0.f;
+  }
+  pdl_launch_dependents();
+  pdl_wait();
+
+  // ---------------- token operand
+  if (p.ln_x) {
+    // LN(x) from the fp32 rows: warp w normalises rows w, w + 8; lane l holds
+    // features 4l + 128 i (every load in flight before the first sum)
+    constexpr int kMaxI = 12;  // K <= 1536
+    const int nI = p.K / 128;
+    for (int r = warp; r < M; r += kSkWarps) {
+      const float *xr = p.ln_x + static_cast<size_t>(r) * p.ln_ld;
+      float4 v[kMaxI];
+#pragma unroll
+      for (int i = 0; i < kMaxI; ++i)
+        if (i < nI) v[i] = __ldcg(reinterpret_cast<const float4 *>(xr + 4 * lane + 128 * i));
+      float s = 0.f;
+#pragma unroll
+      for (int i = 0; i < kMaxI; ++i)
+        if (i < nI) s += (v[i].x + v[i].y) + (v[i].z + v[i].w);
+      const float mean = warp_sum(s) / static_cast<float>(p.K);
+      float q = 0.f;
+#pragma unroll
+      for (int i = 0; i < kMaxI; ++i) {
+        if (i < nI) {
+          const float a = v[i].x - mean, b = v[i].y - mean, c = v[i].z - mean, d = v[i].w - mean;
+          q += (a * a + b * b) + (c * c + d * d);
+        }
+      }
+      const float rstd = rsqrtf(warp_sum(q) / static_cast<float>(p.K) + p.ln_eps);
+#pragma unroll
+      for (int i = 0; i < kMaxI; ++i) {
+        if (i < nI) {
+          const int k = 4 * lane + 128 * i;
+          const uint2 gg = *reinterpret_cast<const uint2 *>(p.ln_g + k);
+          const uint2 bb = *reinterpret_cast<const uint2 *>(p.ln_b + k);
+          const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gg);
+          const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&bb);
+          const float2 ms = make_float2(mean, rstd);
+          const __nv_bfloat162 o0 = __floats2bfloat162_rn(ln_apply(v[i].x, ms, __low2float(g2[0]), __low2float(b2[0])),
+                                                          ln_apply(v[i].y, ms, __high2float(g2[0]), __high2float(b2[0])));
+          const __nv_bfloat162 o1 = __floats2bfloat162_rn(ln_apply(v[i].z, ms, __low2float(g2[1]), __low2float(b2[1])),
+                                                          ln_apply(v[i].w, ms, __high2float(g2[1]), __high2float(b2[1])));
+          uint2 o;
+          o.x = *reinterpret_cast<const uint32_t *>(&o0);
+          o.y = *reinterpret_cast<const uint32_t *>(&o1);
+          *reinterpret_cast<uint2 *>(sA + a_off(M, r, k)) = o;
+        }
+      }
+    }
+  } else {
+    // bf16 rows [M][ld_x], columns [split * Ks, (split + 1) * Ks)
+    const int chunks = M * (Ks / 8);
+    const bf16 *x0 = p.x + static_cast<size_t>(split) * Ks;
+    for (int c = tid; c < chunks; c += kSkThreads) {
+      const int r = c / (Ks / 8), k = (c - r * (Ks / 8)) * 8;
+      const uint4 v = __ldcg(reinterpret_cast<const uint4 *>(x0 + static_cast<size_t>(r) * p.ld_x + k));
+      *reinterpret_cast<uint4 *>(sA + a_off(M, r, k)) = v;
+    }
+  }
+  __syncthreads();
+
+  // ---------------- MMAs: warp w takes k-steps [w * ksw, (w + 1) * ksw) of every unit
+  const bool landed = mbar_wait(bar, 0, p.err, p.spin);
+  if (!landed) *s_flag = 1;
+  const int ksteps = Ks / 16, ksw = ksteps / kSkWarps;
+  float acc[8][4];  // per unit (U <= 8): the 16 x 8 tile's fragment
+#pragma unroll
+  for (int u = 0; u < 8; ++u) acc[u][0] = acc[u][1] = acc[u][2] = acc[u][3] = 0.f;
+  if (landed) {
+    const uint32_t a_base = smem_u32(sA), w_base = smem_u32(sW), z_addr = smem_u32(sZero);
+    // A rows for ldmatrix.x4: lanes 0-7 rows 0-7 (k 0-7), 8-15 rows 8-15 (k 0-7),
+    // 16-23 rows 0-7 (k 8-15), 24-31 rows 8-15 (k 8-15); rows >= M read zeros
+    const int ar = (lane & 7) + ((lane >> 3) & 1) * 8, ak = (lane >> 4) * 8;
+    // B for ldmatrix.x4 over two k-steps: lane group g = lane >> 3 -> k offset 8 g
+    const int br = lane & 7, bk = (lane >> 3) * 8;
+    const int s_end = (warp + 1) * ksw;
+    int s = warp * ksw;
+    for (; s + 1 < s_end; s += 2) {  // two k-steps per B load
+      uint32_t a0[4], a1[4];
+      {
+        const int k = s * 16 + ak;
+        const uint32_t ad0 = ar < M ? a_base + a_off(M, ar, k) : z_addr;
+        const uint32_t ad1 = ar < M ? a_base + a_off(M, ar, k + 16) : z_addr;
+        ldsm_x4(ad0, a0[0], a0[1], a0[2], a0[3]);
+        ldsm_x4(ad1, a1[0], a1[1], a1[2], a1[3]);
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        if (u < U) {
+          const int k = s * 16 + bk;  // 32 consecutive k over the four matrices
+          const uint32_t wd = w_base + static_cast<uint32_t>(u * unit_bytes + (k >> 6) * 1024 + br * 128 +
+                                                             ((((k >> 3) & 7) ^ br) << 4));
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4(wd, b0, b1, b2, b3);
+          mma_bf16(acc[u], a0[0], a0[1], a0[2], a0[3], b0, b1);
+          mma_bf16(acc[u], a1[0], a1[1], a1[2], a1[3], b2, b3);
+        }
+      }
+    }
+    if (s < s_end) {  // an odd last k-step
+      uint32_t a0[4];
+      const int k = s * 16 + ak;
+      ldsm_x4(ar < M ? a_base + a_off(M, ar, k) : z_addr, a0[0], a0[1], a0[2], a0[3]);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        if (u < U) {
+          const int kk = s * 16 + (bk & 8);  // lanes 16-31 repeat lanes 0-15's addresses
+          const uint32_t wd = w_base + static_cast<uint32_t>(u * unit_bytes + (kk >> 6) * 1024 + br * 128 +
+                                                             ((((kk >> 3) & 7) ^ br) << 4));
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4(wd, b0, b1, b2, b3);
+          mma_bf16(acc[u], a0[0], a0[1], a0[2], a0[3], b0, b1);
+        }
+      }
+    }
+  }
+  __syncthreads();  // every warp is done with the slab, which now takes the partials
+  // warp partials -> shared memory: lane holds rows g, g+8 and columns 2 c4, 2 c4 + 1
+  {
+    const int g = lane >> 2, c4 = lane & 3;
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      if (u < U) {
+        float *pw = sPart + (warp * U + u) * 128;
+        pw[g * 8 + 2 * c4] = acc[u][0];
+        pw[g * 8 + 2 * c4 + 1] = acc[u][1];
+        pw[(g + 8) * 8 + 2 * c4] = acc[u][2];
+        pw[(g + 8) * 8 + 2 * c4 + 1] = acc[u][3];
+      }
+    }
+  }
+  __syncthreads();
+  // the CTA's sums, warps added in order
+  for (int e = tid; e < U * 128; e += kSkThreads) {
+    const int u = e >> 7, rc = e & 127;
+    float v = 0.f;
+#pragma unroll
+    for (int w = 0; w < kSkWarps; ++w) v += sPart[(w * U + u) * 128 + rc];
+    sSum[e] = v;
+  }
+  // ---------------- S > 1: the cluster's CTAs add their sums in rank order;
+  // rank r finishes the outputs e with e % S == r
+  const bool ok = landed;
+  if (S > 1) cluster_sync();
+  else __syncthreads();
+  for (int e = tid; e < U * M * 8; e += kSkThreads) {
+    if (S > 1 && (e % S) != split) continue;
+    const int u = e / (M * 8), rem = e - u * M * 8, t = rem >> 3, j = rem & 7;
+    const int idx = u * 128 + t * 8 + j;
+    float v;
+    if (S > 1) {
+      v = 0.f;
+      const uint32_t loc = smem_u32(sSum + idx);
+      for (int r = 0; r < S; ++r) v += dsmem_ld_f32(dsmem_map(loc, r));
+    } else {
+      v = sSum[idx];
+    }
+    const int n = n_base + u * 8 + j;
+    if (n >= p.N || !ok) continue;
+    v += sBias[u * 8 + j];
+    if (p.epi == EPI_F32) {
+      p.out_f32[static_cast<size_t>(t) * p.ld_out + n] = v;
+    } else if (p.epi == EPI_BF16) {
+      p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(v);
+    } else if (p.epi == EPI_GELU) {
+      p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(gelu_erf(v));
+    } else if (p.epi == EPI_RESID) {
+      float *xr = p.resid + static_cast<size_t>(t) * p.ld_resid + n;
+      const float nr = __ldcg(xr) + v;
+      *xr = nr;
+      if (p.tap0) p.tap0[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
+      if (p.tap1) p.tap1[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
+    } else if (p.epi == EPI_KV) {
+      if (n < p.q_cols) {
+        p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(v);
+      } else {
+        const int c = n - p.q_cols, which = c / p.d_model, hd = c - which * p.d_model;
+        const int i = t / p.rows_per_seq, jr = t - i * p.rows_per_seq;
+        const int slot = p.seq_slot[i];
+        const int pos = (p.pos_base ? p.pos_base[slot] : 0) + jr;
+        if (pos >= p.ctx) {
+          set_error(p.err, WF_DEV_ERR_CAPACITY);
+        } else {
+          bf16 *dst = which == 0 ? p.kc : p.vc;
+          dst[((static_cast<size_t>(slot) * p.n_heads + (hd >> 6)) * p.ctx + pos) * 64 + (hd & 63)] =
+              __float2bfloat16(v);
+        }
+      }
+    }
+  }
+  if (S > 1) cluster_sync();  // peers may read this CTA's sums until here
+  // after a timeout the slab's copy may still be landing: wait for it (bounded)
+  __syncthreads();
+  if (tid == 0 && *s_flag) mbar_drain(bar, 0);
+}
+
+// ------------------------------------------------------------------ host ----
+namespace {
+size_t skinny_smem(int M, int K, int U, int S) { return 1024 + static_cast<size_t>(SkLayout(M, K / S, U).total); }
+}  // namespace
+
+bool skinny_plan(int M, int N, int K, bool ln, int *U, int *S) {
+  if (M < 1 || M > kSkMaxRows || N % 8 || K % 128) return false;
+  const int units = N / 8;
+  // the fewest CTAs' worth of units that keeps the grid within about one CTA
+  // per SM (160 for 1280 rows of 8) and a CTA within 110 KB of shared memory
+  // (two kernels' CTAs share an SM, so the next one's slab streams in while
+  // this one runs); whole K per CTA unless that does not fit, then K split
+  // over a cluster of S CTAs
+  int best_u = 0, best_s = 0;
+  for (int s = 1; s <= 8; s *= 2) {
+    if (K % (s * 128) || K / s < 256 || (ln && s > 1)) continue;
+    for (int u = 1; u <= 8; ++u) {
+      if (units % u) continue;
+      const int ctas = units / u * s;
+      if (ctas > 160) continue;
+      if (skinny_smem(M, K, u, s) > 110 * 1024) continue;
+      if (!best_u) {
+        best_u = u;
+        best_s = s;
+      }
+      break;
+    }
+    if (best_u) break;
+  }
+  if (!best_u) return false;
+  if (ln && K > 1536) return false;
+  *U = best_u;
+  *S = best_s;
+  return true;
+}
+
+// Unit tensor maps, encoded once per (matrix, k-blocks per copy).
+static const CUtensorMap *skinny_tmap(const void *W, int N, int K, int kblocks) {
+  static std::mutex mu;
+  static std::map<std::tuple<uintptr_t, int, int, int>, CUtensorMap *> cache;
+  std::lock_guard<std::mutex> lock(mu);
+  const auto key = std::make_tuple(reinterpret_cast<uintptr_t>(W), N, K, kblocks);
+  auto it = cache.find(key);
+  if (it != cache.end()) return it->second;
+  CUtensorMap *m = new CUtensorMap;
+  if (!tmap_bf16_units(m, W, N, K, kblocks)) {
+    delete m;
+    return nullptr;
+  }
+  cache.emplace(key, m);
+  return m;
+}
+
+cudaError_t skinny_init() {
+  static cudaError_t status = cudaErrorNotReady;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    status = cudaFuncSetAttribute(skinny_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 110 * 1024);
+    if (status == cudaSuccess)
+      status = cudaFuncSetAttribute(skinny_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  });
+  return status;
+}
+
+cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pdl) {
+  if (p.spin <= 0) p.spin = kSpinLimitCycles;
+  if (!skinny_plan(p.M, p.N, p.K, p.ln_x != nullptr, &p.U, &p.S)) return cudaErrorInvalidValue;
+  if (p.ln_x && (!p.ln_g || !p.ln_b || p.ln_ld % 4 || (reinterpret_cast<uintptr_t>(p.ln_x) & 15)))
+    return cudaErrorInvalidValue;
+  if (!p.ln_x && (!p.x || p.ld_x % 8 || (reinterpret_cast<uintptr_t>(p.x) & 15))) return cudaErrorInvalidValue;
+  const CUtensorMap *tm = skinny_tmap(W, p.N, p.K, p.K / p.S / 64);
+  if (!tm) return cudaErrorInvalidValue;
+  const size_t smem = skinny_smem(p.M, p.K, p.U, p.S);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.N / 8 / p.U, 1, p.S);
+  cfg.blockDim = dim3(kSkThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  int na = 0;
+  if (p.S > 1) {
+    attr[na].id = cudaLaunchAttributeClusterDimension;
+    attr[na].val.clusterDim.x = 1;
+    attr[na].val.clusterDim.y = 1;
+    attr[na].val.clusterDim.z = p.S;
+    ++na;
+  }
+  if (pdl) {
+    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = na;
+  return cudaLaunchKernelEx(&cfg, skinny_kernel, *tm, p);
+}
+
+}  // namespace wf

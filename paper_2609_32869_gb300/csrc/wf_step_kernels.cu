@@ -137,7 +137,25 @@ __global__ void __launch_bounds__(128) layernorm_kernel(const float *__restrict_
       bv[k] = br[k * 32 + lane];
     }
   }
-  const float2 ms = merge_tile_stats(stats + row * chunks, chunks, eps);
+  float2 ms;
+  if (stats) {
+    ms = merge_tile_stats(stats + row * chunks, chunks, eps);
+  } else {  // the row's own mean and variance (two passes over the registers)
+    float sum = 0.f;
+#pragma unroll
+    for (int k = 0; k < kMaxStatTiles; ++k)
+      if (k < chunks) sum += (v[k].x + v[k].y) + (v[k].z + v[k].w);
+    const float mean = warp_sum(sum) / static_cast<float>(d);
+    float q = 0.f;
+#pragma unroll
+    for (int k = 0; k < kMaxStatTiles; ++k) {
+      if (k < chunks) {
+        const float a = v[k].x - mean, b = v[k].y - mean, c = v[k].z - mean, e = v[k].w - mean;
+        q += (a * a + b * b) + (c * c + e * e);
+      }
+    }
+    ms = make_float2(mean, rsqrtf(warp_sum(q) / static_cast<float>(d) + eps));
+  }
   uint2 *yr = reinterpret_cast<uint2 *>(y + static_cast<size_t>(warp) * d);
 #pragma unroll
   for (int k = 0; k < kMaxStatTiles; ++k) {
@@ -163,7 +181,7 @@ __global__ void __launch_bounds__(128) layernorm_kernel(const float *__restrict_
 cudaError_t launch_layernorm(const float *x, const float2 *stats, int in_stride, int in_off,
                              const bf16 *g, const bf16 *b, bf16 *y, int rows, int d, float eps,
                              cudaStream_t s, bool pdl) {
-  if (d % 128 || d / 128 > kMaxStatTiles || !stats) return cudaErrorInvalidValue;
+  if (d % 128 || d / 128 > kMaxStatTiles) return cudaErrorInvalidValue;
   void *args[] = {&x, &stats, &in_stride, &in_off, &g, &b, &y, &rows, &d, &eps};
   const int threads = 128;
   const int blocks = (rows * 32 + threads - 1) / threads;
