@@ -268,6 +268,8 @@ def measure_greedy(args, wl_name, dev, host_ws, rank, world, steps, warmup, e2e=
     sess = Session(cfg, dev, max_batch=Bn, max_ctx=cfg.max_pos)
     if args.persist:
         B.wf_set_option(sess.h, B.WF_OPT_PERSIST, 1)
+    if args.no_skinny:
+        B.wf_set_option(sess.h, B.WF_OPT_SKINNY, 0)
     slots = np.arange(Bn, dtype=np.int32)
     stream = sess.stream
 
@@ -875,6 +877,8 @@ def main():
                     help="cudaProfilerStart/Stop around the timed steps (for ncu)")
     ap.add_argument("--budget", type=int, default=0,
                     help="override every transcript budget (short profiling runs)")
+    ap.add_argument("--no-skinny", action="store_true",
+                    help="single-sequence handles use the tcgen05 projections (WF_OPT_SKINNY 0)")
     ap.add_argument("--no-per-batch", action="store_true",
                     help="skip the batch-16 and batch-96 entries of the default line")
     ap.add_argument("--batch-steps", type=int, default=20,
