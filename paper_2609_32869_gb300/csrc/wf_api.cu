@@ -912,6 +912,7 @@ wf_status wf_create(const wf_config *cfg, const wf_target_weights *tw, const wf_
   h->skinny_ok = skinny_shapes_fit(h->d, h->F, h->sk_rows);
   h->skinny = h->skinny_ok;
   ok = ok && gemm_init() == cudaSuccess && skinny_init() == cudaSuccess && attention_init() == cudaSuccess &&
+       step_kernels_init() == cudaSuccess &&
        cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) == cudaSuccess;
   if (ok && h->mk_ok) ok = persist_setup(h, s) == cudaSuccess;
   if (!ok) {

@@ -467,6 +467,7 @@ cudaError_t attention_init() {
   std::call_once(once, [] {
     status = cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   kSmemAttnSpread);
+    if (status == cudaSuccess) status = prefer_max_shared(reinterpret_cast<const void *>(attention_kernel));
   });
   return status;
 }

@@ -812,6 +812,9 @@ cudaError_t gemm_init() {
     for (const void *f : fns)
       if (status == cudaSuccess)
         status = cudaFuncSetAttribute(f, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    for (const void *f : fns)
+      if (status == cudaSuccess) status = prefer_max_shared(f);
+    if (status == cudaSuccess) status = prefer_max_shared(reinterpret_cast<const void *>(gemm_tc_kernel<EPI_HEAD>));
   });
   return status;
 }

@@ -12,6 +12,17 @@ namespace wf {
 
 using bf16 = __nv_bfloat16;
 
+// Every kernel of the library runs with the same shared-memory carveout (the
+// largest), so consecutive kernels of a pass, whose CTAs overlap under
+// programmatic dependent launch, can share an SM without it first draining
+// to change its L1 / shared-memory split.
+inline cudaError_t prefer_max_shared(const void *fn) {
+  return cudaFuncSetAttribute(fn, cudaFuncAttributePreferredSharedMemoryCarveout,
+                              cudaSharedmemCarveoutMaxShared);
+}
+// The row-wise kernels of wf_step_kernels.cu (once per process).
+cudaError_t step_kernels_init();
+
 // ------------------------------------------------------------------ GEMM --
 // Y[t, n] = sum_k X[t, k] W[n, k] for token rows t < M and features n < N,
 // computed as a 128 x BT tile of D = W_tile * X_tile^T on tcgen05 ("swap-AB":

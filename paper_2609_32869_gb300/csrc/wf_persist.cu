@@ -1251,6 +1251,7 @@ cudaError_t persist_init(int *G) {
   if (!ready[dev]) {
     int n_sm = 0, per_sm = 0;
     e = cudaFuncSetAttribute(persist_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMk);
+    if (e == cudaSuccess) e = prefer_max_shared(reinterpret_cast<const void *>(persist_kernel));
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
     if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, persist_kernel, kThr, kSmemMk);
     if (e == cudaSuccess && per_sm < 1) e = cudaErrorInvalidConfiguration;

@@ -49,8 +49,9 @@ __device__ __forceinline__ void tma_load_3d(void *smem_dst, const CUtensorMap *m
 // Shared-memory layout of one CTA (offsets from the 1024-aligned base).  The
 // warps' partial sums reuse the weight slab once every MMA has read it.
 struct SkLayout {
-  int unit_bytes, w_bytes, a_off, a_bytes, sum_off, bias_off, bar_off, zero_off, flag_off, total;
-  __host__ __device__ SkLayout(int M, int Ks, int U) {
+  int unit_bytes, w_bytes, a_off, a_bytes, sum_off, bias_off, gb_off, bar_off, zero_off, flag_off, total;
+  // K_ln: features of a LayerNorm operand (its gain and bias are staged), else 0
+  __host__ __device__ SkLayout(int M, int Ks, int U, int K_ln) {
     const int kb = Ks / 64;
     unit_bytes = kb * 1024;
     w_bytes = U * unit_bytes;
@@ -58,7 +59,8 @@ struct SkLayout {
     a_bytes = kb * M * 128;
     sum_off = (a_off + a_bytes + 15) & ~15;
     bias_off = sum_off + U * 128 * 4;
-    bar_off = (bias_off + U * 8 * 4 + 15) & ~15;
+    gb_off = (bias_off + U * 8 * 4 + 15) & ~15;
+    bar_off = (gb_off + K_ln * 4 + 15) & ~15;
     zero_off = bar_off + 16;
     flag_off = zero_off + 16;
     total = flag_off + 16;
@@ -73,7 +75,7 @@ __device__ __forceinline__ uint32_t a_off(int M, int r, int k) {
 
 }  // namespace
 
-__global__ void __launch_bounds__(kSkThreads, 1) skinny_kernel(const __grid_constant__ CUtensorMap tmW,
+__global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_constant__ CUtensorMap tmW,
                                                                const SkinnyParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -81,13 +83,15 @@ __global__ void __launch_bounds__(kSkThreads, 1) skinny_kernel(const __grid_cons
   const int M = p.M, U = p.U, S = p.S;
   const int Ks = p.K / S;  // K range of this CTA
   const int kb = Ks / 64;  // 64-wide k-blocks
-  const SkLayout L(M, Ks, U);
+  const SkLayout L(M, Ks, U, p.ln_x ? p.K : 0);
   const int unit_bytes = L.unit_bytes;             // one unit: [kb][8 rows][128 B]
   uint8_t *sW = smem;
   uint8_t *sA = smem + L.a_off;                    // [kb][M][128 B]
   float *sPart = reinterpret_cast<float *>(smem);  // [warps][U][16][8], over the slab after the MMAs
   float *sSum = reinterpret_cast<float *>(smem + L.sum_off);    // [U][16][8]
   float *sBias = reinterpret_cast<float *>(smem + L.bias_off);  // [U * 8]
+  bf16 *sG = reinterpret_cast<bf16 *>(smem + L.gb_off);         // [K] LayerNorm gain, then [K] bias
+  bf16 *sB = sG + p.K;
   uint64_t *bar = reinterpret_cast<uint64_t *>(smem + L.bar_off);
   uint4 *sZero = reinterpret_cast<uint4 *>(smem + L.zero_off);
   int *s_flag = reinterpret_cast<int *>(smem + L.flag_off);
@@ -112,48 +116,62 @@ __global__ void __launch_bounds__(kSkThreads, 1) skinny_kernel(const __grid_cons
     const int n = n_base + i;
     sBias[i] = (p.bias && n < p.N) ? bf2f(p.bias[n]) : 0.f;
   }
+  if (p.ln_x) {  // parameters, not activations: staged before the wait
+    for (int i = tid; i < p.K / 8; i += kSkThreads) {
+      reinterpret_cast<uint4 *>(sG)[i] = reinterpret_cast<const uint4 *>(p.ln_g)[i];
+      reinterpret_cast<uint4 *>(sB)[i] = reinterpret_cast<const uint4 *>(p.ln_b)[i];
+    }
+  }
   pdl_launch_dependents();
   pdl_wait();
 
   // ---------------- token operand
   if (p.ln_x) {
-    // LN(x) from the fp32 rows: warp w normalises rows w, w + 8; lane l holds
-    // features 4l + 128 i (every load in flight before the first sum)
+    // LN(x) from the fp32 rows: warp w normalises rows w and w + 8 together
+    // (every load of both rows in flight before the first sum); lane l holds
+    // features 4l + 128 i
     constexpr int kMaxI = 12;  // K <= 1536
     const int nI = p.K / 128;
-    for (int r = warp; r < M; r += kSkWarps) {
-      const float *xr = p.ln_x + static_cast<size_t>(r) * p.ln_ld;
-      float4 v[kMaxI];
+    const int r0 = warp, r1 = warp + kSkWarps;
+    float4 v[2][kMaxI];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int r = h ? r1 : r0;
+      const float *xr = p.ln_x + static_cast<size_t>(r < M ? r : 0) * p.ln_ld;
 #pragma unroll
       for (int i = 0; i < kMaxI; ++i)
-        if (i < nI) v[i] = __ldcg(reinterpret_cast<const float4 *>(xr + 4 * lane + 128 * i));
-      float s = 0.f;
+        if (i < nI && r < M) v[h][i] = __ldcg(reinterpret_cast<const float4 *>(xr + 4 * lane + 128 * i));
+    }
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int r = h ? r1 : r0;
+      if (r >= M) continue;
+      float sum = 0.f;
 #pragma unroll
       for (int i = 0; i < kMaxI; ++i)
-        if (i < nI) s += (v[i].x + v[i].y) + (v[i].z + v[i].w);
-      const float mean = warp_sum(s) / static_cast<float>(p.K);
+        if (i < nI) sum += (v[h][i].x + v[h][i].y) + (v[h][i].z + v[h][i].w);
+      const float mean = warp_sum(sum) / static_cast<float>(p.K);
       float q = 0.f;
 #pragma unroll
       for (int i = 0; i < kMaxI; ++i) {
         if (i < nI) {
-          const float a = v[i].x - mean, b = v[i].y - mean, c = v[i].z - mean, d = v[i].w - mean;
+          const float a = v[h][i].x - mean, b = v[h][i].y - mean, c = v[h][i].z - mean, d = v[h][i].w - mean;
           q += (a * a + b * b) + (c * c + d * d);
         }
       }
-      const float rstd = rsqrtf(warp_sum(q) / static_cast<float>(p.K) + p.ln_eps);
+      const float2 ms = make_float2(mean, rsqrtf(warp_sum(q) / static_cast<float>(p.K) + p.ln_eps));
 #pragma unroll
       for (int i = 0; i < kMaxI; ++i) {
         if (i < nI) {
           const int k = 4 * lane + 128 * i;
-          const uint2 gg = *reinterpret_cast<const uint2 *>(p.ln_g + k);
-          const uint2 bb = *reinterpret_cast<const uint2 *>(p.ln_b + k);
+          const uint2 gg = *reinterpret_cast<const uint2 *>(sG + k);
+          const uint2 bb = *reinterpret_cast<const uint2 *>(sB + k);
           const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gg);
           const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&bb);
-          const float2 ms = make_float2(mean, rstd);
-          const __nv_bfloat162 o0 = __floats2bfloat162_rn(ln_apply(v[i].x, ms, __low2float(g2[0]), __low2float(b2[0])),
-                                                          ln_apply(v[i].y, ms, __high2float(g2[0]), __high2float(b2[0])));
-          const __nv_bfloat162 o1 = __floats2bfloat162_rn(ln_apply(v[i].z, ms, __low2float(g2[1]), __low2float(b2[1])),
-                                                          ln_apply(v[i].w, ms, __high2float(g2[1]), __high2float(b2[1])));
+          const __nv_bfloat162 o0 = __floats2bfloat162_rn(ln_apply(v[h][i].x, ms, __low2float(g2[0]), __low2float(b2[0])),
+                                                          ln_apply(v[h][i].y, ms, __high2float(g2[0]), __high2float(b2[0])));
+          const __nv_bfloat162 o1 = __floats2bfloat162_rn(ln_apply(v[h][i].z, ms, __low2float(g2[1]), __low2float(b2[1])),
+                                                          ln_apply(v[h][i].w, ms, __high2float(g2[1]), __high2float(b2[1])));
           uint2 o;
           o.x = *reinterpret_cast<const uint32_t *>(&o0);
           o.y = *reinterpret_cast<const uint32_t *>(&o1);
@@ -162,13 +180,29 @@ __global__ void __launch_bounds__(kSkThreads, 1) skinny_kernel(const __grid_cons
       }
     }
   } else {
-    // bf16 rows [M][ld_x], columns [split * Ks, (split + 1) * Ks)
-    const int chunks = M * (Ks / 8);
+    // bf16 rows [M][ld_x], columns [split * Ks, (split + 1) * Ks): up to eight
+    // 16-byte loads per thread in flight before their stores
+    const int cpr = Ks / 8, chunks = M * cpr;
     const bf16 *x0 = p.x + static_cast<size_t>(split) * Ks;
-    for (int c = tid; c < chunks; c += kSkThreads) {
-      const int r = c / (Ks / 8), k = (c - r * (Ks / 8)) * 8;
-      const uint4 v = __ldcg(reinterpret_cast<const uint4 *>(x0 + static_cast<size_t>(r) * p.ld_x + k));
-      *reinterpret_cast<uint4 *>(sA + a_off(M, r, k)) = v;
+    constexpr int kU = 8;
+    for (int c0 = 0; c0 < chunks; c0 += kU * kSkThreads) {
+      uint4 v[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int c = c0 + u * kSkThreads + tid;
+        if (c < chunks) {
+          const int r = c / cpr, k = (c - r * cpr) * 8;
+          v[u] = __ldcg(reinterpret_cast<const uint4 *>(x0 + static_cast<size_t>(r) * p.ld_x + k));
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int c = c0 + u * kSkThreads + tid;
+        if (c < chunks) {
+          const int r = c / cpr, k = (c - r * cpr) * 8;
+          *reinterpret_cast<uint4 *>(sA + a_off(M, r, k)) = v[u];
+        }
+      }
     }
   }
   __syncthreads();
@@ -310,7 +344,9 @@ __global__ void __launch_bounds__(kSkThreads, 1) skinny_kernel(const __grid_cons
 
 // ------------------------------------------------------------------ host ----
 namespace {
-size_t skinny_smem(int M, int K, int U, int S) { return 1024 + static_cast<size_t>(SkLayout(M, K / S, U).total); }
+size_t skinny_smem(int M, int K, int U, int S, bool ln) {
+  return 1024 + static_cast<size_t>(SkLayout(M, K / S, U, ln ? K : 0).total);
+}
 }  // namespace
 
 bool skinny_plan(int M, int N, int K, bool ln, int *U, int *S) {
@@ -328,7 +364,7 @@ bool skinny_plan(int M, int N, int K, bool ln, int *U, int *S) {
       if (units % u) continue;
       const int ctas = units / u * s;
       if (ctas > 160) continue;
-      if (skinny_smem(M, K, u, s) > 110 * 1024) continue;
+      if (skinny_smem(M, K, u, s, ln) > 110 * 1024) continue;
       if (!best_u) {
         best_u = u;
         best_s = s;
@@ -368,6 +404,7 @@ cudaError_t skinny_init() {
     status = cudaFuncSetAttribute(skinny_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 110 * 1024);
     if (status == cudaSuccess)
       status = cudaFuncSetAttribute(skinny_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (status == cudaSuccess) status = prefer_max_shared(reinterpret_cast<const void *>(skinny_kernel));
   });
   return status;
 }
@@ -380,7 +417,7 @@ cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pd
   if (!p.ln_x && (!p.x || p.ld_x % 8 || (reinterpret_cast<uintptr_t>(p.x) & 15))) return cudaErrorInvalidValue;
   const CUtensorMap *tm = skinny_tmap(W, p.N, p.K, p.K / p.S / 64);
   if (!tm) return cudaErrorInvalidValue;
-  const size_t smem = skinny_smem(p.M, p.K, p.U, p.S);
+  const size_t smem = skinny_smem(p.M, p.K, p.U, p.S, p.ln_x != nullptr);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.N / 8 / p.U, 1, p.S);
   cfg.blockDim = dim3(kSkThreads, 1, 1);

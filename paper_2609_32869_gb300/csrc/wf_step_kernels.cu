@@ -2,6 +2,8 @@
 // drafter; token + learned position for the target), LayerNorm, the
 // cross-tile reduction of the output head, the per-sequence accept/rollback
 // rule (Sec. 3.1, App. A.1, A.4) and per-slot state bookkeeping.
+#include <mutex>
+
 #include "wf_device.cuh"
 #include "wf_internal.h"
 
@@ -541,6 +543,20 @@ __global__ void compact_kernel(const int32_t *done, int max_batch, int32_t *acti
       if (!done[s]) active[c++] = s;
     *n_active = c;
   }
+}
+
+cudaError_t step_kernels_init() {
+  static cudaError_t status = cudaErrorNotReady;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    const void *fns[] = {reinterpret_cast<const void *>(embed_kernel), reinterpret_cast<const void *>(layernorm_kernel),
+                         reinterpret_cast<const void *>(head_reduce_kernel), reinterpret_cast<const void *>(accept_kernel),
+                         reinterpret_cast<const void *>(state_kernel), reinterpret_cast<const void *>(compact_kernel)};
+    status = cudaSuccess;
+    for (const void *f : fns)
+      if (status == cudaSuccess) status = prefer_max_shared(f);
+  });
+  return status;
 }
 
 cudaError_t launch_compact(const int32_t *done, int max_batch, int32_t *active,
