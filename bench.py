@@ -268,8 +268,15 @@ def measure_greedy(args, wl_name, dev, host_ws, rank, world, steps, warmup, e2e=
     sess = Session(cfg, dev, max_batch=Bn, max_ctx=cfg.max_pos)
     if args.persist:
         B.wf_set_option(sess.h, B.WF_OPT_PERSIST, 1)
+    proj_path = "tcgen05"
     if args.no_skinny:
         B.wf_set_option(sess.h, B.WF_OPT_SKINNY, 0)
+    else:
+        try:
+            B.wf_set_option(sess.h, B.WF_OPT_SKINNY, 1)
+            proj_path = "skinny"
+        except B.WfError:
+            pass
     slots = np.arange(Bn, dtype=np.int32)
     stream = sess.stream
 
@@ -413,7 +420,7 @@ def measure_greedy(args, wl_name, dev, host_ws, rank, world, steps, warmup, e2e=
                 prof=prof, n_prof=n_prof, clocks=clocks, consistent=consistent, err=err,
                 launches=launches, wbytes=wbytes, kvbytes=float(np.mean(pl["kv"][warmup:])),
                 ctx=(min(pl["ctx"][warmup:]), float(np.mean(pl["ctx"][warmup:])), max(pl["ctx"][warmup:])),
-                budgets=budgets, acc=acc, enc=enc, prompt=prompt)
+                budgets=budgets, acc=acc, enc=enc, prompt=prompt, proj_path=proj_path)
 
 
 def _step_roofline(m, step_ms, hbm_peak, peak_src):
@@ -444,7 +451,8 @@ def run_ours(args, rank, world):
     fam = max(("gemm", "head", "attn_cross", "attn_self", "persist"), key=lambda f: prof[f]["ms"])
     roof_fam = "persist" if args.persist else "gemm"
     kernel = ("persist_kernel (every block of a pass in one launch; bytes = weights and acoustic K/V)"
-              if args.persist else "gemm_tc_kernel (tcgen05 projections)")
+              if args.persist else ("skinny_kernel (single-sequence projections)" if m["proj_path"] == "skinny"
+                                    else "gemm_tc_kernel (tcgen05 projections)"))
     Bn, Kc = m["batch"], cfg.block_k
     result = {
         "metric": METRIC,
@@ -463,6 +471,7 @@ def run_ours(args, rank, world):
         "config": {"workload": args.workload, "description": wl["text"], "batch": Bn,
                    "block": Kc + 1, "parallelism": f"replicas x{world}",
                    "path": "persistent passes" if args.persist else "launch by launch",
+                   "projections": m["proj_path"],
                    "l2": "inputs larger than L2 (every step streams "
                          f"{(m['wbytes'] + m['kvbytes']) / 1e9:.2f} GB of weights and K/V > 129 MB L2)"},
         "step_us": step_ms * 1e3,

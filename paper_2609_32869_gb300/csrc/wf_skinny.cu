@@ -36,6 +36,9 @@ namespace {
 
 constexpr int kSkThreads = 256;
 constexpr int kSkWarps = kSkThreads / 32;
+// Shared memory a CTA may plan for: two CTAs (of this kernel and the next)
+// fit on one SM's 228 KB with the per-CTA reserve.
+constexpr int kSkSmemBudget = 113 * 1024;
 
 __device__ __forceinline__ void tma_load_3d(void *smem_dst, const CUtensorMap *m, int32_t x, int32_t y,
                                             int32_t z, uint64_t *bar) {
@@ -353,7 +356,7 @@ bool skinny_plan(int M, int N, int K, bool ln, int *U, int *S) {
   if (M < 1 || M > kSkMaxRows || N % 8 || K % 128) return false;
   const int units = N / 8;
   // the fewest CTAs' worth of units that keeps the grid within about one CTA
-  // per SM (160 for 1280 rows of 8) and a CTA within 110 KB of shared memory
+  // per SM (160 for 1280 rows of 8) and a CTA within 113 KB of shared memory
   // (two kernels' CTAs share an SM, so the next one's slab streams in while
   // this one runs); whole K per CTA unless that does not fit, then K split
   // over a cluster of S CTAs
@@ -364,7 +367,7 @@ bool skinny_plan(int M, int N, int K, bool ln, int *U, int *S) {
       if (units % u) continue;
       const int ctas = units / u * s;
       if (ctas > 160) continue;
-      if (skinny_smem(M, K, u, s, ln) > 110 * 1024) continue;
+      if (skinny_smem(M, K, u, s, ln) > kSkSmemBudget) continue;
       if (!best_u) {
         best_u = u;
         best_s = s;
@@ -401,7 +404,7 @@ cudaError_t skinny_init() {
   static cudaError_t status = cudaErrorNotReady;
   static std::once_flag once;
   std::call_once(once, [] {
-    status = cudaFuncSetAttribute(skinny_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 110 * 1024);
+    status = cudaFuncSetAttribute(skinny_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSkSmemBudget);
     if (status == cudaSuccess)
       status = cudaFuncSetAttribute(skinny_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (status == cudaSuccess) status = prefer_max_shared(reinterpret_cast<const void *>(skinny_kernel));
