@@ -78,12 +78,13 @@ __device__ __forceinline__ uint32_t a_off(int M, int r, int k) {
 
 }  // namespace
 
+template <int U>
 __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_constant__ CUtensorMap tmW,
                                                                const SkinnyParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   uint8_t *smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
-  const int M = p.M, U = p.U, S = p.S;
+  const int M = p.M, S = p.S;
   const int Ks = p.K / S;  // K range of this CTA
   const int kb = Ks / 64;  // 64-wide k-blocks
   const SkLayout L(M, Ks, U, p.ln_x ? p.K : 0);
@@ -127,6 +128,22 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   }
   pdl_launch_dependents();
   pdl_wait();
+
+  // ---------------- the residual values this thread will update (loaded with
+  // the operand, so the epilogue only stores)
+  constexpr int kEpi = (U * kSkMaxRows * 8 + kSkThreads - 1) / kSkThreads;
+  const int n_out = U * M * 8;
+  float old[kEpi];
+#pragma unroll
+  for (int i = 0; i < kEpi; ++i) {
+    old[i] = 0.f;
+    const int e = tid + i * kSkThreads;
+    if (p.epi == EPI_RESID && e < n_out && (S == 1 || e % S == split)) {
+      const int u = e / (M * 8), rem = e - u * M * 8, t = rem >> 3, j = rem & 7;
+      const int n = n_base + u * 8 + j;
+      if (n < p.N) old[i] = __ldcg(p.resid + static_cast<size_t>(t) * p.ld_resid + n);
+    }
+  }
 
   // ---------------- token operand
   if (p.ln_x) {
@@ -210,58 +227,48 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   }
   __syncthreads();
 
-  // ---------------- MMAs: warp w takes k-steps [w * ksw, (w + 1) * ksw) of every unit
+  // ---------------- MMAs: warp w takes the k-blocks [w kbc / 8, (w + 1) kbc / 8) of
+  // every unit; within a k-block the k-steps alternate between two accumulators
+  // (shorter dependency chains), added in a fixed order at the end
   const bool landed = mbar_wait(bar, 0, p.err, p.spin);
   if (!landed) *s_flag = 1;
-  const int ksteps = Ks / 16, ksw = ksteps / kSkWarps;
-  float acc[8][4];  // per unit (U <= 8): the 16 x 8 tile's fragment
+  float acc[U][2][4];
 #pragma unroll
-  for (int u = 0; u < 8; ++u) acc[u][0] = acc[u][1] = acc[u][2] = acc[u][3] = 0.f;
+  for (int u = 0; u < U; ++u)
+#pragma unroll
+    for (int h = 0; h < 2; ++h) acc[u][h][0] = acc[u][h][1] = acc[u][h][2] = acc[u][h][3] = 0.f;
   if (landed) {
-    const uint32_t a_base = smem_u32(sA), w_base = smem_u32(sW), z_addr = smem_u32(sZero);
-    // A rows for ldmatrix.x4: lanes 0-7 rows 0-7 (k 0-7), 8-15 rows 8-15 (k 0-7),
-    // 16-23 rows 0-7 (k 8-15), 24-31 rows 8-15 (k 8-15); rows >= M read zeros
-    const int ar = (lane & 7) + ((lane >> 3) & 1) * 8, ak = (lane >> 4) * 8;
-    // B for ldmatrix.x4 over two k-steps: lane group g = lane >> 3 -> k offset 8 g
-    const int br = lane & 7, bk = (lane >> 3) * 8;
-    const int s_end = (warp + 1) * ksw;
-    int s = warp * ksw;
-    for (; s + 1 < s_end; s += 2) {  // two k-steps per B load
-      uint32_t a0[4], a1[4];
-      {
-        const int k = s * 16 + ak;
-        const uint32_t ad0 = ar < M ? a_base + a_off(M, ar, k) : z_addr;
-        const uint32_t ad1 = ar < M ? a_base + a_off(M, ar, k + 16) : z_addr;
-        ldsm_x4(ad0, a0[0], a0[1], a0[2], a0[3]);
-        ldsm_x4(ad1, a1[0], a1[1], a1[2], a1[3]);
-      }
+    const uint32_t w_base = smem_u32(sW);
+    // A (ldmatrix.x4 per k-step): lanes 0-7 rows 0-7 and 16-23 rows 0-7 (second
+    // 8 features), 8-15 and 24-31 rows 8-15; rows >= M read 16 zero bytes
+    const int ar = (lane & 7) + ((lane >> 3) & 1) * 8, c0 = lane >> 4;
+    const bool real = ar < M;
+    const uint32_t a_row = real ? smem_u32(sA) + ar * 128 : smem_u32(sZero);
+    const uint32_t a_kb = real ? M * 128 : 0;
+    uint32_t offA[4];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        if (u < U) {
-          const int k = s * 16 + bk;  // 32 consecutive k over the four matrices
-          const uint32_t wd = w_base + static_cast<uint32_t>(u * unit_bytes + (k >> 6) * 1024 + br * 128 +
-                                                             ((((k >> 3) & 7) ^ br) << 4));
-          uint32_t b0, b1, b2, b3;
-          ldsm_x4(wd, b0, b1, b2, b3);
-          mma_bf16(acc[u], a0[0], a0[1], a0[2], a0[3], b0, b1);
-          mma_bf16(acc[u], a1[0], a1[1], a1[2], a1[3], b2, b3);
-        }
-      }
-    }
-    if (s < s_end) {  // an odd last k-step
-      uint32_t a0[4];
-      const int k = s * 16 + ak;
-      ldsm_x4(ar < M ? a_base + a_off(M, ar, k) : z_addr, a0[0], a0[1], a0[2], a0[3]);
+    for (int j = 0; j < 4; ++j) offA[j] = real ? (((2 * j + c0) ^ (ar & 7)) << 4) : 0u;
+    // B (ldmatrix.x4 per pair of k-steps): lane group g reads 16-byte chunk g
+    // (first pair) or g + 4 (second pair) of weight row lane & 7
+    const int br = lane & 7, bg = lane >> 3;
+    const uint32_t offB0 = br * 128 + (((bg) ^ br) << 4), offB1 = br * 128 + (((bg + 4) ^ br) << 4);
+    const int kbc = kb;
+    const int kb_lo = warp * kbc / kSkWarps, kb_hi = (warp + 1) * kbc / kSkWarps;
+    for (int q = kb_lo; q < kb_hi; ++q) {
+      uint32_t a[4][4];
+      const uint32_t aq = a_row + q * a_kb;
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        if (u < U) {
-          const int kk = s * 16 + (bk & 8);  // lanes 16-31 repeat lanes 0-15's addresses
-          const uint32_t wd = w_base + static_cast<uint32_t>(u * unit_bytes + (kk >> 6) * 1024 + br * 128 +
-                                                             ((((kk >> 3) & 7) ^ br) << 4));
-          uint32_t b0, b1, b2, b3;
-          ldsm_x4(wd, b0, b1, b2, b3);
-          mma_bf16(acc[u], a0[0], a0[1], a0[2], a0[3], b0, b1);
-        }
+      for (int j = 0; j < 4; ++j) ldsm_x4(aq + offA[j], a[j][0], a[j][1], a[j][2], a[j][3]);
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const uint32_t wq = w_base + u * unit_bytes + q * 1024;
+        uint32_t b0, b1, b2, b3, b4, b5, b6, b7;
+        ldsm_x4(wq + offB0, b0, b1, b2, b3);
+        ldsm_x4(wq + offB1, b4, b5, b6, b7);
+        mma_bf16(acc[u][0], a[0][0], a[0][1], a[0][2], a[0][3], b0, b1);
+        mma_bf16(acc[u][1], a[1][0], a[1][1], a[1][2], a[1][3], b2, b3);
+        mma_bf16(acc[u][0], a[2][0], a[2][1], a[2][2], a[2][3], b4, b5);
+        mma_bf16(acc[u][1], a[3][0], a[3][1], a[3][2], a[3][3], b6, b7);
       }
     }
   }
@@ -270,14 +277,12 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   {
     const int g = lane >> 2, c4 = lane & 3;
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      if (u < U) {
-        float *pw = sPart + (warp * U + u) * 128;
-        pw[g * 8 + 2 * c4] = acc[u][0];
-        pw[g * 8 + 2 * c4 + 1] = acc[u][1];
-        pw[(g + 8) * 8 + 2 * c4] = acc[u][2];
-        pw[(g + 8) * 8 + 2 * c4 + 1] = acc[u][3];
-      }
+    for (int u = 0; u < U; ++u) {
+      float *pw = sPart + (warp * U + u) * 128;
+      pw[g * 8 + 2 * c4] = acc[u][0][0] + acc[u][1][0];
+      pw[g * 8 + 2 * c4 + 1] = acc[u][0][1] + acc[u][1][1];
+      pw[(g + 8) * 8 + 2 * c4] = acc[u][0][2] + acc[u][1][2];
+      pw[(g + 8) * 8 + 2 * c4 + 1] = acc[u][0][3] + acc[u][1][3];
     }
   }
   __syncthreads();
@@ -294,8 +299,10 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   const bool ok = landed;
   if (S > 1) cluster_sync();
   else __syncthreads();
-  for (int e = tid; e < U * M * 8; e += kSkThreads) {
-    if (S > 1 && (e % S) != split) continue;
+#pragma unroll
+  for (int i = 0; i < kEpi; ++i) {
+    const int e = tid + i * kSkThreads;
+    if (e >= n_out || (S > 1 && (e % S) != split)) continue;
     const int u = e / (M * 8), rem = e - u * M * 8, t = rem >> 3, j = rem & 7;
     const int idx = u * 128 + t * 8 + j;
     float v;
@@ -316,9 +323,8 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
     } else if (p.epi == EPI_GELU) {
       p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(gelu_erf(v));
     } else if (p.epi == EPI_RESID) {
-      float *xr = p.resid + static_cast<size_t>(t) * p.ld_resid + n;
-      const float nr = __ldcg(xr) + v;
-      *xr = nr;
+      const float nr = old[i] + v;
+      p.resid[static_cast<size_t>(t) * p.ld_resid + n] = nr;
       if (p.tap0) p.tap0[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
       if (p.tap1) p.tap1[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
     } else if (p.epi == EPI_KV) {
@@ -400,14 +406,28 @@ static const CUtensorMap *skinny_tmap(const void *W, int N, int K, int kblocks) 
   return m;
 }
 
+template <int U>
+static cudaError_t skinny_attrs() {
+  const void *f = reinterpret_cast<const void *>(skinny_kernel<U>);
+  cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, kSkSmemBudget);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(f, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e == cudaSuccess) e = prefer_max_shared(f);
+  return e;
+}
+
 cudaError_t skinny_init() {
   static cudaError_t status = cudaErrorNotReady;
   static std::once_flag once;
   std::call_once(once, [] {
-    status = cudaFuncSetAttribute(skinny_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSkSmemBudget);
-    if (status == cudaSuccess)
-      status = cudaFuncSetAttribute(skinny_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    if (status == cudaSuccess) status = prefer_max_shared(reinterpret_cast<const void *>(skinny_kernel));
+    cudaError_t e = skinny_attrs<1>();
+    if (e == cudaSuccess) e = skinny_attrs<2>();
+    if (e == cudaSuccess) e = skinny_attrs<3>();
+    if (e == cudaSuccess) e = skinny_attrs<4>();
+    if (e == cudaSuccess) e = skinny_attrs<5>();
+    if (e == cudaSuccess) e = skinny_attrs<6>();
+    if (e == cudaSuccess) e = skinny_attrs<7>();
+    if (e == cudaSuccess) e = skinny_attrs<8>();
+    status = e;
   });
   return status;
 }
@@ -442,7 +462,17 @@ cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pd
   }
   cfg.attrs = attr;
   cfg.numAttrs = na;
-  return cudaLaunchKernelEx(&cfg, skinny_kernel, *tm, p);
+  switch (p.U) {
+    case 1: return cudaLaunchKernelEx(&cfg, skinny_kernel<1>, *tm, p);
+    case 2: return cudaLaunchKernelEx(&cfg, skinny_kernel<2>, *tm, p);
+    case 3: return cudaLaunchKernelEx(&cfg, skinny_kernel<3>, *tm, p);
+    case 4: return cudaLaunchKernelEx(&cfg, skinny_kernel<4>, *tm, p);
+    case 5: return cudaLaunchKernelEx(&cfg, skinny_kernel<5>, *tm, p);
+    case 6: return cudaLaunchKernelEx(&cfg, skinny_kernel<6>, *tm, p);
+    case 7: return cudaLaunchKernelEx(&cfg, skinny_kernel<7>, *tm, p);
+    case 8: return cudaLaunchKernelEx(&cfg, skinny_kernel<8>, *tm, p);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 }  // namespace wf
