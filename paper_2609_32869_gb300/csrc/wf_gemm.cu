@@ -708,6 +708,20 @@ bool tmap_bf16_units(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t co
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool tmap_bf16_rows(CUtensorMap *m, const void *ptr, uint32_t rows, uint64_t cols, uint64_t ld, uint32_t kblocks) {
+  auto fn = encode_fn();
+  if (!fn || (reinterpret_cast<uintptr_t>(ptr) & 15) || cols % 64 || (ld * 2) % 16 || ld < cols || rows == 0 ||
+      rows > 256 || kblocks == 0 || kblocks > 256 || kblocks > cols / 64)
+    return false;
+  cuuint64_t gdim[3] = {64, rows, cols / 64};
+  cuuint64_t gstride[2] = {ld * 2, 128};
+  cuuint32_t box[3] = {64, rows, kblocks};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), gdim, gstride, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 void gemm_token_tiling(int M, int *BT, int *n_tt) {
   const int nt = (M + kMaxBT - 1) / kMaxBT;
   const int per = (M + nt - 1) / nt;

@@ -95,6 +95,9 @@ struct GemmParams {
 const CUtensorMap *tmap_bf16_2d(const void *ptr, uint64_t rows, uint64_t cols, uint32_t box_rows);
 // A whole 8-row unit of a [rows][cols] matrix per copy: box {64, 8, kblocks}.
 bool tmap_bf16_units(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint32_t kblocks);
+// All `rows` rows of a [rows][cols] matrix (row stride ld elements) over
+// kblocks 64-column blocks per copy: box {64, rows, kblocks}.
+bool tmap_bf16_rows(CUtensorMap *m, const void *ptr, uint32_t rows, uint64_t cols, uint64_t ld, uint32_t kblocks);
 
 // Token tile for M rows: a multiple of 16, at most 128.
 void gemm_token_tiling(int M, int *BT, int *n_tt);
@@ -121,7 +124,7 @@ bool gemm_ln_fits(int M, int N, int K, int epi);
 constexpr int kSkMaxRows = 16;
 struct SkinnyParams {
   int M, N, K;
-  int U, S;  // set by launch_skinny
+  int U, S, C;  // set by launch_skinny (C: CTAs of a cluster sharing a LayerNorm operand)
   int epi;
   const bf16 *x;
   int ld_x;

@@ -10,9 +10,11 @@
 //    with TMA before griddepcontrol.wait, one 3-D tensor copy per unit that
 //    lands 128-byte swizzled ([k-block][8 rows][64 features]); the slab
 //    streams while the previous kernels run;
-//  - after the wait the token operand is built in shared memory: LN(x) from
-//    the fp32 residual rows (each warp computes its rows' mean and variance
-//    itself, so no statistics travel between kernels), or plain bf16 rows;
+//  - after the wait the token operand lands in shared memory: bf16 rows by
+//    one TMA copy, or LN(x) from the fp32 residual rows, where the CTAs of a
+//    cluster split the rows (each computes its rows' mean and variance, so no
+//    statistics travel between kernels) and write the normalised bf16 rows
+//    into every CTA of the cluster over distributed shared memory;
 //  - all eight warps issue mma.sync m16n8k16 at once (tokens on the 16-row
 //    side, weight rows on the 8-column side), each over its own slice of K;
 //    the slices are summed in warp order, then (S > 1) the S CTAs' sums in
@@ -58,7 +60,7 @@ struct SkLayout {
     const int kb = Ks / 64;
     unit_bytes = kb * 1024;
     w_bytes = U * unit_bytes;
-    a_off = w_bytes;
+    a_off = w_bytes;  // 1024-aligned: the operand's TMA copy swizzles by address
     a_bytes = kb * M * 128;
     sum_off = (a_off + a_bytes + 15) & ~15;
     bias_off = sum_off + U * 128 * 4;
@@ -70,24 +72,36 @@ struct SkLayout {
   }
 };
 
-// byte offset of element k of token row r in the operand tile: [k-block][M rows][128 B],
-// 16-byte chunk j of a row stored at chunk j ^ (r & 7) (the TMA's 128-byte swizzle)
+// Byte offset of element k of token row r in the operand tile [k-block][M
+// rows][128 B]: 128-byte line l = kb * M + r holds 16-byte chunk j at
+// position j ^ (l & 7), the pattern a 128-byte-swizzled TMA copy writes into
+// a 1024-aligned destination.
 __device__ __forceinline__ uint32_t a_off(int M, int r, int k) {
-  return static_cast<uint32_t>(((k >> 6) * M + r) * 128 + ((((k >> 3) & 7) ^ (r & 7)) << 4) + (k & 7) * 2);
+  const int line = (k >> 6) * M + r;
+  return static_cast<uint32_t>(line * 128 + ((((k >> 3) & 7) ^ (line & 7)) << 4) + (k & 7) * 2);
+}
+
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void dsmem_st_u32x2(uint32_t cluster_addr, uint32_t a, uint32_t b) {
+  asm volatile("st.shared::cluster.v2.b32 [%0], {%1, %2};" ::"r"(cluster_addr), "r"(a), "r"(b) : "memory");
 }
 
 }  // namespace
 
 template <int U>
 __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_constant__ CUtensorMap tmW,
+                                                               const __grid_constant__ CUtensorMap tmX,
                                                                const SkinnyParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   uint8_t *smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
-  const int M = p.M, S = p.S;
+  const int M = p.M, S = p.S, C = p.C;
+  const bool ln = p.ln_x != nullptr;
   const int Ks = p.K / S;  // K range of this CTA
   const int kb = Ks / 64;  // 64-wide k-blocks
-  const SkLayout L(M, Ks, U, p.ln_x ? p.K : 0);
+  const SkLayout L(M, Ks, U, ln ? p.K : 0);
   const int unit_bytes = L.unit_bytes;             // one unit: [kb][8 rows][128 B]
   uint8_t *sW = smem;
   uint8_t *sA = smem + L.a_off;                    // [kb][M][128 B]
@@ -96,7 +110,7 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   float *sBias = reinterpret_cast<float *>(smem + L.bias_off);  // [U * 8]
   bf16 *sG = reinterpret_cast<bf16 *>(smem + L.gb_off);         // [K] LayerNorm gain, then [K] bias
   bf16 *sB = sG + p.K;
-  uint64_t *bar = reinterpret_cast<uint64_t *>(smem + L.bar_off);
+  uint64_t *bar = reinterpret_cast<uint64_t *>(smem + L.bar_off);  // [0] weights, [1] operand
   uint4 *sZero = reinterpret_cast<uint4 *>(smem + L.zero_off);
   int *s_flag = reinterpret_cast<int *>(smem + L.flag_off);
 
@@ -104,35 +118,63 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   const int cta = blockIdx.x, split = blockIdx.z;
   const int unit0 = cta * U;  // first 8-row unit of this CTA
   const int n_base = unit0 * 8;
+  const uint32_t crank = C > 1 ? cluster_ctarank() : 0u;  // cluster (C, 1, 1) when C > 1
 
+  if (C > 1) cluster_arrive_relaxed();  // this CTA has started (peers write into it later)
   if (tid == 0) {
     *s_flag = 0;
     tma_prefetch_desc(&tmW);
-    mbar_init(bar, 1);
+    if (!ln) tma_prefetch_desc(&tmX);
+    mbar_init(&bar[0], 1);
+    mbar_init(&bar[1], 1);
     fence_barrier_init();
     *sZero = make_uint4(0u, 0u, 0u, 0u);
     // the whole weight slab: one copy per unit, before the dependency wait
-    mbar_arrive_expect_tx(bar, static_cast<uint32_t>(U * unit_bytes));
+    mbar_arrive_expect_tx(&bar[0], static_cast<uint32_t>(U * unit_bytes));
     for (int u = 0; u < U; ++u)
-      tma_load_3d(sW + static_cast<size_t>(u) * unit_bytes, &tmW, 0, (unit0 + u) * 8, split * kb, bar);
+      tma_load_3d(sW + static_cast<size_t>(u) * unit_bytes, &tmW, 0, (unit0 + u) * 8, split * kb, &bar[0]);
   }
   for (int i = tid; i < U * 8; i += kSkThreads) {
     const int n = n_base + i;
     sBias[i] = (p.bias && n < p.N) ? bf2f(p.bias[n]) : 0.f;
   }
-  if (p.ln_x) {  // parameters, not activations: staged before the wait
+  if (ln) {  // parameters, not activations: staged before the wait
     for (int i = tid; i < p.K / 8; i += kSkThreads) {
       reinterpret_cast<uint4 *>(sG)[i] = reinterpret_cast<const uint4 *>(p.ln_g)[i];
       reinterpret_cast<uint4 *>(sB)[i] = reinterpret_cast<const uint4 *>(p.ln_b)[i];
     }
   }
+  // epilogue outputs of this thread: element e = tid + i * threads of the
+  // U x M x 8 tile; the cache slot and position of a key/value row are fixed
+  // for the step, so they are read before the wait
+  constexpr int kEpi = (U * kSkMaxRows * 8 + kSkThreads - 1) / kSkThreads;
+  const int n_out = U * M * 8;
+  int kv_dst[kEpi];  // EPI_KV: cache row index (slot * heads + head) * ctx + position, or -1
+#pragma unroll
+  for (int i = 0; i < kEpi; ++i) {
+    kv_dst[i] = -1;
+    const int e = tid + i * kSkThreads;
+    if (p.epi == EPI_KV && e < n_out) {
+      const int u = e / (M * 8), rem = e - u * M * 8, t = rem >> 3, j = rem & 7;
+      const int n = n_base + u * 8 + j;
+      if (n >= p.q_cols && n < p.N) {
+        const int c = n - p.q_cols, hd = c % p.d_model;
+        const int ii = t / p.rows_per_seq, jr = t - ii * p.rows_per_seq;
+        const int slot = p.seq_slot[ii];
+        const int pos = (p.pos_base ? p.pos_base[slot] : 0) + jr;
+        kv_dst[i] = pos < p.ctx ? (slot * p.n_heads + (hd >> 6)) * p.ctx + pos : -2;
+      }
+    }
+  }
   pdl_launch_dependents();
   pdl_wait();
 
-  // ---------------- the residual values this thread will update (loaded with
-  // the operand, so the epilogue only stores)
-  constexpr int kEpi = (U * kSkMaxRows * 8 + kSkThreads - 1) / kSkThreads;
-  const int n_out = U * M * 8;
+  // ---------------- operand: bf16 rows by one TMA copy (issued first), the
+  // residual values this thread will update, or LN(x) shared by the cluster
+  if (!ln && tid == 0) {
+    mbar_arrive_expect_tx(&bar[1], static_cast<uint32_t>(L.a_bytes));
+    tma_load_3d(sA, &tmX, 0, 0, split * kb, &bar[1]);
+  }
   float old[kEpi];
 #pragma unroll
   for (int i = 0; i < kEpi; ++i) {
@@ -144,38 +186,33 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
       if (n < p.N) old[i] = __ldcg(p.resid + static_cast<size_t>(t) * p.ld_resid + n);
     }
   }
-
-  // ---------------- token operand
-  if (p.ln_x) {
-    // LN(x) from the fp32 rows: warp w normalises rows w and w + 8 together
-    // (every load of both rows in flight before the first sum); lane l holds
-    // features 4l + 128 i
+  bool op_ok = true;
+  if (ln) {
+    // rows r = crank + C q of the cluster's operand belong to this CTA; warp w
+    // normalises its rows q = w, w + 8 (lane l holds features 4l + 128 i) and
+    // writes them into every CTA of the cluster
     constexpr int kMaxI = 12;  // K <= 1536
     const int nI = p.K / 128;
-    const int r0 = warp, r1 = warp + kSkWarps;
-    float4 v[2][kMaxI];
-#pragma unroll
+    if (C > 1) cluster_wait();  // every CTA of the cluster has started
+    const uint32_t a_loc = smem_u32(sA);
     for (int h = 0; h < 2; ++h) {
-      const int r = h ? r1 : r0;
-      const float *xr = p.ln_x + static_cast<size_t>(r < M ? r : 0) * p.ln_ld;
+      const int r = static_cast<int>(crank) + C * (warp + kSkWarps * h);
+      if (r >= M) break;
+      const float *xr = p.ln_x + static_cast<size_t>(r) * p.ln_ld;
+      float4 v[kMaxI];
 #pragma unroll
       for (int i = 0; i < kMaxI; ++i)
-        if (i < nI && r < M) v[h][i] = __ldcg(reinterpret_cast<const float4 *>(xr + 4 * lane + 128 * i));
-    }
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int r = h ? r1 : r0;
-      if (r >= M) continue;
+        if (i < nI) v[i] = __ldcg(reinterpret_cast<const float4 *>(xr + 4 * lane + 128 * i));
       float sum = 0.f;
 #pragma unroll
       for (int i = 0; i < kMaxI; ++i)
-        if (i < nI) sum += (v[h][i].x + v[h][i].y) + (v[h][i].z + v[h][i].w);
+        if (i < nI) sum += (v[i].x + v[i].y) + (v[i].z + v[i].w);
       const float mean = warp_sum(sum) / static_cast<float>(p.K);
       float q = 0.f;
 #pragma unroll
       for (int i = 0; i < kMaxI; ++i) {
         if (i < nI) {
-          const float a = v[h][i].x - mean, b = v[h][i].y - mean, c = v[h][i].z - mean, d = v[h][i].w - mean;
+          const float a = v[i].x - mean, b = v[i].y - mean, c = v[i].z - mean, d = v[i].w - mean;
           q += (a * a + b * b) + (c * c + d * d);
         }
       }
@@ -188,49 +225,31 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
           const uint2 bb = *reinterpret_cast<const uint2 *>(sB + k);
           const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gg);
           const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&bb);
-          const __nv_bfloat162 o0 = __floats2bfloat162_rn(ln_apply(v[h][i].x, ms, __low2float(g2[0]), __low2float(b2[0])),
-                                                          ln_apply(v[h][i].y, ms, __high2float(g2[0]), __high2float(b2[0])));
-          const __nv_bfloat162 o1 = __floats2bfloat162_rn(ln_apply(v[h][i].z, ms, __low2float(g2[1]), __low2float(b2[1])),
-                                                          ln_apply(v[h][i].w, ms, __high2float(g2[1]), __high2float(b2[1])));
-          uint2 o;
-          o.x = *reinterpret_cast<const uint32_t *>(&o0);
-          o.y = *reinterpret_cast<const uint32_t *>(&o1);
-          *reinterpret_cast<uint2 *>(sA + a_off(M, r, k)) = o;
+          const __nv_bfloat162 o0 = __floats2bfloat162_rn(ln_apply(v[i].x, ms, __low2float(g2[0]), __low2float(b2[0])),
+                                                          ln_apply(v[i].y, ms, __high2float(g2[0]), __high2float(b2[0])));
+          const __nv_bfloat162 o1 = __floats2bfloat162_rn(ln_apply(v[i].z, ms, __low2float(g2[1]), __low2float(b2[1])),
+                                                          ln_apply(v[i].w, ms, __high2float(g2[1]), __high2float(b2[1])));
+          const uint32_t w0 = *reinterpret_cast<const uint32_t *>(&o0), w1 = *reinterpret_cast<const uint32_t *>(&o1);
+          const uint32_t off = a_off(M, r, k);
+          if (C > 1) {
+            for (int d = 0; d < C; ++d) dsmem_st_u32x2(dsmem_map(a_loc + off, static_cast<uint32_t>(d)), w0, w1);
+          } else {
+            *reinterpret_cast<uint2 *>(sA + off) = make_uint2(w0, w1);
+          }
         }
       }
     }
+    if (C > 1) cluster_sync();  // every row has landed in every CTA
+    else __syncthreads();
   } else {
-    // bf16 rows [M][ld_x], columns [split * Ks, (split + 1) * Ks): up to eight
-    // 16-byte loads per thread in flight before their stores
-    const int cpr = Ks / 8, chunks = M * cpr;
-    const bf16 *x0 = p.x + static_cast<size_t>(split) * Ks;
-    constexpr int kU = 8;
-    for (int c0 = 0; c0 < chunks; c0 += kU * kSkThreads) {
-      uint4 v[kU];
-#pragma unroll
-      for (int u = 0; u < kU; ++u) {
-        const int c = c0 + u * kSkThreads + tid;
-        if (c < chunks) {
-          const int r = c / cpr, k = (c - r * cpr) * 8;
-          v[u] = __ldcg(reinterpret_cast<const uint4 *>(x0 + static_cast<size_t>(r) * p.ld_x + k));
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < kU; ++u) {
-        const int c = c0 + u * kSkThreads + tid;
-        if (c < chunks) {
-          const int r = c / cpr, k = (c - r * cpr) * 8;
-          *reinterpret_cast<uint4 *>(sA + a_off(M, r, k)) = v[u];
-        }
-      }
-    }
+    op_ok = mbar_wait(&bar[1], 0, p.err, p.spin);
+    if (!op_ok) *s_flag = 1;
   }
-  __syncthreads();
 
-  // ---------------- MMAs: warp w takes the k-blocks [w kbc / 8, (w + 1) kbc / 8) of
+  // ---------------- MMAs: warp w takes the k-blocks [w kb / 8, (w + 1) kb / 8) of
   // every unit; within a k-block the k-steps alternate between two accumulators
   // (shorter dependency chains), added in a fixed order at the end
-  const bool landed = mbar_wait(bar, 0, p.err, p.spin);
+  const bool landed = mbar_wait(&bar[0], 0, p.err, p.spin) && op_ok;
   if (!landed) *s_flag = 1;
   float acc[U][2][4];
 #pragma unroll
@@ -243,22 +262,19 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
     // 8 features), 8-15 and 24-31 rows 8-15; rows >= M read 16 zero bytes
     const int ar = (lane & 7) + ((lane >> 3) & 1) * 8, c0 = lane >> 4;
     const bool real = ar < M;
-    const uint32_t a_row = real ? smem_u32(sA) + ar * 128 : smem_u32(sZero);
-    const uint32_t a_kb = real ? M * 128 : 0;
-    uint32_t offA[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) offA[j] = real ? (((2 * j + c0) ^ (ar & 7)) << 4) : 0u;
+    const uint32_t a_base = smem_u32(sA), z_addr = smem_u32(sZero);
     // B (ldmatrix.x4 per pair of k-steps): lane group g reads 16-byte chunk g
     // (first pair) or g + 4 (second pair) of weight row lane & 7
     const int br = lane & 7, bg = lane >> 3;
     const uint32_t offB0 = br * 128 + (((bg) ^ br) << 4), offB1 = br * 128 + (((bg + 4) ^ br) << 4);
-    const int kbc = kb;
-    const int kb_lo = warp * kbc / kSkWarps, kb_hi = (warp + 1) * kbc / kSkWarps;
+    const int kb_lo = warp * kb / kSkWarps, kb_hi = (warp + 1) * kb / kSkWarps;
     for (int q = kb_lo; q < kb_hi; ++q) {
       uint32_t a[4][4];
-      const uint32_t aq = a_row + q * a_kb;
+      const int line = q * M + ar;
+      const uint32_t aq = a_base + line * 128, sw = line & 7;
 #pragma unroll
-      for (int j = 0; j < 4; ++j) ldsm_x4(aq + offA[j], a[j][0], a[j][1], a[j][2], a[j][3]);
+      for (int j = 0; j < 4; ++j)
+        ldsm_x4(real ? aq + (((2 * j + c0) ^ sw) << 4) : z_addr, a[j][0], a[j][1], a[j][2], a[j][3]);
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         const uint32_t wq = w_base + u * unit_bytes + q * 1024;
@@ -307,9 +323,15 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
     const int idx = u * 128 + t * 8 + j;
     float v;
     if (S > 1) {
-      v = 0.f;
+      float part[8];
       const uint32_t loc = smem_u32(sSum + idx);
-      for (int r = 0; r < S; ++r) v += dsmem_ld_f32(dsmem_map(loc, r));
+#pragma unroll
+      for (int r = 0; r < 8; ++r)  // every load in flight before the sum
+        part[r] = r < S ? dsmem_ld_f32(dsmem_map(loc, r)) : 0.f;
+      v = 0.f;
+#pragma unroll
+      for (int r = 0; r < 8; ++r)
+        if (r < S) v += part[r];
     } else {
       v = sSum[idx];
     }
@@ -330,25 +352,22 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
     } else if (p.epi == EPI_KV) {
       if (n < p.q_cols) {
         p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(v);
+      } else if (kv_dst[i] == -2) {
+        set_error(p.err, WF_DEV_ERR_CAPACITY);
       } else {
-        const int c = n - p.q_cols, which = c / p.d_model, hd = c - which * p.d_model;
-        const int i = t / p.rows_per_seq, jr = t - i * p.rows_per_seq;
-        const int slot = p.seq_slot[i];
-        const int pos = (p.pos_base ? p.pos_base[slot] : 0) + jr;
-        if (pos >= p.ctx) {
-          set_error(p.err, WF_DEV_ERR_CAPACITY);
-        } else {
-          bf16 *dst = which == 0 ? p.kc : p.vc;
-          dst[((static_cast<size_t>(slot) * p.n_heads + (hd >> 6)) * p.ctx + pos) * 64 + (hd & 63)] =
-              __float2bfloat16(v);
-        }
+        const int c = n - p.q_cols, which = c / p.d_model;
+        bf16 *dst = which == 0 ? p.kc : p.vc;
+        dst[static_cast<size_t>(kv_dst[i]) * 64 + ((c - which * p.d_model) & 63)] = __float2bfloat16(v);
       }
     }
   }
   if (S > 1) cluster_sync();  // peers may read this CTA's sums until here
-  // after a timeout the slab's copy may still be landing: wait for it (bounded)
+  // after a timeout a copy may still be landing: wait for it (bounded)
   __syncthreads();
-  if (tid == 0 && *s_flag) mbar_drain(bar, 0);
+  if (tid == 0 && *s_flag) {
+    mbar_drain(&bar[0], 0);
+    if (!ln) mbar_drain(&bar[1], 0);
+  }
 }
 
 // ------------------------------------------------------------------ host ----
@@ -432,6 +451,25 @@ cudaError_t skinny_init() {
   return status;
 }
 
+// Operand tensor maps: the M bf16 rows of X [M][K] (row stride ld) as
+// (64 columns, row, 64-column block), one copy of {64, M, kblocks} per CTA
+// landing as [k-block][M][128 B], 128-byte swizzled.
+static const CUtensorMap *skinny_xmap(const void *X, int M, int K, int ld, int kblocks) {
+  static std::mutex mu;
+  static std::map<std::tuple<uintptr_t, int, int, int, int>, CUtensorMap *> cache;
+  std::lock_guard<std::mutex> lock(mu);
+  const auto key = std::make_tuple(reinterpret_cast<uintptr_t>(X), M, K, ld, kblocks);
+  auto it = cache.find(key);
+  if (it != cache.end()) return it->second;
+  CUtensorMap *m = new CUtensorMap;
+  if (!tmap_bf16_rows(m, X, M, K, ld, kblocks)) {
+    delete m;
+    return nullptr;
+  }
+  cache.emplace(key, m);
+  return m;
+}
+
 cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pdl) {
   if (p.spin <= 0) p.spin = kSpinLimitCycles;
   if (!skinny_plan(p.M, p.N, p.K, p.ln_x != nullptr, &p.U, &p.S)) return cudaErrorInvalidValue;
@@ -440,6 +478,17 @@ cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pd
   if (!p.ln_x && (!p.x || p.ld_x % 8 || (reinterpret_cast<uintptr_t>(p.x) & 15))) return cudaErrorInvalidValue;
   const CUtensorMap *tm = skinny_tmap(W, p.N, p.K, p.K / p.S / 64);
   if (!tm) return cudaErrorInvalidValue;
+  const CUtensorMap *tx = p.ln_x ? tm : skinny_xmap(p.x, p.M, p.K, p.ld_x, p.K / p.S / 64);
+  if (!tx) return cudaErrorInvalidValue;
+  // LayerNorm operands: the CTAs of a cluster share the rows (at most 8)
+  const int gx = p.N / 8 / p.U;
+  p.C = 1;
+  if (p.ln_x && p.S == 1)
+    for (int c = 8; c >= 2; c >>= 1)
+      if (gx % c == 0) {
+        p.C = c;
+        break;
+      }
   const size_t smem = skinny_smem(p.M, p.K, p.U, p.S, p.ln_x != nullptr);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.N / 8 / p.U, 1, p.S);
@@ -448,9 +497,9 @@ cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pd
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   int na = 0;
-  if (p.S > 1) {
+  if (p.S > 1 || p.C > 1) {
     attr[na].id = cudaLaunchAttributeClusterDimension;
-    attr[na].val.clusterDim.x = 1;
+    attr[na].val.clusterDim.x = p.C;
     attr[na].val.clusterDim.y = 1;
     attr[na].val.clusterDim.z = p.S;
     ++na;
@@ -463,14 +512,14 @@ cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pd
   cfg.attrs = attr;
   cfg.numAttrs = na;
   switch (p.U) {
-    case 1: return cudaLaunchKernelEx(&cfg, skinny_kernel<1>, *tm, p);
-    case 2: return cudaLaunchKernelEx(&cfg, skinny_kernel<2>, *tm, p);
-    case 3: return cudaLaunchKernelEx(&cfg, skinny_kernel<3>, *tm, p);
-    case 4: return cudaLaunchKernelEx(&cfg, skinny_kernel<4>, *tm, p);
-    case 5: return cudaLaunchKernelEx(&cfg, skinny_kernel<5>, *tm, p);
-    case 6: return cudaLaunchKernelEx(&cfg, skinny_kernel<6>, *tm, p);
-    case 7: return cudaLaunchKernelEx(&cfg, skinny_kernel<7>, *tm, p);
-    case 8: return cudaLaunchKernelEx(&cfg, skinny_kernel<8>, *tm, p);
+    case 1: return cudaLaunchKernelEx(&cfg, skinny_kernel<1>, *tm, *tx, p);
+    case 2: return cudaLaunchKernelEx(&cfg, skinny_kernel<2>, *tm, *tx, p);
+    case 3: return cudaLaunchKernelEx(&cfg, skinny_kernel<3>, *tm, *tx, p);
+    case 4: return cudaLaunchKernelEx(&cfg, skinny_kernel<4>, *tm, *tx, p);
+    case 5: return cudaLaunchKernelEx(&cfg, skinny_kernel<5>, *tm, *tx, p);
+    case 6: return cudaLaunchKernelEx(&cfg, skinny_kernel<6>, *tm, *tx, p);
+    case 7: return cudaLaunchKernelEx(&cfg, skinny_kernel<7>, *tm, *tx, p);
+    case 8: return cudaLaunchKernelEx(&cfg, skinny_kernel<8>, *tm, *tx, p);
     default: return cudaErrorInvalidValue;
   }
 }
