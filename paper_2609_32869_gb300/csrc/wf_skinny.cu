@@ -84,8 +84,10 @@ __device__ __forceinline__ uint32_t a_off(int M, int r, int k) {
 __device__ __forceinline__ void cluster_arrive_relaxed() {
   asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
 }
-__device__ __forceinline__ void dsmem_st_u32x2(uint32_t cluster_addr, uint32_t a, uint32_t b) {
-  asm volatile("st.shared::cluster.v2.b32 [%0], {%1, %2};" ::"r"(cluster_addr), "r"(a), "r"(b) : "memory");
+__device__ __forceinline__ void dsmem_st_u32x4(uint32_t cluster_addr, uint4 v) {
+  asm volatile("st.shared::cluster.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(cluster_addr), "r"(v.x), "r"(v.y),
+               "r"(v.z), "r"(v.w)
+               : "memory");
 }
 
 }  // namespace
@@ -189,8 +191,8 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   bool op_ok = true;
   if (ln) {
     // rows r = crank + C q of the cluster's operand belong to this CTA; warp w
-    // normalises its rows q = w, w + 8 (lane l holds features 4l + 128 i) and
-    // writes them into every CTA of the cluster
+    // normalises its rows q = w, w + 8 (lane l holds features 4l + 128 i)
+    // into its own operand tile, then the CTA copies them to its peers
     constexpr int kMaxI = 12;  // K <= 1536
     const int nI = p.K / 128;
     if (C > 1) cluster_wait();  // every CTA of the cluster has started
@@ -229,13 +231,25 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
                                                           ln_apply(v[i].y, ms, __high2float(g2[0]), __high2float(b2[0])));
           const __nv_bfloat162 o1 = __floats2bfloat162_rn(ln_apply(v[i].z, ms, __low2float(g2[1]), __low2float(b2[1])),
                                                           ln_apply(v[i].w, ms, __high2float(g2[1]), __high2float(b2[1])));
-          const uint32_t w0 = *reinterpret_cast<const uint32_t *>(&o0), w1 = *reinterpret_cast<const uint32_t *>(&o1);
-          const uint32_t off = a_off(M, r, k);
-          if (C > 1) {
-            for (int d = 0; d < C; ++d) dsmem_st_u32x2(dsmem_map(a_loc + off, static_cast<uint32_t>(d)), w0, w1);
-          } else {
-            *reinterpret_cast<uint2 *>(sA + off) = make_uint2(w0, w1);
-          }
+          *reinterpret_cast<uint2 *>(sA + a_off(M, r, k)) =
+              make_uint2(*reinterpret_cast<const uint32_t *>(&o0), *reinterpret_cast<const uint32_t *>(&o1));
+        }
+      }
+    }
+    if (C > 1) {
+      // fan this CTA's rows out to the other CTAs of the cluster: warp w
+      // copies them to rank (crank + 1 + w) % C, 16 bytes per lane and store
+      __syncthreads();
+      const int my_rows = (M - static_cast<int>(crank) + C - 1) / C;  // rows crank, crank + C, ...
+      const int lines = my_rows * kb;                                  // 128-byte lines to copy
+      for (int w = warp; w < C - 1; w += kSkWarps) {
+        const uint32_t dst = (crank + 1 + w) % C;
+        for (int c = lane; c < lines * 8; c += 32) {
+          const int li = c >> 3, ch = c & 7;
+          const int rr = static_cast<int>(crank) + C * (li / kb), q = li % kb;
+          const uint32_t off = static_cast<uint32_t>((q * M + rr) * 128 + ch * 16);
+          const uint4 v4 = *reinterpret_cast<const uint4 *>(sA + off);
+          dsmem_st_u32x4(dsmem_map(a_loc + off, dst), v4);
         }
       }
     }
