@@ -35,6 +35,7 @@ struct wf_handle {
   // per row and 128-feature tile (mean, M2) of x, xd, hproj for their LayerNorms
   float2 *st_x, *st_xd, *st_hp;
   bf16 *xn, *q, *att, *h1, *taps, *hn;
+  bf16 *xb;  // bf16 copy of the residual stream of a skinny pass (the next LayerNorm's input)
   // scratch
   float *apart;
   int32_t *attn_counters;
@@ -174,6 +175,7 @@ size_t layout(wf_handle *h, const wf_config *c, int Bmax, int ctx, char *base) {
   o->st_xd = cv.take<float2>(M * (d / 128));
   o->st_hp = cv.take<float2>(M * (d / 128));
   o->xn = cv.take<bf16>(M * d);
+  o->xb = cv.take<bf16>(M * d);
   o->q = cv.take<bf16>(M * d);
   o->att = cv.take<bf16>(M * d);
   o->hn = cv.take<bf16>(M * d);
@@ -328,12 +330,16 @@ cudaError_t gemm(wf_handle *h, const void *X, const void *W, GemmParams p, cudaS
   return e;
 }
 
-// A skinny projection: operand LN(ln_x) (g, b) when ln_x is set, else bf16 rows X.
+// A skinny projection: operand LN of the residual (g, b) when g is set --
+// from its bf16 copy h->xb, or from the fp32 rows ln_x when given -- else the
+// bf16 rows X.  EPI_RESID also refreshes h->xb for the next LayerNorm.
 cudaError_t skinny(wf_handle *h, const void *X, const float *ln_x, const void *g, const void *b,
                    const void *W, const GemmParams &gp, cudaStream_t s) {
   SkinnyParams p = skinny_of(gp);
-  if (ln_x) {
-    p.ln_x = ln_x;
+  if (gp.epi == EPI_RESID) p.resid_b = h->xb;
+  if (g) {
+    if (ln_x) p.ln_x = ln_x;
+    else p.ln_xb = h->xb;
     p.ln_ld = h->d;
     p.ln_g = static_cast<const bf16 *>(g);
     p.ln_b = static_cast<const bf16 *>(b);
@@ -464,7 +470,7 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.rows_per_seq = ps.rps;
     p.seq_slot = ps.slots;
     p.pos_base = h->L;
-    e = ps.sk ? skinny(h, nullptr, ps.x, lw.ln1_g, lw.ln1_b, lw.qkv_w, p, s)
+    e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln1_g, lw.ln1_b, lw.qkv_w, p, s)
               : ln_gemm(h, ps.x, ps.st, lw.ln1_g, lw.ln1_b, lw.qkv_w, p, s);
     if (e != cudaSuccess) return e;
   }
@@ -486,7 +492,7 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.bias = static_cast<const bf16 *>(lw.xq_b);
     p.out_bf16 = h->q;
     p.ld_out = d;
-    e = ps.sk ? skinny(h, nullptr, ps.x, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s)
+    e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s)
               : ln_gemm(h, ps.x, ps.st, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s);
     if (e != cudaSuccess) return e;
   }
@@ -508,7 +514,7 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.bias = static_cast<const bf16 *>(lw.fc1_b);
     p.out_bf16 = h->h1;
     p.ld_out = h->F;
-    e = ps.sk ? skinny(h, nullptr, ps.x, lw.ln3_g, lw.ln3_b, lw.fc1_w, p, s)
+    e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln3_g, lw.ln3_b, lw.fc1_w, p, s)
               : ln_gemm(h, ps.x, ps.st, lw.ln3_g, lw.ln3_b, lw.fc1_w, p, s);
     if (e != cudaSuccess) return e;
   }
@@ -640,6 +646,7 @@ cudaError_t target_pass(wf_handle *h, int n_seq, int rps, const int32_t *slots, 
   ep.forced = forced;
   ep.prompt = prompt;
   ep.x = h->x;
+  ep.xb = use_skinny(h, n_seq * rps) ? h->xb : nullptr;
   ep.stats_out = h->st_x;
   ep.n_seq = n_seq;
   ep.rps = rps;
@@ -1111,6 +1118,7 @@ static wf_status draft_body(wf_handle *h, const wf_sample_params *sp, cudaStream
   ep.seq_slot = h->active;
   ep.anchor = h->anchor;
   ep.x = h->xd;
+  ep.xb = use_skinny(h, n * rps) ? h->xb : nullptr;
   ep.stats_out = h->st_xd;
   ep.n_seq = n;
   ep.rps = rps;

@@ -132,12 +132,16 @@ struct SkinnyParams {
   int ln_ld;
   const bf16 *ln_g, *ln_b;
   float ln_eps;
+  // LN operand from bf16 rows (the residual's bf16 copy, row stride ln_ld),
+  // loaded by TMA and normalised in shared memory; takes precedence over ln_x
+  const bf16 *ln_xb;
   const bf16 *bias;
   float *out_f32;
   bf16 *out_bf16;
   int ld_out;
   float *resid;
   int ld_resid;
+  bf16 *resid_b;  // EPI_RESID: nullable bf16 copy of the updated residual (row stride ld_resid)
   bf16 *tap0, *tap1;
   int ld_tap;
   int q_cols, d_model, n_heads, ctx, rows_per_seq;
@@ -180,6 +184,7 @@ struct EmbedParams {
   const int32_t *seq_slot, *L, *anchor, *cand_in, *forced, *prompt;
   int32_t *cand_out;   // effective proposals (after forcing) [slot][K]
   float *x;
+  bf16 *xb;           // nullable: bf16 copy of x
   float2 *stats_out;  // nullable: per row and 128-feature tile (mean, M2) of x
   int n_seq, rps, d, K, P, vocab, src, drafter;
   uint32_t *err;

@@ -100,7 +100,9 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   const uint32_t raw = smem_u32(smem_raw);
   uint8_t *smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
   const int M = p.M, S = p.S, C = p.C;
-  const bool ln = p.ln_x != nullptr;
+  const bool lnb = p.ln_xb != nullptr;     // LN over the residual's bf16 copy (TMA + in place)
+  const bool ln = p.ln_x != nullptr || lnb;  // a LayerNorm operand (its gain and bias staged)
+  const bool tma_op = !ln || lnb;          // the operand's rows arrive by one TMA copy
   const int Ks = p.K / S;  // K range of this CTA
   const int kb = Ks / 64;  // 64-wide k-blocks
   const SkLayout L(M, Ks, U, ln ? p.K : 0);
@@ -126,7 +128,7 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   if (tid == 0) {
     *s_flag = 0;
     tma_prefetch_desc(&tmW);
-    if (!ln) tma_prefetch_desc(&tmX);
+    if (tma_op) tma_prefetch_desc(&tmX);
     mbar_init(&bar[0], 1);
     mbar_init(&bar[1], 1);
     fence_barrier_init();
@@ -173,7 +175,7 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
 
   // ---------------- operand: bf16 rows by one TMA copy (issued first), the
   // residual values this thread will update, or LN(x) shared by the cluster
-  if (!ln && tid == 0) {
+  if (tma_op && tid == 0) {
     mbar_arrive_expect_tx(&bar[1], static_cast<uint32_t>(L.a_bytes));
     tma_load_3d(sA, &tmX, 0, 0, split * kb, &bar[1]);
   }
@@ -189,7 +191,71 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
     }
   }
   bool op_ok = true;
-  if (ln) {
+  if (lnb) {
+    // LN in place over the bf16 rows in shared memory: warp w normalises rows
+    // w and w + 8; lane l holds 16-byte chunks l + 32 i of a row (chunk c =
+    // features 8c .. 8c + 7, at line (c / 8) M + r of the swizzled tile)
+    op_ok = mbar_wait(&bar[1], 0, p.err, p.spin);
+    if (!op_ok) *s_flag = 1;
+    constexpr int kMaxC = 6;  // K <= 1536: at most 192 chunks, 6 per lane
+    const int nch = p.K / 8;
+    for (int h = 0; h < 2 && op_ok; ++h) {
+      const int r = warp + kSkWarps * h;
+      if (r >= M) break;
+      float f[kMaxC][8];
+      uint32_t off[kMaxC];
+#pragma unroll
+      for (int i = 0; i < kMaxC; ++i) {
+        const int c = lane + 32 * i;
+        if (c < nch) {
+          const int line = (c >> 3) * M + r;
+          off[i] = static_cast<uint32_t>(line * 128 + (((c & 7) ^ (line & 7)) << 4));
+          const uint4 raw4 = *reinterpret_cast<const uint4 *>(sA + off[i]);
+          const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&raw4);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            f[i][2 * e] = __low2float(h2[e]);
+            f[i][2 * e + 1] = __high2float(h2[e]);
+          }
+        }
+      }
+      float sum = 0.f;
+#pragma unroll
+      for (int i = 0; i < kMaxC; ++i)
+        if (lane + 32 * i < nch)
+          sum += ((f[i][0] + f[i][1]) + (f[i][2] + f[i][3])) + ((f[i][4] + f[i][5]) + (f[i][6] + f[i][7]));
+      const float mean = warp_sum(sum) / static_cast<float>(p.K);
+      float q = 0.f;
+#pragma unroll
+      for (int i = 0; i < kMaxC; ++i) {
+        if (lane + 32 * i < nch) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const float dv = f[i][e] - mean;
+            q = __fmaf_rn(dv, dv, q);
+          }
+        }
+      }
+      const float2 ms = make_float2(mean, rsqrtf(warp_sum(q) / static_cast<float>(p.K) + p.ln_eps));
+#pragma unroll
+      for (int i = 0; i < kMaxC; ++i) {
+        const int c = lane + 32 * i;
+        if (c < nch) {
+          const uint4 gg = *reinterpret_cast<const uint4 *>(sG + 8 * c);
+          const uint4 bb = *reinterpret_cast<const uint4 *>(sB + 8 * c);
+          const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gg);
+          const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&bb);
+          __nv_bfloat162 o[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e)
+            o[e] = __floats2bfloat162_rn(ln_apply(f[i][2 * e], ms, __low2float(g2[e]), __low2float(b2[e])),
+                                         ln_apply(f[i][2 * e + 1], ms, __high2float(g2[e]), __high2float(b2[e])));
+          *reinterpret_cast<uint4 *>(sA + off[i]) = *reinterpret_cast<const uint4 *>(o);
+        }
+      }
+    }
+    __syncthreads();
+  } else if (ln) {
     // rows r = crank + C q of the cluster's operand belong to this CTA; warp w
     // normalises its rows q = w, w + 8 (lane l holds features 4l + 128 i)
     // into its own operand tile, then the CTA copies them to its peers
@@ -361,6 +427,7 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
     } else if (p.epi == EPI_RESID) {
       const float nr = old[i] + v;
       p.resid[static_cast<size_t>(t) * p.ld_resid + n] = nr;
+      if (p.resid_b) p.resid_b[static_cast<size_t>(t) * p.ld_resid + n] = __float2bfloat16(nr);
       if (p.tap0) p.tap0[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
       if (p.tap1) p.tap1[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
     } else if (p.epi == EPI_KV) {
@@ -380,7 +447,7 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   __syncthreads();
   if (tid == 0 && *s_flag) {
     mbar_drain(&bar[0], 0);
-    if (!ln) mbar_drain(&bar[1], 0);
+    if (tma_op) mbar_drain(&bar[1], 0);
   }
 }
 
@@ -486,24 +553,29 @@ static const CUtensorMap *skinny_xmap(const void *X, int M, int K, int ld, int k
 
 cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pdl) {
   if (p.spin <= 0) p.spin = kSpinLimitCycles;
-  if (!skinny_plan(p.M, p.N, p.K, p.ln_x != nullptr, &p.U, &p.S)) return cudaErrorInvalidValue;
-  if (p.ln_x && (!p.ln_g || !p.ln_b || p.ln_ld % 4 || (reinterpret_cast<uintptr_t>(p.ln_x) & 15)))
+  const bool ln = p.ln_x || p.ln_xb;
+  if (!skinny_plan(p.M, p.N, p.K, ln, &p.U, &p.S)) return cudaErrorInvalidValue;
+  if (ln && (!p.ln_g || !p.ln_b || p.ln_ld % 8 || (reinterpret_cast<uintptr_t>(p.ln_x) & 15) ||
+             (reinterpret_cast<uintptr_t>(p.ln_xb) & 15)))
     return cudaErrorInvalidValue;
-  if (!p.ln_x && (!p.x || p.ld_x % 8 || (reinterpret_cast<uintptr_t>(p.x) & 15))) return cudaErrorInvalidValue;
+  if (!ln && (!p.x || p.ld_x % 8 || (reinterpret_cast<uintptr_t>(p.x) & 15))) return cudaErrorInvalidValue;
+  if (p.resid_b && (reinterpret_cast<uintptr_t>(p.resid_b) & 15)) return cudaErrorInvalidValue;
   const CUtensorMap *tm = skinny_tmap(W, p.N, p.K, p.K / p.S / 64);
   if (!tm) return cudaErrorInvalidValue;
-  const CUtensorMap *tx = p.ln_x ? tm : skinny_xmap(p.x, p.M, p.K, p.ld_x, p.K / p.S / 64);
+  const bool lnb = p.ln_xb != nullptr;
+  const CUtensorMap *tx = lnb ? skinny_xmap(p.ln_xb, p.M, p.K, p.ln_ld, p.K / p.S / 64)
+                        : p.ln_x ? tm : skinny_xmap(p.x, p.M, p.K, p.ld_x, p.K / p.S / 64);
   if (!tx) return cudaErrorInvalidValue;
-  // LayerNorm operands: the CTAs of a cluster share the rows (at most 8)
+  // fp32 LayerNorm operands: the CTAs of a cluster share the rows (at most 8)
   const int gx = p.N / 8 / p.U;
   p.C = 1;
-  if (p.ln_x && p.S == 1)
+  if (p.ln_x && !lnb && p.S == 1)
     for (int c = 8; c >= 2; c >>= 1)
       if (gx % c == 0) {
         p.C = c;
         break;
       }
-  const size_t smem = skinny_smem(p.M, p.K, p.U, p.S, p.ln_x != nullptr);
+  const size_t smem = skinny_smem(p.M, p.K, p.U, p.S, ln);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.N / 8 / p.U, 1, p.S);
   cfg.blockDim = dim3(kSkThreads, 1, 1);

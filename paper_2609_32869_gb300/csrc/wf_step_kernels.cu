@@ -66,6 +66,7 @@ __global__ void embed_kernel(const EmbedParams p) {
     }
     v[k] = val;
     x[e] = val;
+    if (p.xb) p.xb[static_cast<size_t>(r) * p.d + e] = __float2bfloat16(val);
   }
   if (!p.stats_out) return;
   // per-tile (mean, M2) of the row for the next LayerNorm
