@@ -192,81 +192,66 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   }
   bool op_ok = true;
   if (lnb) {
-    // LN in place over the bf16 rows in shared memory.  Statistics: warp w
-    // takes rows w and w + 8, lane l the 16-byte chunks l + 32 i of a row
-    // (chunk c = features 8c .. 8c + 7, at line (c / 8) M + r of the swizzled
-    // tile).  Then every thread normalises (row, chunk) tasks tid + 256 j.
+    // LN in place over the bf16 rows in shared memory: warp w normalises rows
+    // w and w + 8; lane l holds 16-byte chunks l + 32 i of a row (chunk c =
+    // features 8c .. 8c + 7, at line (c / 8) M + r of the swizzled tile)
     op_ok = mbar_wait(&bar[1], 0, p.err, p.spin);
     if (!op_ok) *s_flag = 1;
     constexpr int kMaxC = 6;  // K <= 1536: at most 192 chunks, 6 per lane
     const int nch = p.K / 8;
-    float2 *sStat = reinterpret_cast<float2 *>(sSum);  // [M] (mean, rstd); sSum is free until the MMAs
-    auto chunk_off = [&](int r, int c) {
-      const int line = (c >> 3) * M + r;
-      return static_cast<uint32_t>(line * 128 + (((c & 7) ^ (line & 7)) << 4));
-    };
     for (int h = 0; h < 2 && op_ok; ++h) {
       const int r = warp + kSkWarps * h;
       if (r >= M) break;
       float f[kMaxC][8];
+      uint32_t off[kMaxC];
 #pragma unroll
       for (int i = 0; i < kMaxC; ++i) {
         const int c = lane + 32 * i;
         if (c < nch) {
-          const uint4 raw4 = *reinterpret_cast<const uint4 *>(sA + chunk_off(r, c));
+          const int line = (c >> 3) * M + r;
+          off[i] = static_cast<uint32_t>(line * 128 + (((c & 7) ^ (line & 7)) << 4));
+          const uint4 raw4 = *reinterpret_cast<const uint4 *>(sA + off[i]);
           const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&raw4);
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
             f[i][2 * e] = __low2float(h2[e]);
             f[i][2 * e + 1] = __high2float(h2[e]);
           }
-        } else {
-#pragma unroll
-          for (int e = 0; e < 8; ++e) f[i][e] = 0.f;
         }
       }
-      float part[8];
+      float sum = 0.f;
 #pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        part[e] = f[0][e];
+      for (int i = 0; i < kMaxC; ++i)
+        if (lane + 32 * i < nch)
+          sum += ((f[i][0] + f[i][1]) + (f[i][2] + f[i][3])) + ((f[i][4] + f[i][5]) + (f[i][6] + f[i][7]));
+      const float mean = warp_sum(sum) / static_cast<float>(p.K);
+      float q = 0.f;
 #pragma unroll
-        for (int i = 1; i < kMaxC; ++i) part[e] += f[i][e];
-      }
-      const float mean =
-          warp_sum(((part[0] + part[1]) + (part[2] + part[3])) + ((part[4] + part[5]) + (part[6] + part[7]))) /
-          static_cast<float>(p.K);
+      for (int i = 0; i < kMaxC; ++i) {
+        if (lane + 32 * i < nch) {
 #pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        part[e] = 0.f;
-#pragma unroll
-        for (int i = 0; i < kMaxC; ++i) {
-          const float dv = lane + 32 * i < nch ? f[i][e] - mean : 0.f;
-          part[e] = __fmaf_rn(dv, dv, part[e]);
+          for (int e = 0; e < 8; ++e) {
+            const float dv = f[i][e] - mean;
+            q = __fmaf_rn(dv, dv, q);
+          }
         }
       }
-      const float var =
-          warp_sum(((part[0] + part[1]) + (part[2] + part[3])) + ((part[4] + part[5]) + (part[6] + part[7]))) /
-          static_cast<float>(p.K);
-      if (lane == 0) sStat[r] = make_float2(mean, rsqrtf(var + p.ln_eps));
-    }
-    __syncthreads();
-    if (op_ok) {
-      for (int task = tid; task < M * nch; task += kSkThreads) {
-        const int r = task / nch, c = task - r * nch;
-        const float2 ms = sStat[r];
-        const uint32_t off = chunk_off(r, c);
-        const uint4 raw4 = *reinterpret_cast<const uint4 *>(sA + off);
-        const uint4 gg = *reinterpret_cast<const uint4 *>(sG + 8 * c);
-        const uint4 bb = *reinterpret_cast<const uint4 *>(sB + 8 * c);
-        const __nv_bfloat162 *x2 = reinterpret_cast<const __nv_bfloat162 *>(&raw4);
-        const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gg);
-        const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&bb);
-        __nv_bfloat162 o[4];
+      const float2 ms = make_float2(mean, rsqrtf(warp_sum(q) / static_cast<float>(p.K) + p.ln_eps));
 #pragma unroll
-        for (int e = 0; e < 4; ++e)
-          o[e] = __floats2bfloat162_rn(ln_apply(__low2float(x2[e]), ms, __low2float(g2[e]), __low2float(b2[e])),
-                                       ln_apply(__high2float(x2[e]), ms, __high2float(g2[e]), __high2float(b2[e])));
-        *reinterpret_cast<uint4 *>(sA + off) = *reinterpret_cast<const uint4 *>(o);
+      for (int i = 0; i < kMaxC; ++i) {
+        const int c = lane + 32 * i;
+        if (c < nch) {
+          const uint4 gg = *reinterpret_cast<const uint4 *>(sG + 8 * c);
+          const uint4 bb = *reinterpret_cast<const uint4 *>(sB + 8 * c);
+          const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gg);
+          const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&bb);
+          __nv_bfloat162 o[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e)
+            o[e] = __floats2bfloat162_rn(ln_apply(f[i][2 * e], ms, __low2float(g2[e]), __low2float(b2[e])),
+                                         ln_apply(f[i][2 * e + 1], ms, __high2float(g2[e]), __high2float(b2[e])));
+          *reinterpret_cast<uint4 *>(sA + off[i]) = *reinterpret_cast<const uint4 *>(o);
+        }
       }
     }
     __syncthreads();
