@@ -35,7 +35,13 @@ struct wf_handle {
   // per row and 128-feature tile (mean, M2) of x, xd, hproj for their LayerNorms
   float2 *st_x, *st_xd, *st_hp;
   bf16 *xn, *q, *att, *h1, *taps, *hn;
-  bf16 *xb;  // bf16 copy of the residual stream of a skinny pass (the next LayerNorm's input)
+  // skinny passes: the next projection's folded LayerNorm operand (rows g, b,
+  // then g . x of every token row) and the residual's partial row sums
+  // (sum x, sum x^2), fold_np of them per row, written by the residual's
+  // producer
+  bf16 *xg;
+  float2 *fpart;
+  int fold_np = 0;
   // scratch
   float *apart;
   int32_t *attn_counters;
@@ -175,7 +181,8 @@ size_t layout(wf_handle *h, const wf_config *c, int Bmax, int ctx, char *base) {
   o->st_xd = cv.take<float2>(M * (d / 128));
   o->st_hp = cv.take<float2>(M * (d / 128));
   o->xn = cv.take<bf16>(M * d);
-  o->xb = cv.take<bf16>(M * d);
+  o->xg = cv.take<bf16>(static_cast<size_t>(kSkMaxRows) * d);
+  o->fpart = cv.take<float2>(static_cast<size_t>(kSkMaxRows) * kSkMaxParts);
   o->q = cv.take<bf16>(M * d);
   o->att = cv.take<bf16>(M * d);
   o->hn = cv.take<bf16>(M * d);
@@ -330,19 +337,36 @@ cudaError_t gemm(wf_handle *h, const void *X, const void *W, GemmParams p, cudaS
   return e;
 }
 
-// A skinny projection: operand LN of the residual (g, b) when g is set --
-// from its bf16 copy h->xb, or from the fp32 rows ln_x when given -- else the
-// bf16 rows X.  EPI_RESID also refreshes h->xb for the next LayerNorm.
+// A skinny projection.  Operand: LN(ln_x) of fp32 rows with gain g and bias
+// b when ln_x is given; the folded LayerNorm of the residual when only g is
+// (rows h->xg and partial sums h->fpart left by the residual's producer; the
+// gain and bias are in those rows); else the bf16 rows X.  An EPI_RESID
+// projection followed by a LayerNorm with gain g_next and bias b_next writes
+// that LayerNorm's folded operand.
 cudaError_t skinny(wf_handle *h, const void *X, const float *ln_x, const void *g, const void *b,
-                   const void *W, const GemmParams &gp, cudaStream_t s) {
+                   const void *W, const GemmParams &gp, cudaStream_t s, const void *g_next = nullptr,
+                   const void *b_next = nullptr) {
   SkinnyParams p = skinny_of(gp);
-  if (gp.epi == EPI_RESID) p.resid_b = h->xb;
-  if (g) {
-    if (ln_x) p.ln_x = ln_x;
-    else p.ln_xb = h->xb;
+  if (g_next) {
+    p.xg_out = h->xg;
+    p.g_next = static_cast<const bf16 *>(g_next);
+    p.b_next = static_cast<const bf16 *>(b_next);
+    p.part_out = h->fpart;
+    p.part_stride = kSkMaxParts;
+  }
+  if (g && ln_x) {
+    p.ln_x = ln_x;
     p.ln_ld = h->d;
     p.ln_g = static_cast<const bf16 *>(g);
     p.ln_b = static_cast<const bf16 *>(b);
+    p.ln_eps = h->cfg.ln_eps;
+  } else if (g) {
+    p.fold = 1;
+    p.x = h->xg;
+    p.ld_x = h->d;
+    p.fold_part = h->fpart;
+    p.n_part = h->fold_np;
+    p.part_stride = kSkMaxParts;
     p.ln_eps = h->cfg.ln_eps;
   } else {
     p.x = static_cast<const bf16 *>(X);
@@ -352,15 +376,22 @@ cudaError_t skinny(wf_handle *h, const void *X, const float *ln_x, const void *g
   prof_begin(h, s);
   cudaError_t e = launch_skinny(W, p, s, kPDL);
   prof_end(h, s, WF_FAM_GEMM, gemm_bytes(gp));
+  if (e == cudaSuccess && g_next) {  // partials per row: one per CTA of the plan
+    int U = 0, S = 0;
+    if (!skinny_plan(p.M, p.N, p.K, false, false, &U, &S)) return cudaErrorInvalidValue;
+    h->fold_np = p.N / 8 / U * S;
+  }
   return e;
 }
 
 // Whether every projection of a pass of up to M rows has a skinny plan.
 bool skinny_shapes_fit(int d, int F, int M) {
+  // folded LayerNorm operands carry two more rows (g and b)
   int U = 0, S = 0;
-  return M <= kSkMaxRows && skinny_plan(M, 3 * d, d, true, &U, &S) && skinny_plan(M, d, d, false, &U, &S) &&
-         skinny_plan(M, d, d, true, &U, &S) && skinny_plan(M, F, d, true, &U, &S) &&
-         skinny_plan(M, d, F, false, &U, &S) && skinny_plan(M, 2 * d, d, true, &U, &S);
+  return M <= kSkMaxFoldRows && skinny_plan(M + 2, 3 * d, d, false, true, &U, &S) &&
+         skinny_plan(M, d, d, false, false, &U, &S) && skinny_plan(M + 2, d, d, false, true, &U, &S) &&
+         skinny_plan(M + 2, F, d, false, true, &U, &S) && skinny_plan(M, d, F, false, false, &U, &S) &&
+         skinny_plan(M, 2 * d, d, true, false, &U, &S);
 }
 
 // Whether a pass of M rows takes the skinny projections.
@@ -440,9 +471,10 @@ struct Pass {
   bool sk;     // skinny projections (no statistics travel)
 };
 
-// One pre-LayerNorm Whisper block over the pass's rows.
+// One pre-LayerNorm Whisper block over the pass's rows; next: the following
+// block of the pass (whose first LayerNorm a skinny pass folds), or null.
 cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, int layer,
-                      cudaStream_t s) {
+                      const wf_layer_weights *next, cudaStream_t s) {
   const int M = ps.n_seq * ps.rps, d = h->d;
   cudaError_t e;
   bf16 *kc, *vc, *xkc, *xvc;
@@ -483,7 +515,8 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.resid = ps.x;
     p.ld_resid = d;
     p.stats_out = ps.st;
-    e = ps.sk ? skinny(h, h->att, nullptr, nullptr, nullptr, lw.out_w, p, s) : gemm(h, h->att, lw.out_w, p, s);
+    e = ps.sk ? skinny(h, h->att, nullptr, nullptr, nullptr, lw.out_w, p, s, lw.ln2_g, lw.ln2_b)
+              : gemm(h, h->att, lw.out_w, p, s);
     if (e != cudaSuccess) return e;
   }
   // cross-attention
@@ -505,7 +538,8 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.resid = ps.x;
     p.ld_resid = d;
     p.stats_out = ps.st;
-    e = ps.sk ? skinny(h, h->att, nullptr, nullptr, nullptr, lw.xout_w, p, s) : gemm(h, h->att, lw.xout_w, p, s);
+    e = ps.sk ? skinny(h, h->att, nullptr, nullptr, nullptr, lw.xout_w, p, s, lw.ln3_g, lw.ln3_b)
+              : gemm(h, h->att, lw.xout_w, p, s);
     if (e != cudaSuccess) return e;
   }
   // feed-forward
@@ -536,7 +570,9 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
       }
       p.ld_tap = h->cfg.n_taps * d;
     }
-    e = ps.sk ? skinny(h, h->h1, nullptr, nullptr, nullptr, lw.fc2_w, p, s) : gemm(h, h->h1, lw.fc2_w, p, s);
+    e = ps.sk ? skinny(h, h->h1, nullptr, nullptr, nullptr, lw.fc2_w, p, s, next ? next->ln1_g : nullptr,
+                       next ? next->ln1_b : nullptr)
+              : gemm(h, h->h1, lw.fc2_w, p, s);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
@@ -646,7 +682,14 @@ cudaError_t target_pass(wf_handle *h, int n_seq, int rps, const int32_t *slots, 
   ep.forced = forced;
   ep.prompt = prompt;
   ep.x = h->x;
-  ep.xb = use_skinny(h, n_seq * rps) ? h->xb : nullptr;
+  if (use_skinny(h, n_seq * rps)) {  // the first block's folded LN1 operand
+    ep.xg = h->xg;
+    ep.g_next = static_cast<const bf16 *>(h->tl[0].ln1_g);
+    ep.b_next = static_cast<const bf16 *>(h->tl[0].ln1_b);
+    ep.part_out = h->fpart;
+    ep.part_stride = kSkMaxParts;
+    h->fold_np = 1;
+  }
   ep.stats_out = h->st_x;
   ep.n_seq = n_seq;
   ep.rps = rps;
@@ -664,7 +707,8 @@ cudaError_t target_pass(wf_handle *h, int n_seq, int rps, const int32_t *slots, 
   if (e != cudaSuccess) return e;
   Pass ps{n_seq, rps, slots, false, h->x, h->st_x, taps, use_skinny(h, n_seq * rps)};
   for (int l = 0; l < h->nl; ++l)
-    if ((e = run_block(h, ps, h->tl[l], l, s)) != cudaSuccess) return e;
+    if ((e = run_block(h, ps, h->tl[l], l, l + 1 < h->nl ? &h->tl[l + 1] : nullptr, s)) != cudaSuccess)
+      return e;
   return cudaSuccess;
 }
 
@@ -1118,7 +1162,14 @@ static wf_status draft_body(wf_handle *h, const wf_sample_params *sp, cudaStream
   ep.seq_slot = h->active;
   ep.anchor = h->anchor;
   ep.x = h->xd;
-  ep.xb = use_skinny(h, n * rps) ? h->xb : nullptr;
+  if (use_skinny(h, n * rps)) {  // the first block's folded LN1 operand
+    ep.xg = h->xg;
+    ep.g_next = static_cast<const bf16 *>(h->dl[0].ln1_g);
+    ep.b_next = static_cast<const bf16 *>(h->dl[0].ln1_b);
+    ep.part_out = h->fpart;
+    ep.part_stride = kSkMaxParts;
+    h->fold_np = 1;
+  }
   ep.stats_out = h->st_xd;
   ep.n_seq = n;
   ep.rps = rps;
@@ -1133,7 +1184,7 @@ static wf_status draft_body(wf_handle *h, const wf_sample_params *sp, cudaStream
   WF_TRY(launch_embed(ep, s, kPDL));
   prof_end(h, s, WF_FAM_OTHER, 0.0);
   Pass ps{n, rps, h->active, true, h->xd, h->st_xd, false, use_skinny(h, n * rps)};
-  for (int l = 0; l < h->nd; ++l) WF_TRY(run_block(h, ps, h->dl[l], l, s));
+  for (int l = 0; l < h->nd; ++l) WF_TRY(run_block(h, ps, h->dl[l], l, l + 1 < h->nd ? &h->dl[l + 1] : nullptr, s));
   WF_TRY(head(h, h->xd, ps.sk ? nullptr : h->st_xd, 1, 0, n * rps, h->active, rps, h->recs_d, h->hout_d,
               h->logits_d, sp, kTagDraft, h->cand, s));
   return WF_OK;

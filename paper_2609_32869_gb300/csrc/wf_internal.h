@@ -118,10 +118,13 @@ bool gemm_ln_fits(int M, int N, int K, int epi);
 // ------------------------------------------------------ skinny projections --
 // Y = X W^T for M <= 16 token rows (wf_skinny.cu): each CTA prefetches its
 // whole weight slab (U units of 8 rows over K / S) with TMA before the
-// dependency wait and reduces K in a fixed order.  The operand is LN(ln_x)
-// computed in the kernel (row statistics included) or bf16 rows x.  Epilogues
-// as EpiMode (no EPI_HEAD; EPI_RESID writes no statistics).
+// dependency wait and reduces K in a fixed order.  The operand is bf16 rows
+// x, the folded LayerNorm of a residual (rows written by its producer), or
+// LN(ln_x) computed in the kernel from fp32 rows.  Epilogues as EpiMode (no
+// EPI_HEAD; EPI_RESID writes no tile statistics).
 constexpr int kSkMaxRows = 16;
+constexpr int kSkMaxFoldRows = kSkMaxRows - 2;  // token rows of a folded LayerNorm operand
+constexpr int kSkMaxParts = 160;                // partial row sums of one residual update
 struct SkinnyParams {
   int M, N, K;
   int U, S, C;  // set by launch_skinny (C: CTAs of a cluster sharing a LayerNorm operand)
@@ -132,16 +135,29 @@ struct SkinnyParams {
   int ln_ld;
   const bf16 *ln_g, *ln_b;
   float ln_eps;
-  // LN operand from bf16 rows (the residual's bf16 copy, row stride ln_ld),
-  // loaded by TMA and normalised in shared memory; takes precedence over ln_x
-  const bf16 *ln_xb;
+  // Folded LayerNorm (fold != 0): LN(x) W^T = r (W (g . x)) - r mu (W g) + W b
+  // per row, with the row's mean mu and r = 1 / sqrt(var + eps).  The
+  // operand x holds M + 2 bf16 rows (row stride ld_x): g, b, then g . x of
+  // every token row, all written by the residual's producer, so one MMA gives
+  // W g and W b beside the token rows.  The row statistics are the sums of
+  // n_part partials (sum x, sum x^2) per row, fold_part[t * part_stride + i].
+  int fold;
+  const float2 *fold_part;
+  int n_part, part_stride;
   const bf16 *bias;
   float *out_f32;
   bf16 *out_bf16;
   int ld_out;
   float *resid;
   int ld_resid;
-  bf16 *resid_b;  // EPI_RESID: nullable bf16 copy of the updated residual (row stride ld_resid)
+  // EPI_RESID, for a folded LayerNorm next (nullable): the next projection's
+  // operand rows into xg_out (row stride ld_resid): g_next, b_next, then
+  // bf16 (g_next . x) of every row; and per row the (sum x, sum x^2) of the
+  // outputs this CTA finishes into part_out[t * part_stride + blockIdx.x * S
+  // + rank]
+  bf16 *xg_out;
+  const bf16 *g_next, *b_next;
+  float2 *part_out;  // (row stride part_stride, shared with fold_part)
   bf16 *tap0, *tap1;
   int ld_tap;
   int q_cols, d_model, n_heads, ctx, rows_per_seq;
@@ -150,9 +166,10 @@ struct SkinnyParams {
   uint32_t *err;
   long long spin;
 };
-// Whether a projection of M rows, N outputs and K inputs has a skinny plan
-// (units per CTA U, K split S); LN operands need S == 1.
-bool skinny_plan(int M, int N, int K, bool ln, int *U, int *S);
+// Whether a projection of M operand rows, N outputs and K inputs has a
+// skinny plan (units per CTA U, K split S).  ln: an fp32 LayerNorm operand
+// (gain and bias staged, S == 1); whole_k: S == 1 (a folded LayerNorm).
+bool skinny_plan(int M, int N, int K, bool ln, bool whole_k, int *U, int *S);
 cudaError_t skinny_init();
 cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pdl);
 
@@ -184,7 +201,13 @@ struct EmbedParams {
   const int32_t *seq_slot, *L, *anchor, *cand_in, *forced, *prompt;
   int32_t *cand_out;   // effective proposals (after forcing) [slot][K]
   float *x;
-  bf16 *xb;           // nullable: bf16 copy of x
+  // nullable: the operand rows of a folded LayerNorm over x (g_next, b_next,
+  // then bf16 g_next . x per row; row stride d) and each row's (sum x, sum
+  // x^2) as its one partial (part_out[r * part_stride])
+  bf16 *xg;
+  const bf16 *g_next, *b_next;
+  float2 *part_out;
+  int part_stride;
   float2 *stats_out;  // nullable: per row and 128-feature tile (mean, M2) of x
   int n_seq, rps, d, K, P, vocab, src, drafter;
   uint32_t *err;

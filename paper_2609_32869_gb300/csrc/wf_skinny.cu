@@ -10,11 +10,18 @@
 //    with TMA before griddepcontrol.wait, one 3-D tensor copy per unit that
 //    lands 128-byte swizzled ([k-block][8 rows][64 features]); the slab
 //    streams while the previous kernels run;
-//  - after the wait the token operand lands in shared memory: bf16 rows by
-//    one TMA copy, or LN(x) from the fp32 residual rows, where the CTAs of a
-//    cluster split the rows (each computes its rows' mean and variance, so no
-//    statistics travel between kernels) and write the normalised bf16 rows
-//    into every CTA of the cluster over distributed shared memory;
+//  - after the wait the token operand lands in shared memory by one TMA
+//    copy.  A LayerNorm operand is folded into the projection: with the
+//    row's mean mu and r = 1 / sqrt(var + eps),
+//      LN(x) W^T = r (W (g . x) - mu W g) + W b,
+//    so the producer of the residual writes the bf16 rows g, b and g . x
+//    (and per row its partial sums of x and x^2), one MMA over those rows
+//    gives W g and W b beside the token rows, and the row statistics are
+//    applied in the epilogue: no normalisation sits between the operand's
+//    arrival and the MMAs.  (The history memory's LN_h, over fp32 rows, is
+//    computed in the kernel instead: the CTAs of a cluster split the rows and
+//    write the normalised bf16 rows into every CTA over distributed shared
+//    memory.);
 //  - all eight warps issue mma.sync m16n8k16 at once (tokens on the 16-row
 //    side, weight rows on the 8-column side), each over its own slice of K;
 //    the slices are summed in warp order, then (S > 1) the S CTAs' sums in
@@ -54,8 +61,10 @@ __device__ __forceinline__ void tma_load_3d(void *smem_dst, const CUtensorMap *m
 // Shared-memory layout of one CTA (offsets from the 1024-aligned base).  The
 // warps' partial sums reuse the weight slab once every MMA has read it.
 struct SkLayout {
-  int unit_bytes, w_bytes, a_off, a_bytes, sum_off, bias_off, gb_off, bar_off, zero_off, flag_off, total;
-  // K_ln: features of a LayerNorm operand (its gain and bias are staged), else 0
+  int unit_bytes, w_bytes, a_off, a_bytes, sum_off, bias_off, gb_off, stat_off, bar_off, zero_off, flag_off,
+      total;
+  // M: operand rows; K_ln: features of an fp32 LayerNorm operand (its gain
+  // and bias are staged), else 0
   __host__ __device__ SkLayout(int M, int Ks, int U, int K_ln) {
     const int kb = Ks / 64;
     unit_bytes = kb * 1024;
@@ -65,7 +74,8 @@ struct SkLayout {
     sum_off = (a_off + a_bytes + 15) & ~15;
     bias_off = sum_off + U * 128 * 4;
     gb_off = (bias_off + U * 8 * 4 + 15) & ~15;
-    bar_off = (gb_off + K_ln * 4 + 15) & ~15;
+    stat_off = (gb_off + K_ln * 4 + 15) & ~15;
+    bar_off = stat_off + kSkMaxRows * 8;
     zero_off = bar_off + 16;
     flag_off = zero_off + 16;
     total = flag_off + 16;
@@ -100,20 +110,23 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   const uint32_t raw = smem_u32(smem_raw);
   uint8_t *smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
   const int M = p.M, S = p.S, C = p.C;
-  const bool lnb = p.ln_xb != nullptr;     // LN over the residual's bf16 copy (TMA + in place)
-  const bool ln = p.ln_x != nullptr || lnb;  // a LayerNorm operand (its gain and bias staged)
-  const bool tma_op = !ln || lnb;          // the operand's rows arrive by one TMA copy
+  const bool ln = p.ln_x != nullptr;  // LayerNorm of fp32 rows computed here (gain and bias staged)
+  const bool fold = p.fold != 0;      // folded LayerNorm: rows g, b, then the M token rows
+  const bool tma_op = !ln;            // the operand's rows arrive by one TMA copy
+  const int t0 = fold ? 2 : 0;        // first token row of the operand
+  const int Mr = M + t0;              // operand rows
   const int Ks = p.K / S;  // K range of this CTA
   const int kb = Ks / 64;  // 64-wide k-blocks
-  const SkLayout L(M, Ks, U, ln ? p.K : 0);
+  const SkLayout L(Mr, Ks, U, ln ? p.K : 0);
   const int unit_bytes = L.unit_bytes;             // one unit: [kb][8 rows][128 B]
   uint8_t *sW = smem;
-  uint8_t *sA = smem + L.a_off;                    // [kb][M][128 B]
+  uint8_t *sA = smem + L.a_off;                    // [kb][Mr][128 B]
   float *sPart = reinterpret_cast<float *>(smem);  // [warps][U][16][8], over the slab after the MMAs
   float *sSum = reinterpret_cast<float *>(smem + L.sum_off);    // [U][16][8]
   float *sBias = reinterpret_cast<float *>(smem + L.bias_off);  // [U * 8]
   bf16 *sG = reinterpret_cast<bf16 *>(smem + L.gb_off);         // [K] LayerNorm gain, then [K] bias
   bf16 *sB = sG + p.K;
+  float2 *sStat = reinterpret_cast<float2 *>(smem + L.stat_off);  // [M] (mu, r) of a folded LayerNorm
   uint64_t *bar = reinterpret_cast<uint64_t *>(smem + L.bar_off);  // [0] weights, [1] operand
   uint4 *sZero = reinterpret_cast<uint4 *>(smem + L.zero_off);
   int *s_flag = reinterpret_cast<int *>(smem + L.flag_off);
@@ -154,10 +167,21 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   constexpr int kEpi = (U * kSkMaxRows * 8 + kSkThreads - 1) / kSkThreads;
   const int n_out = U * M * 8;
   int kv_dst[kEpi];  // EPI_KV: cache row index (slot * heads + head) * ctx + position, or -1
+  // EPI_RESID with a folded LayerNorm next: its gain (and, on token row 0,
+  // its bias) at this thread's outputs
+  float g_nx[kEpi], b_nx[kEpi];
 #pragma unroll
   for (int i = 0; i < kEpi; ++i) {
     kv_dst[i] = -1;
     const int e = tid + i * kSkThreads;
+    g_nx[i] = b_nx[i] = 0.f;
+    if (p.xg_out && e < n_out) {
+      const int n = n_base + e / (M * 8) * 8 + (e & 7);
+      if (n < p.N) {
+        g_nx[i] = bf2f(p.g_next[n]);
+        if ((e % (M * 8)) < 8) b_nx[i] = bf2f(p.b_next[n]);
+      }
+    }
     if (p.epi == EPI_KV && e < n_out) {
       const int u = e / (M * 8), rem = e - u * M * 8, t = rem >> 3, j = rem & 7;
       const int n = n_base + u * 8 + j;
@@ -190,72 +214,40 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
       if (n < p.N) old[i] = __ldcg(p.resid + static_cast<size_t>(t) * p.ld_resid + n);
     }
   }
-  bool op_ok = true;
-  if (lnb) {
-    // LN in place over the bf16 rows in shared memory: warp w normalises rows
-    // w and w + 8; lane l holds 16-byte chunks l + 32 i of a row (chunk c =
-    // features 8c .. 8c + 7, at line (c / 8) M + r of the swizzled tile)
-    op_ok = mbar_wait(&bar[1], 0, p.err, p.spin);
-    if (!op_ok) *s_flag = 1;
-    constexpr int kMaxC = 6;  // K <= 1536: at most 192 chunks, 6 per lane
-    const int nch = p.K / 8;
-    for (int h = 0; h < 2 && op_ok; ++h) {
-      const int r = warp + kSkWarps * h;
-      if (r >= M) break;
-      float f[kMaxC][8];
-      uint32_t off[kMaxC];
+  if (fold) {
+    // row statistics of a folded LayerNorm: warp w sums the partials of rows
+    // w and w + 8, lane l the partials l + 32 i (every load in flight at
+    // once), added in order of i, then across lanes
+    constexpr int kPL = (kSkMaxParts + 31) / 32;
+    float2 v[2][kPL];
 #pragma unroll
-      for (int i = 0; i < kMaxC; ++i) {
-        const int c = lane + 32 * i;
-        if (c < nch) {
-          const int line = (c >> 3) * M + r;
-          off[i] = static_cast<uint32_t>(line * 128 + (((c & 7) ^ (line & 7)) << 4));
-          const uint4 raw4 = *reinterpret_cast<const uint4 *>(sA + off[i]);
-          const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&raw4);
+    for (int h = 0; h < 2; ++h) {
+      const int t = warp + kSkWarps * h;
+      const float2 *pr = p.fold_part + static_cast<size_t>(t) * p.part_stride;
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            f[i][2 * e] = __low2float(h2[e]);
-            f[i][2 * e + 1] = __high2float(h2[e]);
-          }
-        }
-      }
-      float sum = 0.f;
-#pragma unroll
-      for (int i = 0; i < kMaxC; ++i)
-        if (lane + 32 * i < nch)
-          sum += ((f[i][0] + f[i][1]) + (f[i][2] + f[i][3])) + ((f[i][4] + f[i][5]) + (f[i][6] + f[i][7]));
-      const float mean = warp_sum(sum) / static_cast<float>(p.K);
-      float q = 0.f;
-#pragma unroll
-      for (int i = 0; i < kMaxC; ++i) {
-        if (lane + 32 * i < nch) {
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const float dv = f[i][e] - mean;
-            q = __fmaf_rn(dv, dv, q);
-          }
-        }
-      }
-      const float2 ms = make_float2(mean, rsqrtf(warp_sum(q) / static_cast<float>(p.K) + p.ln_eps));
-#pragma unroll
-      for (int i = 0; i < kMaxC; ++i) {
-        const int c = lane + 32 * i;
-        if (c < nch) {
-          const uint4 gg = *reinterpret_cast<const uint4 *>(sG + 8 * c);
-          const uint4 bb = *reinterpret_cast<const uint4 *>(sB + 8 * c);
-          const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gg);
-          const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&bb);
-          __nv_bfloat162 o[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e)
-            o[e] = __floats2bfloat162_rn(ln_apply(f[i][2 * e], ms, __low2float(g2[e]), __low2float(b2[e])),
-                                         ln_apply(f[i][2 * e + 1], ms, __high2float(g2[e]), __high2float(b2[e])));
-          *reinterpret_cast<uint4 *>(sA + off[i]) = *reinterpret_cast<const uint4 *>(o);
-        }
+      for (int q = 0; q < kPL; ++q) {
+        const int i = lane + 32 * q;
+        v[h][q] = (t < M && i < p.n_part) ? __ldcg(pr + i) : make_float2(0.f, 0.f);
       }
     }
-    __syncthreads();
-  } else if (ln) {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int t = warp + kSkWarps * h;
+      float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+      for (int q = 0; q < kPL; ++q) {
+        s1 += v[h][q].x;
+        s2 += v[h][q].y;
+      }
+      s1 = warp_sum(s1);
+      s2 = warp_sum(s2);
+      const float mu = s1 / static_cast<float>(p.K);
+      const float var = fmaxf(s2 / static_cast<float>(p.K) - mu * mu, 0.f);
+      if (lane == 0 && t < M) sStat[t] = make_float2(mu, rsqrtf(var + p.ln_eps));
+    }
+  }
+  bool op_ok = true;
+  if (ln) {
     // rows r = crank + C q of the cluster's operand belong to this CTA; warp w
     // normalises its rows q = w, w + 8 (lane l holds features 4l + 128 i)
     // into its own operand tile, then the CTA copies them to its peers
@@ -325,7 +317,6 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
     op_ok = mbar_wait(&bar[1], 0, p.err, p.spin);
     if (!op_ok) *s_flag = 1;
   }
-
   // ---------------- MMAs: warp w takes the k-blocks [w kb / 8, (w + 1) kb / 8) of
   // every unit; within a k-block the k-steps alternate between two accumulators
   // (shorter dependency chains), added in a fixed order at the end
@@ -339,9 +330,9 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   if (landed) {
     const uint32_t w_base = smem_u32(sW);
     // A (ldmatrix.x4 per k-step): lanes 0-7 rows 0-7 and 16-23 rows 0-7 (second
-    // 8 features), 8-15 and 24-31 rows 8-15; rows >= M read 16 zero bytes
+    // 8 features), 8-15 and 24-31 rows 8-15; rows >= Mr read 16 zero bytes
     const int ar = (lane & 7) + ((lane >> 3) & 1) * 8, c0 = lane >> 4;
-    const bool real = ar < M;
+    const bool real = ar < Mr;
     const uint32_t a_base = smem_u32(sA), z_addr = smem_u32(sZero);
     // B (ldmatrix.x4 per pair of k-steps): lane group g reads 16-byte chunk g
     // (first pair) or g + 4 (second pair) of weight row lane & 7
@@ -350,7 +341,7 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
     const int kb_lo = warp * kb / kSkWarps, kb_hi = (warp + 1) * kb / kSkWarps;
     for (int q = kb_lo; q < kb_hi; ++q) {
       uint32_t a[4][4];
-      const int line = q * M + ar;
+      const int line = q * Mr + ar;
       const uint32_t aq = a_base + line * 128, sw = line & 7;
 #pragma unroll
       for (int j = 0; j < 4; ++j)
@@ -400,7 +391,7 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
     const int e = tid + i * kSkThreads;
     if (e >= n_out || (S > 1 && (e % S) != split)) continue;
     const int u = e / (M * 8), rem = e - u * M * 8, t = rem >> 3, j = rem & 7;
-    const int idx = u * 128 + t * 8 + j;
+    const int idx = u * 128 + (t + t0) * 8 + j;
     float v;
     if (S > 1) {
       float part[8];
@@ -417,6 +408,10 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
     }
     const int n = n_base + u * 8 + j;
     if (n >= p.N || !ok) continue;
+    if (fold) {  // r (W (g . x) - mu W g) + W b; rows 0 and 1 of the sums hold W g and W b
+      const float2 ms = sStat[t];
+      v = __fmaf_rn(ms.y, __fmaf_rn(-ms.x, sSum[u * 128 + j], v), sSum[u * 128 + 8 + j]);
+    }
     v += sBias[u * 8 + j];
     if (p.epi == EPI_F32) {
       p.out_f32[static_cast<size_t>(t) * p.ld_out + n] = v;
@@ -427,7 +422,14 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
     } else if (p.epi == EPI_RESID) {
       const float nr = old[i] + v;
       p.resid[static_cast<size_t>(t) * p.ld_resid + n] = nr;
-      if (p.resid_b) p.resid_b[static_cast<size_t>(t) * p.ld_resid + n] = __float2bfloat16(nr);
+      if (p.xg_out) {
+        p.xg_out[static_cast<size_t>(t + 2) * p.ld_resid + n] = __float2bfloat16(nr * g_nx[i]);
+        if (t == 0) {  // bf16 values, converted back exactly
+          p.xg_out[n] = __float2bfloat16(g_nx[i]);
+          p.xg_out[static_cast<size_t>(p.ld_resid) + n] = __float2bfloat16(b_nx[i]);
+        }
+        sPart[u * 128 + t * 8 + j] = nr;  // the slab is free: the CTA's sums are in sSum
+      }
       if (p.tap0) p.tap0[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
       if (p.tap1) p.tap1[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
     } else if (p.epi == EPI_KV) {
@@ -440,6 +442,25 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
         bf16 *dst = which == 0 ? p.kc : p.vc;
         dst[static_cast<size_t>(kv_dst[i]) * 64 + ((c - which * p.d_model) & 63)] = __float2bfloat16(v);
       }
+    }
+  }
+  if (p.xg_out) {
+    // this CTA's partial (sum x, sum x^2) of every row over the outputs it
+    // finished: warp w takes rows w and w + 8, lane l the outputs (u, j) with
+    // u = l / 8 + 4 i and j = l % 8, added in order of i, then across lanes
+    __syncthreads();
+    for (int t = warp; t < M; t += kSkWarps) {
+      float s1 = 0.f, s2 = 0.f;
+      for (int u = lane >> 3; u < U; u += 4) {
+        const int j = lane & 7, e = u * M * 8 + t * 8 + j;
+        if ((S > 1 && e % S != split) || n_base + u * 8 + j >= p.N || !ok) continue;
+        const float x = sPart[u * 128 + t * 8 + j];
+        s1 += x;
+        s2 = __fmaf_rn(x, x, s2);
+      }
+      s1 = warp_sum(s1);
+      s2 = warp_sum(s2);
+      if (lane == 0) p.part_out[static_cast<size_t>(t) * p.part_stride + cta * S + split] = make_float2(s1, s2);
     }
   }
   if (S > 1) cluster_sync();  // peers may read this CTA's sums until here
@@ -458,7 +479,7 @@ size_t skinny_smem(int M, int K, int U, int S, bool ln) {
 }
 }  // namespace
 
-bool skinny_plan(int M, int N, int K, bool ln, int *U, int *S) {
+bool skinny_plan(int M, int N, int K, bool ln, bool whole_k, int *U, int *S) {
   if (M < 1 || M > kSkMaxRows || N % 8 || K % 128) return false;
   const int units = N / 8;
   // the fewest CTAs' worth of units that keeps the grid within about one CTA
@@ -468,11 +489,11 @@ bool skinny_plan(int M, int N, int K, bool ln, int *U, int *S) {
   // over a cluster of S CTAs
   int best_u = 0, best_s = 0;
   for (int s = 1; s <= 8; s *= 2) {
-    if (K % (s * 128) || K / s < 256 || (ln && s > 1)) continue;
+    if (K % (s * 128) || K / s < 256 || ((ln || whole_k) && s > 1)) continue;
     for (int u = 1; u <= 8; ++u) {
       if (units % u) continue;
       const int ctas = units / u * s;
-      if (ctas > 160) continue;
+      if (ctas > kSkMaxParts) continue;
       if (skinny_smem(M, K, u, s, ln) > kSkSmemBudget) continue;
       if (!best_u) {
         best_u = u;
@@ -553,29 +574,32 @@ static const CUtensorMap *skinny_xmap(const void *X, int M, int K, int ld, int k
 
 cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pdl) {
   if (p.spin <= 0) p.spin = kSpinLimitCycles;
-  const bool ln = p.ln_x || p.ln_xb;
-  if (!skinny_plan(p.M, p.N, p.K, ln, &p.U, &p.S)) return cudaErrorInvalidValue;
-  if (ln && (!p.ln_g || !p.ln_b || p.ln_ld % 8 || (reinterpret_cast<uintptr_t>(p.ln_x) & 15) ||
-             (reinterpret_cast<uintptr_t>(p.ln_xb) & 15)))
+  const bool ln = p.ln_x != nullptr;
+  const bool fold = p.fold != 0;
+  if (fold && (ln || p.M > kSkMaxFoldRows || !p.fold_part || p.n_part < 1 || p.n_part > p.part_stride))
+    return cudaErrorInvalidValue;
+  const int Mr = p.M + (fold ? 2 : 0);  // operand rows
+  if (!skinny_plan(Mr, p.N, p.K, ln, fold, &p.U, &p.S)) return cudaErrorInvalidValue;
+  if (ln && (!p.ln_g || !p.ln_b || p.ln_ld % 4 || (reinterpret_cast<uintptr_t>(p.ln_x) & 15)))
     return cudaErrorInvalidValue;
   if (!ln && (!p.x || p.ld_x % 8 || (reinterpret_cast<uintptr_t>(p.x) & 15))) return cudaErrorInvalidValue;
-  if (p.resid_b && (reinterpret_cast<uintptr_t>(p.resid_b) & 15)) return cudaErrorInvalidValue;
+  if (p.xg_out && (p.epi != EPI_RESID || !p.g_next || !p.b_next || !p.part_out ||
+                   p.N / 8 / p.U * p.S > p.part_stride))
+    return cudaErrorInvalidValue;
   const CUtensorMap *tm = skinny_tmap(W, p.N, p.K, p.K / p.S / 64);
   if (!tm) return cudaErrorInvalidValue;
-  const bool lnb = p.ln_xb != nullptr;
-  const CUtensorMap *tx = lnb ? skinny_xmap(p.ln_xb, p.M, p.K, p.ln_ld, p.K / p.S / 64)
-                        : p.ln_x ? tm : skinny_xmap(p.x, p.M, p.K, p.ld_x, p.K / p.S / 64);
+  const CUtensorMap *tx = ln ? tm : skinny_xmap(p.x, Mr, p.K, p.ld_x, p.K / p.S / 64);
   if (!tx) return cudaErrorInvalidValue;
   // fp32 LayerNorm operands: the CTAs of a cluster share the rows (at most 8)
   const int gx = p.N / 8 / p.U;
   p.C = 1;
-  if (p.ln_x && !lnb && p.S == 1)
+  if (ln && p.S == 1)
     for (int c = 8; c >= 2; c >>= 1)
       if (gx % c == 0) {
         p.C = c;
         break;
       }
-  const size_t smem = skinny_smem(p.M, p.K, p.U, p.S, ln);
+  const size_t smem = skinny_smem(Mr, p.K, p.U, p.S, ln);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.N / 8 / p.U, 1, p.S);
   cfg.blockDim = dim3(kSkThreads, 1, 1);

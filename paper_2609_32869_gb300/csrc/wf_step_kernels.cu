@@ -66,7 +66,35 @@ __global__ void embed_kernel(const EmbedParams p) {
     }
     v[k] = val;
     x[e] = val;
-    if (p.xb) p.xb[static_cast<size_t>(r) * p.d + e] = __float2bfloat16(val);
+    if (p.xg) {
+      p.xg[static_cast<size_t>(r + 2) * p.d + e] = __float2bfloat16(val * bf2f(p.g_next[e]));
+      if (r == 0) {
+        p.xg[e] = p.g_next[e];
+        p.xg[static_cast<size_t>(p.d) + e] = p.b_next[e];
+      }
+    }
+  }
+  if (p.part_out) {  // the whole row's (sum x, sum x^2), summed in a fixed order
+    __shared__ float red2[4][2];
+    float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+    for (int k = 0; k < kMaxStatTiles; ++k)
+      if (k < tiles) {
+        s1 += v[k];
+        s2 = __fmaf_rn(v[k], v[k], s2);
+      }
+    s1 = warp_sum(s1);
+    s2 = warp_sum(s2);
+    const int w = threadIdx.x >> 5;
+    if ((threadIdx.x & 31) == 0) {
+      red2[w][0] = s1;
+      red2[w][1] = s2;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0)
+      p.part_out[static_cast<size_t>(r) * p.part_stride] =
+          make_float2((red2[0][0] + red2[1][0]) + (red2[2][0] + red2[3][0]),
+                      (red2[0][1] + red2[1][1]) + (red2[2][1] + red2[3][1]));
   }
   if (!p.stats_out) return;
   // per-tile (mean, M2) of the row for the next LayerNorm
