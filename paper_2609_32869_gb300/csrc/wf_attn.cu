@@ -334,13 +334,18 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
   float L = 0.f, acc[kDPT];
 #pragma unroll
   for (int e = 0; e < kDPT; ++e) acc[e] = 0.f;
+  static_assert(kDPT == 4, "one float4 of O per warp and thread");
 #pragma unroll
   for (int w = 0; w < kWarps; ++w) {
     const float mw = sm[w * kQG + qi];
     const float wt = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
     L += sl[w * kQG + qi] * wt;
-#pragma unroll
-    for (int e = 0; e < kDPT; ++e) acc[e] += so[(w * kQG + qi) * 64 + ((d0 + e) ^ ((qi & 3) << 3))] * wt;
+    // dims d0..d0+3 stay contiguous under the swizzle (it flips bits 3 and 4)
+    const float4 o4 = *reinterpret_cast<const float4 *>(so + (w * kQG + qi) * 64 + (d0 ^ ((qi & 3) << 3)));
+    acc[0] += o4.x * wt;
+    acc[1] += o4.y * wt;
+    acc[2] += o4.z * wt;
+    acc[3] += o4.w * wt;
   }
 
   if (n_blocks == 1) {
@@ -366,18 +371,31 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
     cluster_sync();
     float MM = -INFINITY, LL = 0.f, oo[kDPT];
     if (blk == 0) {
+      // every peer's (m, l, o) load in flight at once (at most 8 blocks), then
+      // merged in block order; an absent block adds exact zeros
       const uint32_t pb_u32 = smem_u32(pb);
-      for (int u = 0; u < p.n_chunks; ++u)
-        MM = fmaxf(MM, dsmem_ld_f32(dsmem_map(pb_u32 + 4u * (qi * 68), u)));
+      float mc[8], lc[8];
+      float4 o4[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        mc[u] = -INFINITY;
+        lc[u] = 0.f;
+        o4[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (u < p.n_chunks) {
+          mc[u] = dsmem_ld_f32(dsmem_map(pb_u32 + 4u * (qi * 68), u));
+          lc[u] = dsmem_ld_f32(dsmem_map(pb_u32 + 4u * (qi * 68 + 1), u));
+          o4[u] = dsmem_ld_f32x4(dsmem_map(pb_u32 + 4u * (qi * 68 + 4 + d0), u));
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) MM = fmaxf(MM, mc[u]);
 #pragma unroll
       for (int e = 0; e < kDPT; ++e) oo[e] = 0.f;
-      for (int u = 0; u < p.n_chunks; ++u) {
-        const float mc = dsmem_ld_f32(dsmem_map(pb_u32 + 4u * (qi * 68), u));
-        const float lc = dsmem_ld_f32(dsmem_map(pb_u32 + 4u * (qi * 68 + 1), u));
-        const float4 o4 = dsmem_ld_f32x4(dsmem_map(pb_u32 + 4u * (qi * 68 + 4 + d0), u));
-        const float ov[4] = {o4.x, o4.y, o4.z, o4.w};
-        const float wt = (mc == -INFINITY) ? 0.f : exp2f(mc - MM);
-        LL = __fmaf_rn(lc, wt, LL);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const float ov[4] = {o4[u].x, o4[u].y, o4[u].z, o4[u].w};
+        const float wt = (mc[u] == -INFINITY) ? 0.f : exp2f(mc[u] - MM);
+        LL = __fmaf_rn(lc[u], wt, LL);
 #pragma unroll
         for (int e = 0; e < kDPT; ++e) oo[e] = __fmaf_rn(ov[e], wt, oo[e]);
       }
@@ -416,22 +434,43 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
   // weight 0, so it adds exact zeros; the loads of all blocks are independent.
   if (qi < nq) {
     const float *pg = p.part + static_cast<size_t>(group_id) * p.n_chunks * kQG * kPartStride;
+    // blocks in groups of 8 with every load of a group in flight, merged in
+    // block order; a block past n_blocks adds exact zeros
     float MM = -INFINITY;
-    for (int u = 0; u < n_blocks; ++u) MM = fmaxf(MM, __ldcg(pg + (u * kQG + qi) * kPartStride));
+    for (int u0 = 0; u0 < n_blocks; u0 += 8) {
+      float mc[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        mc[u] = u0 + u < n_blocks ? __ldcg(pg + ((u0 + u) * kQG + qi) * kPartStride) : -INFINITY;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) MM = fmaxf(MM, mc[u]);
+    }
     float LL = 0.f, oo[kDPT];
 #pragma unroll
     for (int e = 0; e < kDPT; ++e) oo[e] = 0.f;
-    for (int u = 0; u < n_blocks; ++u) {
-      const float *pe = pg + (u * kQG + qi) * kPartStride;
-      const float mc = __ldcg(pe);
-      const float lc = __ldcg(pe + 1);
-      float ov[kDPT];
+    for (int u0 = 0; u0 < n_blocks; u0 += 8) {
+      float mc[8], lc[8], ov[8][kDPT];
 #pragma unroll
-      for (int e = 0; e < kDPT; ++e) ov[e] = __ldcg(pe + 2 + d0 + e);
-      const float wt = (mc == -INFINITY) ? 0.f : exp2f(mc - MM);
-      LL = __fmaf_rn(lc, wt, LL);
+      for (int u = 0; u < 8; ++u) {
+        mc[u] = -INFINITY;
+        lc[u] = 0.f;
 #pragma unroll
-      for (int e = 0; e < kDPT; ++e) oo[e] = __fmaf_rn(ov[e], wt, oo[e]);
+        for (int e = 0; e < kDPT; ++e) ov[u][e] = 0.f;
+        if (u0 + u < n_blocks) {
+          const float *pe = pg + ((u0 + u) * kQG + qi) * kPartStride;
+          mc[u] = __ldcg(pe);
+          lc[u] = __ldcg(pe + 1);
+#pragma unroll
+          for (int e = 0; e < kDPT; ++e) ov[u][e] = __ldcg(pe + 2 + d0 + e);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const float wt = (mc[u] == -INFINITY) ? 0.f : exp2f(mc[u] - MM);
+        LL = __fmaf_rn(lc[u], wt, LL);
+#pragma unroll
+        for (int e = 0; e < kDPT; ++e) oo[e] = __fmaf_rn(ov[u][e], wt, oo[e]);
+      }
     }
     const float inv = 1.0f / LL;
     bf16 *orow = p.out + static_cast<size_t>(i * p.rps + q0 + qi) * d_model + h * 64 + d0;
