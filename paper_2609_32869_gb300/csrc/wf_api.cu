@@ -342,11 +342,14 @@ cudaError_t gemm(wf_handle *h, const void *X, const void *W, GemmParams p, cudaS
 // (rows h->xg and partial sums h->fpart left by the residual's producer; the
 // gain and bias are in those rows); else the bf16 rows X.  An EPI_RESID
 // projection followed by a LayerNorm with gain g_next and bias b_next writes
-// that LayerNorm's folded operand.
+// that LayerNorm's folded operand.  pf: the next projection's weights (pf_n
+// rows of pf_k), brought into L2 while this one waits for its inputs.
 cudaError_t skinny(wf_handle *h, const void *X, const float *ln_x, const void *g, const void *b,
                    const void *W, const GemmParams &gp, cudaStream_t s, const void *g_next = nullptr,
-                   const void *b_next = nullptr) {
+                   const void *b_next = nullptr, const void *pf = nullptr, int pf_n = 0, int pf_k = 0) {
   SkinnyParams p = skinny_of(gp);
+  p.pf = pf;
+  p.pf_bytes = pf ? static_cast<size_t>(pf_n) * pf_k * sizeof(bf16) : 0;
   if (g_next) {
     p.xg_out = h->xg;
     p.g_next = static_cast<const bf16 *>(g_next);
@@ -448,6 +451,8 @@ cudaError_t attention(wf_handle *h, const bf16 *q, const bf16 *kc, const bf16 *v
   p.n_heads = h->H;
   p.ctx = ctx;
   p.mode = mode;
+  p.spin = h->spin;
+  p.outer = h->Bmax * h->H;
   if (attn_partial_floats(n_seq, rps, h->H, ctx) > h->apart_floats) return cudaErrorInvalidValue;
   if (attn_counter_slots(n_seq, rps, h->H) > h->attn_counter_cap) return cudaErrorInvalidValue;
   h->launches++;
@@ -502,7 +507,7 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.rows_per_seq = ps.rps;
     p.seq_slot = ps.slots;
     p.pos_base = h->L;
-    e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln1_g, lw.ln1_b, lw.qkv_w, p, s)
+    e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln1_g, lw.ln1_b, lw.qkv_w, p, s, nullptr, nullptr, lw.out_w, d, d)
               : ln_gemm(h, ps.x, ps.st, lw.ln1_g, lw.ln1_b, lw.qkv_w, p, s);
     if (e != cudaSuccess) return e;
   }
@@ -515,7 +520,7 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.resid = ps.x;
     p.ld_resid = d;
     p.stats_out = ps.st;
-    e = ps.sk ? skinny(h, h->att, nullptr, nullptr, nullptr, lw.out_w, p, s, lw.ln2_g, lw.ln2_b)
+    e = ps.sk ? skinny(h, h->att, nullptr, nullptr, nullptr, lw.out_w, p, s, lw.ln2_g, lw.ln2_b, lw.xq_w, d, d)
               : gemm(h, h->att, lw.out_w, p, s);
     if (e != cudaSuccess) return e;
   }
@@ -525,7 +530,7 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.bias = static_cast<const bf16 *>(lw.xq_b);
     p.out_bf16 = h->q;
     p.ld_out = d;
-    e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s)
+    e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s, nullptr, nullptr, lw.xout_w, d, d)
               : ln_gemm(h, ps.x, ps.st, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s);
     if (e != cudaSuccess) return e;
   }
@@ -538,7 +543,8 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.resid = ps.x;
     p.ld_resid = d;
     p.stats_out = ps.st;
-    e = ps.sk ? skinny(h, h->att, nullptr, nullptr, nullptr, lw.xout_w, p, s, lw.ln3_g, lw.ln3_b)
+    e = ps.sk ? skinny(h, h->att, nullptr, nullptr, nullptr, lw.xout_w, p, s, lw.ln3_g, lw.ln3_b, lw.fc1_w,
+                       h->F, d)
               : gemm(h, h->att, lw.xout_w, p, s);
     if (e != cudaSuccess) return e;
   }
@@ -548,7 +554,8 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.bias = static_cast<const bf16 *>(lw.fc1_b);
     p.out_bf16 = h->h1;
     p.ld_out = h->F;
-    e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln3_g, lw.ln3_b, lw.fc1_w, p, s)
+    e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln3_g, lw.ln3_b, lw.fc1_w, p, s, nullptr, nullptr, lw.fc2_w, d,
+                       h->F)
               : ln_gemm(h, ps.x, ps.st, lw.ln3_g, lw.ln3_b, lw.fc1_w, p, s);
     if (e != cudaSuccess) return e;
   }
@@ -571,7 +578,7 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
       p.ld_tap = h->cfg.n_taps * d;
     }
     e = ps.sk ? skinny(h, h->h1, nullptr, nullptr, nullptr, lw.fc2_w, p, s, next ? next->ln1_g : nullptr,
-                       next ? next->ln1_b : nullptr)
+                       next ? next->ln1_b : nullptr, next ? next->qkv_w : nullptr, 3 * d, d)
               : gemm(h, h->h1, lw.fc2_w, p, s);
     if (e != cudaSuccess) return e;
   }

@@ -11,8 +11,10 @@
 //  - mode 2, cross: all encoder frames (cross-attention, Sec. 3.2).
 //
 // A CTA takes one (sequence, head, group of <= 16 query rows, block of 256
-// keys).  Keys and values stream into XOR-swizzled shared memory with
-// cp.async (rows past the cache length are zero-filled); each of the eight
+// keys).  Keys and values arrive as two TMA copies of 32 KB (the caches are
+// 3-D tensors (64, position, slot * heads), 128-byte swizzled in shared
+// memory; rows past the cache are zero-filled by the copy, value rows past
+// the visible keys are zeroed after it); each of the eight
 // warps multiplies the 16 query rows against its 32 keys on the tensor cores
 // (mma.sync m16n8k16, bf16 in, fp32 accumulate), keeps the row maxima and
 // sums in fp32 and forms P V the same way.  Warps combine in order, and the
@@ -20,7 +22,9 @@
 // order.  Blocks and warps are aligned to absolute key positions and a key a
 // query cannot see contributes an exact zero, so a query's result does not
 // depend on how many other rows run with it.
+#include <map>
 #include <mutex>
+#include <tuple>
 
 #include "wf_device.cuh"
 #include "wf_internal.h"
@@ -41,8 +45,9 @@ constexpr int kPartStride = 2 + 64;   // m, l, o[64]
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr int kSmemK = kKB * 128;     // bytes
 constexpr int kSmemQ = kQG * 128;
-// K, V, Q, then the warps' (m, l); the warps' O partials reuse the K tile
-constexpr int kSmemAttn = 2 * kSmemK + kSmemQ + kWarps * kQG * 2 * 4 + 16;
+// K, V, Q, then the warps' (m, l); the warps' O partials reuse the K tile.
+// The K and V tiles start 1024-aligned (the copies swizzle by address).
+constexpr int kSmemAttn = 1024 + 2 * kSmemK + kSmemQ + kWarps * kQG * 2 * 4 + 16;
 static_assert(kWarps * kQG * 64 * 4 <= kSmemK, "O partials must fit in the key tile");
 static_assert(kQG * 8 <= kThreadsA && kDPT * kThreadsA == kQG * 64, "thread mapping");
 // A launch with fewer CTAs than SMs asks for enough shared memory that no two
@@ -50,18 +55,6 @@ static_assert(kQG * 8 <= kThreadsA && kDPT * kThreadsA == kQG * 64, "thread mapp
 // under programmatic dependent launch); a larger one packs three per SM.
 constexpr int kSmemAttnSpread = 116 * 1024;
 
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, bool valid) {
-  const int n = valid ? 16 : 0;  // zero-fill when the source row is past the cache
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(n)
-               : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() {
-  asm volatile("cp.async.commit_group;" ::: "memory");
-}
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
 // kDPT consecutive output dims (scaled by inv) as bf16
 __device__ __forceinline__ void store_row(bf16 *orow, const float (&v)[kDPT], float inv) {
   uint32_t w[kDPT / 2];
@@ -74,8 +67,12 @@ __device__ __forceinline__ void store_row(bf16 *orow, const float (&v)[kDPT], fl
     *reinterpret_cast<uint2 *>(orow) = make_uint2(w[0], w[1]);
   }
 }
-__global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p) {
-  extern __shared__ __align__(128) uint8_t smem[];
+__global__ void __launch_bounds__(kThreadsA) attention_kernel(const __grid_constant__ CUtensorMap tmK,
+                                                              const __grid_constant__ CUtensorMap tmV,
+                                                              const AttnParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_u32 = smem_u32(smem_raw);
+  uint8_t *smem = smem_raw + (((raw_u32 + 1023u) & ~1023u) - raw_u32);
   uint8_t *sK = smem;
   uint8_t *sV = smem + kSmemK;
   uint8_t *sQ = smem + 2 * kSmemK;
@@ -83,6 +80,7 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
   float *sl = sm + kWarps * kQG;                                     // [kWarps][16]
   float *so = reinterpret_cast<float *>(sK);  // [kWarps][16][64], once every warp is done with K
   __shared__ int s_last;
+  __shared__ uint64_t s_bar[2];  // [0] keys, [1] values
 
   const int blk = blockIdx.x;
   const int h = blockIdx.y % p.n_heads;
@@ -124,48 +122,37 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
   const size_t cache_off = (static_cast<size_t>(slot) * p.n_heads + h) * p.ctx;
   const int key0 = blk * kKB;
 
-  // ---- keys and values: cp.async, zero-filled past the cache length.  Rows
-  // below `fresh` are settled before this kernel starts; rows from `fresh`
-  // on are written by this step's projection and load after the wait.
+  // ---- keys and values: one TMA copy each.  A block holding rows that this
+  // step's projection writes (positions from `fresh` on) loads after the
+  // wait; a block of settled rows streams in while the producer of the
+  // queries finishes.
   const int fresh = p.mode == 2 ? n_keys : base;
-  {
-    const uint32_t k_u32 = smem_u32(sK), v_u32 = smem_u32(sV);
-#pragma unroll 4
-    for (int idx = tid; idx < kKB * 8; idx += kThreadsA) {
-      const int kr = idx >> 3, ch = idx & 7;
-      const int pos = key0 + kr;
-      if (pos >= fresh && pos < n_keys) continue;
-      const bool valid = pos < n_keys;
-      const size_t off = (cache_off + (valid ? pos : 0)) * 64 + ch * 8;
-      cp_async16(k_u32 + swz(kr, ch), p.kc + off, valid);
+  const bool any_keys = key0 < n_keys;
+  const bool has_fresh = any_keys && fresh < n_keys && key0 + kKB > fresh;
+  const int cache_row = slot * p.n_heads + h;
+  const uint32_t tile_bytes = static_cast<uint32_t>(min(kKB, p.ctx)) * 128u;  // the maps' box
+  if (tid == 0) {
+    mbar_init(&s_bar[0], 1);
+    mbar_init(&s_bar[1], 1);
+    fence_barrier_init();
+    if (any_keys && !has_fresh) {
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmV);
+      mbar_arrive_expect_tx(&s_bar[0], tile_bytes);
+      tma_load_3d(sK, &tmK, 0, key0, cache_row, &s_bar[0]);
+      mbar_arrive_expect_tx(&s_bar[1], tile_bytes);
+      tma_load_3d(sV, &tmV, 0, key0, cache_row, &s_bar[1]);
     }
-    cp_async_commit();
-#pragma unroll 4
-    for (int idx = tid; idx < kKB * 8; idx += kThreadsA) {
-      const int kr = idx >> 3, ch = idx & 7;
-      const int pos = key0 + kr;
-      if (pos >= fresh && pos < n_keys) continue;
-      const bool valid = pos < n_keys;
-      const size_t off = (cache_off + (valid ? pos : 0)) * 64 + ch * 8;
-      cp_async16(v_u32 + swz(kr, ch), p.vc + off, valid);
-    }
-    cp_async_commit();
   }
   pdl_wait();
   pdl_launch_dependents();
-  const bool has_fresh = fresh < n_keys && key0 + kKB > fresh;
-  if (has_fresh) {
-    const uint32_t k_u32 = smem_u32(sK), v_u32 = smem_u32(sV);
-    for (int idx = tid; idx < kKB * 8; idx += kThreadsA) {
-      const int kr = idx >> 3, ch = idx & 7;
-      const int pos = key0 + kr;
-      if (pos < fresh || pos >= n_keys) continue;
-      const size_t off = (cache_off + pos) * 64 + ch * 8;
-      cp_async16(k_u32 + swz(kr, ch), p.kc + off, true);
-      cp_async16(v_u32 + swz(kr, ch), p.vc + off, true);
-    }
-    cp_async_commit();
+  if (tid == 0 && has_fresh) {
+    mbar_arrive_expect_tx(&s_bar[0], tile_bytes);
+    tma_load_3d(sK, &tmK, 0, key0, cache_row, &s_bar[0]);
+    mbar_arrive_expect_tx(&s_bar[1], tile_bytes);
+    tma_load_3d(sV, &tmV, 0, key0, cache_row, &s_bar[1]);
   }
+  const long long spin = p.spin > 0 ? p.spin : kSpinLimitCycles;
   // ---- queries, pre-scaled by 1/8 = 1/sqrt(64) (exact in binary), RoPE in fp32
   if (tid < kQG * 8) {
     const int r = tid >> 3, ch = tid & 7;
@@ -196,11 +183,14 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
     o.w = pack_bf16(f[6], f[7]);
     *reinterpret_cast<uint4 *>(sQ + swz(r, ch)) = o;
   }
-  // keys (and this step's rows) first; the acoustic values keep streaming
-  // while the scores are formed
-  if (has_fresh) cp_async_wait<0>();
-  else cp_async_wait<1>();
+  // keys first; the values keep streaming while the scores are formed.  After
+  // a timeout thread 0 waits (bounded) for both copies before going on, so
+  // no copy lands in a CTA that has exited.
   __syncthreads();
+  if (any_keys && !mbar_wait(&s_bar[0], 0, p.err, spin) && tid == 0) {
+    mbar_drain(&s_bar[0], 0);
+    mbar_drain(&s_bar[1], 0);
+  }
 
   // ---- RoPE on the keys (drafter): dims i and i+32 rotate by pos * base^(-2i/64)
   if (p.rope_tab) {
@@ -284,10 +274,16 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const AttnParams p
     lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 1);
     lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 2);
   }
-  if (!has_fresh) {
-    cp_async_wait<0>();  // the values
-    __syncthreads();
+  // the values; rows past the visible keys (stale cache rows, rows past the
+  // copy, or a block with no visible key at all) become zeros, so P V adds
+  // exact zeros there
+  if (any_keys && !mbar_wait(&s_bar[1], 0, p.err, spin) && tid == 0) mbar_drain(&s_bar[1], 0);
+  {
+    const int z0 = min(max(n_keys - key0, 0), kKB);
+    for (int idx = tid; idx < (kKB - z0) * 8; idx += kThreadsA)
+      *reinterpret_cast<uint4 *>(sV + swz(z0 + (idx >> 3), idx & 7)) = make_uint4(0u, 0u, 0u, 0u);
   }
+  __syncthreads();
   // O = P V (P rounded to bf16 as the A operand)
   float o[8][4];
 #pragma unroll
@@ -500,6 +496,27 @@ int attn_counter_slots(int n_seq, int rps, int n_heads) {
   return n_seq * n_heads * ((rps + kQG - 1) / kQG);
 }
 
+// Tensor maps of the caches, encoded once per (cache, ctx, outer): 3-D
+// (64 dims, ctx positions, outer = slot * heads + head) with a box of one
+// (slot, head)'s 256 positions, 128-byte swizzled; positions past ctx read
+// as zeros.
+static const CUtensorMap *attn_tmap(const void *cache, int ctx, int outer) {
+  static std::mutex mu;
+  static std::map<std::tuple<uintptr_t, int, int>, CUtensorMap *> maps;
+  std::lock_guard<std::mutex> lock(mu);
+  const auto key = std::make_tuple(reinterpret_cast<uintptr_t>(cache), ctx, outer);
+  auto it = maps.find(key);
+  if (it != maps.end()) return it->second;
+  CUtensorMap *m = new CUtensorMap;
+  if (!tmap_bf16_cache(m, cache, static_cast<uint64_t>(ctx), static_cast<uint64_t>(outer),
+                       static_cast<uint32_t>(ctx < kKB ? ctx : kKB))) {
+    delete m;
+    return nullptr;
+  }
+  maps.emplace(key, m);
+  return m;
+}
+
 cudaError_t attention_init() {
   static cudaError_t status = cudaErrorNotReady;
   static std::once_flag once;
@@ -548,7 +565,10 @@ cudaError_t launch_attention(const AttnParams &p0, cudaStream_t s, bool pdl) {
   }
   cfg.attrs = attr;
   cfg.numAttrs = na;
-  return cudaLaunchKernelEx(&cfg, attention_kernel, p);
+  if (p.outer < 1) return cudaErrorInvalidValue;
+  const CUtensorMap *tk = attn_tmap(p.kc, p.ctx, p.outer), *tv = attn_tmap(p.vc, p.ctx, p.outer);
+  if (!tk || !tv) return cudaErrorInvalidValue;
+  return cudaLaunchKernelEx(&cfg, attention_kernel, *tk, *tv, p);
 }
 
 cudaError_t launch_rope_table(float2 *tab, int max_pos, float base, cudaStream_t s) {
@@ -592,6 +612,7 @@ extern "C" wf_status wf_attention(const void *d_q, const void *d_kc, const void 
   p.n_heads = n_heads;
   p.ctx = ctx;
   p.mode = mode;
+  p.outer = wf::kAttnOuterBound;
   const size_t pf = wf::attn_partial_floats(n_seq, RPS, n_heads, ctx);
   p.part = static_cast<float *>(d_scratch);
   p.counters = reinterpret_cast<int32_t *>(static_cast<char *>(d_scratch) + pf * sizeof(float));
@@ -673,6 +694,7 @@ extern "C" wf_status wf_attention_noalloc(const void *d_q, const void *d_kc, con
   p.n_heads = n_heads;
   p.ctx = ctx;
   p.mode = mode;
+  p.outer = wf::kAttnOuterBound;
   const size_t pf = wf::attn_partial_floats(n_seq, RPS, n_heads, ctx);
   const size_t counters = static_cast<size_t>(wf::attn_counter_slots(n_seq, RPS, n_heads)) * 4;
   p.part = static_cast<float *>(scratch);

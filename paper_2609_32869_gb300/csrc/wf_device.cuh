@@ -91,6 +91,15 @@ __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap *m) {
 }
 // 2-D tiled bulk-tensor load into shared memory; completes tx bytes on `bar`.
 // x is the innermost coordinate (elements), y the row.
+// 3-D tiled bulk-tensor load into shared memory; completes tx bytes on `bar`.
+__device__ __forceinline__ void tma_load_3d(void *smem_dst, const CUtensorMap *m, int32_t x, int32_t y,
+                                            int32_t z, uint64_t *bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      : "memory");
+}
 __device__ __forceinline__ void tma_load_2d(void *smem_dst, const CUtensorMap *m, int32_t x,
                                             int32_t y, uint64_t *bar) {
   asm volatile(

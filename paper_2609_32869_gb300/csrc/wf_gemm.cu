@@ -722,6 +722,20 @@ bool tmap_bf16_rows(CUtensorMap *m, const void *ptr, uint32_t rows, uint64_t col
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool tmap_bf16_cache(CUtensorMap *m, const void *ptr, uint64_t ctx, uint64_t outer, uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn || (reinterpret_cast<uintptr_t>(ptr) & 15) || ctx == 0 || outer == 0 || box_rows == 0 || box_rows > 256 ||
+      box_rows > ctx)
+    return false;
+  cuuint64_t gdim[3] = {64, ctx, outer};
+  cuuint64_t gstride[2] = {128, ctx * 128};
+  cuuint32_t box[3] = {64, box_rows, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), gdim, gstride, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 void gemm_token_tiling(int M, int *BT, int *n_tt) {
   const int nt = (M + kMaxBT - 1) / kMaxBT;
   const int per = (M + nt - 1) / nt;

@@ -98,6 +98,9 @@ bool tmap_bf16_units(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t co
 // All `rows` rows of a [rows][cols] matrix (row stride ld elements) over
 // kblocks 64-column blocks per copy: box {64, rows, kblocks}.
 bool tmap_bf16_rows(CUtensorMap *m, const void *ptr, uint32_t rows, uint64_t cols, uint64_t ld, uint32_t kblocks);
+// A key/value cache [outer][ctx][64] bf16 as (64 dims, position, outer) with a
+// box of {64, box_rows, 1}, 128-byte swizzled; positions past ctx read as 0.
+bool tmap_bf16_cache(CUtensorMap *m, const void *ptr, uint64_t ctx, uint64_t outer, uint32_t box_rows);
 
 // Token tile for M rows: a multiple of 16, at most 128.
 void gemm_token_tiling(int M, int *BT, int *n_tt);
@@ -163,6 +166,10 @@ struct SkinnyParams {
   int q_cols, d_model, n_heads, ctx, rows_per_seq;
   bf16 *kc, *vc;
   const int32_t *seq_slot, *pos_base;
+  // nullable: weights of the next projection in the chain, brought into L2
+  // in the prologue (pf_bytes, a multiple of 16, 16-byte aligned)
+  const void *pf;
+  size_t pf_bytes;
   uint32_t *err;
   long long spin;
 };
@@ -183,11 +190,16 @@ struct AttnParams {
   float *part;
   int32_t *counters;
   uint32_t *err;
+  long long spin;  // bounded-wait limit (clock cycles; 0: the default)
   int n_seq, rps, n_heads, ctx, mode, n_chunks, qgroups;
+  int outer;    // bound on slot * n_heads + head (the caches' tensor maps)
   int cluster;  // the n_chunks blocks of a (sequence, head, group) form a cluster
 };
 constexpr int kAttnKeysPerCTA = 256;  // keys per CTA (32 per warp), aligned to absolute positions
 constexpr int kAttnQGroup = 16;       // query rows per CTA
+// slot * n_heads + head stays below this in calls that do not state the
+// number of cache slots (the kernel-level entry points)
+constexpr int kAttnOuterBound = 1 << 20;
 cudaError_t attention_init();
 size_t attn_partial_floats(int n_seq, int rps, int n_heads, int ctx);
 int attn_counter_slots(int n_seq, int rps, int n_heads);

@@ -168,15 +168,6 @@ __device__ __forceinline__ bool wait_bar_idle(uint64_t *bar, uint32_t parity, ui
   }
   return true;
 }
-// 3-D tiled bulk-tensor load (a whole projection unit) into shared memory.
-__device__ __forceinline__ void tma_load_3d(void *smem_dst, const CUtensorMap *m, int32_t x, int32_t y,
-                                            int32_t z, uint64_t *bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(smem_dst)),
-      "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
-      : "memory");
-}
 __device__ __forceinline__ void mbar_arrive1(uint64_t *bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }

@@ -49,13 +49,27 @@ constexpr int kSkWarps = kSkThreads / 32;
 // fit on one SM's 228 KB with the per-CTA reserve.
 constexpr int kSkSmemBudget = 113 * 1024;
 
-__device__ __forceinline__ void tma_load_3d(void *smem_dst, const CUtensorMap *m, int32_t x, int32_t y,
-                                            int32_t z, uint64_t *bar) {
+
+// The same copy marked evict-first in L2: a step streams every weight once
+// (far more bytes than L2 holds), so the weights should not push out the
+// small activations and statistics that the next launches read.
+__device__ __forceinline__ void tma_load_3d_stream(void *smem_dst, const CUtensorMap *m, int32_t x,
+                                                   int32_t y, int32_t z, uint64_t *bar, uint64_t policy) {
   asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(smem_dst)),
-      "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_u32(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "l"(policy)
       : "memory");
+}
+__device__ __forceinline__ uint64_t l2_evict_first_policy() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+// Bring [src, src + bytes) into L2 (16-byte aligned, size a multiple of 16).
+__device__ __forceinline__ void l2_prefetch_bulk(const void *src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(src)), "r"(bytes)
+               : "memory");
 }
 
 // Shared-memory layout of one CTA (offsets from the 1024-aligned base).  The
@@ -148,8 +162,19 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
     *sZero = make_uint4(0u, 0u, 0u, 0u);
     // the whole weight slab: one copy per unit, before the dependency wait
     mbar_arrive_expect_tx(&bar[0], static_cast<uint32_t>(U * unit_bytes));
+    const uint64_t pol = l2_evict_first_policy();
     for (int u = 0; u < U; ++u)
-      tma_load_3d(sW + static_cast<size_t>(u) * unit_bytes, &tmW, 0, (unit0 + u) * 8, split * kb, &bar[0]);
+      tma_load_3d_stream(sW + static_cast<size_t>(u) * unit_bytes, &tmW, 0, (unit0 + u) * 8, split * kb, &bar[0],
+                         pol);
+    // this CTA's share of the next projection's weights, into L2
+    if (p.pf) {
+      const size_t n_cta = static_cast<size_t>(gridDim.x) * gridDim.z;
+      const size_t share = ((p.pf_bytes + n_cta - 1) / n_cta + 15) & ~static_cast<size_t>(15);
+      const size_t lo = (static_cast<size_t>(split) * gridDim.x + cta) * share;
+      const size_t hi = lo + share < p.pf_bytes ? lo + share : p.pf_bytes;
+      for (size_t off = lo; off < hi; off += 32768)
+        l2_prefetch_bulk(static_cast<const uint8_t *>(p.pf) + off, static_cast<uint32_t>(hi - off < 32768 ? hi - off : 32768));
+    }
   }
   for (int i = tid; i < U * 8; i += kSkThreads) {
     const int n = n_base + i;
