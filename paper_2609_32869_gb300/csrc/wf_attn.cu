@@ -119,7 +119,6 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const __grid_const
   if (blk >= n_blocks && !(p.cluster && n_blocks > 1)) return;
 
   const int d_model = p.n_heads * 64;
-  const size_t cache_off = (static_cast<size_t>(slot) * p.n_heads + h) * p.ctx;
   const int key0 = blk * kKB;
 
   // ---- keys and values: one TMA copy each.  A block holding rows that this
@@ -417,15 +416,18 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const __grid_const
 #pragma unroll
     for (int e = 0; e < kDPT; ++e) pe[2 + d0 + e] = acc[e];
   }
-  __threadfence();
+  // one fence per CTA: after the barrier thread 0 releases the whole CTA's
+  // partial at GPU scope and counts it; the last CTA's thread 0 fences again
+  // (acquire) before the barrier that releases its threads into the combine
   __syncthreads();
   if (tid == 0) {
-    const int prev = atomicAdd(&p.counters[group_id], 1);
-    s_last = (prev == n_blocks - 1);
+    __threadfence();
+    const int last = atomicAdd(&p.counters[group_id], 1) == n_blocks - 1;
+    if (last) __threadfence();
+    s_last = last;
   }
   __syncthreads();
   if (!s_last) return;
-  __threadfence();
   // A block the query cannot see carries m = -inf, l = 0, o = 0 and gets
   // weight 0, so it adds exact zeros; the loads of all blocks are independent.
   if (qi < nq) {
