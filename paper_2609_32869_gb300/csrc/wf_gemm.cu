@@ -17,7 +17,12 @@
 // its own shared memory and, past a cluster barrier, reduces a slice of the
 // tile by reading the S partials over distributed shared memory in split
 // order, so results are deterministic and independent of M, and no partial
-// ever travels through global memory.
+// ever travels through global memory.  When the token tiles alone give
+// enough CTAs (many sequences), one CTA computes all S splits of its tile in
+// turn ("fold"): the MMA thread alternates the splits between two TMEM
+// accumulators while four warps add each finished partial, in split order,
+// into a third -- the same sums in the same order as the cluster reduction,
+// without its S-fold CTAs, barriers and partial tiles.
 //
 // With programmatic dependent launch the weight tiles of the first pipeline
 // stages are requested before griddepcontrol.wait: they do not depend on the
@@ -41,10 +46,12 @@ constexpr int kStageA = kBlockN * kBlockK * 2;  // 16 KB
 // Shared memory a CTA plans for: two CTAs fit on an SM, so one CTA's
 // epilogue overlaps the other's weight stream.
 constexpr int kSmemBudget = 110 * 1024;
+constexpr int kSmemBudgetAlone = 200 * 1024;  // a CTA that holds all 512 TMEM columns
 constexpr int kSmemBudgetLn = 110 * 1024;  // LN mode: resident token tiles + weight ring
 constexpr int kMaxBT = 128;                // token rows per tile (MMA N)
 constexpr size_t kSmemPerSM = 228 * 1024;  // shared memory of one SM
 constexpr int kLnFuseMaxM = 256;              // token rows up to which LN is fused
+constexpr int kFoldMinTiles = 64;             // output tiles from which split-K folds into one CTA
 
 __device__ __forceinline__ void head_combine(float &m, float &s, int &arg, float &gm, int &garg,
                                              float m2, float s2, int arg2, float gm2, int garg2) {
@@ -289,9 +296,11 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
   uint64_t *full = reinterpret_cast<uint64_t *>(smem + p.pipe_bytes);
   uint64_t *empty = full + stages;
   uint64_t *done = empty + stages;
-  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
+  uint64_t *part_bar = done + 1;  // fold: split partial r finished in accumulator r % 2
+  uint64_t *free_bar = done + 3;  // fold: accumulator r % 2 added into the sum, free again
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 5);
   // per-token (slot, position) for EPI_KV, (slot, step) for sampling heads
-  int2 *tok = reinterpret_cast<int2 *>(smem + p.pipe_bytes + (2 * stages + 1) * 8 + 16 + 16);
+  int2 *tok = reinterpret_cast<int2 *>(smem + p.pipe_bytes + (2 * stages + 5) * 8 + 16 + 16);
   float2 *lnst = reinterpret_cast<float2 *>(tok + BT);  // per-token (mean, rstd), LN mode
   const bool ln = p.ln_x != nullptr;
   // a bounded wait of this CTA gave up (in the 32 bytes reserved after the
@@ -300,7 +309,9 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int tt = blockIdx.x, ntile = blockIdx.y, split = blockIdx.z;
-  const int n0 = ntile * kBlockN, t0 = tt * BT, kit0 = split * kps;
+  const bool fold = p.fold != 0;
+  const int nk = fold ? kps * p.splits : kps;  // k-steps of this CTA
+  const int n0 = ntile * kBlockN, t0 = tt * BT, kit0 = fold ? 0 : split * kps;
 
   if (threadIdx.x == 0) {
     s_timed_out = 0;
@@ -311,6 +322,10 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
       mbar_init(&empty[s], 1);
     }
     mbar_init(done, 1);
+    mbar_init(&part_bar[0], 1);
+    mbar_init(&part_bar[1], 1);
+    mbar_init(&free_bar[0], 4);
+    mbar_init(&free_bar[1], 4);
     fence_barrier_init();
     fence_proxy_async();
   }
@@ -324,7 +339,7 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
   // Weight tiles of the first stages do not depend on the previous kernel:
   // request them before the dependency wait.  In LN mode each stage carries
   // only its weight tile; the token operand is built once for all k-steps.
-  const int npre = kps < stages ? kps : stages;
+  const int npre = nk < stages ? nk : stages;
   const uint32_t tx = ln ? static_cast<uint32_t>(kStageA) : kStageA + stageB;
   if (threadIdx.x == 0) {
     for (int i = 0; i < npre; ++i) {
@@ -347,7 +362,7 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
       for (int i = 0; i < npre; ++i)
         tma_load_2d(sB + static_cast<size_t>(i) * stageB, &tmX, (kit0 + i) * kBlockK, t0, &full[i]);
     }
-    for (int it = npre; it < kps; ++it) {
+    for (int it = npre; it < nk; ++it) {
       const int s = it % stages;
       const uint32_t ph = static_cast<uint32_t>((it / stages) - 1) & 1u;
       if (!mbar_wait(&empty[s], ph, p.err, p.spin)) {
@@ -369,7 +384,7 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
     // rate, so the loop keeps everything but the MMAs out of the way.
     const uint32_t idesc = umma_idesc_bf16(kBlockN, BT);
     const uint64_t a_base = umma_desc_sw128(smem_u32(sA)), b_base = umma_desc_sw128(smem_u32(sB));
-    if (kps <= stages) {
+    if (!fold && kps <= stages) {
       // every k-step has its own stage and none is refilled: wait for all
       // of them, then issue the MMAs back to back (no per-stage commit)
       bool landed = true;
@@ -386,27 +401,72 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
         }
       }
     } else {
-      for (int it = 0; it < kps; ++it) {
+      for (int it = 0; it < nk; ++it) {
         const int s = it % stages;
         const uint32_t ph = static_cast<uint32_t>(it / stages) & 1u;
         if (!mbar_wait(&full[s], ph, p.err, p.spin)) {
           s_timed_out = 1;
           break;
         }
+        // fold: split r = it / kps accumulates in columns (r % 2) acc_cols,
+        // once the sum has taken split r - 2 out of them
+        const int r = it / kps, kin = it - r * kps;
+        if (fold && kin == 0 && r >= 2 &&
+            !mbar_wait(&free_bar[r & 1], static_cast<uint32_t>((r >> 1) - 1) & 1u, p.err, p.spin)) {
+          s_timed_out = 1;
+          break;
+        }
         tc_fence_after();
+        const uint32_t dacc = tmem + (fold ? static_cast<uint32_t>(r & 1) * p.acc_cols : 0u);
         const uint64_t ad = a_base + static_cast<uint64_t>((s * kStageA) >> 4);
         const uint64_t bd = b_base + static_cast<uint64_t>(((ln ? it : s) * stageB) >> 4);
 #pragma unroll
         for (int kk = 0; kk < kBlockK / 16; ++kk)
-          umma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (it | kk) != 0 ? 1u : 0u);
+          umma_bf16(dacc, ad + 2 * kk, bd + 2 * kk, idesc, (kin | kk) != 0 ? 1u : 0u);
         umma_commit(&empty[s]);
+        if (fold && kin == kps - 1) umma_commit(&part_bar[r & 1]);
       }
     }
     umma_commit(done);
   }
   __syncwarp();
 
+  // ---------------- fold: warps 4..7 (TMEM lane quarters 0..3) add each split
+  // partial into the sum columns 2 acc_cols.., in split order from zero
+  if (fold && warp >= 4) {
+    const uint32_t lbase = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+    const uint32_t sum_col = lbase + 2 * p.acc_cols;
+    const int n_ch = BT / 16;
+    for (int r = 0; r < p.splits; ++r) {
+      if (!mbar_wait(&part_bar[r & 1], static_cast<uint32_t>(r >> 1) & 1u, p.err, p.spin)) {
+        s_timed_out = 1;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t part_col = lbase + static_cast<uint32_t>(r & 1) * p.acc_cols;
+      for (int c = 0; c < n_ch; ++c) {
+        float v[16], a[16];
+        tmem_ld16(part_col + c * 16, v);
+        if (r == 0) {
+#pragma unroll
+          for (int e = 0; e < 16; ++e) a[e] = 0.f + v[e];
+        } else {
+          tmem_ld16(sum_col + c * 16, a);
+#pragma unroll
+          for (int e = 0; e < 16; ++e) a[e] += v[e];
+        }
+        tmem_st16(sum_col + c * 16, a);
+      }
+      tmem_st_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cta(&free_bar[r & 1]);
+    }
+  }
+
   // ---------------- epilogue: warp w owns TMEM lanes [32w, 32w+32) = weight rows
+  // (fold: the sum columns; S_eff = 1, the CTA finishes every row of its tile)
+  const int S_eff = fold ? 1 : p.splits;
   pdl_wait();
   if constexpr (EPI == EPI_HEAD) {
     if (p.temperature > 0.f) {
@@ -441,14 +501,14 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
   float b4[4] = {0.f, 0.f, 0.f, 0.f};
   float4 pre = make_float4(0.f, 0.f, 0.f, 0.f);
   bool has_pre = false;
-  if (EPI != EPI_HEAD && (p.splits > 1 || p.stats_out)) {
+  if (EPI != EPI_HEAD && (S_eff > 1 || p.stats_out)) {
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const int nn = n0 + 4 * lane + i;
       b4[i] = (p.bias && nn < p.N) ? bf2f(p.bias[nn]) : 0.f;
     }
     if constexpr (EPI == EPI_RESID) {
-      const int S = p.splits, tl = cols * split / S + warp;
+      const int S = S_eff, tl = cols * split / S + warp;
       if (tl < cols * (split + 1) / S) {
         pre = *reinterpret_cast<const float4 *>(p.resid + static_cast<size_t>(t0 + tl) * p.ld_resid +
                                                 n0 + 4 * lane);
@@ -465,7 +525,8 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
   // token-column chunks [c_lo, c_hi) of its half of the tile
   const int quarter = warp & 3, half = warp >> 2;
   const int n = n0 + quarter * 32 + lane;
-  const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+  const uint32_t trow =
+      tmem + (static_cast<uint32_t>(quarter * 32) << 16) + (fold ? 2 * p.acc_cols : 0u);
   const int n_chunks = BT / 16, c_per = (n_chunks + 1) / 2;
   const int c_lo = half * c_per, c_hi = min(n_chunks, c_lo + c_per);
 
@@ -527,7 +588,7 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
         p.recs[static_cast<size_t>(t) * n_tiles + ntile] = rec;
       }
     }
-  } else if (p.splits == 1 && !p.stats_out) {
+  } else if (S_eff == 1 && !p.stats_out) {
     const float bn = (p.bias && n < p.N) ? bf2f(p.bias[n]) : 0.f;
     for (int c = c_lo; c < c_hi; ++c) {
       float v[16];
@@ -538,8 +599,8 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
     // Four-feature epilogue: a warp owns a token row (lane l: features
     // 4l..4l+3), so the row's LayerNorm statistics over this 128-feature tile
     // are two warp reductions.  Split-K partials are summed in split order.
-    const int S = p.splits;
-    const int rank = split;  // cluster (1, 1, S) over gridDim.z == S: rank == blockIdx.z
+    const int S = S_eff;
+    const int rank = fold ? 0 : split;  // cluster (1, 1, S) over gridDim.z == S: rank == blockIdx.z
     const int rlo = cols * rank / S, rhi = cols * (rank + 1) / S;
     const int stat_tiles = p.N / kBlockN;
     // the residual row a warp updates next (EPI_RESID; the first one was
@@ -786,8 +847,9 @@ static cudaError_t cluster_fits(int splits, size_t smem, dim3 grid) {
 template <int EPI>
 static cudaError_t launch_typed(const CUtensorMap *tw, const CUtensorMap *tx, const GemmParams &p,
                                 size_t smem, cudaStream_t s, bool pdl) {
-  const dim3 grid(p.n_tt, (p.N + kBlockN - 1) / kBlockN, p.splits);
-  if (p.splits > 1) {
+  const bool clustered = p.splits > 1 && !p.fold;
+  const dim3 grid(p.n_tt, (p.N + kBlockN - 1) / kBlockN, clustered ? p.splits : 1);
+  if (clustered) {
     cudaError_t e = cluster_fits<EPI>(p.splits, smem, grid);
     if (e != cudaSuccess) return e;
   }
@@ -798,7 +860,7 @@ static cudaError_t launch_typed(const CUtensorMap *tw, const CUtensorMap *tx, co
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   int na = 0;
-  if (p.splits > 1) {
+  if (clustered) {
     attr[na].id = cudaLaunchAttributeClusterDimension;
     attr[na].val.clusterDim.x = 1;
     attr[na].val.clusterDim.y = 1;
@@ -857,9 +919,24 @@ static bool plan_gemm(GemmParams &p, size_t *smem_out) {
   if (k_iters % p.splits) return false;
   p.kps = k_iters / p.splits;
   const bool ln = p.ln_x != nullptr;
+  // fold the splits into one CTA when the token tiles alone fill the GPU
+  const int n_tiles = (p.N + kBlockN - 1) / kBlockN;
+  p.fold = (!ln && p.epi != EPI_HEAD && p.splits > 1 && p.n_tt * n_tiles >= kFoldMinTiles) ? 1 : 0;
   const size_t stageA = kStageA, stageB = static_cast<size_t>(p.BT) * kBlockK * 2;
   const size_t red = static_cast<size_t>(p.BT) * sizeof(int2) * (ln ? 2 : 1);
   const size_t fixed = red;
+  uint32_t cols = 32;
+  while (cols < static_cast<uint32_t>(p.BT)) cols <<= 1;
+  p.acc_cols = cols;
+  if (p.fold) {  // two split accumulators and their sum
+    uint32_t all = 32;
+    while (all < 3 * cols) all <<= 1;
+    if (all > 512) return false;
+    cols = all;
+  }
+  p.tmem_cols = cols;
+  // a CTA that holds all of TMEM is alone on its SM: it may take a deeper ring
+  const size_t budget = cols == 512 ? kSmemBudgetAlone : kSmemBudget;
   int stages;
   size_t pipe;
   if (ln) {
@@ -871,20 +948,18 @@ static bool plan_gemm(GemmParams &p, size_t *smem_out) {
     if (stages > 16) stages = 16;
     pipe = stages * stageA + btiles;
   } else {
-    if (fixed + stageA + stageB > kSmemBudget) return false;
-    stages = static_cast<int>((kSmemBudget - fixed) / (stageA + stageB));
-    if (stages > p.kps) stages = p.kps;
+    if (fixed + stageA + stageB > budget) return false;
+    stages = static_cast<int>((budget - fixed) / (stageA + stageB));
+    const int nk = p.fold ? p.kps * p.splits : p.kps;
+    if (stages > nk) stages = nk;
     if (stages > 16) stages = 16;
     pipe = stages * (stageA + stageB);
   }
   p.stages = stages;
-  uint32_t cols = 32;
-  while (cols < static_cast<uint32_t>(p.BT)) cols <<= 1;
-  p.tmem_cols = cols;
   // the staged epilogues reuse the pipeline buffers for a [BT][128] fp32 tile
-  if (p.splits > 1 || p.stats_out || p.epi == EPI_HEAD)
+  if ((p.splits > 1 && !p.fold) || p.stats_out || p.epi == EPI_HEAD)
     pipe = std::max<size_t>(pipe, 512 * static_cast<size_t>(p.BT));
-  size_t smem = 1024 + pipe + (2 * stages + 1) * 8 + 32 + 16 + red;
+  size_t smem = 1024 + pipe + (2 * stages + 5) * 8 + 32 + 16 + red;
   // A CTA blocks in tcgen05.alloc while co-resident CTAs hold the SM's 512
   // TMEM columns; CTAs of one cluster wait for each other, so no more CTAs
   // may fit on an SM (by shared memory) than can hold TMEM at once.

@@ -50,6 +50,12 @@ struct GemmParams {
   int M, N, K;
   int BT, n_tt, splits, kps, stages, pipe_bytes;
   uint32_t tmem_cols;
+  // fold != 0: one CTA computes every split of its tile in turn (the split
+  // partials alternate between two TMEM accumulators of acc_cols columns and
+  // are added in split order into a third), with the same arithmetic as the
+  // cluster reduction
+  int fold;
+  uint32_t acc_cols;
   int epi;
   const bf16 *bias;
   float *out_f32;

@@ -56,14 +56,16 @@ def test_gemm_matches_oracle(M, N, K):
 
 def test_gemm_rows_do_not_depend_on_batch():
     """A row's result is bit-identical whether it runs alone, among 9 rows, or
-    among 300 (fixed split-K and token-tile-independent reduction order)."""
+    among 300 or 1000 (fixed split-K and token-tile-independent reduction
+    order; at 1000 rows the 10 splits of a tile run in one CTA and are added
+    in the same order as the cluster reduction of the smaller launches)."""
     import torch
     from paper_2609_32869_gb300 import binding as B
     N, K = 1280, 1280
-    x = syn.normal_bf16(21, "xb", (300, K), 1.0)
+    x = syn.normal_bf16(21, "xb", (1000, K), 1.0)
     w = _dev(syn.normal_bf16(22, "wb", (N, K), 0.02))
     outs = {}
-    for M in (1, 9, 64, 65, 300):
+    for M in (1, 9, 64, 65, 300, 1000):
         y = torch.empty(M, N, dtype=torch.float32, device="cuda")
         nb = B.wf_gemm_scratch_bytes(M, N, K)
         sc = torch.empty(max(nb, 256), dtype=torch.uint8, device="cuda")
@@ -73,6 +75,7 @@ def test_gemm_rows_do_not_depend_on_batch():
     np.testing.assert_array_equal(outs[9], outs[300][:9])
     np.testing.assert_array_equal(outs[64], outs[300][:64])
     np.testing.assert_array_equal(outs[65], outs[300][:65])
+    np.testing.assert_array_equal(outs[300], outs[1000][:300])
 
 
 def _cache(n_slots, H, ctx, seed, name, std=1.0):
