@@ -476,6 +476,47 @@ struct Pass {
   bool sk;     // skinny projections (no statistics travel)
 };
 
+// The cross-query projection (LN2 folded, one sequence) fused with the
+// cross-attention of its queries over the acoustic memory xkc/xvc; the
+// attention output lands in h->att for the cross-out projection.
+cudaError_t skinny_xattn(wf_handle *h, const wf_layer_weights &lw, const bf16 *xkc, const bf16 *xvc,
+                         const Pass &ps, cudaStream_t s) {
+  const int M = ps.n_seq * ps.rps, d = h->d;
+  SkinnyParams p = {};
+  p.M = M;
+  p.N = d;
+  p.K = d;
+  p.epi = EPI_BF16;
+  p.fold = 1;
+  p.x = h->xg;
+  p.ld_x = d;
+  p.fold_part = h->fpart;
+  p.n_part = h->fold_np;
+  p.part_stride = kSkMaxParts;
+  p.ln_eps = h->cfg.ln_eps;
+  p.bias = static_cast<const bf16 *>(lw.xq_b);
+  p.out_bf16 = h->att;
+  p.ld_out = d;
+  p.kc = const_cast<bf16 *>(xkc);
+  p.vc = const_cast<bf16 *>(xvc);
+  p.ctx = h->cfg.enc_frames;
+  p.seq_slot = ps.slots;
+  p.n_heads = h->H;
+  p.d_model = d;
+  p.xa_outer = h->Bmax * h->H;
+  p.pf = lw.xout_w;
+  p.pf_bytes = static_cast<size_t>(d) * d * sizeof(bf16);
+  p.err = h->err;
+  p.spin = h->spin;
+  h->launches++;
+  prof_begin(h, s);
+  cudaError_t e = launch_skinny_xattn(lw.xq_w, p, s, kPDL);
+  // the projection's weights and operand plus the acoustic keys and values read
+  const double kv = 2.0 * ps.n_seq * h->H * static_cast<double>(h->cfg.enc_frames) * 64 * sizeof(bf16);
+  prof_end(h, s, WF_FAM_ATTN_CROSS, static_cast<double>(d) * d * sizeof(bf16) + kv);
+  return e;
+}
+
 // One pre-LayerNorm Whisper block over the pass's rows; next: the following
 // block of the pass (whose first LayerNorm a skinny pass folds), or null.
 cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, int layer,
@@ -524,19 +565,24 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
               : gemm(h, h->att, lw.out_w, p, s);
     if (e != cudaSuccess) return e;
   }
-  // cross-attention
-  {
-    GemmParams p = gemm_base(h, M, d, d, EPI_BF16);
-    p.bias = static_cast<const bf16 *>(lw.xq_b);
-    p.out_bf16 = h->q;
-    p.ld_out = d;
-    e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s, nullptr, nullptr, lw.xout_w, d, d)
-              : ln_gemm(h, ps.x, ps.st, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s);
-    if (e != cudaSuccess) return e;
+  // cross-attention: for one sequence on the skinny path, the query
+  // projection and the attention run as one kernel (a cluster per head)
+  if (ps.sk && ps.n_seq == 1 && skinny_xattn_fits(M, d, h->H, h->cfg.enc_frames)) {
+    if ((e = skinny_xattn(h, lw, xkc, xvc, ps, s)) != cudaSuccess) return e;
+  } else {
+    {
+      GemmParams p = gemm_base(h, M, d, d, EPI_BF16);
+      p.bias = static_cast<const bf16 *>(lw.xq_b);
+      p.out_bf16 = h->q;
+      p.ld_out = d;
+      e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s, nullptr, nullptr, lw.xout_w, d, d)
+                : ln_gemm(h, ps.x, ps.st, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s);
+      if (e != cudaSuccess) return e;
+    }
+    if ((e = attention(h, h->q, xkc, xvc, ps.slots, ps.n_seq, ps.rps, h->cfg.enc_frames, 2, false,
+                       s)) != cudaSuccess)
+      return e;
   }
-  if ((e = attention(h, h->q, xkc, xvc, ps.slots, ps.n_seq, ps.rps, h->cfg.enc_frames, 2, false,
-                     s)) != cudaSuccess)
-    return e;
   {
     GemmParams p = gemm_base(h, M, d, d, EPI_RESID);
     p.bias = static_cast<const bf16 *>(lw.xout_b);

@@ -172,6 +172,10 @@ struct SkinnyParams {
   int q_cols, d_model, n_heads, ctx, rows_per_seq;
   bf16 *kc, *vc;
   const int32_t *seq_slot, *pos_base;
+  // skinny_xattn: frames per CTA of the fused cross-attention (kc, vc: the
+  // acoustic keys and values, ctx frames; out_bf16: the attention output)
+  int xa_kpc;
+  int xa_outer;  // bound on slot * n_heads + head (the caches' tensor maps)
   // nullable: weights of the next projection in the chain, brought into L2
   // in the prologue (pf_bytes, a multiple of 16, 16-byte aligned)
   const void *pf;
@@ -185,6 +189,11 @@ struct SkinnyParams {
 bool skinny_plan(int M, int N, int K, bool ln, bool whole_k, int *U, int *S);
 cudaError_t skinny_init();
 cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pdl);
+// The cross-query projection (folded LN2, one sequence) fused with the
+// cross-attention of its queries: one cluster of 8 CTAs per 64-dim head.
+// False when the shapes do not allow it (then run the two separately).
+bool skinny_xattn_fits(int M, int d, int n_heads, int frames);
+cudaError_t launch_skinny_xattn(const void *W, SkinnyParams p, cudaStream_t s, bool pdl);
 
 // ------------------------------------------------------------- attention --
 struct AttnParams {

@@ -108,6 +108,9 @@ __device__ __forceinline__ uint32_t a_off(int M, int r, int k) {
 __device__ __forceinline__ void cluster_arrive_relaxed() {
   asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
 }
+__device__ __forceinline__ void dsmem_st_f32(uint32_t cluster_addr, float v) {
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(cluster_addr), "f"(v) : "memory");
+}
 __device__ __forceinline__ void dsmem_st_u32x4(uint32_t cluster_addr, uint4 v) {
   asm volatile("st.shared::cluster.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(cluster_addr), "r"(v.x), "r"(v.y),
                "r"(v.z), "r"(v.w)
@@ -497,6 +500,388 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   }
 }
 
+// ------------------------------------------- cross-query + cross-attention --
+// The cross-attention of a single sequence fused into the projection that
+// forms its queries (Sec. 3.2: the drafter and the target attend to the
+// acoustic memory; the query projection is LN2(x) W_q^T + b_q, folded as in
+// the skinny projection).  A head's 64 query columns are 8 units of 8 weight
+// rows, i.e. 8 CTAs with U = 1: the kernel runs them as one cluster per head.
+// Each CTA projects its 8 columns for the M rows (MMA as above), scales them
+// by 1/8 and writes them as one 16-byte chunk per row into the query tile of
+// every CTA of the cluster.  Each CTA then attends to its own kpc frames
+// (kpc = ceil(frames / 8) rounded up to 32; keys and values requested by TMA
+// before the dependency wait: the acoustic memory is written once, at
+// prefill), with the attention kernel's per-warp arithmetic (32 frames per
+// warp, base-2 softmax, P rounded to bf16 for P V) and its in-order warp
+// merge; the 8 CTAs' (m, l, o) then merge in rank order over distributed
+// shared memory: each CTA pushes its partial of dims 8c .. 8c + 7 into CTA c,
+// which merges the 8 it receives.  No query
+// row and no partial leaves the cluster, and a row's result depends only on
+// its own query (frames are split by position, not by rows).
+namespace {
+struct XaLayout {
+  int w_off, a_off, k_off, v_off, q_off, pb_off, sum_off, bias_off, stat_off, ml_off, bar_off, zero_off, flag_off,
+      total;
+  __host__ __device__ XaLayout(int Mr, int K, int kpc) {
+    const int kb = K / 64;
+    w_off = 0;
+    a_off = kb * 1024;
+    k_off = (a_off + kb * Mr * 128 + 1023) & ~1023;
+    v_off = k_off + kpc * 128;  // kpc a multiple of 32: 1024-aligned
+    q_off = v_off + kpc * 128;
+    pb_off = q_off + 16 * 128;
+    sum_off = pb_off + 8 * 16 * 12 * 4;
+    bias_off = sum_off + 128 * 4;
+    stat_off = bias_off + 8 * 4;
+    ml_off = stat_off + kSkMaxRows * 8;
+    bar_off = ml_off + 2 * 8 * 16 * 4;
+    zero_off = bar_off + 4 * 8;
+    flag_off = zero_off + 16;
+    total = flag_off + 16;
+  }
+};
+constexpr float kXaLog2e = 1.4426950408889634f;
+}  // namespace
+
+__global__ void __launch_bounds__(kSkThreads, 1) skinny_xattn_kernel(const __grid_constant__ CUtensorMap tmW,
+                                                                     const __grid_constant__ CUtensorMap tmX,
+                                                                     const __grid_constant__ CUtensorMap tmK,
+                                                                     const __grid_constant__ CUtensorMap tmV,
+                                                                     const SkinnyParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  uint8_t *smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+  const int M = p.M, Mr = M + 2, K = p.K, kb = K / 64, kpc = p.xa_kpc, ctx = p.ctx;
+  const XaLayout L(Mr, K, kpc);
+  uint8_t *sW = smem + L.w_off;
+  uint8_t *sA = smem + L.a_off;
+  uint8_t *sK = smem + L.k_off;
+  uint8_t *sV = smem + L.v_off;
+  uint8_t *sQ = smem + L.q_off;
+  // [8 source CTAs][16 rows][12]: m, l, -, -, o[8] of this CTA's 8 dims, pushed by each CTA
+  float *pin = reinterpret_cast<float *>(smem + L.pb_off);
+  float *sPart = reinterpret_cast<float *>(smem + L.w_off);  // [8 warps][16][8], over the slab after the MMAs
+  float *sSum = reinterpret_cast<float *>(smem + L.sum_off);  // [16][8]
+  float *sBias = reinterpret_cast<float *>(smem + L.bias_off);
+  float2 *sStat = reinterpret_cast<float2 *>(smem + L.stat_off);
+  float *sm = reinterpret_cast<float *>(smem + L.ml_off);  // [8][16]
+  float *sl = sm + 8 * 16;                                 // [8][16]
+  float *so = reinterpret_cast<float *>(sK);               // [warps][16][64], once every warp is done with K
+  uint64_t *bar = reinterpret_cast<uint64_t *>(smem + L.bar_off);  // weights, operand, keys, values
+  uint4 *sZero = reinterpret_cast<uint4 *>(smem + L.zero_off);
+  int *s_flag = reinterpret_cast<int *>(smem + L.flag_off);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int cta = blockIdx.x, head = cta >> 3;
+  const uint32_t crank = cluster_ctarank();  // == cta % 8: this CTA's 8 dims of the head
+  const int n_base = cta * 8;
+  const int nw = kpc / 32;                   // warps with frames
+  const int key0 = static_cast<int>(crank) * kpc;
+  const bool any_keys = key0 < ctx;
+  const long long spin = p.spin > 0 ? p.spin : kSpinLimitCycles;
+
+  cluster_arrive_relaxed();  // this CTA has started (peers write into it later)
+  if (tid == 0) {
+    *s_flag = 0;
+    tma_prefetch_desc(&tmW);
+    tma_prefetch_desc(&tmX);
+    for (int i = 0; i < 4; ++i) mbar_init(&bar[i], 1);
+    fence_barrier_init();
+    *sZero = make_uint4(0u, 0u, 0u, 0u);
+    mbar_arrive_expect_tx(&bar[0], static_cast<uint32_t>(kb * 1024));
+    tma_load_3d_stream(sW, &tmW, 0, n_base, 0, &bar[0], l2_evict_first_policy());
+    if (any_keys) {  // the acoustic memory of this CTA's frames
+      const int slot = p.seq_slot[0];
+      const int outer = slot * p.n_heads + head;
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmV);
+      mbar_arrive_expect_tx(&bar[2], static_cast<uint32_t>(kpc * 128));
+      tma_load_3d(sK, &tmK, 0, key0, outer, &bar[2]);
+      mbar_arrive_expect_tx(&bar[3], static_cast<uint32_t>(kpc * 128));
+      tma_load_3d(sV, &tmV, 0, key0, outer, &bar[3]);
+    }
+    if (p.pf) {  // this CTA's share of the next projection's weights, into L2
+      const size_t share = ((p.pf_bytes + gridDim.x - 1) / gridDim.x + 15) & ~static_cast<size_t>(15);
+      const size_t lo = static_cast<size_t>(cta) * share;
+      const size_t hi = lo + share < p.pf_bytes ? lo + share : p.pf_bytes;
+      for (size_t off = lo; off < hi; off += 32768)
+        l2_prefetch_bulk(static_cast<const uint8_t *>(p.pf) + off,
+                         static_cast<uint32_t>(hi - off < 32768 ? hi - off : 32768));
+    }
+  }
+  if (tid < 8) sBias[tid] = p.bias ? bf2f(p.bias[n_base + tid]) : 0.f;
+  pdl_launch_dependents();
+  pdl_wait();
+
+  // ---------------- operand (rows g, b, then g . x) and the row statistics
+  if (tid == 0) {
+    mbar_arrive_expect_tx(&bar[1], static_cast<uint32_t>(kb * Mr * 128));
+    tma_load_3d(sA, &tmX, 0, 0, 0, &bar[1]);
+  }
+  {
+    constexpr int kPL = (kSkMaxParts + 31) / 32;
+    float2 v[2][kPL];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int t = warp + kSkWarps * h;
+      const float2 *pr = p.fold_part + static_cast<size_t>(t) * p.part_stride;
+#pragma unroll
+      for (int q = 0; q < kPL; ++q) {
+        const int i = lane + 32 * q;
+        v[h][q] = (t < M && i < p.n_part) ? __ldcg(pr + i) : make_float2(0.f, 0.f);
+      }
+    }
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int t = warp + kSkWarps * h;
+      float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+      for (int q = 0; q < kPL; ++q) {
+        s1 += v[h][q].x;
+        s2 += v[h][q].y;
+      }
+      s1 = warp_sum(s1);
+      s2 = warp_sum(s2);
+      const float mu = s1 / static_cast<float>(K);
+      const float var = fmaxf(s2 / static_cast<float>(K) - mu * mu, 0.f);
+      if (lane == 0 && t < M) sStat[t] = make_float2(mu, rsqrtf(var + p.ln_eps));
+    }
+  }
+  bool ok = mbar_wait(&bar[1], 0, p.err, spin);
+  ok = mbar_wait(&bar[0], 0, p.err, spin) && ok;
+  if (!ok) *s_flag = 1;
+
+  // ---------------- the 8 query columns: warp w over k-blocks [w kb / 8, (w + 1) kb / 8)
+  float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+  if (ok) {
+    const int ar = (lane & 7) + ((lane >> 3) & 1) * 8, c0 = lane >> 4;
+    const bool real = ar < Mr;
+    const uint32_t a_base = smem_u32(sA), z_addr = smem_u32(sZero), w_base = smem_u32(sW);
+    const int br = lane & 7, bg = lane >> 3;
+    const uint32_t offB0 = br * 128 + (((bg) ^ br) << 4), offB1 = br * 128 + (((bg + 4) ^ br) << 4);
+    const int kb_lo = warp * kb / kSkWarps, kb_hi = (warp + 1) * kb / kSkWarps;
+    for (int q = kb_lo; q < kb_hi; ++q) {
+      uint32_t a[4][4];
+      const int line = q * Mr + ar;
+      const uint32_t aq = a_base + line * 128, sw = line & 7;
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        ldsm_x4(real ? aq + (((2 * j + c0) ^ sw) << 4) : z_addr, a[j][0], a[j][1], a[j][2], a[j][3]);
+      const uint32_t wq = w_base + q * 1024;
+      uint32_t b0, b1, b2, b3, b4, b5, b6, b7;
+      ldsm_x4(wq + offB0, b0, b1, b2, b3);
+      ldsm_x4(wq + offB1, b4, b5, b6, b7);
+      mma_bf16(acc[0], a[0][0], a[0][1], a[0][2], a[0][3], b0, b1);
+      mma_bf16(acc[1], a[1][0], a[1][1], a[1][2], a[1][3], b2, b3);
+      mma_bf16(acc[0], a[2][0], a[2][1], a[2][2], a[2][3], b4, b5);
+      mma_bf16(acc[1], a[3][0], a[3][1], a[3][2], a[3][3], b6, b7);
+    }
+  }
+  __syncthreads();  // the slab now takes the warps' partials
+  {
+    const int g = lane >> 2, c4 = lane & 3;
+    float *pw = sPart + warp * 128;
+    pw[g * 8 + 2 * c4] = acc[0][0] + acc[1][0];
+    pw[g * 8 + 2 * c4 + 1] = acc[0][1] + acc[1][1];
+    pw[(g + 8) * 8 + 2 * c4] = acc[0][2] + acc[1][2];
+    pw[(g + 8) * 8 + 2 * c4 + 1] = acc[0][3] + acc[1][3];
+  }
+  __syncthreads();
+  if (tid < 128) {
+    float v = 0.f;
+#pragma unroll
+    for (int w = 0; w < kSkWarps; ++w) v += sPart[w * 128 + tid];
+    sSum[tid] = v;
+  }
+  __syncthreads();
+
+  // ---------------- queries into every CTA of the cluster: a lane group of 8
+  // holds one row's 8 values; lane j of the group stores the row's chunk into
+  // CTA j
+  cluster_wait();  // every CTA of the cluster has started
+  if (warp < (M * 8 + 31) / 32) {
+    const int e = tid, t = e >> 3, j = e & 7;
+    float qv = 0.f;
+    if (t < M) {
+      const float2 ms = sStat[t];
+      float v = __fmaf_rn(ms.y, __fmaf_rn(-ms.x, sSum[j], sSum[(t + 2) * 8 + j]), sSum[8 + j]);
+      v += sBias[j];
+      qv = __bfloat162float(__float2bfloat16(v)) * 0.125f;  // the query in bf16, scaled by 1/sqrt(64)
+    }
+    const float nx = __shfl_down_sync(0xffffffffu, qv, 1);
+    const uint32_t pr = pack_bf16(qv, nx);
+    const int base = lane & ~7;
+    uint4 chunk;
+    chunk.x = __shfl_sync(0xffffffffu, pr, base + 0);
+    chunk.y = __shfl_sync(0xffffffffu, pr, base + 2);
+    chunk.z = __shfl_sync(0xffffffffu, pr, base + 4);
+    chunk.w = __shfl_sync(0xffffffffu, pr, base + 6);
+    if (t < M) dsmem_st_u32x4(dsmem_map(smem_u32(sQ) + swz(t, static_cast<int>(crank)), j), chunk);
+  }
+  cluster_sync();  // every row's 8 chunks have landed in every CTA
+
+  // ---------------- attention over this CTA's frames (warps < nw, 32 each)
+  const bool k_ok = !any_keys || mbar_wait(&bar[2], 0, p.err, spin);
+  if (!k_ok) *s_flag = 1;
+  const int g = lane >> 2, c4 = lane & 3;
+  const int kw = warp * 32;
+  float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
+  float o[8][4];
+#pragma unroll
+  for (int nd = 0; nd < 8; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
+  // warp-uniform: the MMAs below need the whole warp
+  const bool mine = __all_sync(0xffffffffu, any_keys && warp < nw && k_ok && ok);
+  float sc[4][4];
+  if (mine) {
+    const uint32_t q_u32 = smem_u32(sQ), k_u32 = smem_u32(sK);
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
+#pragma unroll
+    for (int ks = 0; ks < 4; ++ks) {
+      uint32_t a0, a1, a2, a3;
+      const int mi = lane >> 3;
+      ldsm_x4(q_u32 + swz((mi & 1) * 8 + (lane & 7), 2 * ks + (mi >> 1)), a0, a1, a2, a3);
+#pragma unroll
+      for (int np = 0; np < 2; ++np) {
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4(k_u32 + swz(kw + np * 16 + (mi >> 1) * 8 + (lane & 7), 2 * ks + (mi & 1)), b0, b1, b2, b3);
+        mma_bf16(sc[2 * np], a0, a1, a2, a3, b0, b1);
+        mma_bf16(sc[2 * np + 1], a0, a1, a2, a3, b2, b3);
+      }
+    }
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int row = g + (e >> 1) * 8;
+        const int pos = key0 + kw + nt * 8 + c4 * 2 + (e & 1);
+        const bool vis = row < M && pos < ctx;
+        sc[nt][e] = vis ? sc[nt][e] * kXaLog2e : -INFINITY;
+        mrow[e >> 1] = fmaxf(mrow[e >> 1], sc[nt][e]);
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      mrow[r] = fmaxf(mrow[r], __shfl_xor_sync(0xffffffffu, mrow[r], 1));
+      mrow[r] = fmaxf(mrow[r], __shfl_xor_sync(0xffffffffu, mrow[r], 2));
+    }
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float v = sc[nt][e] == -INFINITY ? 0.f : exp2f(sc[nt][e] - mrow[e >> 1]);
+        sc[nt][e] = v;
+        lrow[e >> 1] += v;
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 1);
+      lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 2);
+    }
+    if (!mbar_wait(&bar[3], 0, p.err, spin)) *s_flag = 1;
+    const uint32_t v_u32 = smem_u32(sV);
+#pragma unroll
+    for (int kk = 0; kk < 2; ++kk) {
+      const uint32_t a0 = pack_bf16(sc[2 * kk][0], sc[2 * kk][1]);
+      const uint32_t a1 = pack_bf16(sc[2 * kk][2], sc[2 * kk][3]);
+      const uint32_t a2 = pack_bf16(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+      const uint32_t a3 = pack_bf16(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+#pragma unroll
+      for (int dp = 0; dp < 4; ++dp) {
+        uint32_t b0, b1, b2, b3;
+        const int mi = lane >> 3;
+        ldsm_x4_t(v_u32 + swz(kw + kk * 16 + (mi & 1) * 8 + (lane & 7), 2 * dp + (mi >> 1)), b0, b1, b2, b3);
+        mma_bf16(o[2 * dp], a0, a1, a2, a3, b0, b1);
+        mma_bf16(o[2 * dp + 1], a0, a1, a2, a3, b2, b3);
+      }
+    }
+  } else if (any_keys && warp < nw) {
+    // a wait gave up: this warp still waits (bounded) for the values it would read
+    mbar_wait(&bar[3], 0, p.err, spin);
+  }
+  __syncthreads();  // every warp is done with the key tile, which now holds O
+  if (warp < nw) {
+    if (c4 == 0) {
+      sm[warp * 16 + g] = mrow[0];
+      sm[warp * 16 + g + 8] = mrow[1];
+      sl[warp * 16 + g] = lrow[0];
+      sl[warp * 16 + g + 8] = lrow[1];
+    }
+#pragma unroll
+    for (int nd = 0; nd < 8; ++nd) {
+      const int col = (nd ^ (g & 3)) * 8 + c4 * 2;
+      *reinterpret_cast<float2 *>(so + (warp * 16 + g) * 64 + col) = make_float2(o[nd][0], o[nd][1]);
+      *reinterpret_cast<float2 *>(so + (warp * 16 + g + 8) * 64 + col) = make_float2(o[nd][2], o[nd][3]);
+    }
+  }
+  __syncthreads();
+  // the CTA's (m, l, o) per row: thread -> (row qi, dims d0 .. d0 + 3), warps in order
+  {
+    const int qi = tid >> 4, d0 = (tid & 15) * 4;
+    float Mx = -INFINITY;
+    for (int w = 0; w < nw; ++w) Mx = fmaxf(Mx, sm[w * 16 + qi]);
+    float Ls = 0.f, a4[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int w = 0; w < nw; ++w) {
+      const float mw = sm[w * 16 + qi];
+      const float wt = (mw == -INFINITY) ? 0.f : exp2f(mw - Mx);
+      Ls += sl[w * 16 + qi] * wt;
+      const float4 o4 = *reinterpret_cast<const float4 *>(so + (w * 16 + qi) * 64 + (d0 ^ ((qi & 3) << 3)));
+      a4[0] += o4.x * wt;
+      a4[1] += o4.y * wt;
+      a4[2] += o4.z * wt;
+      a4[3] += o4.w * wt;
+    }
+    if (!any_keys) {  // no frame here: the empty partial
+      Mx = -INFINITY;
+      Ls = 0.f;
+      a4[0] = a4[1] = a4[2] = a4[3] = 0.f;
+    }
+    // push to the CTA that owns dims d0 .. d0 + 3 (rank d0 / 8)
+    const uint32_t dst = static_cast<uint32_t>(d0 >> 3);
+    const uint32_t base = smem_u32(pin) + 4u * ((crank * 16 + qi) * 12);
+    if ((d0 & 7) == 0) {
+      dsmem_st_f32(dsmem_map(base, dst), Mx);
+      dsmem_st_f32(dsmem_map(base + 4u, dst), Ls);
+    }
+    dsmem_st_u32x4(dsmem_map(base + 4u * (4 + (d0 & 7)), dst),
+                   make_uint4(__float_as_uint(a4[0]), __float_as_uint(a4[1]), __float_as_uint(a4[2]),
+                              __float_as_uint(a4[3])));
+  }
+  cluster_sync();  // every CTA's partial of this CTA's dims has arrived
+  // ---------------- merge the 8 partials in rank order: thread -> (row, 4 of the 8 dims)
+  if (tid < 2 * M) {
+    const int qi = tid >> 1, half = tid & 1;
+    float MM = -INFINITY;
+#pragma unroll
+    for (int r = 0; r < 8; ++r) MM = fmaxf(MM, pin[(r * 16 + qi) * 12]);
+    float LL = 0.f, oo[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+      const float *pr = pin + (r * 16 + qi) * 12;
+      const float mc = pr[0];
+      const float wt = (mc == -INFINITY) ? 0.f : exp2f(mc - MM);
+      const float4 o4 = *reinterpret_cast<const float4 *>(pr + 4 + 4 * half);
+      LL = __fmaf_rn(pr[1], wt, LL);
+      oo[0] = __fmaf_rn(o4.x, wt, oo[0]);
+      oo[1] = __fmaf_rn(o4.y, wt, oo[1]);
+      oo[2] = __fmaf_rn(o4.z, wt, oo[2]);
+      oo[3] = __fmaf_rn(o4.w, wt, oo[3]);
+    }
+    if (!*s_flag) {
+      const float inv = 1.0f / LL;
+      const int d0 = static_cast<int>(crank) * 8 + 4 * half;
+      *reinterpret_cast<uint2 *>(p.out_bf16 + static_cast<size_t>(qi) * p.ld_out + head * 64 + d0) =
+          make_uint2(pack_bf16(oo[0] * inv, oo[1] * inv), pack_bf16(oo[2] * inv, oo[3] * inv));
+    }
+  }
+  __syncthreads();
+  if (tid == 0 && *s_flag) {  // after a timeout a copy may still be landing
+    for (int i = 0; i < 4; ++i)
+      if (i < 2 || any_keys) mbar_drain(&bar[i], 0);
+  }
+}
+
 // ------------------------------------------------------------------ host ----
 namespace {
 size_t skinny_smem(int M, int K, int U, int S, bool ln) {
@@ -565,7 +950,10 @@ cudaError_t skinny_init() {
   static cudaError_t status = cudaErrorNotReady;
   static std::once_flag once;
   std::call_once(once, [] {
-    cudaError_t e = skinny_attrs<1>();
+    const void *xa = reinterpret_cast<const void *>(skinny_xattn_kernel);
+    cudaError_t e = cudaFuncSetAttribute(xa, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+    if (e == cudaSuccess) e = prefer_max_shared(xa);
+    if (e == cudaSuccess) e = skinny_attrs<1>();
     if (e == cudaSuccess) e = skinny_attrs<2>();
     if (e == cudaSuccess) e = skinny_attrs<3>();
     if (e == cudaSuccess) e = skinny_attrs<4>();
@@ -657,6 +1045,78 @@ cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pd
     case 8: return cudaLaunchKernelEx(&cfg, skinny_kernel<8>, *tm, *tx, p);
     default: return cudaErrorInvalidValue;
   }
+}
+
+// ------------------------------------------- fused cross-attention, host ----
+namespace {
+// frames per CTA: an eighth of the memory, rounded up to whole warps of 32
+int xattn_kpc(int frames) { return ((frames + 7) / 8 + 31) / 32 * 32; }
+size_t xattn_smem(int Mr, int K, int kpc) { return 1024 + static_cast<size_t>(XaLayout(Mr, K, kpc).total); }
+// Tensor maps of the acoustic caches with a box of kpc frames.
+const CUtensorMap *xattn_tmap(const void *cache, int ctx, int outer, int kpc) {
+  static std::mutex mu;
+  static std::map<std::tuple<uintptr_t, int, int, int>, CUtensorMap *> maps;
+  std::lock_guard<std::mutex> lock(mu);
+  const auto key = std::make_tuple(reinterpret_cast<uintptr_t>(cache), ctx, outer, kpc);
+  auto it = maps.find(key);
+  if (it != maps.end()) return it->second;
+  CUtensorMap *m = new CUtensorMap;
+  if (!tmap_bf16_cache(m, cache, static_cast<uint64_t>(ctx), static_cast<uint64_t>(outer),
+                       static_cast<uint32_t>(kpc))) {
+    delete m;
+    return nullptr;
+  }
+  maps.emplace(key, m);
+  return m;
+}
+}  // namespace
+
+bool skinny_xattn_fits(int M, int d, int n_heads, int frames) {
+  if (M < 1 || M > kSkMaxFoldRows || n_heads < 1 || d != n_heads * 64 || d % 128 || frames < 1) return false;
+  const int kpc = xattn_kpc(frames);
+  if (kpc > 256 || kpc > frames) return false;
+  int U = 0, S = 0;
+  if (!skinny_plan(M + 2, d, d, false, true, &U, &S)) return false;
+  return xattn_smem(M + 2, d, kpc) <= 227 * 1024;
+}
+
+cudaError_t launch_skinny_xattn(const void *W, SkinnyParams p, cudaStream_t s, bool pdl) {
+  if (p.spin <= 0) p.spin = kSpinLimitCycles;
+  if (!p.fold || !p.x || !p.fold_part || p.n_part < 1 || p.n_part > p.part_stride || !p.kc || !p.vc ||
+      !p.seq_slot || !p.out_bf16 || p.K != p.N || p.ld_out % 4 || p.ld_x % 8 || p.xa_outer < 1 ||
+      (reinterpret_cast<uintptr_t>(p.x) & 15) || (reinterpret_cast<uintptr_t>(p.out_bf16) & 7) ||
+      !skinny_xattn_fits(p.M, p.N, p.n_heads, p.ctx))
+    return cudaErrorInvalidValue;
+  p.U = 1;
+  p.S = 1;
+  p.C = 8;
+  p.xa_kpc = xattn_kpc(p.ctx);
+  const int Mr = p.M + 2;
+  const CUtensorMap *tm = skinny_tmap(W, p.N, p.K, p.K / 64);
+  const CUtensorMap *tx = skinny_xmap(p.x, Mr, p.K, p.ld_x, p.K / 64);
+  const CUtensorMap *tk = xattn_tmap(p.kc, p.ctx, p.xa_outer, p.xa_kpc);
+  const CUtensorMap *tv = xattn_tmap(p.vc, p.ctx, p.xa_outer, p.xa_kpc);
+  if (!tm || !tx || !tk || !tv) return cudaErrorInvalidValue;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.N / 8, 1, 1);
+  cfg.blockDim = dim3(kSkThreads, 1, 1);
+  cfg.dynamicSmemBytes = xattn_smem(Mr, p.K, p.xa_kpc);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  int na = 0;
+  attr[na].id = cudaLaunchAttributeClusterDimension;
+  attr[na].val.clusterDim.x = 8;
+  attr[na].val.clusterDim.y = 1;
+  attr[na].val.clusterDim.z = 1;
+  ++na;
+  if (pdl) {
+    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = na;
+  return cudaLaunchKernelEx(&cfg, skinny_xattn_kernel, *tm, *tx, *tk, *tv, p);
 }
 
 }  // namespace wf
