@@ -517,6 +517,49 @@ cudaError_t skinny_xattn(wf_handle *h, const wf_layer_weights &lw, const bf16 *x
   return e;
 }
 
+// The QKV projection (LN1 folded, one sequence) fused with the self-attention
+// of its rows over the cache kc/vc (target: causal; drafter: the history
+// memory and the block, with RoPE); the new keys and values are written to
+// the cache at L + j and the attention output lands in h->att.
+cudaError_t skinny_sattn(wf_handle *h, const wf_layer_weights &lw, bf16 *kc, bf16 *vc, const Pass &ps,
+                         cudaStream_t s) {
+  const int M = ps.n_seq * ps.rps, d = h->d;
+  SkinnyParams p = {};
+  p.M = M;
+  p.N = 3 * d;
+  p.K = d;
+  p.epi = EPI_KV;
+  p.fold = 1;
+  p.x = h->xg;
+  p.ld_x = d;
+  p.fold_part = h->fpart;
+  p.n_part = h->fold_np;
+  p.part_stride = kSkMaxParts;
+  p.ln_eps = h->cfg.ln_eps;
+  p.bias = static_cast<const bf16 *>(lw.qkv_b);
+  p.out_bf16 = h->att;
+  p.ld_out = d;
+  p.kc = kc;
+  p.vc = vc;
+  p.ctx = h->ctx;
+  p.seq_slot = ps.slots;
+  p.pos_base = h->L;
+  p.n_heads = h->H;
+  p.d_model = d;
+  p.xa_outer = h->Bmax * h->H;
+  p.xa_mode = ps.drafter ? 1 : 0;
+  p.rope_tab = ps.drafter ? h->rope : nullptr;
+  p.pf = lw.out_w;
+  p.pf_bytes = static_cast<size_t>(d) * d * sizeof(bf16);
+  p.err = h->err;
+  p.spin = h->spin;
+  h->launches++;
+  prof_begin(h, s);
+  cudaError_t e = launch_skinny_sattn(lw.qkv_w, p, s, kPDL);
+  prof_end(h, s, WF_FAM_ATTN_SELF, 3.0 * d * d * sizeof(bf16));
+  return e;
+}
+
 // One pre-LayerNorm Whisper block over the pass's rows; next: the following
 // block of the pass (whose first LayerNorm a skinny pass folds), or null.
 cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, int layer,
@@ -535,7 +578,11 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     xkc = h->cross_k + layer_cache_off(h, layer, h->cfg.enc_frames);
     xvc = h->cross_v + layer_cache_off(h, layer, h->cfg.enc_frames);
   }
-  // self-attention
+  // self-attention: for one sequence on the skinny path, the QKV projection
+  // and the attention run as one kernel (a cluster per head)
+  if (ps.sk && ps.n_seq == 1 && skinny_sattn_fits(M, d, h->H, h->ctx)) {
+    if ((e = skinny_sattn(h, lw, kc, vc, ps, s)) != cudaSuccess) return e;
+  } else {
   {
     GemmParams p = gemm_base(h, M, 3 * d, d, EPI_KV);
     p.bias = static_cast<const bf16 *>(lw.qkv_b);
@@ -555,6 +602,7 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
   if ((e = attention(h, h->q, kc, vc, ps.slots, ps.n_seq, ps.rps, h->ctx, ps.drafter ? 1 : 0,
                      ps.drafter, s)) != cudaSuccess)
     return e;
+  }
   {
     GemmParams p = gemm_base(h, M, d, d, EPI_RESID);
     p.bias = static_cast<const bf16 *>(lw.out_b);

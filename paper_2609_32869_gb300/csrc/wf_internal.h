@@ -176,6 +176,9 @@ struct SkinnyParams {
   // acoustic keys and values, ctx frames; out_bf16: the attention output)
   int xa_kpc;
   int xa_outer;  // bound on slot * n_heads + head (the caches' tensor maps)
+  // skinny_sattn: 0 causal (target), 1 block (drafter: all of [0, L + M), RoPE)
+  int xa_mode;
+  const float2 *rope_tab;  // [max_pos][32] (cos, sin), mode 1
   // nullable: weights of the next projection in the chain, brought into L2
   // in the prologue (pf_bytes, a multiple of 16, 16-byte aligned)
   const void *pf;
@@ -194,6 +197,11 @@ cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pd
 // False when the shapes do not allow it (then run the two separately).
 bool skinny_xattn_fits(int M, int d, int n_heads, int frames);
 cudaError_t launch_skinny_xattn(const void *W, SkinnyParams p, cudaStream_t s, bool pdl);
+// The QKV projection (folded LN1, one sequence) fused with the self-attention
+// of its rows: one cluster of 8 CTAs per head, each projecting 8 query, 8 key
+// and 8 value columns; the new keys and values also go to the cache.
+bool skinny_sattn_fits(int M, int d, int n_heads, int ctx);
+cudaError_t launch_skinny_sattn(const void *W, SkinnyParams p, cudaStream_t s, bool pdl);
 
 // ------------------------------------------------------------- attention --
 struct AttnParams {

@@ -529,8 +529,11 @@ struct XaLayout {
     k_off = (a_off + kb * Mr * 128 + 1023) & ~1023;
     v_off = k_off + kpc * 128;  // kpc a multiple of 32: 1024-aligned
     q_off = v_off + kpc * 128;
-    pb_off = q_off + 16 * 128;
-    sum_off = pb_off + 8 * 16 * 12 * 4;
+    // the partial inbox reuses the operand tile (dead in every CTA of the
+    // cluster before the first partial is pushed) when it is large enough
+    const bool inbox_in_a = kb * Mr * 128 >= 8 * 16 * 12 * 4;
+    pb_off = inbox_in_a ? a_off : q_off + 16 * 128;
+    sum_off = q_off + 16 * 128 + (inbox_in_a ? 0 : 8 * 16 * 12 * 4);
     bias_off = sum_off + 128 * 4;
     stat_off = bias_off + 8 * 4;
     ml_off = stat_off + kSkMaxRows * 8;
@@ -543,7 +546,7 @@ struct XaLayout {
 constexpr float kXaLog2e = 1.4426950408889634f;
 }  // namespace
 
-__global__ void __launch_bounds__(kSkThreads, 1) skinny_xattn_kernel(const __grid_constant__ CUtensorMap tmW,
+__global__ void __launch_bounds__(kSkThreads, 2) skinny_xattn_kernel(const __grid_constant__ CUtensorMap tmW,
                                                                      const __grid_constant__ CUtensorMap tmX,
                                                                      const __grid_constant__ CUtensorMap tmK,
                                                                      const __grid_constant__ CUtensorMap tmV,
@@ -882,6 +885,472 @@ __global__ void __launch_bounds__(kSkThreads, 1) skinny_xattn_kernel(const __gri
   }
 }
 
+// ------------------------------------------------ QKV + self-attention --
+// The self-attention of a single sequence fused into its QKV projection
+// (Sec. 3.1: the verify block's causal pass, query j seeing positions
+// 0 .. L + j; Sec. 3.2, App. A.2: the drafter's joint softmax over its
+// history memory and the bidirectional block, RoPE on queries and keys).  A
+// cluster of 8 CTAs owns a head: CTA c projects query, key and value columns
+// 8c .. 8c + 7 of the head (three units of 8 weight rows) for the M rows.
+// The new keys and values go to the cache at positions L + j, as in the
+// unfused projection, and, as 16-byte chunks over distributed shared memory,
+// straight into the key/value tile of the CTA that attends to position
+// L + j (CTA c attends to positions c kpc .. (c + 1) kpc - 1, its settled
+// rows requested by TMA before the dependency wait; the chunks are written
+// only after every CTA's copy has landed).  The query chunks go to every
+// CTA.  Attention, warp merge and the rank-order merge of the 8 CTAs are
+// those of the cross-attention kernel above.
+namespace {
+struct SaLayout {
+  int w_off, a_off, k_off, v_off, q_off, pb_off, sum_off, bias_off, stat_off, ml_off, bar_off, zero_off, flag_off,
+      total;
+  __host__ __device__ SaLayout(int Mr, int K, int kpc) {
+    const int kb = K / 64;
+    w_off = 0;
+    a_off = 3 * kb * 1024;
+    k_off = (a_off + kb * Mr * 128 + 1023) & ~1023;
+    v_off = k_off + kpc * 128;
+    q_off = v_off + kpc * 128;
+    // the partial inbox reuses the operand tile, as in the cross-attention kernel
+    const bool inbox_in_a = kb * Mr * 128 >= 8 * 16 * 12 * 4;
+    pb_off = inbox_in_a ? a_off : q_off + 16 * 128;
+    sum_off = q_off + 16 * 128 + (inbox_in_a ? 0 : 8 * 16 * 12 * 4);
+    bias_off = sum_off + 3 * 128 * 4;
+    stat_off = bias_off + 24 * 4;
+    ml_off = stat_off + kSkMaxRows * 8;
+    bar_off = ml_off + 2 * 8 * 16 * 4;
+    zero_off = bar_off + 4 * 8;
+    flag_off = zero_off + 16;
+    total = flag_off + 16;
+  }
+};
+}  // namespace
+
+__global__ void __launch_bounds__(kSkThreads, 2) skinny_sattn_kernel(const __grid_constant__ CUtensorMap tmW,
+                                                                     const __grid_constant__ CUtensorMap tmX,
+                                                                     const __grid_constant__ CUtensorMap tmK,
+                                                                     const __grid_constant__ CUtensorMap tmV,
+                                                                     const SkinnyParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  uint8_t *smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+  const int M = p.M, Mr = M + 2, K = p.K, kb = K / 64, kpc = p.xa_kpc, ctx = p.ctx, H = p.n_heads;
+  const SaLayout L(Mr, K, kpc);
+  uint8_t *sW = smem + L.w_off;
+  uint8_t *sA = smem + L.a_off;
+  uint8_t *sK = smem + L.k_off;
+  uint8_t *sV = smem + L.v_off;
+  uint8_t *sQ = smem + L.q_off;
+  float *pin = reinterpret_cast<float *>(smem + L.pb_off);   // [8 source CTAs][16][12]
+  float *sPart = reinterpret_cast<float *>(smem + L.w_off);  // [8 warps][3 units][16][8]
+  float *sSum = reinterpret_cast<float *>(smem + L.sum_off);  // [3][16][8]
+  float *sBias = reinterpret_cast<float *>(smem + L.bias_off);  // [3][8]
+  float2 *sStat = reinterpret_cast<float2 *>(smem + L.stat_off);
+  float *sm = reinterpret_cast<float *>(smem + L.ml_off);
+  float *sl = sm + 8 * 16;
+  float *so = reinterpret_cast<float *>(sK);
+  uint64_t *bar = reinterpret_cast<uint64_t *>(smem + L.bar_off);
+  uint4 *sZero = reinterpret_cast<uint4 *>(smem + L.zero_off);
+  int *s_flag = reinterpret_cast<int *>(smem + L.flag_off);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int cta = blockIdx.x, head = cta >> 3;
+  const uint32_t crank = cluster_ctarank();
+  const int nw = kpc / 32;
+  const int key0 = static_cast<int>(crank) * kpc;
+  const long long spin = p.spin > 0 ? p.spin : kSpinLimitCycles;
+  // query, key and value units of this CTA (rows of the [3 d][d] weight)
+  auto unit_row = [&](int u) { return (u * H * 8 + head * 8 + static_cast<int>(crank)) * 8; };
+  // the cache length and slot are fixed for the step (read before the wait)
+  const int slot = p.seq_slot[0];
+  const int Lc = p.pos_base[slot];
+  const int n_keys = Lc + M;
+  const bool fits = n_keys <= ctx;
+  const bool any_keys = fits && key0 < n_keys;
+  const int outer = slot * H + head;
+
+  if (tid == 0) {
+    *s_flag = fits ? 0 : 1;
+    if (!fits) set_error(p.err, WF_DEV_ERR_CAPACITY);
+    tma_prefetch_desc(&tmW);
+    tma_prefetch_desc(&tmX);
+    for (int i = 0; i < 4; ++i) mbar_init(&bar[i], 1);
+    fence_barrier_init();
+    *sZero = make_uint4(0u, 0u, 0u, 0u);
+    mbar_arrive_expect_tx(&bar[0], static_cast<uint32_t>(3 * kb * 1024));
+    const uint64_t pol = l2_evict_first_policy();
+    for (int u = 0; u < 3; ++u) tma_load_3d_stream(sW + u * kb * 1024, &tmW, 0, unit_row(u), 0, &bar[0], pol);
+    if (any_keys) {  // this CTA's positions; rows from L on are replaced below
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmV);
+      mbar_arrive_expect_tx(&bar[2], static_cast<uint32_t>(kpc * 128));
+      tma_load_3d(sK, &tmK, 0, key0, outer, &bar[2]);
+      mbar_arrive_expect_tx(&bar[3], static_cast<uint32_t>(kpc * 128));
+      tma_load_3d(sV, &tmV, 0, key0, outer, &bar[3]);
+    }
+    if (p.pf) {
+      const size_t share = ((p.pf_bytes + gridDim.x - 1) / gridDim.x + 15) & ~static_cast<size_t>(15);
+      const size_t lo = static_cast<size_t>(cta) * share;
+      const size_t hi = lo + share < p.pf_bytes ? lo + share : p.pf_bytes;
+      for (size_t off = lo; off < hi; off += 32768)
+        l2_prefetch_bulk(static_cast<const uint8_t *>(p.pf) + off,
+                         static_cast<uint32_t>(hi - off < 32768 ? hi - off : 32768));
+    }
+  }
+  if (tid < 24) sBias[tid] = p.bias ? bf2f(p.bias[unit_row(tid >> 3) + (tid & 7)]) : 0.f;
+  pdl_launch_dependents();
+  pdl_wait();
+
+  // ---------------- operand (rows g, b, then g . x) and the row statistics
+  if (tid == 0) {
+    mbar_arrive_expect_tx(&bar[1], static_cast<uint32_t>(kb * Mr * 128));
+    tma_load_3d(sA, &tmX, 0, 0, 0, &bar[1]);
+  }
+  {
+    constexpr int kPL = (kSkMaxParts + 31) / 32;
+    float2 v[2][kPL];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int t = warp + kSkWarps * h;
+      const float2 *pr = p.fold_part + static_cast<size_t>(t) * p.part_stride;
+#pragma unroll
+      for (int q = 0; q < kPL; ++q) {
+        const int i = lane + 32 * q;
+        v[h][q] = (t < M && i < p.n_part) ? __ldcg(pr + i) : make_float2(0.f, 0.f);
+      }
+    }
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int t = warp + kSkWarps * h;
+      float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+      for (int q = 0; q < kPL; ++q) {
+        s1 += v[h][q].x;
+        s2 += v[h][q].y;
+      }
+      s1 = warp_sum(s1);
+      s2 = warp_sum(s2);
+      const float mu = s1 / static_cast<float>(K);
+      const float var = fmaxf(s2 / static_cast<float>(K) - mu * mu, 0.f);
+      if (lane == 0 && t < M) sStat[t] = make_float2(mu, rsqrtf(var + p.ln_eps));
+    }
+  }
+  bool ok = mbar_wait(&bar[1], 0, p.err, spin);
+  ok = mbar_wait(&bar[0], 0, p.err, spin) && ok;
+  if (!ok) *s_flag = 1;
+
+  // ---------------- query, key and value columns: warp w over k-blocks [w kb / 8, (w + 1) kb / 8)
+  float acc[3][2][4];
+#pragma unroll
+  for (int u = 0; u < 3; ++u)
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) acc[u][hh][0] = acc[u][hh][1] = acc[u][hh][2] = acc[u][hh][3] = 0.f;
+  if (ok) {
+    const int ar = (lane & 7) + ((lane >> 3) & 1) * 8, c0 = lane >> 4;
+    const bool real = ar < Mr;
+    const uint32_t a_base = smem_u32(sA), z_addr = smem_u32(sZero), w_base = smem_u32(sW);
+    const int br = lane & 7, bg = lane >> 3;
+    const uint32_t offB0 = br * 128 + (((bg) ^ br) << 4), offB1 = br * 128 + (((bg + 4) ^ br) << 4);
+    const int kb_lo = warp * kb / kSkWarps, kb_hi = (warp + 1) * kb / kSkWarps;
+    for (int q = kb_lo; q < kb_hi; ++q) {
+      uint32_t a[4][4];
+      const int line = q * Mr + ar;
+      const uint32_t aq = a_base + line * 128, sw = line & 7;
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        ldsm_x4(real ? aq + (((2 * j + c0) ^ sw) << 4) : z_addr, a[j][0], a[j][1], a[j][2], a[j][3]);
+#pragma unroll
+      for (int u = 0; u < 3; ++u) {
+        const uint32_t wq = w_base + u * kb * 1024 + q * 1024;
+        uint32_t b0, b1, b2, b3, b4, b5, b6, b7;
+        ldsm_x4(wq + offB0, b0, b1, b2, b3);
+        ldsm_x4(wq + offB1, b4, b5, b6, b7);
+        mma_bf16(acc[u][0], a[0][0], a[0][1], a[0][2], a[0][3], b0, b1);
+        mma_bf16(acc[u][1], a[1][0], a[1][1], a[1][2], a[1][3], b2, b3);
+        mma_bf16(acc[u][0], a[2][0], a[2][1], a[2][2], a[2][3], b4, b5);
+        mma_bf16(acc[u][1], a[3][0], a[3][1], a[3][2], a[3][3], b6, b7);
+      }
+    }
+  }
+  __syncthreads();  // the slab now takes the warps' partials
+  {
+    const int g = lane >> 2, c4 = lane & 3;
+#pragma unroll
+    for (int u = 0; u < 3; ++u) {
+      float *pw = sPart + (warp * 3 + u) * 128;
+      pw[g * 8 + 2 * c4] = acc[u][0][0] + acc[u][1][0];
+      pw[g * 8 + 2 * c4 + 1] = acc[u][0][1] + acc[u][1][1];
+      pw[(g + 8) * 8 + 2 * c4] = acc[u][0][2] + acc[u][1][2];
+      pw[(g + 8) * 8 + 2 * c4 + 1] = acc[u][0][3] + acc[u][1][3];
+    }
+  }
+  __syncthreads();
+  for (int e = tid; e < 3 * 128; e += kSkThreads) {
+    const int u = e >> 7, rc = e & 127;
+    float v = 0.f;
+#pragma unroll
+    for (int w = 0; w < kSkWarps; ++w) v += sPart[(w * 3 + u) * 128 + rc];
+    sSum[e] = v;
+  }
+  // this CTA's keys and values have landed before any peer writes into them
+  bool kv_ok = true;
+  if (any_keys) {
+    kv_ok = mbar_wait(&bar[2], 0, p.err, spin);
+    kv_ok = mbar_wait(&bar[3], 0, p.err, spin) && kv_ok;
+  }
+  if (!kv_ok) *s_flag = 1;
+  __syncthreads();
+  cluster_arrive();
+  cluster_wait();
+
+  // ---------------- the new rows: a lane group of 8 holds one (unit, row)'s
+  // 8 values.  Queries: lane j stores the chunk into CTA j.  Keys and values:
+  // every lane writes its value to the cache, lane 0 the chunk into the CTA
+  // attending to position L + t.
+  const int n_el = 3 * M * 8;
+  for (int e0 = 0; e0 < n_el; e0 += kSkThreads) {
+    if (e0 + warp * 32 >= n_el) break;  // warp-uniform
+    const int e = e0 + tid, u = e / (M * 8), rem = e - u * M * 8, t = rem >> 3, j = rem & 7;
+    const bool live = e < n_el;
+    float val = 0.f;
+    if (live) {
+      const float *su = sSum + (u < 3 ? u : 0) * 128;
+      const float2 ms = sStat[t];
+      float v = __fmaf_rn(ms.y, __fmaf_rn(-ms.x, su[j], su[(t + 2) * 8 + j]), su[8 + j]);
+      v += sBias[u * 8 + j];
+      val = __bfloat162float(__float2bfloat16(v));
+      if (u > 0 && fits && !*s_flag) {
+        bf16 *dst = u == 1 ? p.kc : p.vc;
+        dst[(static_cast<size_t>(outer) * ctx + Lc + t) * 64 + static_cast<int>(crank) * 8 + j] = __float2bfloat16(v);
+      }
+    }
+    const float nx = __shfl_down_sync(0xffffffffu, val, 1);
+    const uint32_t pr = pack_bf16(val, nx);
+    const int base = lane & ~7;
+    uint4 chunk;
+    chunk.x = __shfl_sync(0xffffffffu, pr, base + 0);
+    chunk.y = __shfl_sync(0xffffffffu, pr, base + 2);
+    chunk.z = __shfl_sync(0xffffffffu, pr, base + 4);
+    chunk.w = __shfl_sync(0xffffffffu, pr, base + 6);
+    if (live && fits) {
+      if (u == 0) {
+        dsmem_st_u32x4(dsmem_map(smem_u32(sQ) + swz(t, static_cast<int>(crank)), j), chunk);
+      } else if (j == 0) {
+        const int pos = Lc + t, owner = pos / kpc, r = pos - owner * kpc;
+        dsmem_st_u32x4(dsmem_map(smem_u32(u == 1 ? sK : sV) + swz(r, static_cast<int>(crank)),
+                                 static_cast<uint32_t>(owner)),
+                       chunk);
+      }
+    }
+  }
+  cluster_sync();  // every chunk has landed
+
+  // ---------------- queries: RoPE (drafter) at L + r, then the 1/8 scale;
+  // keys: RoPE at their positions; values past the visible keys: zeros
+  const bool rope = p.xa_mode == 1 && p.rope_tab;
+  if (tid < 16 * 4) {
+    const int r = tid >> 2, c = tid & 3;  // chunk c pairs with chunk c + 4 (dims i and i + 32)
+    uint4 *lo = reinterpret_cast<uint4 *>(sQ + swz(r, c));
+    uint4 *hi = reinterpret_cast<uint4 *>(sQ + swz(r, c + 4));
+    uint4 a = *lo, b = *hi;
+    bf16 *av = reinterpret_cast<bf16 *>(&a);
+    bf16 *bv = reinterpret_cast<bf16 *>(&b);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      float x1 = bf2f(av[e]), x2 = bf2f(bv[e]);
+      if (rope && r < M) {
+        const float2 cs = __ldg(p.rope_tab + (Lc + r) * 32 + c * 8 + e);
+        const float y1 = x1 * cs.x - x2 * cs.y, y2 = x2 * cs.x + x1 * cs.y;
+        x1 = y1;
+        x2 = y2;
+      }
+      av[e] = __float2bfloat16(x1 * 0.125f);
+      bv[e] = __float2bfloat16(x2 * 0.125f);
+    }
+    *lo = a;
+    *hi = b;
+  }
+  if (rope && any_keys) {
+    for (int idx = tid; idx < kpc * 4; idx += kSkThreads) {
+      const int kr = idx >> 2, c = idx & 3;
+      const int pos = key0 + kr;
+      if (pos >= n_keys) continue;
+      uint4 *lo = reinterpret_cast<uint4 *>(sK + swz(kr, c));
+      uint4 *hi = reinterpret_cast<uint4 *>(sK + swz(kr, c + 4));
+      uint4 a = *lo, b = *hi;
+      bf16 *av = reinterpret_cast<bf16 *>(&a);
+      bf16 *bv = reinterpret_cast<bf16 *>(&b);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        const float2 cs = __ldg(p.rope_tab + pos * 32 + c * 8 + e);
+        const float x1 = bf2f(av[e]), x2 = bf2f(bv[e]);
+        av[e] = __float2bfloat16(x1 * cs.x - x2 * cs.y);
+        bv[e] = __float2bfloat16(x2 * cs.x + x1 * cs.y);
+      }
+      *lo = a;
+      *hi = b;
+    }
+  }
+  {
+    const int z0 = min(max(n_keys - key0, 0), kpc);
+    for (int idx = tid; idx < (kpc - z0) * 8; idx += kSkThreads)
+      *reinterpret_cast<uint4 *>(sV + swz(z0 + (idx >> 3), idx & 7)) = make_uint4(0u, 0u, 0u, 0u);
+  }
+  __syncthreads();
+
+  // ---------------- attention over this CTA's positions (warps < nw, 32 each)
+  const int g = lane >> 2, c4 = lane & 3;
+  const int kw = warp * 32;
+  float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
+  float o[8][4];
+#pragma unroll
+  for (int nd = 0; nd < 8; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
+  const bool mine = __all_sync(0xffffffffu, any_keys && warp < nw && key0 + kw < n_keys && ok && kv_ok);
+  if (mine) {
+    float sc[4][4];
+    const uint32_t q_u32 = smem_u32(sQ), k_u32 = smem_u32(sK);
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
+#pragma unroll
+    for (int ks = 0; ks < 4; ++ks) {
+      uint32_t a0, a1, a2, a3;
+      const int mi = lane >> 3;
+      ldsm_x4(q_u32 + swz((mi & 1) * 8 + (lane & 7), 2 * ks + (mi >> 1)), a0, a1, a2, a3);
+#pragma unroll
+      for (int np = 0; np < 2; ++np) {
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4(k_u32 + swz(kw + np * 16 + (mi >> 1) * 8 + (lane & 7), 2 * ks + (mi & 1)), b0, b1, b2, b3);
+        mma_bf16(sc[2 * np], a0, a1, a2, a3, b0, b1);
+        mma_bf16(sc[2 * np + 1], a0, a1, a2, a3, b2, b3);
+      }
+    }
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int row = g + (e >> 1) * 8;
+        const int pos = key0 + kw + nt * 8 + c4 * 2 + (e & 1);
+        bool vis = row < M && pos < n_keys;
+        if (p.xa_mode == 0) vis = vis && pos <= Lc + row;
+        sc[nt][e] = vis ? sc[nt][e] * kXaLog2e : -INFINITY;
+        mrow[e >> 1] = fmaxf(mrow[e >> 1], sc[nt][e]);
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      mrow[r] = fmaxf(mrow[r], __shfl_xor_sync(0xffffffffu, mrow[r], 1));
+      mrow[r] = fmaxf(mrow[r], __shfl_xor_sync(0xffffffffu, mrow[r], 2));
+    }
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float v = sc[nt][e] == -INFINITY ? 0.f : exp2f(sc[nt][e] - mrow[e >> 1]);
+        sc[nt][e] = v;
+        lrow[e >> 1] += v;
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 1);
+      lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 2);
+    }
+    const uint32_t v_u32 = smem_u32(sV);
+#pragma unroll
+    for (int kk = 0; kk < 2; ++kk) {
+      const uint32_t a0 = pack_bf16(sc[2 * kk][0], sc[2 * kk][1]);
+      const uint32_t a1 = pack_bf16(sc[2 * kk][2], sc[2 * kk][3]);
+      const uint32_t a2 = pack_bf16(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+      const uint32_t a3 = pack_bf16(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+#pragma unroll
+      for (int dp = 0; dp < 4; ++dp) {
+        uint32_t b0, b1, b2, b3;
+        const int mi = lane >> 3;
+        ldsm_x4_t(v_u32 + swz(kw + kk * 16 + (mi & 1) * 8 + (lane & 7), 2 * dp + (mi >> 1)), b0, b1, b2, b3);
+        mma_bf16(o[2 * dp], a0, a1, a2, a3, b0, b1);
+        mma_bf16(o[2 * dp + 1], a0, a1, a2, a3, b2, b3);
+      }
+    }
+  }
+  __syncthreads();  // every warp is done with the key tile, which now holds O
+  if (warp < nw) {
+    if (c4 == 0) {
+      sm[warp * 16 + g] = mrow[0];
+      sm[warp * 16 + g + 8] = mrow[1];
+      sl[warp * 16 + g] = lrow[0];
+      sl[warp * 16 + g + 8] = lrow[1];
+    }
+#pragma unroll
+    for (int nd = 0; nd < 8; ++nd) {
+      const int col = (nd ^ (g & 3)) * 8 + c4 * 2;
+      *reinterpret_cast<float2 *>(so + (warp * 16 + g) * 64 + col) = make_float2(o[nd][0], o[nd][1]);
+      *reinterpret_cast<float2 *>(so + (warp * 16 + g + 8) * 64 + col) = make_float2(o[nd][2], o[nd][3]);
+    }
+  }
+  __syncthreads();
+  {
+    const int qi = tid >> 4, d0 = (tid & 15) * 4;
+    float Mx = -INFINITY;
+    for (int w = 0; w < nw; ++w) Mx = fmaxf(Mx, sm[w * 16 + qi]);
+    float Ls = 0.f, a4[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int w = 0; w < nw; ++w) {
+      const float mw = sm[w * 16 + qi];
+      const float wt = (mw == -INFINITY) ? 0.f : exp2f(mw - Mx);
+      Ls += sl[w * 16 + qi] * wt;
+      const float4 o4 = *reinterpret_cast<const float4 *>(so + (w * 16 + qi) * 64 + (d0 ^ ((qi & 3) << 3)));
+      a4[0] += o4.x * wt;
+      a4[1] += o4.y * wt;
+      a4[2] += o4.z * wt;
+      a4[3] += o4.w * wt;
+    }
+    if (!any_keys) {
+      Mx = -INFINITY;
+      Ls = 0.f;
+      a4[0] = a4[1] = a4[2] = a4[3] = 0.f;
+    }
+    const uint32_t dst = static_cast<uint32_t>(d0 >> 3);
+    const uint32_t base = smem_u32(pin) + 4u * ((crank * 16 + qi) * 12);
+    if ((d0 & 7) == 0) {
+      dsmem_st_f32(dsmem_map(base, dst), Mx);
+      dsmem_st_f32(dsmem_map(base + 4u, dst), Ls);
+    }
+    dsmem_st_u32x4(dsmem_map(base + 4u * (4 + (d0 & 7)), dst),
+                   make_uint4(__float_as_uint(a4[0]), __float_as_uint(a4[1]), __float_as_uint(a4[2]),
+                              __float_as_uint(a4[3])));
+  }
+  cluster_sync();  // every CTA's partial of this CTA's dims has arrived
+  if (tid < 2 * M) {
+    const int qi = tid >> 1, half = tid & 1;
+    float MM = -INFINITY;
+#pragma unroll
+    for (int r = 0; r < 8; ++r) MM = fmaxf(MM, pin[(r * 16 + qi) * 12]);
+    float LL = 0.f, oo[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+      const float *pr = pin + (r * 16 + qi) * 12;
+      const float mc = pr[0];
+      const float wt = (mc == -INFINITY) ? 0.f : exp2f(mc - MM);
+      const float4 o4 = *reinterpret_cast<const float4 *>(pr + 4 + 4 * half);
+      LL = __fmaf_rn(pr[1], wt, LL);
+      oo[0] = __fmaf_rn(o4.x, wt, oo[0]);
+      oo[1] = __fmaf_rn(o4.y, wt, oo[1]);
+      oo[2] = __fmaf_rn(o4.z, wt, oo[2]);
+      oo[3] = __fmaf_rn(o4.w, wt, oo[3]);
+    }
+    if (!*s_flag) {
+      const float inv = 1.0f / LL;
+      const int d0 = static_cast<int>(crank) * 8 + 4 * half;
+      *reinterpret_cast<uint2 *>(p.out_bf16 + static_cast<size_t>(qi) * p.ld_out + head * 64 + d0) =
+          make_uint2(pack_bf16(oo[0] * inv, oo[1] * inv), pack_bf16(oo[2] * inv, oo[3] * inv));
+    }
+  }
+  __syncthreads();
+  if (tid == 0 && *s_flag) {  // after a timeout a copy may still be landing
+    for (int i = 0; i < 4; ++i)
+      if (i < 2 || any_keys) mbar_drain(&bar[i], 0);
+  }
+}
+
 // ------------------------------------------------------------------ host ----
 namespace {
 size_t skinny_smem(int M, int K, int U, int S, bool ln) {
@@ -951,8 +1420,11 @@ cudaError_t skinny_init() {
   static std::once_flag once;
   std::call_once(once, [] {
     const void *xa = reinterpret_cast<const void *>(skinny_xattn_kernel);
+    const void *sa = reinterpret_cast<const void *>(skinny_sattn_kernel);
     cudaError_t e = cudaFuncSetAttribute(xa, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
     if (e == cudaSuccess) e = prefer_max_shared(xa);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(sa, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+    if (e == cudaSuccess) e = prefer_max_shared(sa);
     if (e == cudaSuccess) e = skinny_attrs<1>();
     if (e == cudaSuccess) e = skinny_attrs<2>();
     if (e == cudaSuccess) e = skinny_attrs<3>();
@@ -1117,6 +1589,53 @@ cudaError_t launch_skinny_xattn(const void *W, SkinnyParams p, cudaStream_t s, b
   cfg.attrs = attr;
   cfg.numAttrs = na;
   return cudaLaunchKernelEx(&cfg, skinny_xattn_kernel, *tm, *tx, *tk, *tv, p);
+}
+
+bool skinny_sattn_fits(int M, int d, int n_heads, int ctx) {
+  if (M < 1 || M > kSkMaxFoldRows || n_heads < 1 || d != n_heads * 64 || d % 128 || ctx < 1) return false;
+  const int kpc = xattn_kpc(ctx);
+  if (kpc > 256 || kpc > ctx) return false;
+  return 1024 + static_cast<size_t>(SaLayout(M + 2, d, kpc).total) <= 227 * 1024;
+}
+
+cudaError_t launch_skinny_sattn(const void *W, SkinnyParams p, cudaStream_t s, bool pdl) {
+  if (p.spin <= 0) p.spin = kSpinLimitCycles;
+  if (!p.fold || !p.x || !p.fold_part || p.n_part < 1 || p.n_part > p.part_stride || !p.kc || !p.vc ||
+      !p.seq_slot || !p.pos_base || !p.out_bf16 || p.N != 3 * p.K || p.ld_out % 4 || p.ld_x % 8 ||
+      p.xa_outer < 1 || (p.xa_mode != 0 && p.xa_mode != 1) || (p.xa_mode == 1 && !p.rope_tab) ||
+      (reinterpret_cast<uintptr_t>(p.x) & 15) || (reinterpret_cast<uintptr_t>(p.out_bf16) & 7) ||
+      !skinny_sattn_fits(p.M, p.K, p.n_heads, p.ctx))
+    return cudaErrorInvalidValue;
+  p.U = 3;
+  p.S = 1;
+  p.C = 8;
+  p.xa_kpc = xattn_kpc(p.ctx);
+  const int Mr = p.M + 2;
+  const CUtensorMap *tm = skinny_tmap(W, p.N, p.K, p.K / 64);
+  const CUtensorMap *tx = skinny_xmap(p.x, Mr, p.K, p.ld_x, p.K / 64);
+  const CUtensorMap *tk = xattn_tmap(p.kc, p.ctx, p.xa_outer, p.xa_kpc);
+  const CUtensorMap *tv = xattn_tmap(p.vc, p.ctx, p.xa_outer, p.xa_kpc);
+  if (!tm || !tx || !tk || !tv) return cudaErrorInvalidValue;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.K / 8, 1, 1);  // 8 CTAs per head
+  cfg.blockDim = dim3(kSkThreads, 1, 1);
+  cfg.dynamicSmemBytes = 1024 + static_cast<size_t>(SaLayout(Mr, p.K, p.xa_kpc).total);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  int na = 0;
+  attr[na].id = cudaLaunchAttributeClusterDimension;
+  attr[na].val.clusterDim.x = 8;
+  attr[na].val.clusterDim.y = 1;
+  attr[na].val.clusterDim.z = 1;
+  ++na;
+  if (pdl) {
+    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = na;
+  return cudaLaunchKernelEx(&cfg, skinny_sattn_kernel, *tm, *tx, *tk, *tv, p);
 }
 
 }  // namespace wf
