@@ -342,14 +342,11 @@ cudaError_t gemm(wf_handle *h, const void *X, const void *W, GemmParams p, cudaS
 // (rows h->xg and partial sums h->fpart left by the residual's producer; the
 // gain and bias are in those rows); else the bf16 rows X.  An EPI_RESID
 // projection followed by a LayerNorm with gain g_next and bias b_next writes
-// that LayerNorm's folded operand.  pf: the next projection's weights (pf_n
-// rows of pf_k), brought into L2 while this one waits for its inputs.
+// that LayerNorm's folded operand.
 cudaError_t skinny(wf_handle *h, const void *X, const float *ln_x, const void *g, const void *b,
                    const void *W, const GemmParams &gp, cudaStream_t s, const void *g_next = nullptr,
-                   const void *b_next = nullptr, const void *pf = nullptr, int pf_n = 0, int pf_k = 0) {
+                   const void *b_next = nullptr) {
   SkinnyParams p = skinny_of(gp);
-  p.pf = pf;
-  p.pf_bytes = pf ? static_cast<size_t>(pf_n) * pf_k * sizeof(bf16) : 0;
   if (g_next) {
     p.xg_out = h->xg;
     p.g_next = static_cast<const bf16 *>(g_next);
@@ -504,8 +501,6 @@ cudaError_t skinny_xattn(wf_handle *h, const wf_layer_weights &lw, const bf16 *x
   p.n_heads = h->H;
   p.d_model = d;
   p.xa_outer = h->Bmax * h->H;
-  p.pf = lw.xout_w;
-  p.pf_bytes = static_cast<size_t>(d) * d * sizeof(bf16);
   p.err = h->err;
   p.spin = h->spin;
   h->launches++;
@@ -549,8 +544,6 @@ cudaError_t skinny_sattn(wf_handle *h, const wf_layer_weights &lw, bf16 *kc, bf1
   p.xa_outer = h->Bmax * h->H;
   p.xa_mode = ps.drafter ? 1 : 0;
   p.rope_tab = ps.drafter ? h->rope : nullptr;
-  p.pf = lw.out_w;
-  p.pf_bytes = static_cast<size_t>(d) * d * sizeof(bf16);
   p.err = h->err;
   p.spin = h->spin;
   h->launches++;
@@ -595,7 +588,7 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.rows_per_seq = ps.rps;
     p.seq_slot = ps.slots;
     p.pos_base = h->L;
-    e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln1_g, lw.ln1_b, lw.qkv_w, p, s, nullptr, nullptr, lw.out_w, d, d)
+    e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln1_g, lw.ln1_b, lw.qkv_w, p, s)
               : ln_gemm(h, ps.x, ps.st, lw.ln1_g, lw.ln1_b, lw.qkv_w, p, s);
     if (e != cudaSuccess) return e;
   }
@@ -609,7 +602,7 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.resid = ps.x;
     p.ld_resid = d;
     p.stats_out = ps.st;
-    e = ps.sk ? skinny(h, h->att, nullptr, nullptr, nullptr, lw.out_w, p, s, lw.ln2_g, lw.ln2_b, lw.xq_w, d, d)
+    e = ps.sk ? skinny(h, h->att, nullptr, nullptr, nullptr, lw.out_w, p, s, lw.ln2_g, lw.ln2_b)
               : gemm(h, h->att, lw.out_w, p, s);
     if (e != cudaSuccess) return e;
   }
@@ -623,7 +616,7 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
       p.bias = static_cast<const bf16 *>(lw.xq_b);
       p.out_bf16 = h->q;
       p.ld_out = d;
-      e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s, nullptr, nullptr, lw.xout_w, d, d)
+      e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s)
                 : ln_gemm(h, ps.x, ps.st, lw.ln2_g, lw.ln2_b, lw.xq_w, p, s);
       if (e != cudaSuccess) return e;
     }
@@ -637,8 +630,7 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.resid = ps.x;
     p.ld_resid = d;
     p.stats_out = ps.st;
-    e = ps.sk ? skinny(h, h->att, nullptr, nullptr, nullptr, lw.xout_w, p, s, lw.ln3_g, lw.ln3_b, lw.fc1_w,
-                       h->F, d)
+    e = ps.sk ? skinny(h, h->att, nullptr, nullptr, nullptr, lw.xout_w, p, s, lw.ln3_g, lw.ln3_b)
               : gemm(h, h->att, lw.xout_w, p, s);
     if (e != cudaSuccess) return e;
   }
@@ -648,8 +640,7 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     p.bias = static_cast<const bf16 *>(lw.fc1_b);
     p.out_bf16 = h->h1;
     p.ld_out = h->F;
-    e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln3_g, lw.ln3_b, lw.fc1_w, p, s, nullptr, nullptr, lw.fc2_w, d,
-                       h->F)
+    e = ps.sk ? skinny(h, nullptr, nullptr, lw.ln3_g, lw.ln3_b, lw.fc1_w, p, s)
               : ln_gemm(h, ps.x, ps.st, lw.ln3_g, lw.ln3_b, lw.fc1_w, p, s);
     if (e != cudaSuccess) return e;
   }
@@ -672,7 +663,7 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
       p.ld_tap = h->cfg.n_taps * d;
     }
     e = ps.sk ? skinny(h, h->h1, nullptr, nullptr, nullptr, lw.fc2_w, p, s, next ? next->ln1_g : nullptr,
-                       next ? next->ln1_b : nullptr, next ? next->qkv_w : nullptr, 3 * d, d)
+                       next ? next->ln1_b : nullptr)
               : gemm(h, h->h1, lw.fc2_w, p, s);
     if (e != cudaSuccess) return e;
   }

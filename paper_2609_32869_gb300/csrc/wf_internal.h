@@ -179,10 +179,6 @@ struct SkinnyParams {
   // skinny_sattn: 0 causal (target), 1 block (drafter: all of [0, L + M), RoPE)
   int xa_mode;
   const float2 *rope_tab;  // [max_pos][32] (cos, sin), mode 1
-  // nullable: weights of the next projection in the chain, brought into L2
-  // in the prologue (pf_bytes, a multiple of 16, 16-byte aligned)
-  const void *pf;
-  size_t pf_bytes;
   uint32_t *err;
   long long spin;
 };

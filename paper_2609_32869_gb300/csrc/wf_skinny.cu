@@ -1,10 +1,12 @@
 // Low-latency projections for a handful of token rows (M <= 16: one
 // speculative block of K + 1 = 9 rows, a plain greedy step, a short prompt).
 //
-// At batch 1 a decoder block is a chain of eight dependent steps over 46 MB
-// of weights (Sec. 3.1: one verify pass; Sec. 3.2: one drafter pass), so each
+// At batch 1 a decoder block is a chain of dependent steps over 46 MB of
+// weights (Sec. 3.1: one verify pass; Sec. 3.2: one drafter pass), so each
 // projection's time after its dependency wait, not its weight stream, sets
-// the step time.  This kernel is shaped for that:
+// the step time.  The kernels here are shaped for that (the QKV and the
+// cross-query projections of one sequence also carry their attention, in
+// skinny_sattn_kernel and skinny_xattn_kernel below):
 //  - every CTA owns U units of 8 weight rows over a K range (the whole K, or
 //    1/S of it inside a cluster of S CTAs) and requests its entire weight slab
 //    with TMA before griddepcontrol.wait, one 3-D tensor copy per unit that
@@ -21,7 +23,7 @@
 //    arrival and the MMAs.  (The history memory's LN_h, over fp32 rows, is
 //    computed in the kernel instead: the CTAs of a cluster split the rows and
 //    write the normalised bf16 rows into every CTA over distributed shared
-//    memory.);
+//    memory.)
 //  - all eight warps issue mma.sync m16n8k16 at once (tokens on the 16-row
 //    side, weight rows on the 8-column side), each over its own slice of K;
 //    the slices are summed in warp order, then (S > 1) the S CTAs' sums in
@@ -49,28 +51,6 @@ constexpr int kSkWarps = kSkThreads / 32;
 // fit on one SM's 228 KB with the per-CTA reserve.
 constexpr int kSkSmemBudget = 113 * 1024;
 
-
-// The same copy marked evict-first in L2: a step streams every weight once
-// (far more bytes than L2 holds), so the weights should not push out the
-// small activations and statistics that the next launches read.
-__device__ __forceinline__ void tma_load_3d_stream(void *smem_dst, const CUtensorMap *m, int32_t x,
-                                                   int32_t y, int32_t z, uint64_t *bar, uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-      " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_u32(smem_dst)),
-      "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "l"(policy)
-      : "memory");
-}
-__device__ __forceinline__ uint64_t l2_evict_first_policy() {
-  uint64_t pol;
-  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
-  return pol;
-}
-// Bring [src, src + bytes) into L2 (16-byte aligned, size a multiple of 16).
-__device__ __forceinline__ void l2_prefetch_bulk(const void *src, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(src)), "r"(bytes)
-               : "memory");
-}
 
 // Shared-memory layout of one CTA (offsets from the 1024-aligned base).  The
 // warps' partial sums reuse the weight slab once every MMA has read it.
@@ -165,19 +145,8 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
     *sZero = make_uint4(0u, 0u, 0u, 0u);
     // the whole weight slab: one copy per unit, before the dependency wait
     mbar_arrive_expect_tx(&bar[0], static_cast<uint32_t>(U * unit_bytes));
-    const uint64_t pol = l2_evict_first_policy();
     for (int u = 0; u < U; ++u)
-      tma_load_3d_stream(sW + static_cast<size_t>(u) * unit_bytes, &tmW, 0, (unit0 + u) * 8, split * kb, &bar[0],
-                         pol);
-    // this CTA's share of the next projection's weights, into L2
-    if (p.pf) {
-      const size_t n_cta = static_cast<size_t>(gridDim.x) * gridDim.z;
-      const size_t share = ((p.pf_bytes + n_cta - 1) / n_cta + 15) & ~static_cast<size_t>(15);
-      const size_t lo = (static_cast<size_t>(split) * gridDim.x + cta) * share;
-      const size_t hi = lo + share < p.pf_bytes ? lo + share : p.pf_bytes;
-      for (size_t off = lo; off < hi; off += 32768)
-        l2_prefetch_bulk(static_cast<const uint8_t *>(p.pf) + off, static_cast<uint32_t>(hi - off < 32768 ? hi - off : 32768));
-    }
+      tma_load_3d(sW + static_cast<size_t>(u) * unit_bytes, &tmW, 0, (unit0 + u) * 8, split * kb, &bar[0]);
   }
   for (int i = tid; i < U * 8; i += kSkThreads) {
     const int n = n_base + i;
@@ -592,7 +561,7 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_xattn_kernel(const __gri
     fence_barrier_init();
     *sZero = make_uint4(0u, 0u, 0u, 0u);
     mbar_arrive_expect_tx(&bar[0], static_cast<uint32_t>(kb * 1024));
-    tma_load_3d_stream(sW, &tmW, 0, n_base, 0, &bar[0], l2_evict_first_policy());
+    tma_load_3d(sW, &tmW, 0, n_base, 0, &bar[0]);
     if (any_keys) {  // the acoustic memory of this CTA's frames
       const int slot = p.seq_slot[0];
       const int outer = slot * p.n_heads + head;
@@ -602,14 +571,6 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_xattn_kernel(const __gri
       tma_load_3d(sK, &tmK, 0, key0, outer, &bar[2]);
       mbar_arrive_expect_tx(&bar[3], static_cast<uint32_t>(kpc * 128));
       tma_load_3d(sV, &tmV, 0, key0, outer, &bar[3]);
-    }
-    if (p.pf) {  // this CTA's share of the next projection's weights, into L2
-      const size_t share = ((p.pf_bytes + gridDim.x - 1) / gridDim.x + 15) & ~static_cast<size_t>(15);
-      const size_t lo = static_cast<size_t>(cta) * share;
-      const size_t hi = lo + share < p.pf_bytes ? lo + share : p.pf_bytes;
-      for (size_t off = lo; off < hi; off += 32768)
-        l2_prefetch_bulk(static_cast<const uint8_t *>(p.pf) + off,
-                         static_cast<uint32_t>(hi - off < 32768 ? hi - off : 32768));
     }
   }
   if (tid < 8) sBias[tid] = p.bias ? bf2f(p.bias[n_base + tid]) : 0.f;
@@ -978,8 +939,7 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_sattn_kernel(const __gri
     fence_barrier_init();
     *sZero = make_uint4(0u, 0u, 0u, 0u);
     mbar_arrive_expect_tx(&bar[0], static_cast<uint32_t>(3 * kb * 1024));
-    const uint64_t pol = l2_evict_first_policy();
-    for (int u = 0; u < 3; ++u) tma_load_3d_stream(sW + u * kb * 1024, &tmW, 0, unit_row(u), 0, &bar[0], pol);
+    for (int u = 0; u < 3; ++u) tma_load_3d(sW + u * kb * 1024, &tmW, 0, unit_row(u), 0, &bar[0]);
     if (any_keys) {  // this CTA's positions; rows from L on are replaced below
       tma_prefetch_desc(&tmK);
       tma_prefetch_desc(&tmV);
@@ -987,14 +947,6 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_sattn_kernel(const __gri
       tma_load_3d(sK, &tmK, 0, key0, outer, &bar[2]);
       mbar_arrive_expect_tx(&bar[3], static_cast<uint32_t>(kpc * 128));
       tma_load_3d(sV, &tmV, 0, key0, outer, &bar[3]);
-    }
-    if (p.pf) {
-      const size_t share = ((p.pf_bytes + gridDim.x - 1) / gridDim.x + 15) & ~static_cast<size_t>(15);
-      const size_t lo = static_cast<size_t>(cta) * share;
-      const size_t hi = lo + share < p.pf_bytes ? lo + share : p.pf_bytes;
-      for (size_t off = lo; off < hi; off += 32768)
-        l2_prefetch_bulk(static_cast<const uint8_t *>(p.pf) + off,
-                         static_cast<uint32_t>(hi - off < 32768 ? hi - off : 32768));
     }
   }
   if (tid < 24) sBias[tid] = p.bias ? bf2f(p.bias[unit_row(tid >> 3) + (tid & 7)]) : 0.f;
