@@ -863,8 +863,8 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_xattn_kernel(const __gri
 // those of the cross-attention kernel above.
 namespace {
 struct SaLayout {
-  int w_off, a_off, k_off, v_off, q_off, pb_off, sum_off, bias_off, stat_off, ml_off, bar_off, zero_off, flag_off,
-      total;
+  int w_off, a_off, k_off, v_off, q_off, new_off, pb_off, sum_off, bias_off, stat_off, ml_off, bar_off, zero_off,
+      flag_off, total;
   __host__ __device__ SaLayout(int Mr, int K, int kpc) {
     const int kb = K / 64;
     w_off = 0;
@@ -872,11 +872,13 @@ struct SaLayout {
     k_off = (a_off + kb * Mr * 128 + 1023) & ~1023;
     v_off = k_off + kpc * 128;
     q_off = v_off + kpc * 128;
-    // the partial inbox reuses the operand tile, as in the cross-attention kernel
+    new_off = q_off + 16 * 128;  // the new key rows, then the new value rows: [2][16][128 B]
+    // the partial inbox reuses the operand tile, as in the cross-attention
+    // kernel, and the CTA sums sit in the slab behind the warps' partials
     const bool inbox_in_a = kb * Mr * 128 >= 8 * 16 * 12 * 4;
-    pb_off = inbox_in_a ? a_off : q_off + 16 * 128;
-    sum_off = q_off + 16 * 128 + (inbox_in_a ? 0 : 8 * 16 * 12 * 4);
-    bias_off = sum_off + 3 * 128 * 4;
+    pb_off = inbox_in_a ? a_off : new_off + 2 * 16 * 128;
+    sum_off = w_off + 8 * 3 * 128 * 4;
+    bias_off = new_off + 2 * 16 * 128 + (inbox_in_a ? 0 : 8 * 16 * 12 * 4);
     stat_off = bias_off + 24 * 4;
     ml_off = stat_off + kSkMaxRows * 8;
     bar_off = ml_off + 2 * 8 * 16 * 4;
@@ -902,6 +904,7 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_sattn_kernel(const __gri
   uint8_t *sK = smem + L.k_off;
   uint8_t *sV = smem + L.v_off;
   uint8_t *sQ = smem + L.q_off;
+  uint8_t *sKn = smem + L.new_off, *sVn = sKn + 16 * 128;  // new key / value rows, by block row
   float *pin = reinterpret_cast<float *>(smem + L.pb_off);   // [8 source CTAs][16][12]
   float *sPart = reinterpret_cast<float *>(smem + L.w_off);  // [8 warps][3 units][16][8]
   float *sSum = reinterpret_cast<float *>(smem + L.sum_off);  // [3][16][8]
@@ -930,6 +933,7 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_sattn_kernel(const __gri
   const bool any_keys = fits && key0 < n_keys;
   const int outer = slot * H + head;
 
+  cluster_arrive_relaxed();  // this CTA has started (peers write into it later)
   if (tid == 0) {
     *s_flag = fits ? 0 : 1;
     if (!fits) set_error(p.err, WF_DEV_ERR_CAPACITY);
@@ -1044,21 +1048,13 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_sattn_kernel(const __gri
     for (int w = 0; w < kSkWarps; ++w) v += sPart[(w * 3 + u) * 128 + rc];
     sSum[e] = v;
   }
-  // this CTA's keys and values have landed before any peer writes into them
-  bool kv_ok = true;
-  if (any_keys) {
-    kv_ok = mbar_wait(&bar[2], 0, p.err, spin);
-    kv_ok = mbar_wait(&bar[3], 0, p.err, spin) && kv_ok;
-  }
-  if (!kv_ok) *s_flag = 1;
   __syncthreads();
-  cluster_arrive();
-  cluster_wait();
+  cluster_wait();  // every CTA of the cluster has started
 
   // ---------------- the new rows: a lane group of 8 holds one (unit, row)'s
-  // 8 values.  Queries: lane j stores the chunk into CTA j.  Keys and values:
-  // every lane writes its value to the cache, lane 0 the chunk into the CTA
-  // attending to position L + t.
+  // 8 values; lane j stores the row's chunk into CTA j (queries into the
+  // query tile, keys and values into the new-row buffers), and every lane
+  // writes its key or value to the cache
   const int n_el = 3 * M * 8;
   for (int e0 = 0; e0 < n_el; e0 += kSkThreads) {
     if (e0 + warp * 32 >= n_el) break;  // warp-uniform
@@ -1085,17 +1081,29 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_sattn_kernel(const __gri
     chunk.z = __shfl_sync(0xffffffffu, pr, base + 4);
     chunk.w = __shfl_sync(0xffffffffu, pr, base + 6);
     if (live && fits) {
-      if (u == 0) {
-        dsmem_st_u32x4(dsmem_map(smem_u32(sQ) + swz(t, static_cast<int>(crank)), j), chunk);
-      } else if (j == 0) {
-        const int pos = Lc + t, owner = pos / kpc, r = pos - owner * kpc;
-        dsmem_st_u32x4(dsmem_map(smem_u32(u == 1 ? sK : sV) + swz(r, static_cast<int>(crank)),
-                                 static_cast<uint32_t>(owner)),
-                       chunk);
-      }
+      uint8_t *dst = u == 0 ? sQ : (u == 1 ? sKn : sVn);
+      dsmem_st_u32x4(dsmem_map(smem_u32(dst) + swz(t, static_cast<int>(crank)), j), chunk);
     }
   }
   cluster_sync();  // every chunk has landed
+  // this CTA's settled keys and values have landed: the new rows it attends
+  // to (positions L + t in its range) replace the stale cache rows there
+  bool kv_ok = true;
+  if (any_keys) {
+    kv_ok = mbar_wait(&bar[2], 0, p.err, spin);
+    kv_ok = mbar_wait(&bar[3], 0, p.err, spin) && kv_ok;
+  }
+  if (!kv_ok) *s_flag = 1;
+  {
+    const int t = tid >> 4, c = (tid >> 1) & 7, kv = tid & 1;  // 16 rows x 8 chunks x {K, V}
+    const int pos = Lc + t;
+    if (t < M && any_keys && pos >= key0 && pos < key0 + kpc) {
+      const uint8_t *src = kv ? sVn : sKn;
+      uint8_t *dst = kv ? sV : sK;
+      *reinterpret_cast<uint4 *>(dst + swz(pos - key0, c)) = *reinterpret_cast<const uint4 *>(src + swz(t, c));
+    }
+  }
+  __syncthreads();
 
   // ---------------- queries: RoPE (drafter) at L + r, then the 1/8 scale;
   // keys: RoPE at their positions; values past the visible keys: zeros
