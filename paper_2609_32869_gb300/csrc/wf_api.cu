@@ -379,7 +379,7 @@ cudaError_t skinny(wf_handle *h, const void *X, const float *ln_x, const void *g
   if (e == cudaSuccess && g_next) {  // partials per row: one per CTA of the plan
     int U = 0, S = 0;
     if (!skinny_plan(p.M, p.N, p.K, false, false, &U, &S)) return cudaErrorInvalidValue;
-    h->fold_np = p.N / 8 / U * S;
+    h->fold_np = p.N / 8 / U;  // one partial per CTA column block (its rank that finishes the row)
   }
   return e;
 }

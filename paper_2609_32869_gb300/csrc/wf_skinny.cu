@@ -158,11 +158,22 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
       reinterpret_cast<uint4 *>(sB)[i] = reinterpret_cast<const uint4 *>(p.ln_b)[i];
     }
   }
-  // epilogue outputs of this thread: element e = tid + i * threads of the
-  // U x M x 8 tile; the cache slot and position of a key/value row are fixed
-  // for the step, so they are read before the wait
+  // epilogue outputs: rank `split` finishes the token rows [r_lo, r_hi) (all
+  // of them when S == 1), every column u * 8 + j of each; its element
+  // f = (t - r_lo) * U * 8 + u * 8 + j goes to thread f % threads, so a
+  // warp holds whole rows when U * 8 divides 32.  The cache slot and
+  // position of a key/value row are fixed for the step, so they are read
+  // before the wait.
   constexpr int kEpi = (U * kSkMaxRows * 8 + kSkThreads - 1) / kSkThreads;
-  const int n_out = U * M * 8;
+  constexpr int kUC = U * 8;  // columns of this CTA
+  const int r_lo = M * split / S, r_hi = M * (split + 1) / S;
+  const int n_out = (r_hi - r_lo) * kUC;
+  auto elem = [&](int f, int &u, int &t, int &j) {
+    t = r_lo + f / kUC;
+    const int c = f - (t - r_lo) * kUC;
+    u = c >> 3;
+    j = c & 7;
+  };
   int kv_dst[kEpi];  // EPI_KV: cache row index (slot * heads + head) * ctx + position, or -1
   // EPI_RESID with a folded LayerNorm next: its gain (and, on token row 0,
   // its bias) at this thread's outputs
@@ -170,17 +181,20 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
 #pragma unroll
   for (int i = 0; i < kEpi; ++i) {
     kv_dst[i] = -1;
-    const int e = tid + i * kSkThreads;
+    const int f = tid + i * kSkThreads;
     g_nx[i] = b_nx[i] = 0.f;
-    if (p.xg_out && e < n_out) {
-      const int n = n_base + e / (M * 8) * 8 + (e & 7);
+    if (p.xg_out && f < n_out) {
+      int u, t, j;
+      elem(f, u, t, j);
+      const int n = n_base + u * 8 + j;
       if (n < p.N) {
         g_nx[i] = bf2f(p.g_next[n]);
-        if ((e % (M * 8)) < 8) b_nx[i] = bf2f(p.b_next[n]);
+        if (t == 0) b_nx[i] = bf2f(p.b_next[n]);
       }
     }
-    if (p.epi == EPI_KV && e < n_out) {
-      const int u = e / (M * 8), rem = e - u * M * 8, t = rem >> 3, j = rem & 7;
+    if (p.epi == EPI_KV && f < n_out) {
+      int u, t, j;
+      elem(f, u, t, j);
       const int n = n_base + u * 8 + j;
       if (n >= p.q_cols && n < p.N) {
         const int c = n - p.q_cols, hd = c % p.d_model;
@@ -204,9 +218,10 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
 #pragma unroll
   for (int i = 0; i < kEpi; ++i) {
     old[i] = 0.f;
-    const int e = tid + i * kSkThreads;
-    if (p.epi == EPI_RESID && e < n_out && (S == 1 || e % S == split)) {
-      const int u = e / (M * 8), rem = e - u * M * 8, t = rem >> 3, j = rem & 7;
+    const int f = tid + i * kSkThreads;
+    if (p.epi == EPI_RESID && f < n_out) {
+      int u, t, j;
+      elem(f, u, t, j);
       const int n = n_base + u * 8 + j;
       if (n < p.N) old[i] = __ldcg(p.resid + static_cast<size_t>(t) * p.ld_resid + n);
     }
@@ -383,81 +398,101 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
   const bool ok = landed;
   if (S > 1) cluster_sync();
   else __syncthreads();
+  // this CTA's partial (sum x, sum x^2) of each row it finishes, for the next
+  // LayerNorm: reduced over the row's lanes when a warp holds whole rows
+  constexpr bool kRowWarps = 32 % kUC == 0;
 #pragma unroll
   for (int i = 0; i < kEpi; ++i) {
-    const int e = tid + i * kSkThreads;
-    if (e >= n_out || (S > 1 && (e % S) != split)) continue;
-    const int u = e / (M * 8), rem = e - u * M * 8, t = rem >> 3, j = rem & 7;
-    const int idx = u * 128 + (t + t0) * 8 + j;
-    float v;
-    if (S > 1) {
-      float part[8];
-      const uint32_t loc = smem_u32(sSum + idx);
+    const int f = tid + i * kSkThreads;
+    float px = 0.f;  // the updated residual value this lane adds to its row's partial
+    bool pv = false;
+    if (f < n_out) {
+      int u, t, j;
+      elem(f, u, t, j);
+      const int idx = u * 128 + (t + t0) * 8 + j;
+      float v;
+      if (S > 1) {
+        float part[8];
+        const uint32_t loc = smem_u32(sSum + idx);
 #pragma unroll
-      for (int r = 0; r < 8; ++r)  // every load in flight before the sum
-        part[r] = r < S ? dsmem_ld_f32(dsmem_map(loc, r)) : 0.f;
-      v = 0.f;
+        for (int r = 0; r < 8; ++r)  // every load in flight before the sum
+          part[r] = r < S ? dsmem_ld_f32(dsmem_map(loc, r)) : 0.f;
+        v = 0.f;
 #pragma unroll
-      for (int r = 0; r < 8; ++r)
-        if (r < S) v += part[r];
-    } else {
-      v = sSum[idx];
-    }
-    const int n = n_base + u * 8 + j;
-    if (n >= p.N || !ok) continue;
-    if (fold) {  // r (W (g . x) - mu W g) + W b; rows 0 and 1 of the sums hold W g and W b
-      const float2 ms = sStat[t];
-      v = __fmaf_rn(ms.y, __fmaf_rn(-ms.x, sSum[u * 128 + j], v), sSum[u * 128 + 8 + j]);
-    }
-    v += sBias[u * 8 + j];
-    if (p.epi == EPI_F32) {
-      p.out_f32[static_cast<size_t>(t) * p.ld_out + n] = v;
-    } else if (p.epi == EPI_BF16) {
-      p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(v);
-    } else if (p.epi == EPI_GELU) {
-      p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(gelu_erf(v));
-    } else if (p.epi == EPI_RESID) {
-      const float nr = old[i] + v;
-      p.resid[static_cast<size_t>(t) * p.ld_resid + n] = nr;
-      if (p.xg_out) {
-        p.xg_out[static_cast<size_t>(t + 2) * p.ld_resid + n] = __float2bfloat16(nr * g_nx[i]);
-        if (t == 0) {  // bf16 values, converted back exactly
-          p.xg_out[n] = __float2bfloat16(g_nx[i]);
-          p.xg_out[static_cast<size_t>(p.ld_resid) + n] = __float2bfloat16(b_nx[i]);
-        }
-        sPart[u * 128 + t * 8 + j] = nr;  // the slab is free: the CTA's sums are in sSum
-      }
-      if (p.tap0) p.tap0[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
-      if (p.tap1) p.tap1[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
-    } else if (p.epi == EPI_KV) {
-      if (n < p.q_cols) {
-        p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(v);
-      } else if (kv_dst[i] == -2) {
-        set_error(p.err, WF_DEV_ERR_CAPACITY);
+        for (int r = 0; r < 8; ++r)
+          if (r < S) v += part[r];
       } else {
-        const int c = n - p.q_cols, which = c / p.d_model;
-        bf16 *dst = which == 0 ? p.kc : p.vc;
-        dst[static_cast<size_t>(kv_dst[i]) * 64 + ((c - which * p.d_model) & 63)] = __float2bfloat16(v);
+        v = sSum[idx];
       }
+      const int n = n_base + u * 8 + j;
+      if (n < p.N && ok) {
+        if (fold) {  // r (W (g . x) - mu W g) + W b; rows 0 and 1 of the sums hold W g and W b
+          const float2 ms = sStat[t];
+          v = __fmaf_rn(ms.y, __fmaf_rn(-ms.x, sSum[u * 128 + j], v), sSum[u * 128 + 8 + j]);
+        }
+        v += sBias[u * 8 + j];
+        if (p.epi == EPI_F32) {
+          p.out_f32[static_cast<size_t>(t) * p.ld_out + n] = v;
+        } else if (p.epi == EPI_BF16) {
+          p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(v);
+        } else if (p.epi == EPI_GELU) {
+          p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(gelu_erf(v));
+        } else if (p.epi == EPI_RESID) {
+          const float nr = old[i] + v;
+          p.resid[static_cast<size_t>(t) * p.ld_resid + n] = nr;
+          if (p.xg_out) {
+            p.xg_out[static_cast<size_t>(t + 2) * p.ld_resid + n] = __float2bfloat16(nr * g_nx[i]);
+            if (t == 0) {  // bf16 values, converted back exactly
+              p.xg_out[n] = __float2bfloat16(g_nx[i]);
+              p.xg_out[static_cast<size_t>(p.ld_resid) + n] = __float2bfloat16(b_nx[i]);
+            }
+            px = nr;
+            pv = true;
+            if (!kRowWarps) sPart[u * 128 + t * 8 + j] = nr;  // the slab is free: the sums are in sSum
+          }
+          if (p.tap0) p.tap0[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
+          if (p.tap1) p.tap1[static_cast<size_t>(t) * p.ld_tap + n] = __float2bfloat16(nr);
+        } else if (p.epi == EPI_KV) {
+          if (n < p.q_cols) {
+            p.out_bf16[static_cast<size_t>(t) * p.ld_out + n] = __float2bfloat16(v);
+          } else if (kv_dst[i] == -2) {
+            set_error(p.err, WF_DEV_ERR_CAPACITY);
+          } else {
+            const int c = n - p.q_cols, which = c / p.d_model;
+            bf16 *dst = which == 0 ? p.kc : p.vc;
+            dst[static_cast<size_t>(kv_dst[i]) * 64 + ((c - which * p.d_model) & 63)] = __float2bfloat16(v);
+          }
+        }
+      }  // n < N && ok
+    }  // f < n_out
+    if (kRowWarps && p.xg_out && i * kSkThreads + warp * 32 < n_out) {  // warp-uniform
+      float s1 = pv ? px : 0.f, s2 = pv ? px * px : 0.f;
+#pragma unroll
+      for (int off = kUC / 2; off > 0; off >>= 1) {
+        s1 += __shfl_xor_sync(0xffffffffu, s1, off);
+        s2 += __shfl_xor_sync(0xffffffffu, s2, off);
+      }
+      if (f < n_out && (f % kUC) == 0 && ok)
+        p.part_out[static_cast<size_t>(r_lo + f / kUC) * p.part_stride + cta] = make_float2(s1, s2);
     }
   }
-  if (p.xg_out) {
-    // this CTA's partial (sum x, sum x^2) of every row over the outputs it
-    // finished: warp w takes rows w and w + 8, lane l the outputs (u, j) with
-    // u = l / 8 + 4 i and j = l % 8, added in order of i, then across lanes
+  if (!kRowWarps && p.xg_out) {
+    // rows wider than a warp: warp w takes this rank's rows r_lo + w, + 8, ..,
+    // lane l the outputs (u, j) with u = l / 8 + 4 i and j = l % 8, added in
+    // order of i, then across lanes
     __syncthreads();
-    for (int t = warp; t < M; t += kSkWarps) {
+    for (int t = r_lo + warp; t < r_hi; t += kSkWarps) {
       float s1 = 0.f, s2 = 0.f;
       for (int u = lane >> 3; u < U; u += 4) {
-        const int j = lane & 7, e = u * M * 8 + t * 8 + j;
-        if ((S > 1 && e % S != split) || n_base + u * 8 + j >= p.N || !ok) continue;
+        const int j = lane & 7;
+        if (n_base + u * 8 + j >= p.N || !ok) continue;
         const float x = sPart[u * 128 + t * 8 + j];
         s1 += x;
-        s2 = __fmaf_rn(x, x, s2);
+        s2 += x * x;
       }
       s1 = warp_sum(s1);
       s2 = warp_sum(s2);
-      if (lane == 0) p.part_out[static_cast<size_t>(t) * p.part_stride + cta * S + split] = make_float2(s1, s2);
+      if (lane == 0) p.part_out[static_cast<size_t>(t) * p.part_stride + cta] = make_float2(s1, s2);
     }
   }
   if (S > 1) cluster_sync();  // peers may read this CTA's sums until here
@@ -1429,7 +1464,7 @@ cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pd
     return cudaErrorInvalidValue;
   if (!ln && (!p.x || p.ld_x % 8 || (reinterpret_cast<uintptr_t>(p.x) & 15))) return cudaErrorInvalidValue;
   if (p.xg_out && (p.epi != EPI_RESID || !p.g_next || !p.b_next || !p.part_out ||
-                   p.N / 8 / p.U * p.S > p.part_stride))
+                   p.N / 8 / p.U > p.part_stride))
     return cudaErrorInvalidValue;
   const CUtensorMap *tm = skinny_tmap(W, p.N, p.K, p.K / p.S / 64);
   if (!tm) return cudaErrorInvalidValue;
