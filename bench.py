@@ -491,8 +491,9 @@ def run_ours(args, rank, world):
         "consistent": m["consistent"],
         "device_error": m["err"],
     }
-    if args.workload == "large_b1" and not args.no_per_batch and not args.budget:
-        # the metric's other batch sizes, timed in the same run on the same weights
+    if args.workload == "large_b1" and not args.no_per_batch and not args.budget and not args.persist:
+        # the metric's other batch sizes, timed in the same run on the same
+        # weights (launch by launch: the persistent passes serve <= 16 rows)
         per = {}
         for name in ("large_b16", "large_b96"):
             mb = measure_greedy(args, name, dev, None, rank, world, args.batch_steps, args.warmup, e2e=False)

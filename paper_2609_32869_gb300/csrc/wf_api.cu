@@ -347,6 +347,7 @@ cudaError_t skinny(wf_handle *h, const void *X, const float *ln_x, const void *g
                    const void *W, const GemmParams &gp, cudaStream_t s, const void *g_next = nullptr,
                    const void *b_next = nullptr) {
   SkinnyParams p = skinny_of(gp);
+  p.plan_M = h->sk_rows;
   if (g_next) {
     p.xg_out = h->xg;
     p.g_next = static_cast<const bf16 *>(g_next);
@@ -378,7 +379,7 @@ cudaError_t skinny(wf_handle *h, const void *X, const float *ln_x, const void *g
   prof_end(h, s, WF_FAM_GEMM, gemm_bytes(gp));
   if (e == cudaSuccess && g_next) {  // partials per row: one per CTA of the plan
     int U = 0, S = 0;
-    if (!skinny_plan(p.M, p.N, p.K, false, false, &U, &S)) return cudaErrorInvalidValue;
+    if (!skinny_plan(p.plan_M, p.N, p.K, false, false, &U, &S)) return cudaErrorInvalidValue;
     h->fold_np = p.N / 8 / U;  // one partial per CTA column block (its rank that finishes the row)
   }
   return e;

@@ -136,6 +136,10 @@ constexpr int kSkMaxFoldRows = kSkMaxRows - 2;  // token rows of a folded LayerN
 constexpr int kSkMaxParts = 160;                // partial row sums of one residual update
 struct SkinnyParams {
   int M, N, K;
+  // token rows the plan (U, S) is chosen for, >= M (0: M): every pass of a
+  // handle plans for its largest, so a row's arithmetic (K split, partial
+  // sums) does not depend on how many rows run with it
+  int plan_M;
   int U, S, C;  // set by launch_skinny (C: CTAs of a cluster sharing a LayerNorm operand)
   int epi;
   const bf16 *x;

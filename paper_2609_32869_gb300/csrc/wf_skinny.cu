@@ -1459,7 +1459,9 @@ cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pd
   if (fold && (ln || p.M > kSkMaxFoldRows || !p.fold_part || p.n_part < 1 || p.n_part > p.part_stride))
     return cudaErrorInvalidValue;
   const int Mr = p.M + (fold ? 2 : 0);  // operand rows
-  if (!skinny_plan(Mr, p.N, p.K, ln, fold, &p.U, &p.S)) return cudaErrorInvalidValue;
+  if (p.plan_M && p.plan_M < p.M) return cudaErrorInvalidValue;
+  const int Mp = (p.plan_M ? p.plan_M : p.M) + (fold ? 2 : 0);  // operand rows of the plan
+  if (!skinny_plan(Mp, p.N, p.K, ln, fold, &p.U, &p.S)) return cudaErrorInvalidValue;
   if (ln && (!p.ln_g || !p.ln_b || p.ln_ld % 4 || (reinterpret_cast<uintptr_t>(p.ln_x) & 15)))
     return cudaErrorInvalidValue;
   if (!ln && (!p.x || p.ld_x % 8 || (reinterpret_cast<uintptr_t>(p.x) & 15))) return cudaErrorInvalidValue;

@@ -196,6 +196,7 @@ def test_persistent_large_shapes_match_oracle():
     prompt = syn.prompts(cfg, 1, length=4, seed=1)
     budget = 60
     s = Session(cfg, ws, max_batch=1, keep_logits=True)
+    B.wf_set_option(s.h, B.WF_OPT_PERSIST, 1)
     first = int(s.prefill([0], enc, prompt, np.array([budget], np.int32)).cpu()[0])
     o = WhisperFlashOracle(syn.weights_as_float(ws, np.float64), cfg)
     encf = syn.bf16_bits_to_f32(enc[0]).astype(np.float64)
