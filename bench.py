@@ -77,11 +77,24 @@ WORKLOADS = {
 # same per-layer shapes (profiles/dram_per_kernel_large_b1_4l.md and
 # profiles/dram_per_kernel_large_b96_2l.md); None where no capture covers the
 # workload's shapes.
-GEMM_DRAM_BYTES_PER_LAUNCH = {}
+GEMM_DRAM_BYTES_PER_LAUNCH = {
+    # 68 x out/cross-out (3.404 MB), 34 x fc1 (13.219), 34 x fc2 (13.313),
+    # 2 x history K/V (6.662), 1 x history projection (16.572) per step
+    "large_b1": 8.370e6,
+    # 34 x QKV (12.077 MB), 102 x out/cross-out/fc2 (15.296), 34 x cross-query
+    # (5.514), 34 x fc1 (15.354), 2 x history K/V (8.796), 1 x history
+    # projection (27.283) per step, captured at 94 sequences
+    "large_b96": 13.165e6,
+}
 
 # Tensor-pipe activity of the projections at batch 96 from the committed ncu
 # capture of the same kernels (profiles/), or absent until one is taken.
-TENSOR_PIPE_FROM_PROFILE = {}
+TENSOR_PIPE_FROM_PROFILE = {
+    "large_b96": {"pct_of_peak_elapsed_time_weighted": 7.8,
+                  "by_projection": {"fc1": 12.0, "QKV": 9.1, "cross_query": 6.2,
+                                    "out_crossout_fc2": 5.7, "history_kv": 10.1},
+                  "source": "profiles/dram_per_kernel_large_b96_2l.md (ncu, 94 sequences, 2 target blocks)"},
+}
 
 
 def aggregate_ranks(times, counts, world, device):
