@@ -52,6 +52,8 @@ typedef enum wf_status {
 #define WF_DEV_ERR_TIMEOUT 0x1u  /* a bounded spin-wait gave up; results are invalid */
 #define WF_DEV_ERR_CAPACITY 0x2u /* a sequence would pass max_ctx; it was frozen */
 #define WF_DEV_ERR_TOKEN 0x4u    /* a token id outside [0, vocab) was clamped */
+#define WF_DEV_ERR_LAUNCH 0x8u   /* a kernel found its launch inconsistent with its plan
+                                    (grid, cluster or shared memory) and did nothing */
 
 #define WF_MAX_TAPS 8
 #define WF_MAX_LAYERS 64
@@ -242,11 +244,13 @@ int32_t wf_last_launch_count(const wf_handle *h);
                                 restores about 1 s (projections) and 0.2 s (persistent pass).
                                 Meant for tests of the failure path: a limit below a wait's
                                 normal duration makes the results of that call invalid. */
-#define WF_OPT_SKINNY 7      /* 1 (default when max_batch * (block_k + 1) <= 16): passes of at
-                                most 16 token rows run their projections as low-latency
-                                kernels that hold a CTA's whole weight slab in shared memory
-                                and reduce K in a fixed order; 0: the tcgen05 projections.
-                                Setting 1 on a larger handle returns WF_ERR_UNSUPPORTED.
+#define WF_OPT_SKINNY 7      /* 1 (default when max_batch * (block_k + 1) <= 144): passes of
+                                at most that many token rows run their projections as
+                                low-latency kernels that hold a CTA's whole weight slab in
+                                shared memory and reduce K in a fixed order (up to 16 rows
+                                with the whole token operand resident, more with it streamed
+                                by k-block); 0: the tcgen05 projections.  Setting 1 on a
+                                larger handle returns WF_ERR_UNSUPPORTED.
                                 The two forms agree within the method's tolerances, not bit
                                 for bit; a handle's speculative and plain greedy steps
                                 always take the same form. */

@@ -16,7 +16,7 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libwf.so")
 _lib = None
 
 WF_OK, WF_ERR_INVALID, WF_ERR_CAPACITY, WF_ERR_CUDA, WF_ERR_UNSUPPORTED, WF_ERR_DEVICE = range(6)
-WF_DEV_ERR_TIMEOUT, WF_DEV_ERR_CAPACITY, WF_DEV_ERR_TOKEN = 1, 2, 4
+WF_DEV_ERR_TIMEOUT, WF_DEV_ERR_CAPACITY, WF_DEV_ERR_TOKEN, WF_DEV_ERR_LAUNCH = 1, 2, 4, 8
 WF_MAX_TAPS = 8
 WF_OPT_KEEP_LOGITS = 1
 WF_OPT_PROFILE = 2

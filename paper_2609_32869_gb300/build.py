@@ -20,7 +20,8 @@ BUILD_DIR = os.path.join(PKG, "_build")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "--expt-relaxed-constexpr", "-I", os.path.join(ROOT, "include")]
-SOURCES = ["wf_gemm.cu", "wf_skinny.cu", "wf_attn.cu", "wf_step_kernels.cu", "wf_persist.cu", "wf_api.cu"]
+SOURCES = ["wf_gemm.cu", "wf_skinny.cu", "wf_skinny_mt.cu", "wf_attn.cu", "wf_step_kernels.cu", "wf_persist.cu",
+           "wf_api.cu"]
 
 
 def _nvcc() -> str:

@@ -181,8 +181,11 @@ size_t layout(wf_handle *h, const wf_config *c, int Bmax, int ctx, char *base) {
   o->st_xd = cv.take<float2>(M * (d / 128));
   o->st_hp = cv.take<float2>(M * (d / 128));
   o->xn = cv.take<bf16>(M * d);
-  o->xg = cv.take<bf16>(static_cast<size_t>(kSkMaxRows) * d);
-  o->fpart = cv.take<float2>(static_cast<size_t>(kSkMaxRows) * kSkMaxParts);
+  // the skinny passes' folded operand rows and partial sums: up to the
+  // handle's largest step pass (or kSkMaxRows), plus the rows g and b
+  const size_t xg_rows = static_cast<size_t>(std::max(kSkMaxRows, std::min(Bmax * (K + 1), kMtMaxRows)));
+  o->xg = cv.take<bf16>((xg_rows + 2) * d);
+  o->fpart = cv.take<float2>(xg_rows * kSkMaxParts);
   o->q = cv.take<bf16>(M * d);
   o->att = cv.take<bf16>(M * d);
   o->hn = cv.take<bf16>(M * d);
@@ -256,12 +259,25 @@ cudaEvent_t prof_event(wf_handle *h) {
   }
   return h->ev_pool[h->ev_next++];
 }
+// WF_DEBUG_SYNC in the environment: synchronise after every launch made
+// outside graph capture and name the first that fails on stderr (debugging
+// only: it serialises the launches).
+void debug_sync(cudaStream_t s, const char *what, int M, int N, int K) {
+  static const bool on = getenv("WF_DEBUG_SYNC") != nullptr;
+  if (!on) return;
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(s, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) return;
+  const cudaError_t e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) fprintf(stderr, "libwf: %s (M=%d N=%d K=%d) failed: %s\n", what, M, N, K, cudaGetErrorString(e));
+}
 void prof_begin(wf_handle *h, cudaStream_t s) {
   if (!h->profile) return;
   h->pending = prof_event(h);
   if (h->pending) cudaEventRecord(h->pending, s);
 }
 void prof_end(wf_handle *h, cudaStream_t s, int fam, double bytes) {
+  static const char *const kFam[] = {"gemm", "head", "attn_self", "attn_cross", "layernorm", "other", "persist"};
+  debug_sync(s, fam >= 0 && fam < 7 ? kFam[fam] : "launch", -1, -1, -1);
   if (!h->profile || !h->pending) return;
   cudaEvent_t b = prof_event(h);
   if (!b) return;
@@ -347,7 +363,10 @@ cudaError_t skinny(wf_handle *h, const void *X, const float *ln_x, const void *g
                    const void *W, const GemmParams &gp, cudaStream_t s, const void *g_next = nullptr,
                    const void *b_next = nullptr) {
   SkinnyParams p = skinny_of(gp);
-  p.plan_M = h->sk_rows;
+  // passes of more rows than one operand tile holds stream the operand (an
+  // fp32 LayerNorm operand always fits one tile: it plans for its own rows)
+  const bool mt = h->sk_rows > kSkMaxFoldRows && !ln_x;
+  p.plan_M = (h->sk_rows > kSkMaxFoldRows && ln_x) ? gp.M : h->sk_rows;
   if (g_next) {
     p.xg_out = h->xg;
     p.g_next = static_cast<const bf16 *>(g_next);
@@ -375,20 +394,30 @@ cudaError_t skinny(wf_handle *h, const void *X, const float *ln_x, const void *g
   }
   h->launches++;
   prof_begin(h, s);
-  cudaError_t e = launch_skinny(W, p, s, kPDL);
+  cudaError_t e = mt ? launch_skinny_mt(W, p, s, kPDL) : launch_skinny(W, p, s, kPDL);
+  debug_sync(s, mt ? "skinny_mt" : "skinny", p.M, p.N, p.K);
   prof_end(h, s, WF_FAM_GEMM, gemm_bytes(gp));
-  if (e == cudaSuccess && g_next) {  // partials per row: one per CTA of the plan
-    int U = 0, S = 0;
-    if (!skinny_plan(p.plan_M, p.N, p.K, false, false, &U, &S)) return cudaErrorInvalidValue;
-    h->fold_np = p.N / 8 / U;  // one partial per CTA column block (its rank that finishes the row)
+  if (e == cudaSuccess && g_next) {  // partials per row: one per CTA column block of the plan
+    int U = 0, S = 0, ns = 0;
+    const bool planned = mt ? skinny_mt_plan(p.plan_M + (p.fold ? 2 : 0), p.N, p.K, p.fold != 0,
+                                             p.epi == EPI_RESID, &U, &S, &ns)
+                            : skinny_plan(p.plan_M, p.N, p.K, false, false, &U, &S);
+    if (!planned) return cudaErrorInvalidValue;
+    h->fold_np = p.N / 8 / U;
   }
   return e;
 }
 
-// Whether every projection of a pass of up to M rows has a skinny plan.
+// Whether every projection of a pass of up to M rows has a skinny plan
+// (one operand tile up to kSkMaxFoldRows rows, a streamed operand up to
+// kMtMaxRows).
 bool skinny_shapes_fit(int d, int F, int M) {
   // folded LayerNorm operands carry two more rows (g and b)
-  int U = 0, S = 0;
+  int U = 0, S = 0, ns = 0;
+  if (M > kSkMaxFoldRows)  // QKV, out (and cross out), cross query, fc1, fc2
+    return M <= kMtMaxRows && skinny_mt_plan(M + 2, 3 * d, d, true, false, &U, &S, &ns) &&
+           skinny_mt_plan(M, d, d, false, true, &U, &S, &ns) && skinny_mt_plan(M + 2, d, d, true, false, &U, &S, &ns) &&
+           skinny_mt_plan(M + 2, F, d, true, false, &U, &S, &ns) && skinny_mt_plan(M, d, F, false, true, &U, &S, &ns);
   return M <= kSkMaxFoldRows && skinny_plan(M + 2, 3 * d, d, false, true, &U, &S) &&
          skinny_plan(M, d, d, false, false, &U, &S) && skinny_plan(M + 2, d, d, false, true, &U, &S) &&
          skinny_plan(M + 2, F, d, false, true, &U, &S) && skinny_plan(M, d, F, false, false, &U, &S) &&
@@ -572,9 +601,11 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
     xkc = h->cross_k + layer_cache_off(h, layer, h->cfg.enc_frames);
     xvc = h->cross_v + layer_cache_off(h, layer, h->cfg.enc_frames);
   }
-  // self-attention: for one sequence on the skinny path, the QKV projection
-  // and the attention run as one kernel (a cluster per head)
-  if (ps.sk && ps.n_seq == 1 && skinny_sattn_fits(M, d, h->H, h->ctx)) {
+  // self-attention: for one sequence on a single-sequence handle's skinny
+  // path, the QKV projection and the attention run as one kernel (a cluster
+  // per head); a batched handle keeps its one projection form at any n_seq
+  const bool one_tile = ps.sk && ps.n_seq == 1 && h->sk_rows <= kSkMaxFoldRows;
+  if (one_tile && skinny_sattn_fits(M, d, h->H, h->ctx)) {
     if ((e = skinny_sattn(h, lw, kc, vc, ps, s)) != cudaSuccess) return e;
   } else {
   {
@@ -607,9 +638,8 @@ cudaError_t run_block(wf_handle *h, const Pass &ps, const wf_layer_weights &lw, 
               : gemm(h, h->att, lw.out_w, p, s);
     if (e != cudaSuccess) return e;
   }
-  // cross-attention: for one sequence on the skinny path, the query
-  // projection and the attention run as one kernel (a cluster per head)
-  if (ps.sk && ps.n_seq == 1 && skinny_xattn_fits(M, d, h->H, h->cfg.enc_frames)) {
+  // cross-attention: likewise the query projection and the attention
+  if (one_tile && skinny_xattn_fits(M, d, h->H, h->cfg.enc_frames)) {
     if ((e = skinny_xattn(h, lw, xkc, xvc, ps, s)) != cudaSuccess) return e;
   } else {
     {
@@ -726,7 +756,10 @@ cudaError_t ingest(wf_handle *h, int n_seq, int rps, const int32_t *slots, cudaS
   }
   // LN_h is applied inside each drafter block's key/value projection (or by
   // one LayerNorm kernel ahead of them when their tiles do not fit)
-  const bool sk = use_skinny(h, M);
+  // LN_h over the fp32 projection in the skinny kernel only for one operand
+  // tile that has a plan (whole K per CTA)
+  int sk_u = 0, sk_s = 0;
+  const bool sk = use_skinny(h, M) && M <= kSkMaxRows && skinny_plan(M, 2 * d, d, true, false, &sk_u, &sk_s);
   const bool fused = sk || gemm_ln_fits(M, 2 * d, d, EPI_KV);
   if (!fused &&
       (e = layernorm(h, h->hproj, h->st_hp, 1, 0, h->dw.hln_g, h->dw.hln_b, h->hn, M, s)) != cudaSuccess)
@@ -1055,7 +1088,8 @@ wf_status wf_create(const wf_config *cfg, const wf_target_weights *tw, const wf_
   h->sk_rows = max_batch * (cfg->block_k + 1);
   h->skinny_ok = skinny_shapes_fit(h->d, h->F, h->sk_rows);
   h->skinny = h->skinny_ok;
-  ok = ok && gemm_init() == cudaSuccess && skinny_init() == cudaSuccess && attention_init() == cudaSuccess &&
+  ok = ok && gemm_init() == cudaSuccess && skinny_init() == cudaSuccess && skinny_mt_init() == cudaSuccess &&
+       attention_init() == cudaSuccess &&
        step_kernels_init() == cudaSuccess &&
        cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) == cudaSuccess;
   if (ok && h->mk_ok) ok = persist_setup(h, s) == cudaSuccess;

@@ -141,6 +141,7 @@ struct SkinnyParams {
   // sums) does not depend on how many rows run with it
   int plan_M;
   int U, S, C;  // set by launch_skinny (C: CTAs of a cluster sharing a LayerNorm operand)
+  int ns;       // set by launch_skinny_mt: k-blocks of its operand ring
   int epi;
   const bf16 *x;
   int ld_x;
@@ -192,6 +193,15 @@ struct SkinnyParams {
 bool skinny_plan(int M, int N, int K, bool ln, bool whole_k, int *U, int *S);
 cudaError_t skinny_init();
 cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pdl);
+// The same projections for up to kMtMaxRows token rows (wf_skinny_mt.cu): the
+// weights resident as above, the operand streamed by k-block, warps over
+// units and 16-row tiles.  No fp32 LayerNorm operand (ln_x).  The plan of Mr
+// operand rows (a folded LayerNorm's two included): units per CTA U, K split
+// S, operand ring stages ns.
+constexpr int kMtMaxRows = 144;  // 16 sequences x (1 + 8)
+bool skinny_mt_plan(int Mr, int N, int K, bool fold, bool resid, int *U, int *S, int *ns);
+cudaError_t skinny_mt_init();
+cudaError_t launch_skinny_mt(const void *W, SkinnyParams p, cudaStream_t s, bool pdl);
 // The cross-query projection (folded LN2, one sequence) fused with the
 // cross-attention of its queries: one cluster of 8 CTAs per 64-dim head.
 // False when the shapes do not allow it (then run the two separately).

@@ -205,6 +205,7 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
       }
     }
   }
+  __syncthreads();  // the barriers are initialised before any thread waits on them
   pdl_launch_dependents();
   pdl_wait();
 
@@ -609,6 +610,7 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_xattn_kernel(const __gri
     }
   }
   if (tid < 8) sBias[tid] = p.bias ? bf2f(p.bias[n_base + tid]) : 0.f;
+  __syncthreads();  // the barriers are initialised before any thread waits on them
   pdl_launch_dependents();
   pdl_wait();
 
@@ -989,6 +991,7 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_sattn_kernel(const __gri
     }
   }
   if (tid < 24) sBias[tid] = p.bias ? bf2f(p.bias[unit_row(tid >> 3) + (tid & 7)]) : 0.f;
+  __syncthreads();  // the barriers are initialised before any thread waits on them
   pdl_launch_dependents();
   pdl_wait();
 

@@ -8,8 +8,9 @@ the cache, so the final length is at most max_ctx.  Up to that point the
 speculative transcript must equal plain greedy decoding on a handle of the
 same shape, token for token: on a single-sequence handle (skinny projections
 with the attention fused into them, which attend to the short cache in
-blocks of 32 positions) and on a two-slot handle (tcgen05 projections and
-the separate attention kernel)."""
+blocks of 32 positions) and on a two-slot handle (the batched skinny
+projections, whose K/V epilogue checks each row's position, and the separate
+attention kernel)."""
 import numpy as np
 import pytest
 
@@ -41,7 +42,7 @@ def _run(cfg, dev, enc, prompt, max_batch, spec):
     return out, st, err, B
 
 
-@pytest.mark.parametrize("max_batch", [1, 2], ids=["skinny-fused", "tcgen05"])
+@pytest.mark.parametrize("max_batch", [1, 2], ids=["skinny-fused", "skinny-batched"])
 def test_capacity_freezes_the_sequence_inside_the_cache(max_batch):
     from paper_2609_32869_gb300.session import upload_weights
     cfg = syn.TINY

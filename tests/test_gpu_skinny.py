@@ -1,8 +1,10 @@
 """The low-latency projections of single-sequence handles (GPU).
 
-A handle whose every step pass has at most 16 token rows (max_batch 1: the
-anchor and K = 8 proposals) runs its projections with the skinny kernels
-(wf_skinny.cu, WF_OPT_SKINNY).  Checked against the oracle at the Whisper-tiny
+A handle whose every step pass has at most 144 token rows runs its
+projections with the skinny kernels (WF_OPT_SKINNY): at most 16 rows
+(max_batch 1: the anchor and K = 8 proposals) with the whole operand tile
+resident (wf_skinny.cu), more with the operand streamed by k-block
+(wf_skinny_mt.cu).  Checked against the oracle at the Whisper-tiny
 and Whisper-large shapes with every LayerNorm's gain and bias drawn on its own:
 draft and verify logits within 3e-2, tapped hidden states within 1e-2
 relative, tokens and cache lengths equal wherever the deciding margins
@@ -133,28 +135,35 @@ def test_skinny_speculative_equals_plain_greedy():
         s.close()
 
 
-def test_skinny_and_tcgen05_forms_agree():
+@pytest.mark.parametrize("n", [1, 4], ids=["one-sequence", "batched"])
+def test_skinny_and_tcgen05_forms_agree(n):
+    """The skinny form (one sequence: the whole operand tile resident; four:
+    the operand streamed by k-block) and the tcgen05 form of the same handle
+    agree within the logit tolerance; a handle of more than 144 step rows has
+    no skinny form."""
     import torch
     from paper_2609_32869_gb300 import binding as B
     from paper_2609_32869_gb300.session import Session, upload_weights
-    cfg, ws, enc, prompt = _setup("TINY")
+    cfg, ws, _, _ = _setup("TINY")
     K, V = cfg.block_k, cfg.vocab
+    enc = syn.encoder_output(cfg, n, seed=7)
+    prompt = syn.prompts(cfg, n, length=4, seed=7)
     dev = upload_weights(ws)
-    forced = syn.random_tokens(cfg, (1, K), seed=3)
+    forced = syn.random_tokens(cfg, (n, K), seed=3)
     out = {}
     for sk in (1, 0):
-        s = Session(cfg, dev, max_batch=1, keep_logits=True)
+        s = Session(cfg, dev, max_batch=n, keep_logits=True)
         B.wf_set_option(s.h, B.WF_OPT_SKINNY, sk)
-        s.prefill([0], enc, prompt, np.array([40], np.int32))
+        s.prefill(np.arange(n, dtype=np.int32), enc, prompt, np.full(n, 40, np.int32))
         s.step(forced=forced)
         torch.cuda.synchronize()
-        out[sk] = (s.view(B.WF_VIEW_TARGET_LOGITS, torch.float32, (K + 1, V)).cpu().numpy(),
-                   s.view(B.WF_VIEW_DRAFT_LOGITS, torch.float32, (K + 1, V)).cpu().numpy())
+        out[sk] = (s.view(B.WF_VIEW_TARGET_LOGITS, torch.float32, (n, K + 1, V)).cpu().numpy(),
+                   s.view(B.WF_VIEW_DRAFT_LOGITS, torch.float32, (n, K + 1, V)).cpu().numpy())
         assert s.error() == 0
         s.close()
     assert np.abs(out[1][0] - out[0][0]).max() <= LOGIT_ATOL
-    assert np.abs(out[1][1][1:] - out[0][1][1:]).max() <= LOGIT_ATOL
-    s4 = Session(cfg, dev, max_batch=4)
+    assert np.abs(out[1][1][:, 1:] - out[0][1][:, 1:]).max() <= LOGIT_ATOL
+    big = Session(cfg, dev, max_batch=17)
     with pytest.raises(B.WfError):
-        B.wf_set_option(s4.h, B.WF_OPT_SKINNY, 1)
-    s4.close()
+        B.wf_set_option(big.h, B.WF_OPT_SKINNY, 1)
+    big.close()
