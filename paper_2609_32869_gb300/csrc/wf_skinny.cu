@@ -205,8 +205,8 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_kernel(const __grid_cons
       }
     }
   }
-  __syncthreads();  // the barriers are initialised before any thread waits on them
   pdl_launch_dependents();
+  __syncthreads();  // the barriers are initialised before any thread waits on them
   pdl_wait();
 
   // ---------------- operand: bf16 rows by one TMA copy (issued first), the
@@ -610,8 +610,8 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_xattn_kernel(const __gri
     }
   }
   if (tid < 8) sBias[tid] = p.bias ? bf2f(p.bias[n_base + tid]) : 0.f;
-  __syncthreads();  // the barriers are initialised before any thread waits on them
   pdl_launch_dependents();
+  __syncthreads();  // the barriers are initialised before any thread waits on them
   pdl_wait();
 
   // ---------------- operand (rows g, b, then g . x) and the row statistics
@@ -991,8 +991,8 @@ __global__ void __launch_bounds__(kSkThreads, 2) skinny_sattn_kernel(const __gri
     }
   }
   if (tid < 24) sBias[tid] = p.bias ? bf2f(p.bias[unit_row(tid >> 3) + (tid & 7)]) : 0.f;
-  __syncthreads();  // the barriers are initialised before any thread waits on them
   pdl_launch_dependents();
+  __syncthreads();  // the barriers are initialised before any thread waits on them
   pdl_wait();
 
   // ---------------- operand (rows g, b, then g . x) and the row statistics

@@ -50,13 +50,16 @@ struct MtGrid {
   static constexpr int kUW = U / kWU;                        // units per warp
   static constexpr int kWT = kMtWarps / kWU;                 // tile groups
   static constexpr int kTW = (kMtMaxTiles + kWT - 1) / kWT;  // tiles per warp at most
+  // all of a warp's tiles' A fragments held at once (when few accumulators);
+  // a tile past the operand reads the zero line and its results are dropped
+  static constexpr bool kAllTiles = kTW * kUW <= 8;
 };
 
 // Shared-memory layout: Mr operand rows, Ks inputs, ns ring stages, at most
 // rows_o rows finished per rank.
 struct MtLayout {
-  int w_off, ring_off, stage_bytes, res_ld, part_off, old_off, bias_off, wgb_off, stat_off, bar_off, zero_off,
-      flag_off, total;
+  int w_off, ring_off, stage_bytes, res_ld, part_off, old_off, bias_off, wgb_off, gn_off, stat_off, row_off,
+      bar_off, zero_off, flag_off, total;
   __host__ __device__ MtLayout(int Mr, int Ks, int U, int ns, int rows_o, bool fold, bool resid) {
     const int kb = Ks / 64;
     w_off = 0;
@@ -69,8 +72,10 @@ struct MtLayout {
     old_off = part_off + (fold ? rows_o * kMtStageParts * 8 : 0);
     bias_off = old_off + (resid ? rows_o * U * 8 * 4 : 0);
     wgb_off = bias_off + U * 8 * 4;
-    stat_off = wgb_off + 2 * U * 8 * 4;
-    bar_off = (stat_off + rows_o * 8 + 15) & ~15;
+    gn_off = wgb_off + 2 * U * 8 * 4;
+    stat_off = gn_off + U * 8 * 4;
+    row_off = stat_off + rows_o * 8;
+    bar_off = (row_off + rows_o * 8 + 15) & ~15;
     zero_off = (bar_off + (1 + kMtMaxStages) * 8 + 15) & ~15;
     flag_off = zero_off + 16;
     total = flag_off + 16;
@@ -116,7 +121,9 @@ __global__ void __launch_bounds__(kMtThreads, 2) skinny_mt_kernel(const __grid_c
   float *sOld = reinterpret_cast<float *>(smem + L.old_off);
   float *sBias = reinterpret_cast<float *>(smem + L.bias_off);
   float *sWg = reinterpret_cast<float *>(smem + L.wgb_off);  // W g, then W b, summed over ranks
+  float *sGn = reinterpret_cast<float *>(smem + L.gn_off);   // the next LayerNorm's gain, these columns
   float2 *sStat = reinterpret_cast<float2 *>(smem + L.stat_off);
+  int2 *sRow = reinterpret_cast<int2 *>(smem + L.row_off);   // (cache slot, position) of each row finished
   uint64_t *wbar = reinterpret_cast<uint64_t *>(smem + L.bar_off);
   uint64_t *full = wbar + 1;
   uint4 *sZero = reinterpret_cast<uint4 *>(smem + L.zero_off);
@@ -160,9 +167,20 @@ __global__ void __launch_bounds__(kMtThreads, 2) skinny_mt_kernel(const __grid_c
     for (int u = 0; u < U; ++u)
       tma_load_3d(sW + u * unit_bytes, &tmW, 0, (cta * U + u) * 8, split * kb, wbar);
   }
-  for (int i = tid; i < kUC; i += kMtThreads) sBias[i] = p.bias ? bf2f(p.bias[n_base + i]) : 0.f;
-  __syncthreads();  // the barriers and the zero line are initialised before any thread uses them
+  for (int i = tid; i < kUC; i += kMtThreads) {
+    sBias[i] = p.bias ? bf2f(p.bias[n_base + i]) : 0.f;
+    if (p.xg_out) sGn[i] = bf2f(p.g_next[n_base + i]);
+  }
+  // a key/value row's cache slot and position are fixed for the step (the
+  // kernels before this one in the pass do not write them)
+  if (p.epi == EPI_KV)
+    for (int r = tid; r < rows_o; r += kMtThreads) {
+      const int t = r_lo + r, ii = t / p.rows_per_seq, jr = t - ii * p.rows_per_seq;
+      const int slot = p.seq_slot[ii];
+      sRow[r] = make_int2(slot, (p.pos_base ? p.pos_base[slot] : 0) + jr);
+    }
   pdl_launch_dependents();
+  __syncthreads();  // the barriers and the zero line are initialised before any thread uses them
   pdl_wait();
 
   // ---------------- the first k-blocks of the operand; the partial row sums
@@ -221,23 +239,45 @@ __global__ void __launch_bounds__(kMtThreads, 2) skinny_mt_kernel(const __grid_c
         ldsm_x4(wq + offB0, b[u][0], b[u][1], b[u][2], b[u][3]);
         ldsm_x4(wq + offB1, b[u][4], b[u][5], b[u][6], b[u][7]);
       }
+      // consecutive MMAs go to different accumulators (units, and tiles when
+      // the registers allow): a k-step's result is not waited on before the
+      // next independent MMA issues; each accumulator still adds its k-steps
+      // in order
+      if constexpr (G::kAllTiles) {
+        uint32_t a[G::kTW][4][4];
 #pragma unroll
-      for (int h = 0; h < G::kTW; ++h) {
-        const int tile = wt + G::kWT * h;
-        if (tile >= n_tiles) break;
-        const int row = tile * 16 + ar;
-        const bool real = row < Mr;
-        const uint32_t aq = st + row * 128, sw = row & 7;
-        uint32_t a[4][4];
+        for (int h = 0; h < G::kTW; ++h) {
+          const int row = (wt + G::kWT * h) * 16 + ar;
+          const bool real = row < Mr;
+          const uint32_t aq = st + row * 128, sw = row & 7;
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            ldsm_x4(real ? aq + (((2 * j + c0) ^ sw) << 4) : z_addr, a[h][j][0], a[h][j][1], a[h][j][2], a[h][j][3]);
+        }
 #pragma unroll
         for (int j = 0; j < 4; ++j)
-          ldsm_x4(real ? aq + (((2 * j + c0) ^ sw) << 4) : z_addr, a[j][0], a[j][1], a[j][2], a[j][3]);
 #pragma unroll
-        for (int u = 0; u < G::kUW; ++u) {
-          mma_bf16(acc[h][u], a[0][0], a[0][1], a[0][2], a[0][3], b[u][0], b[u][1]);
-          mma_bf16(acc[h][u], a[1][0], a[1][1], a[1][2], a[1][3], b[u][2], b[u][3]);
-          mma_bf16(acc[h][u], a[2][0], a[2][1], a[2][2], a[2][3], b[u][4], b[u][5]);
-          mma_bf16(acc[h][u], a[3][0], a[3][1], a[3][2], a[3][3], b[u][6], b[u][7]);
+          for (int h = 0; h < G::kTW; ++h)
+#pragma unroll
+            for (int u = 0; u < G::kUW; ++u)
+              mma_bf16(acc[h][u], a[h][j][0], a[h][j][1], a[h][j][2], a[h][j][3], b[u][2 * j], b[u][2 * j + 1]);
+      } else {
+#pragma unroll
+        for (int h = 0; h < G::kTW; ++h) {
+          const int tile = wt + G::kWT * h;
+          if (tile >= n_tiles) break;
+          const int row = tile * 16 + ar;
+          const bool real = row < Mr;
+          const uint32_t aq = st + row * 128, sw = row & 7;
+          uint32_t a[4][4];
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            ldsm_x4(real ? aq + (((2 * j + c0) ^ sw) << 4) : z_addr, a[j][0], a[j][1], a[j][2], a[j][3]);
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+#pragma unroll
+            for (int u = 0; u < G::kUW; ++u)
+              mma_bf16(acc[h][u], a[j][0], a[j][1], a[j][2], a[j][3], b[u][2 * j], b[u][2 * j + 1]);
         }
       }
     }
@@ -267,40 +307,66 @@ __global__ void __launch_bounds__(kMtThreads, 2) skinny_mt_kernel(const __grid_c
   if (S > 1) cluster_sync();  // every rank's results are in its shared memory
   else __syncthreads();
 
-  // ---------------- W g and W b summed over the ranks in rank order; the
-  // statistics of the rows this rank finishes: lane l sums partials
-  // l + 32 i in order of i, then the warp adds across lanes
+  // ---------------- W g and W b summed over the ranks in rank order (warps
+  // 0-3); the statistics of the rows this rank finishes (warps 4-7, four rows
+  // in flight per warp): lane l sums partials l + 32 i in order of i, then
+  // the warp adds across lanes
   const uint32_t res_u32 = smem_u32(sRes);
   if (fold) {
-    for (int i = tid; i < 2 * kUC; i += kMtThreads) {
-      const int e = (i / kUC) * res_ld + (i % kUC);
-      float v = 0.f;
-      if (S > 1) {
-        float part[8];
+    constexpr int kHalf = kMtWarps / 2;
+    if (warp < kHalf) {
+      for (int i = tid; i < 2 * kUC; i += kHalf * 32) {
+        const int e = (i / kUC) * res_ld + (i % kUC);
+        float v = 0.f;
+        if (S > 1) {
+          // every load issued unconditionally (a rank past S reads this
+          // CTA's own value, unused) so none waits on another
+          float part[8];
 #pragma unroll
-        for (int r = 0; r < 8; ++r) part[r] = r < S ? dsmem_ld_f32(dsmem_map(res_u32 + 4u * e, r)) : 0.f;
+          for (int r = 0; r < 8; ++r) part[r] = dsmem_ld_f32(dsmem_map(res_u32 + 4u * e, r < S ? r : split));
 #pragma unroll
-        for (int r = 0; r < 8; ++r)
-          if (r < S) v += part[r];
-      } else {
-        v = sRes[e];
+          for (int r = 0; r < 8; ++r)
+            if (r < S) v += part[r];
+        } else {
+          v = sRes[e];
+        }
+        sWg[i] = v;
       }
-      sWg[i] = v;
-    }
-    for (int r = warp; r < rows_o; r += kMtWarps) {
-      const float2 *src = staged ? sPart + r * kMtStageParts
-                                 : p.fold_part + static_cast<size_t>(r_lo + r) * p.part_stride;
-      float s1 = 0.f, s2 = 0.f;
-      for (int i = lane; i < p.n_part; i += 32) {
-        const float2 v = staged ? src[i] : __ldcg(src + i);
-        s1 += v.x;
-        s2 += v.y;
+    } else {
+      constexpr int kR = 4;
+      for (int r0 = warp - kHalf; r0 < rows_o; r0 += kHalf * kR) {
+        float s1[kR], s2[kR];
+#pragma unroll
+        for (int k = 0; k < kR; ++k) {
+          const int r = r0 + kHalf * k;
+          s1[k] = s2[k] = 0.f;
+          if (r < rows_o) {
+            const float2 *src = staged ? sPart + r * kMtStageParts
+                                       : p.fold_part + static_cast<size_t>(r_lo + r) * p.part_stride;
+            for (int i = lane; i < p.n_part; i += 32) {
+              const float2 v = staged ? src[i] : __ldcg(src + i);
+              s1[k] += v.x;
+              s2[k] += v.y;
+            }
+          }
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1)
+#pragma unroll
+          for (int k = 0; k < kR; ++k) {
+            s1[k] += __shfl_xor_sync(0xffffffffu, s1[k], off);
+            s2[k] += __shfl_xor_sync(0xffffffffu, s2[k], off);
+          }
+        if (lane == 0)
+#pragma unroll
+          for (int k = 0; k < kR; ++k) {
+            const int r = r0 + kHalf * k;
+            if (r >= rows_o) continue;
+            const float mu = s1[k] / static_cast<float>(p.K);
+            const float var = fmaxf(s2[k] / static_cast<float>(p.K) - mu * mu, 0.f);
+            sStat[r] = make_float2(mu, rsqrtf(var + p.ln_eps));
+          }
       }
-      s1 = warp_sum(s1);
-      s2 = warp_sum(s2);
-      const float mu = s1 / static_cast<float>(p.K);
-      const float var = fmaxf(s2 / static_cast<float>(p.K) - mu * mu, 0.f);
-      if (lane == 0) sStat[r] = make_float2(mu, rsqrtf(var + p.ln_eps));
     }
     __syncthreads();
   }
@@ -309,18 +375,23 @@ __global__ void __launch_bounds__(kMtThreads, 2) skinny_mt_kernel(const __grid_c
   // row r_lo + f / kQ (a row's quads in consecutive lanes of one warp)
   const int n_q = rows_o * kQ;
   const bool good = ok && !*s_flag;
+  // a rank arrives at the closing cluster barrier once it has read its
+  // peers' sums for the last time (its own stores then overlap the barrier)
+  bool arrived = false;
   for (int f0 = 0; f0 < n_q; f0 += kMtThreads * kMtQuadsPerPass) {
     float4 val[kMtQuadsPerPass];
     if (S > 1) {
+      // every load issued unconditionally, all in flight before the sums: a
+      // quad past the rows reads row r_lo's first quad and a rank past S this
+      // CTA's own value, neither used
       float4 part[kMtQuadsPerPass][8];
 #pragma unroll
-      for (int e = 0; e < kMtQuadsPerPass; ++e) {  // every load in flight before the sums
+      for (int e = 0; e < kMtQuadsPerPass; ++e) {
         const int f = f0 + e * kMtThreads + tid;
-        const int r = f / kQ, c = (f - r * kQ) * 4;
+        const int r = f < n_q ? f / kQ : 0, c = f < n_q ? (f - r * kQ) * 4 : 0;
         const uint32_t a = res_u32 + 4u * ((r_lo + r + t0) * res_ld + c);
 #pragma unroll
-        for (int k = 0; k < 8; ++k)
-          part[e][k] = (f < n_q && k < S) ? dsmem_ld_f32x4(dsmem_map(a, k)) : make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int k = 0; k < 8; ++k) part[e][k] = dsmem_ld_f32x4(dsmem_map(a, k < S ? k : split));
       }
 #pragma unroll
       for (int e = 0; e < kMtQuadsPerPass; ++e) {
@@ -335,6 +406,10 @@ __global__ void __launch_bounds__(kMtThreads, 2) skinny_mt_kernel(const __grid_c
           }
         }
         val[e] = v;
+      }
+      if (f0 + kMtThreads * kMtQuadsPerPass >= n_q) {
+        cluster_arrive();
+        arrived = true;
       }
     } else {
 #pragma unroll
@@ -375,8 +450,8 @@ __global__ void __launch_bounds__(kMtThreads, 2) skinny_mt_kernel(const __grid_c
           *reinterpret_cast<float4 *>(p.resid + static_cast<size_t>(t) * p.ld_resid + n) =
               make_float4(nr[0], nr[1], nr[2], nr[3]);
           if (p.xg_out) {
-            st_bf16x4(p.xg_out + static_cast<size_t>(t + 2) * p.ld_resid + n, nr[0] * bf2f(p.g_next[n]),
-                      nr[1] * bf2f(p.g_next[n + 1]), nr[2] * bf2f(p.g_next[n + 2]), nr[3] * bf2f(p.g_next[n + 3]));
+            st_bf16x4(p.xg_out + static_cast<size_t>(t + 2) * p.ld_resid + n, nr[0] * sGn[c], nr[1] * sGn[c + 1],
+                      nr[2] * sGn[c + 2], nr[3] * sGn[c + 3]);
             if (t == 0) {
 #pragma unroll
               for (int j = 0; j < 4; ++j) {
@@ -397,9 +472,7 @@ __global__ void __launch_bounds__(kMtThreads, 2) skinny_mt_kernel(const __grid_c
             st_bf16x4(p.out_bf16 + static_cast<size_t>(t) * p.ld_out + n, v[0], v[1], v[2], v[3]);
           } else {
             const int cc = n - p.q_cols, which = cc / p.d_model, hd = cc - which * p.d_model;
-            const int ii = t / p.rows_per_seq, jr = t - ii * p.rows_per_seq;
-            const int slot = p.seq_slot[ii];
-            const int pos = (p.pos_base ? p.pos_base[slot] : 0) + jr;
+            const int slot = sRow[r].x, pos = sRow[r].y;
             if (pos >= p.ctx) {
               set_error(p.err, WF_DEV_ERR_CAPACITY);
             } else {
@@ -422,7 +495,10 @@ __global__ void __launch_bounds__(kMtThreads, 2) skinny_mt_kernel(const __grid_c
       }
     }
   }
-  if (S > 1) cluster_sync();  // peers may read this CTA's results until here
+  if (S > 1) {  // peers may read this CTA's results until they have all arrived
+    if (!arrived) cluster_arrive();
+    cluster_wait();
+  }
   // after a timeout a copy may still be landing
   __syncthreads();
   if (tid == 0 && *s_flag) {
@@ -481,26 +557,88 @@ cudaError_t mt_attrs() {
   return e;
 }
 
-constexpr int kSMs = 152;
+const void *mt_kernel(int U) {
+  switch (U) {
+    case 1: return reinterpret_cast<const void *>(skinny_mt_kernel<1>);
+    case 2: return reinterpret_cast<const void *>(skinny_mt_kernel<2>);
+    case 4: return reinterpret_cast<const void *>(skinny_mt_kernel<4>);
+    case 8: return reinterpret_cast<const void *>(skinny_mt_kernel<8>);
+    default: return nullptr;
+  }
+}
 
-// Estimated SM clock cycles of one launch: mma.sync m16n8k16 at 2 cycles per
-// SM and ldmatrix.x4 at 4 (whichever bounds a k-block), CTAs spread over the
-// SMs, and about 2500 cycles of latency per wave of CTAs (600 more for a
-// cluster reduction).  Two CTAs per SM overlap one's latency with the other.
-double mt_cost(int Mr, int N, int K, int u, int s, bool pair) {
-  const int T = (Mr + 15) / 16, wu = u >= 8 ? 2 : 1, wt = 8 / wu;
+int mt_sms() {
+  static int n = [] {
+    int dev = 0, v = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return 0;
+    return v;
+  }();
+  return n > 0 ? n : 152;
+}
+
+// CTAs (S == 1) or clusters of S CTAs of this shared-memory size that the
+// GPU holds at once (a cluster's CTAs share one GPC, so clusters of 3, 5, 6
+// or 7 CTAs leave SMs idle)
+int mt_resident(int U, int S, size_t smem) {
+  static std::mutex mu;
+  static std::map<std::tuple<int, int, size_t>, int> cache;
+  std::lock_guard<std::mutex> lock(mu);
+  const auto key = std::make_tuple(U, S, smem);
+  auto it = cache.find(key);
+  if (it != cache.end()) return it->second;
+  int n = 0;
+  const void *f = mt_kernel(U);
+  if (S == 1) {
+    int per_sm = 0;
+    if (f && cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, f, kMtThreads, smem) == cudaSuccess)
+      n = per_sm * mt_sms();
+  } else if (f) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(1, 1, S);
+    cfg.blockDim = dim3(kMtThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = 1;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = S;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    if (cudaOccupancyMaxActiveClusters(&n, f, &cfg) != cudaSuccess) n = 0;
+  }
+  cudaGetLastError();  // a failed query leaves no error behind
+  cache.emplace(key, n);
+  return n;
+}
+
+// Estimated SM clock cycles of one launch: the waves of CTAs (clusters) the
+// GPU holds at once, each paying a fixed latency (launch, weights, first
+// operand block, about 4000 cycles; 1500 more for a cluster reduction) and
+// its k-blocks.  A k-block costs the longer of the busiest warp's MMAs (about
+// 10 cycles each with four or more independent accumulators) and the SM's
+// MMA throughput over the CTAs sharing it (about 2.2 cycles per MMA), plus
+// about 300 cycles of waiting and block synchronisation.
+double mt_cost(int Mr, int N, int K, int u, int s, size_t smem) {
+  const int T = (Mr + 15) / 16, wu = u >= 8 ? 2 : 1, wt = 8 / wu, uw = u / wu;
+  const int tw_max = (kMtMaxTiles + wt - 1) / wt;
+  const int tw = tw_max * uw <= 8 ? tw_max : (T + wt - 1) / wt;  // every tile slot, or the real ones
   const int kb = K / 64 / s;
-  const double mma = T * u * 4 * 2.0, ld = (wu * T * 4 + wt * u * 2) * 4.0;
-  const double cta = kb * (mma > ld ? mma : ld);
   const int ctas = N / 8 / u * s;
-  const int per_sm = (ctas + kSMs - 1) / kSMs;
-  const int waves = pair ? (per_sm + 1) / 2 : per_sm;
-  return per_sm * cta + waves * (2500.0 + (s > 1 ? 600.0 : 0.0));
+  const int resident = mt_resident(u, s, smem);
+  if (resident <= 0) return 1e30;
+  const int units = s > 1 ? ctas / s : ctas;  // clusters or CTAs
+  const int waves = (units + resident - 1) / resident;
+  const int per_sm = (ctas / waves + mt_sms() - 1) / mt_sms();  // CTAs sharing an SM in a wave
+  const double warp_mma = tw * uw * 4 * 10.0, sm_mma = per_sm * T * u * 4 * 2.2;
+  const double t_kb = (warp_mma > sm_mma ? warp_mma : sm_mma) + 300.0;
+  return waves * (4000.0 + (s > 1 ? 1500.0 : 0.0) + kb * t_kb);
 }
 }  // namespace
 
 bool skinny_mt_plan(int Mr, int N, int K, bool fold, bool resid, int *U, int *S, int *ns) {
   if (Mr < 1 || Mr > kMtMaxTiles * 16 || N % 8 || K % 64) return false;
+  if (skinny_mt_init() != cudaSuccess) return false;
   const int units = N / 8, kbt = K / 64;
   double best = 0.0;
   bool found = false;
@@ -513,13 +651,12 @@ bool skinny_mt_plan(int Mr, int N, int K, bool fold, bool resid, int *U, int *S,
       const int qmax = kb < kMtMaxStages ? kb : kMtMaxStages, qmin = kb < 2 ? kb : 2;
       // the deepest ring that lets two CTAs share an SM, else the deepest for one
       int pick = 0;
-      bool pair = false;
       for (int q = qmax; q >= qmin && !pick; --q)
-        if (mt_smem(Mr, Mr, K, u, s, q, fold, resid) <= static_cast<size_t>(kMtSmemPair)) pick = q, pair = true;
+        if (mt_smem(Mr, Mr, K, u, s, q, fold, resid) <= static_cast<size_t>(kMtSmemPair)) pick = q;
       for (int q = qmax; q >= qmin && !pick; --q)
         if (mt_smem(Mr, Mr, K, u, s, q, fold, resid) <= static_cast<size_t>(kMtSmemAlone)) pick = q;
       if (!pick) continue;
-      const double c = mt_cost(Mr, N, K, u, s, pair);
+      const double c = mt_cost(Mr, N, K, u, s, mt_smem(Mr, Mr, K, u, s, pick, fold, resid));
       if (!found || c < best) {
         best = c;
         found = true;
