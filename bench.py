@@ -69,14 +69,18 @@ WORKLOADS = {
     "large_b96_2l": dict(cfg="LARGE", layers=2, batch=96, budget=(20, 40), accept="geometric",
                          text="large per-layer shapes cut to 2 target blocks (profiling case), "
                               "batch 96, transcript lengths uniform 20..40"),
+    "large_b16_2l": dict(cfg="LARGE", layers=2, batch=16, budget=(20, 40), accept="geometric",
+                         text="large per-layer shapes cut to 2 target blocks (profiling case), "
+                              "batch 16, transcript lengths uniform 20..40"),
 }
 
 
 # DRAM bytes (read + write) per projection launch, averaged over one step's
 # launch mix, from ncu captures of the depth-reduced profiling cases with the
-# same per-layer shapes (profiles/dram_per_kernel_large_b1_4l.md and
+# same per-layer shapes (profiles/dram_per_kernel_large_b1_4l.md,
+# profiles/dram_per_kernel_large_b16_2l.md and
 # profiles/dram_per_kernel_large_b96_2l.md); None where no capture covers the
-# workload's shapes.
+# workload's shapes and projection path.
 GEMM_DRAM_BYTES_PER_LAUNCH = {
     # 68 x out/cross-out (3.404 MB), 34 x fc1 (13.219), 34 x fc2 (13.313),
     # 2 x history K/V (6.662), 1 x history projection (16.572) per step
@@ -85,7 +89,28 @@ GEMM_DRAM_BYTES_PER_LAUNCH = {
     # (5.514), 34 x fc1 (15.354), 2 x history K/V (8.796), 1 x history
     # projection (27.283) per step, captured at 94 sequences
     "large_b96": 13.165e6,
+    # 204 x batched skinny projections (8.594 MB), 2 x history K/V (7.346), 1 x
+    # history projection (18.182) per step, captured at 16 sequences
+    "large_b16": 8.628e6,
 }
+
+# the projection path each capture above ran on (its traffic describes only that path)
+GEMM_DRAM_CAPTURE_PATH = {"large_b1": "skinny", "large_b16": "skinny", "large_b96": "tcgen05"}
+
+
+def _gemm_traffic(name, path):
+    return GEMM_DRAM_BYTES_PER_LAUNCH.get(name) if GEMM_DRAM_CAPTURE_PATH.get(name) == path else None
+
+
+def _proj_kernel(path, rows):
+    """The kernel that runs a pass's projections: the skinny kernels up to 144
+    step rows (one operand tile up to 14), else the tcgen05 GEMM."""
+    if path != "skinny":
+        return "gemm_tc_kernel (tcgen05 projections)"
+    if rows <= 14:
+        return "skinny_kernel (single-sequence projections)"
+    return "skinny_mt_kernel (batched skinny projections)"
+
 
 # Tensor-pipe activity of the projections at batch 96 from the committed ncu
 # capture of the same kernels (profiles/), or absent until one is taken.
@@ -464,8 +489,7 @@ def run_ours(args, rank, world):
     fam = max(("gemm", "head", "attn_cross", "attn_self", "persist"), key=lambda f: prof[f]["ms"])
     roof_fam = "persist" if args.persist else "gemm"
     kernel = ("persist_kernel (every block of a pass in one launch; bytes = weights and acoustic K/V)"
-              if args.persist else ("skinny_kernel (single-sequence projections)" if m["proj_path"] == "skinny"
-                                    else "gemm_tc_kernel (tcgen05 projections)"))
+              if args.persist else _proj_kernel(m["proj_path"], m["batch"] * (cfg.block_k + 1)))
     Bn, Kc = m["batch"], cfg.block_k
     result = {
         "metric": METRIC,
@@ -492,7 +516,7 @@ def run_ours(args, rank, world):
         "context_len": {"min": m["ctx"][0], "mean": m["ctx"][1], "max": m["ctx"][2]},
         "step_roofline": _step_roofline(m, step_ms, hbm_peak, peak_src),
         "roofline": _family_roofline(prof, n_prof, step_ms, roof_fam, hbm_peak, peak_src, kernel,
-                                     None if args.persist else GEMM_DRAM_BYTES_PER_LAUNCH.get(args.workload)),
+                                     None if args.persist else _gemm_traffic(args.workload, m["proj_path"])),
         "kernel_families_ms_per_step": {k: v["ms"] / n_prof for k, v in prof.items()},
         "kernel_families_launches_per_step": {k: v["launches"] / n_prof for k, v in prof.items()},
         "top_family": fam,
@@ -518,9 +542,10 @@ def run_ours(args, rank, world):
                 "steps": args.batch_steps, "tokens_per_step": btok / args.batch_steps / world,
                 "context_len": {"min": mb["ctx"][0], "mean": mb["ctx"][1], "max": mb["ctx"][2]},
                 "step_roofline": _step_roofline(mb, sms, hbm_peak, peak_src),
+                "projections": mb["proj_path"],
                 "roofline": _family_roofline(mb["prof"], mb["n_prof"], sms, "gemm", hbm_peak, peak_src,
-                                             "gemm_tc_kernel (tcgen05 projections)",
-                                             GEMM_DRAM_BYTES_PER_LAUNCH.get(name)),
+                                             _proj_kernel(mb["proj_path"], mb["batch"] * (cfg.block_k + 1)),
+                                             _gemm_traffic(name, mb["proj_path"])),
                 "kernel_families_ms_per_step": {k: v["ms"] / mb["n_prof"] for k, v in mb["prof"].items()},
                 "clocks": mb["clocks"], "consistent": mb["consistent"], "device_error": mb["err"],
                 "gpu_launches": mb["launches"]}
@@ -731,7 +756,8 @@ def run_sampling(args, rank, world):
         "replayed_identically": replayed,
         "step_roofline": _step_roofline(m, step_ms, hbm_peak, peak_src),
         "roofline": _family_roofline(prof, n_prof, step_ms, "gemm", hbm_peak, peak_src,
-                                     "gemm_tc_kernel (tcgen05 projections)", None),
+                                     _proj_kernel("skinny" if Bn * (Kc + 1) <= 144 else "tcgen05", Bn * (Kc + 1)),
+                                     None),
         "kernel_families_ms_per_step": {k: v["ms"] / n_prof for k, v in prof.items()},
         "e2e": {"value": e2e_tokens / e2e_s, "unit": "tokens/s",
                 "h2d_bytes_per_step": 0,
