@@ -116,41 +116,43 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const __grid_const
   // In a cluster launch every CTA of a multi-block group takes part in the
   // merge; a block past the keys computes over masked keys only and yields
   // the exact empty partial (m = -inf, l = 0, o = 0).
-  if (blk >= n_blocks && !(p.cluster && n_blocks > 1)) return;
+  if (!p.loop && blk >= n_blocks && !(p.cluster && n_blocks > 1)) return;
 
   const int d_model = p.n_heads * 64;
-  const int key0 = blk * kKB;
+  // the key blocks this CTA computes: its own, or (loop) all of its group's
+  // in order, each leaving its partial as a CTA of its own would
+  const int b_first = p.loop ? 0 : blk, b_end = p.loop ? n_blocks : blk + 1;
+  const int group_id = (i * p.n_heads + h) * p.qgroups + qg;
 
   // ---- keys and values: one TMA copy each.  A block holding rows that this
   // step's projection writes (positions from `fresh` on) loads after the
   // wait; a block of settled rows streams in while the producer of the
-  // queries finishes.
+  // queries finishes.  A looping CTA requests each later block once the
+  // previous one is done with the tiles.
   const int fresh = p.mode == 2 ? n_keys : base;
-  const bool any_keys = key0 < n_keys;
-  const bool has_fresh = any_keys && fresh < n_keys && key0 + kKB > fresh;
   const int cache_row = slot * p.n_heads + h;
   const uint32_t tile_bytes = static_cast<uint32_t>(min(kKB, p.ctx)) * 128u;  // the maps' box
+  auto issue = [&](int b) {
+    mbar_arrive_expect_tx(&s_bar[0], tile_bytes);
+    tma_load_3d(sK, &tmK, 0, b * kKB, cache_row, &s_bar[0]);
+    mbar_arrive_expect_tx(&s_bar[1], tile_bytes);
+    tma_load_3d(sV, &tmV, 0, b * kKB, cache_row, &s_bar[1]);
+  };
+  const bool first_keys = b_first * kKB < n_keys;
+  const bool first_fresh = first_keys && fresh < n_keys && b_first * kKB + kKB > fresh;
   if (tid == 0) {
     mbar_init(&s_bar[0], 1);
     mbar_init(&s_bar[1], 1);
     fence_barrier_init();
-    if (any_keys && !has_fresh) {
+    if (first_keys && !first_fresh) {
       tma_prefetch_desc(&tmK);
       tma_prefetch_desc(&tmV);
-      mbar_arrive_expect_tx(&s_bar[0], tile_bytes);
-      tma_load_3d(sK, &tmK, 0, key0, cache_row, &s_bar[0]);
-      mbar_arrive_expect_tx(&s_bar[1], tile_bytes);
-      tma_load_3d(sV, &tmV, 0, key0, cache_row, &s_bar[1]);
+      issue(b_first);
     }
   }
   pdl_wait();
   pdl_launch_dependents();
-  if (tid == 0 && has_fresh) {
-    mbar_arrive_expect_tx(&s_bar[0], tile_bytes);
-    tma_load_3d(sK, &tmK, 0, key0, cache_row, &s_bar[0]);
-    mbar_arrive_expect_tx(&s_bar[1], tile_bytes);
-    tma_load_3d(sV, &tmV, 0, key0, cache_row, &s_bar[1]);
-  }
+  if (tid == 0 && first_fresh) issue(b_first);
   const long long spin = p.spin > 0 ? p.spin : kSpinLimitCycles;
   // ---- queries, pre-scaled by 1/8 = 1/sqrt(64) (exact in binary), RoPE in fp32
   if (tid < kQG * 8) {
@@ -182,13 +184,23 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const __grid_const
     o.w = pack_bf16(f[6], f[7]);
     *reinterpret_cast<uint4 *>(sQ + swz(r, ch)) = o;
   }
+  // thread -> (row qi, dims d0..d0+kDPT-1) in the combines
+  const int qi = tid / (64 / kDPT), d0 = (tid % (64 / kDPT)) * kDPT;
+  for (int bi = b_first; bi < b_end; ++bi) {
+  const int key0 = bi * kKB;
+  const bool any_keys = key0 < n_keys;
+  const uint32_t ph = static_cast<uint32_t>((bi - b_first) & 1);  // the tiles' copy of this block
+  if (bi > b_first && tid == 0) {
+    fence_proxy_async();  // the previous block's generic writes to the tiles come before the copies
+    issue(bi);
+  }
   // keys first; the values keep streaming while the scores are formed.  After
   // a timeout thread 0 waits (bounded) for both copies before going on, so
   // no copy lands in a CTA that has exited.
   __syncthreads();
-  if (any_keys && !mbar_wait(&s_bar[0], 0, p.err, spin) && tid == 0) {
-    mbar_drain(&s_bar[0], 0);
-    mbar_drain(&s_bar[1], 0);
+  if (any_keys && !mbar_wait(&s_bar[0], ph, p.err, spin) && tid == 0) {
+    mbar_drain(&s_bar[0], ph);
+    mbar_drain(&s_bar[1], ph);
   }
 
   // ---- RoPE on the keys (drafter): dims i and i+32 rotate by pos * base^(-2i/64)
@@ -276,7 +288,7 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const __grid_const
   // the values; rows past the visible keys (stale cache rows, rows past the
   // copy, or a block with no visible key at all) become zeros, so P V adds
   // exact zeros there
-  if (any_keys && !mbar_wait(&s_bar[1], 0, p.err, spin) && tid == 0) mbar_drain(&s_bar[1], 0);
+  if (any_keys && !mbar_wait(&s_bar[1], ph, p.err, spin) && tid == 0) mbar_drain(&s_bar[1], ph);
   {
     const int z0 = min(max(n_keys - key0, 0), kKB);
     for (int idx = tid; idx < (kKB - z0) * 8; idx += kThreadsA)
@@ -321,8 +333,7 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const __grid_const
   }
   __syncthreads();
 
-  // ---- combine the warps in order: thread -> (row qi, dims d0..d0+kDPT-1)
-  const int qi = tid / (64 / kDPT), d0 = (tid % (64 / kDPT)) * kDPT;
+  // ---- combine the warps in order
   float M = -INFINITY;
 #pragma unroll
   for (int w = 0; w < kWarps; ++w) M = fmaxf(M, sm[w * kQG + qi]);
@@ -405,8 +416,7 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const __grid_const
   }
 
   // ---- several key blocks: partials to global, the last CTA combines in order
-  const int group_id = (i * p.n_heads + h) * p.qgroups + qg;
-  float *part = p.part + (static_cast<size_t>(group_id) * p.n_chunks + blk) * kQG * kPartStride;
+  float *part = p.part + (static_cast<size_t>(group_id) * p.n_chunks + bi) * kQG * kPartStride;
   if (qi < nq) {
     float *pe = part + qi * kPartStride;
     if (d0 == 0) {
@@ -418,8 +428,11 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const __grid_const
   }
   // one fence per CTA: after the barrier thread 0 releases the whole CTA's
   // partial at GPU scope and counts it; the last CTA's thread 0 fences again
-  // (acquire) before the barrier that releases its threads into the combine
+  // (acquire) before the barrier that releases its threads into the combine.
+  // A looping CTA goes on to its next block once every thread is done with
+  // this one (its partials are then visible to all its threads).
   __syncthreads();
+  if (p.loop) continue;
   if (tid == 0) {
     __threadfence();
     const int last = atomicAdd(&p.counters[group_id], 1) == n_blocks - 1;
@@ -428,6 +441,7 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const __grid_const
   }
   __syncthreads();
   if (!s_last) return;
+  }  // key blocks
   // A block the query cannot see carries m = -inf, l = 0, o = 0 and gets
   // weight 0, so it adds exact zeros; the loads of all blocks are independent.
   if (qi < nq) {
@@ -544,12 +558,22 @@ cudaError_t launch_attention(const AttnParams &p0, cudaStream_t s, bool pdl) {
       return 0;
     return n;
   }();
-  const long long ctas = static_cast<long long>(cfg.gridDim.x) * cfg.gridDim.y * cfg.gridDim.z;
-  cfg.dynamicSmemBytes = ctas <= n_sm ? kSmemAttnSpread : kSmemAttn;
+  long long ctas = static_cast<long long>(cfg.gridDim.x) * cfg.gridDim.y * cfg.gridDim.z;
   // small launches merge their blocks over DSMEM (no global round trip);
   // large ones keep the global partials, where cluster placement costs more
-  // than it saves.  Both paths do the same arithmetic in the same order.
+  // than it saves.  With at least two (sequence, head, query group)s per SM
+  // one CTA per group walks its key blocks in order, leaving the same
+  // partials and merging them itself: a single wave of CTAs streams every
+  // key, with no counter and no second wave.  All three paths do the same
+  // arithmetic in the same order.
   p.cluster = (p.n_chunks > 1 && p.n_chunks <= 8 && ctas <= n_sm) ? 1 : 0;
+  const long long groups = static_cast<long long>(cfg.gridDim.y) * cfg.gridDim.z;
+  p.loop = (!p.cluster && p.n_chunks > 1 && n_sm > 0 && groups >= 2LL * n_sm) ? 1 : 0;
+  if (p.loop) {
+    cfg.gridDim.x = 1;
+    ctas = groups;
+  }
+  cfg.dynamicSmemBytes = ctas <= n_sm ? kSmemAttnSpread : kSmemAttn;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   int na = 0;

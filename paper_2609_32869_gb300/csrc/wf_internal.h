@@ -227,6 +227,7 @@ struct AttnParams {
   int n_seq, rps, n_heads, ctx, mode, n_chunks, qgroups;
   int outer;    // bound on slot * n_heads + head (the caches' tensor maps)
   int cluster;  // the n_chunks blocks of a (sequence, head, group) form a cluster
+  int loop;     // one CTA per (sequence, head, group) walks its key blocks in order
 };
 constexpr int kAttnKeysPerCTA = 256;  // keys per CTA (32 per warp), aligned to absolute positions
 constexpr int kAttnQGroup = 16;       // query rows per CTA

@@ -123,3 +123,48 @@ def test_attention_matches_oracle(mode, rps, ctx, rope):
         # bf16 output rounding (2^-8 relative) dominates the fp32 arithmetic
         np.testing.assert_allclose(g, want, atol=2e-2, rtol=1e-2)
         assert np.abs(g - want).max() < 3 * 2.0 ** -8 * max(1.0, np.abs(want).max())
+
+
+@pytest.mark.parametrize("mode,ctx", [(2, 1500), (0, 448)])
+def test_attention_one_cta_per_group_equals_split_blocks(mode, ctx):
+    """A launch with at least two (sequence, head, query group)s per SM runs
+    one CTA per group that walks its 256-key blocks in order; it leaves the
+    split form's partials and merges them in block order itself, so each
+    sequence's rows equal, bit for bit, those of a launch of that sequence
+    alone (split blocks, merged over a cluster), and the oracle within the
+    attention tolerance.  Whisper-large heads, 16 sequences, 9 query rows."""
+    import torch
+    from paper_2609_32869_gb300 import binding as B
+    H, n_seq, rps = 20, 16, 9
+    d = H * 64
+    slots = np.array([(5 * i + 3) % n_seq for i in range(n_seq)], np.int32)
+    base = np.array([(37 * s + 11) % (ctx - rps) for s in range(n_seq)], np.int32)
+    q = syn.normal_bf16(41, f"ql{mode}", (n_seq * rps, d), 1.0)
+    kc = _cache(n_seq, H, ctx, 42, f"kl{ctx}")
+    vc = _cache(n_seq, H, ctx, 43, f"vl{ctx}")
+    dk, dv, db = _dev(kc), _dev(vc), torch.from_numpy(base).cuda()
+
+    def run(rows, sl):
+        n = len(sl)
+        out = torch.empty(n * rps, d, dtype=torch.bfloat16, device="cuda")
+        nb = B.wf_attention_scratch_bytes(n, rps, H, ctx)
+        sc = torch.empty(nb, dtype=torch.uint8, device="cuda")
+        B.wf_attention(_dev(rows), dk, dv, torch.from_numpy(np.asarray(sl, np.int32)).cuda(), db, n, rps,
+                       H, ctx, mode, 0, 10000.0, out, sc, nb)
+        torch.cuda.synchronize()
+        return out.float().cpu().numpy()
+
+    big = run(q, slots)
+    qf, kf, vf = _f64(q), _f64(kc), _f64(vc)
+    for i in (0, 7, 15):
+        one = run(q[i * rps:(i + 1) * rps], slots[i:i + 1])
+        np.testing.assert_array_equal(big[i * rps:(i + 1) * rps], one)
+        slot = slots[i]
+        L = base[slot]
+        n_keys = ctx if mode == 2 else L + rps
+        keys = kf[slot][:, :n_keys].transpose(1, 0, 2).reshape(n_keys, d)
+        vals = vf[slot][:, :n_keys].transpose(1, 0, 2).reshape(n_keys, d)
+        vis = None if mode == 2 else np.arange(n_keys)[None, :] <= (L + np.arange(rps))[:, None]
+        want = od.multi_head_attention(qf[i * rps:(i + 1) * rps], keys, vals, H, vis)
+        g = big[i * rps:(i + 1) * rps].astype(np.float64)
+        np.testing.assert_allclose(g, want, atol=2e-2, rtol=1e-2)
