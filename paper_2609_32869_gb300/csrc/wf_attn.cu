@@ -78,7 +78,10 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const __grid_const
   uint8_t *sQ = smem + 2 * kSmemK;
   float *sm = reinterpret_cast<float *>(smem + 2 * kSmemK + kSmemQ);  // [kWarps][16]
   float *sl = sm + kWarps * kQG;                                     // [kWarps][16]
-  float *so = reinterpret_cast<float *>(sK);  // [kWarps][16][64], once every warp is done with K
+  // [kWarps][16][64]: the warps' O, in the key tile once every warp is done
+  // with it (in the value tile for a looping CTA, whose next keys are by
+  // then streaming into the key tile)
+  float *so = reinterpret_cast<float *>(p.loop ? sV : sK);
   __shared__ int s_last;
   __shared__ uint64_t s_bar[2];  // [0] keys, [1] values
 
@@ -132,11 +135,17 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const __grid_const
   const int fresh = p.mode == 2 ? n_keys : base;
   const int cache_row = slot * p.n_heads + h;
   const uint32_t tile_bytes = static_cast<uint32_t>(min(kKB, p.ctx)) * 128u;  // the maps' box
-  auto issue = [&](int b) {
+  auto issue_k = [&](int b) {
     mbar_arrive_expect_tx(&s_bar[0], tile_bytes);
     tma_load_3d(sK, &tmK, 0, b * kKB, cache_row, &s_bar[0]);
+  };
+  auto issue_v = [&](int b) {
     mbar_arrive_expect_tx(&s_bar[1], tile_bytes);
     tma_load_3d(sV, &tmV, 0, b * kKB, cache_row, &s_bar[1]);
+  };
+  auto issue = [&](int b) {
+    issue_k(b);
+    issue_v(b);
   };
   const bool first_keys = b_first * kKB < n_keys;
   const bool first_fresh = first_keys && fresh < n_keys && b_first * kKB + kKB > fresh;
@@ -190,9 +199,9 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const __grid_const
   const int key0 = bi * kKB;
   const bool any_keys = key0 < n_keys;
   const uint32_t ph = static_cast<uint32_t>((bi - b_first) & 1);  // the tiles' copy of this block
-  if (bi > b_first && tid == 0) {
-    fence_proxy_async();  // the previous block's generic writes to the tiles come before the copies
-    issue(bi);
+  if (bi > b_first && tid == 0) {  // this block's keys were requested under the previous block's P V
+    fence_proxy_async();  // the previous block's generic writes to the value tile come before the copy
+    issue_v(bi);
   }
   // keys first; the values keep streaming while the scores are formed.  After
   // a timeout thread 0 waits (bounded) for both copies before going on, so
@@ -295,6 +304,11 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const __grid_const
       *reinterpret_cast<uint4 *>(sV + swz(z0 + (idx >> 3), idx & 7)) = make_uint4(0u, 0u, 0u, 0u);
   }
   __syncthreads();
+  // every warp is done with the keys: a looping CTA requests the next block's
+  if (p.loop && bi + 1 < b_end && tid == 0) {
+    fence_proxy_async();  // generic writes to the key tile (RoPE) come before the copy
+    issue_k(bi + 1);
+  }
   // O = P V (P rounded to bf16 as the A operand)
   float o[8][4];
 #pragma unroll
@@ -315,7 +329,7 @@ __global__ void __launch_bounds__(kThreadsA) attention_kernel(const __grid_const
       mma_bf16(o[2 * dp + 1], a0, a1, a2, a3, b2, b3);
     }
   }
-  __syncthreads();  // every warp is done with the key tile, which now holds O
+  __syncthreads();  // every warp is done with the tile that now holds O
   // stage this warp's (m, l, O) for the in-order combine
   if (c4 == 0) {
     sm[warp * kQG + g] = mrow[0];
