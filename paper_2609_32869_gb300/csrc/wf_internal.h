@@ -7,6 +7,7 @@
 #include <stdint.h>
 
 #include "../../include/wf.h"
+#include "wf_skinny_mt_layout.h"
 
 namespace wf {
 
@@ -198,7 +199,6 @@ cudaError_t launch_skinny(const void *W, SkinnyParams p, cudaStream_t s, bool pd
 // units and 16-row tiles.  No fp32 LayerNorm operand (ln_x).  The plan of Mr
 // operand rows (a folded LayerNorm's two included): units per CTA U, K split
 // S, operand ring stages ns.
-constexpr int kMtMaxRows = 144;  // 16 sequences x (1 + 8)
 bool skinny_mt_plan(int Mr, int N, int K, bool fold, bool resid, int *U, int *S, int *ns);
 cudaError_t skinny_mt_init();
 cudaError_t launch_skinny_mt(const void *W, SkinnyParams p, cudaStream_t s, bool pdl);

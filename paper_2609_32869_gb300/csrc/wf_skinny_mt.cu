@@ -27,60 +27,13 @@
 
 #include "wf_device.cuh"
 #include "wf_internal.h"
+#include "wf_skinny_mt_layout.h"
 
 namespace wf {
 
 namespace {
 
-constexpr int kMtThreads = 256;
-constexpr int kMtWarps = kMtThreads / 32;
-constexpr int kMtMaxStages = 4;
-constexpr int kMtMaxTiles = (kMtMaxRows + 2 + 15) / 16;  // 16-row tiles of the largest operand
-constexpr int kMtStageParts = 32;  // partial row sums staged per row (more are read in place)
-// shared memory a CTA may plan for: alone on its SM, or two per SM
-constexpr int kMtSmemAlone = 220 * 1024;
-constexpr int kMtSmemPair = 112 * 1024;
 constexpr int kMtQuadsPerPass = 2;  // epilogue column quads a thread finishes per pass
-
-// warp grid: unit groups x tile groups (fewest ldmatrix bytes per k-block at
-// 10 tiles: 2 x 4 for 8 units, 1 x 8 below)
-template <int U>
-struct MtGrid {
-  static constexpr int kWU = U >= 8 ? 2 : 1;
-  static constexpr int kUW = U / kWU;                        // units per warp
-  static constexpr int kWT = kMtWarps / kWU;                 // tile groups
-  static constexpr int kTW = (kMtMaxTiles + kWT - 1) / kWT;  // tiles per warp at most
-  // all of a warp's tiles' A fragments held at once (when few accumulators);
-  // a tile past the operand reads the zero line and its results are dropped
-  static constexpr bool kAllTiles = kTW * kUW <= 8;
-};
-
-// Shared-memory layout: Mr operand rows, Ks inputs, ns ring stages, at most
-// rows_o rows finished per rank.
-struct MtLayout {
-  int w_off, ring_off, stage_bytes, res_ld, part_off, old_off, bias_off, wgb_off, gn_off, stat_off, row_off,
-      bar_off, zero_off, flag_off, total;
-  __host__ __device__ MtLayout(int Mr, int Ks, int U, int ns, int rows_o, bool fold, bool resid) {
-    const int kb = Ks / 64;
-    w_off = 0;
-    ring_off = U * kb * 1024;
-    stage_bytes = (Mr * 128 + 1023) & ~1023;  // stages start 1024-aligned (the copies swizzle by address)
-    res_ld = U * 8 + 8;                       // fp32 results [Mr][U 8 + 8], over the ring once it is done
-    int region = ns * stage_bytes;
-    if (Mr * res_ld * 4 > region) region = Mr * res_ld * 4;
-    part_off = ring_off + region;
-    old_off = part_off + (fold ? rows_o * kMtStageParts * 8 : 0);
-    bias_off = old_off + (resid ? rows_o * U * 8 * 4 : 0);
-    wgb_off = bias_off + U * 8 * 4;
-    gn_off = wgb_off + 2 * U * 8 * 4;
-    stat_off = gn_off + U * 8 * 4;
-    row_off = stat_off + rows_o * 8;
-    bar_off = (row_off + rows_o * 8 + 15) & ~15;
-    zero_off = (bar_off + (1 + kMtMaxStages) * 8 + 15) & ~15;
-    flag_off = zero_off + 16;
-    total = flag_off + 16;
-  }
-};
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void *src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
@@ -512,7 +465,7 @@ __global__ void __launch_bounds__(kMtThreads, 2) skinny_mt_kernel(const __grid_c
 // ------------------------------------------------------------------ host ----
 namespace {
 size_t mt_smem(int Mr, int M, int K, int U, int S, int ns, bool fold, bool resid) {
-  return 1024 + static_cast<size_t>(MtLayout(Mr, K / S, U, ns, (M + S - 1) / S, fold, resid).total);
+  return static_cast<size_t>(mt_smem_bytes(Mr, M, K, U, S, ns, fold, resid));
 }
 
 const CUtensorMap *mt_wmap(const void *W, int N, int K, int kblocks) {
