@@ -132,7 +132,6 @@ __global__ void __launch_bounds__(kMtThreads, 2) skinny_mt_kernel(const __grid_c
       const int slot = p.seq_slot[ii];
       sRow[r] = make_int2(slot, (p.pos_base ? p.pos_base[slot] : 0) + jr);
     }
-  pdl_launch_dependents();
   __syncthreads();  // the barriers and the zero line are initialised before any thread uses them
   pdl_wait();
 
@@ -240,6 +239,9 @@ __global__ void __launch_bounds__(kMtThreads, 2) skinny_mt_kernel(const __grid_c
       tma_load_3d(ring + s * L.stage_bytes, &tmX, 0, 0, split * kb + q + ns, &full[s]);
     }
   }
+  // the next kernel may start once every CTA is past its MMAs (earlier, its
+  // prefetches slow this kernel's gather of the split-K sums: measured)
+  pdl_launch_dependents();
   // results -> shared memory over the ring (fp32 [Mr][res_ld]); lane holds
   // rows g, g + 8 and columns 2 c4, 2 c4 + 1 of each unit
   {
