@@ -89,9 +89,9 @@ GEMM_DRAM_BYTES_PER_LAUNCH = {
     # (5.514), 34 x fc1 (15.354), 2 x history K/V (8.796), 1 x history
     # projection (27.283) per step, captured at 94 sequences
     "large_b96": 13.165e6,
-    # 204 x batched skinny projections (8.594 MB), 2 x history K/V (7.346), 1 x
-    # history projection (18.182) per step, captured at 16 sequences
-    "large_b16": 8.628e6,
+    # 204 x batched skinny projections (8.593 MB), 2 x history K/V (7.346), 1 x
+    # history projection (18.194) per step, captured at 15 live sequences
+    "large_b16": 8.627e6,
 }
 
 # the projection path each capture above ran on (its traffic describes only that path)
