@@ -90,7 +90,8 @@ GEMM_DRAM_BYTES_PER_LAUNCH = {
     # projection (27.283) per step, captured at 94 sequences
     "large_b96": 13.165e6,
     # 204 x batched skinny projections (8.593 MB), 2 x history K/V (7.346), 1 x
-    # history projection (18.194) per step, captured at 15 live sequences
+    # history projection (18.194) per step, captured at 15 live sequences with
+    # --skinny (the default batch-16 path is tcgen05, which no capture covers)
     "large_b16": 8.627e6,
 }
 
@@ -306,10 +307,12 @@ def measure_greedy(args, wl_name, dev, host_ws, rank, world, steps, warmup, e2e=
     sess = Session(cfg, dev, max_batch=Bn, max_ctx=cfg.max_pos)
     if args.persist:
         B.wf_set_option(sess.h, B.WF_OPT_PERSIST, 1)
+    # the library's default form: skinny projections for single-sequence
+    # handles, tcgen05 above (--skinny: the batched skinny form up to 144 rows)
     proj_path = "tcgen05"
     if args.no_skinny:
         B.wf_set_option(sess.h, B.WF_OPT_SKINNY, 0)
-    else:
+    elif Bn * (cfg.block_k + 1) <= 14 or args.skinny:
         try:
             B.wf_set_option(sess.h, B.WF_OPT_SKINNY, 1)
             proj_path = "skinny"
@@ -756,7 +759,7 @@ def run_sampling(args, rank, world):
         "replayed_identically": replayed,
         "step_roofline": _step_roofline(m, step_ms, hbm_peak, peak_src),
         "roofline": _family_roofline(prof, n_prof, step_ms, "gemm", hbm_peak, peak_src,
-                                     _proj_kernel("skinny" if Bn * (Kc + 1) <= 144 else "tcgen05", Bn * (Kc + 1)),
+                                     _proj_kernel("skinny" if Bn * (Kc + 1) <= 14 else "tcgen05", Bn * (Kc + 1)),
                                      None),
         "kernel_families_ms_per_step": {k: v["ms"] / n_prof for k, v in prof.items()},
         "e2e": {"value": e2e_tokens / e2e_s, "unit": "tokens/s",
@@ -928,6 +931,9 @@ def main():
                     help="override every transcript budget (short profiling runs)")
     ap.add_argument("--no-skinny", action="store_true",
                     help="single-sequence handles use the tcgen05 projections (WF_OPT_SKINNY 0)")
+    ap.add_argument("--skinny", action="store_true",
+                    help="handles of up to 144 step rows use the batched skinny projections "
+                         "(WF_OPT_SKINNY 1; the default there is tcgen05)")
     ap.add_argument("--no-per-batch", action="store_true",
                     help="skip the batch-16 and batch-96 entries of the default line")
     ap.add_argument("--batch-steps", type=int, default=20,

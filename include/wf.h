@@ -244,13 +244,16 @@ int32_t wf_last_launch_count(const wf_handle *h);
                                 restores about 1 s (projections) and 0.2 s (persistent pass).
                                 Meant for tests of the failure path: a limit below a wait's
                                 normal duration makes the results of that call invalid. */
-#define WF_OPT_SKINNY 7      /* 1 (default when max_batch * (block_k + 1) <= 144): passes of
-                                at most that many token rows run their projections as
-                                low-latency kernels that hold a CTA's whole weight slab in
-                                shared memory and reduce K in a fixed order (up to 16 rows
-                                with the whole token operand resident, more with it streamed
-                                by k-block); 0: the tcgen05 projections.  Setting 1 on a
-                                larger handle returns WF_ERR_UNSUPPORTED.
+#define WF_OPT_SKINNY 7      /* 1: passes of at most max_batch * (block_k + 1) <= 144 token
+                                rows run their projections as low-latency kernels that hold
+                                a CTA's whole weight slab in shared memory and reduce K in a
+                                fixed order (up to 14 rows with the whole token operand
+                                resident, more with it streamed by k-block); 0: the tcgen05
+                                projections.  Default 1 when max_batch * (block_k + 1) <= 14
+                                (single-sequence handles), else 0 (the streamed form is
+                                slower than tcgen05 at 2-8 sequences and ties it at 16).
+                                Setting 1 on a handle of more than 144 step rows returns
+                                WF_ERR_UNSUPPORTED.
                                 The two forms agree within the method's tolerances, not bit
                                 for bit; a handle's speculative and plain greedy steps
                                 always take the same form. */

@@ -1087,7 +1087,10 @@ wf_status wf_create(const wf_config *cfg, const wf_target_weights *tw, const wf_
             launch_rope_table(h->rope, cfg->max_pos, cfg->rope_base, s) == cudaSuccess;
   h->sk_rows = max_batch * (cfg->block_k + 1);
   h->skinny_ok = skinny_shapes_fit(h->d, h->F, h->sk_rows);
-  h->skinny = h->skinny_ok;
+  // on by default where one operand tile holds a pass (single-sequence
+  // handles); the batched form (2-16 sequences) is opt-in: it measured 3-12%
+  // slower per step than the tcgen05 projections at 2-8 sequences, a tie at 16
+  h->skinny = h->skinny_ok && h->sk_rows <= kSkMaxFoldRows;
   ok = ok && gemm_init() == cudaSuccess && skinny_init() == cudaSuccess && skinny_mt_init() == cudaSuccess &&
        attention_init() == cudaSuccess &&
        step_kernels_init() == cudaSuccess &&

@@ -8,9 +8,9 @@ the cache, so the final length is at most max_ctx.  Up to that point the
 speculative transcript must equal plain greedy decoding on a handle of the
 same shape, token for token: on a single-sequence handle (skinny projections
 with the attention fused into them, which attend to the short cache in
-blocks of 32 positions) and on a two-slot handle (the batched skinny
-projections, whose K/V epilogue checks each row's position, and the separate
-attention kernel)."""
+blocks of 32 positions) and on a two-slot handle, both with the batched
+skinny projections (whose K/V epilogue checks each row's position) and with
+the tcgen05 projections, and the separate attention kernel."""
 import numpy as np
 import pytest
 
@@ -22,10 +22,12 @@ CTX = 40
 BUDGET = 60
 
 
-def _run(cfg, dev, enc, prompt, max_batch, spec):
+def _run(cfg, dev, enc, prompt, max_batch, spec, skinny):
     from paper_2609_32869_gb300 import binding as B
     from paper_2609_32869_gb300.session import Session
     s = Session(cfg, dev, max_batch=max_batch, max_ctx=CTX)
+    if skinny is not None:
+        B.wf_set_option(s.h, B.WF_OPT_SKINNY, skinny)
     slots = np.arange(max_batch, dtype=np.int32)
     first = s.prefill(slots, enc, prompt, np.full(max_batch, BUDGET, np.int32)).cpu().numpy()
     out = [[int(first[b])] for b in range(max_batch)]
@@ -42,15 +44,16 @@ def _run(cfg, dev, enc, prompt, max_batch, spec):
     return out, st, err, B
 
 
-@pytest.mark.parametrize("max_batch", [1, 2], ids=["skinny-fused", "skinny-batched"])
-def test_capacity_freezes_the_sequence_inside_the_cache(max_batch):
+@pytest.mark.parametrize("max_batch,skinny", [(1, None), (2, 1), (2, 0)],
+                         ids=["skinny-fused", "skinny-batched", "tcgen05"])
+def test_capacity_freezes_the_sequence_inside_the_cache(max_batch, skinny):
     from paper_2609_32869_gb300.session import upload_weights
     cfg = syn.TINY
     dev = upload_weights(syn.make_weights(cfg, seed=0, ln_noise=True))
     enc = syn.encoder_output(cfg, max_batch, seed=3)
     prompt = syn.prompts(cfg, max_batch, length=4, seed=3)
-    spec, st, err, B = _run(cfg, dev, enc, prompt, max_batch, spec=True)
-    plain, _, _, _ = _run(cfg, dev, enc, prompt, max_batch, spec=False)
+    spec, st, err, B = _run(cfg, dev, enc, prompt, max_batch, True, skinny)
+    plain, _, _, _ = _run(cfg, dev, enc, prompt, max_batch, False, skinny)
     K1 = cfg.block_k + 1
     for b in range(max_batch):
         assert st["done"][b]

@@ -28,8 +28,9 @@ def _forced(g, t, a, K, V):
     return cand
 
 
-@pytest.mark.parametrize("ln_noise", [False, True], ids=["ln-unit", "ln-noise"])
-def test_large_shapes_two_steps_match_oracle(ln_noise):
+@pytest.mark.parametrize("ln_noise,skinny", [(False, None), (True, None), (True, 1)],
+                         ids=["ln-unit", "ln-noise", "ln-noise-skinny-batched"])
+def test_large_shapes_two_steps_match_oracle(ln_noise, skinny):
     import torch
     from paper_2609_32869_gb300 import binding as B
     from paper_2609_32869_gb300.session import Session
@@ -43,6 +44,8 @@ def test_large_shapes_two_steps_match_oracle(ln_noise):
     checked = (0, 3)
     accept = {0: (8, 3), 3: (2, 6)}
     s = Session(cfg, ws, max_batch=n, keep_logits=True)
+    if skinny is not None:                    # the batched skinny projections (default: tcgen05)
+        B.wf_set_option(s.h, B.WF_OPT_SKINNY, skinny)
     first = s.prefill(np.arange(n, dtype=np.int32), enc, prompt, budgets).cpu().numpy()
     torch.cuda.synchronize()
     pre_logits = s.view(B.WF_VIEW_TARGET_LOGITS, torch.float32, (n, V)).cpu().numpy()

@@ -1,10 +1,10 @@
 """The low-latency projections of single-sequence handles (GPU).
 
-A handle whose every step pass has at most 144 token rows runs its
-projections with the skinny kernels (WF_OPT_SKINNY): at most 16 rows
-(max_batch 1: the anchor and K = 8 proposals) with the whole operand tile
-resident (wf_skinny.cu), more with the operand streamed by k-block
-(wf_skinny_mt.cu).  Checked against the oracle at the Whisper-tiny
+A handle whose every step pass has at most 144 token rows can run its
+projections with the skinny kernels (WF_OPT_SKINNY, on by default for
+single-sequence handles): at most 14 rows (max_batch 1: the anchor and K = 8
+proposals) with the whole operand tile resident (wf_skinny.cu), more with the
+operand streamed by k-block (wf_skinny_mt.cu).  Checked against the oracle at the Whisper-tiny
 and Whisper-large shapes with every LayerNorm's gain and bias drawn on its own:
 draft and verify logits within 3e-2, tapped hidden states within 1e-2
 relative, tokens and cache lengths equal wherever the deciding margins
