@@ -1,7 +1,8 @@
 // Projections of a batch of up to 16 sequences (Sec. 3.1: one verify block of
 // 9 rows per sequence, up to 146 operand rows with a folded LayerNorm's two
 // extra rows) on the skinny kernels' scheme, for M too large to hold the
-// whole token operand of a CTA's K range beside its weights.
+// whole token operand of a CTA's K range beside its weights.  Opt-in per
+// handle (WF_OPT_SKINNY): the tcgen05 GEMM is the default for such batches.
 //
 // Each CTA owns U units of 8 weight rows over a K range (all of K, or 1/S of
 // it in a cluster of S CTAs) and requests its whole weight slab with TMA

@@ -101,3 +101,19 @@ def test_workspace_grows_with_batch_and_context():
     per_slot = 2 * layers * 448 * d * 2 + 2 * layers * frames * d * 2
     assert two - one >= per_slot
     assert B.wf_workspace_bytes(cfg, 1, 200) < one
+
+
+def test_binding_constants_equal_the_header():
+    """Every numeric #define and status code of include/wf.h that the binding
+    names has the header's value (options, views, error bits, families)."""
+    from paper_2609_32869_gb300 import binding as B
+    src = open(os.path.join(ROOT, "include", "wf.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    values = {m.group(1): int(m.group(2), 0)
+              for m in re.finditer(r"#define\s+(WF_[A-Z0-9_]+)\s+(0x[0-9a-fA-F]+|\d+)u?\b", src)}
+    values.update({m.group(1): int(m.group(2)) for m in re.finditer(r"\b(WF_[A-Z_]+)\s*=\s*(\d+)", src)})
+    assert len(values) >= 20
+    named = {k: v for k, v in values.items() if hasattr(B, k)}
+    assert {"WF_OPT_SKINNY", "WF_DEV_ERR_TIMEOUT", "WF_DEV_ERR_LAUNCH", "WF_ERR_CUDA"} <= set(named)
+    for k, v in named.items():
+        assert getattr(B, k) == v, k
